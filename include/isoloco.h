@@ -1,0 +1,164 @@
+/*
+ * isoloco.h -- C ABI of the GB300-native IsoLoCo / DiLoCo outer step.
+ *
+ * Method: "Can Model Merging Improve Aggregation in DiLoCo?" (arXiv 2607.03011).
+ *   Alg. 1 (DiLoCo):  Delta = (1/R) sum_i (theta^{t-1} - theta_i^{t}); OuterOpt = SGD
+ *                     with Nesterov momentum.
+ *   Alg. 2 (IsoLoCo): mean pseudo-gradient; every 2-D tensor is replaced by its Iso-C
+ *                     correction sigma_bar * U V^T (U S V^T = SVD(Delta),
+ *                     sigma_bar = mean of the singular values); then
+ *                     B <- mu B + Delta, P <- Delta + mu B, theta <- theta - eta_out P.
+ *   Sec. 2.2, Eq. 1:  task-arithmetic merging theta_0 + lambda sum_t tau_t; Iso-C sums
+ *                     the task matrices and flattens their spectrum.
+ *
+ * The polar factor U V^T is computed without an SVD: a batched Newton-Schulz-type
+ * iteration X <- X (a I + b X^T X + c (X^T X)^2) on tcgen05 tensor cores (Sec. 4.3
+ * uses Newton-Schulz for the same purpose), and sigma_bar = tr(Q^T Delta) / min(m, n),
+ * which equals the mean singular value exactly when Q is the polar factor.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - All tensors live in ONE flat fp32 buffer per role (theta, momentum, output),
+ *   described by a parameter table; parameter p occupies elements
+ *   [offset, offset + rows * max(cols, 1)).  cols == 0 marks a 1-D tensor of
+ *   `rows` elements; every other entry is a row-major rows x cols matrix.
+ * - Worker replicas are K more flat buffers of the same layout, fp32 or bf16,
+ *   passed as a HOST array of K DEVICE pointers.  They are only read.
+ * - Pointers are device pointers, 16-byte aligned, unless the name says host.
+ *   The caller owns them; the library never frees or keeps them past a call.
+ * - `stream` is a cudaStream_t (NULL = legacy default stream).  Calls enqueue work
+ *   and return without waiting, unless opts->sync is set.  A plan's workspace is
+ *   used by one call at a time: calls on the same plan from different streams
+ *   must be ordered by the caller.
+ * - Return values are isoloco_status_t codes.  No C++ exception crosses the ABI.
+ *   isoloco_last_error() gives a thread-local message for the last failure.
+ * - Sign convention (Alg. 1/2): Delta_k = theta - theta_k, and theta moves by
+ *   -eta_out * P.  iso_c_merge uses task vectors tau_k = theta_k - theta_base.
+ */
+#ifndef ISOLOCO_H_
+#define ISOLOCO_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct isoloco_plan* isoloco_plan_t;
+
+/* One tensor of the parameter table (see conventions above). */
+typedef struct {
+    int64_t offset;
+    int32_t rows;
+    int32_t cols;
+} isoloco_param_t;
+
+/* Element type of the worker replicas (bf16 is upcast exactly to fp32). */
+typedef enum { ISOLOCO_F32 = 0, ISOLOCO_BF16 = 1 } isoloco_dtype_t;
+
+typedef enum {
+    ISOLOCO_OK = 0,
+    ISOLOCO_ERR_INVALID = -1,       /* bad argument, table or plan; nothing launched */
+    ISOLOCO_ERR_ALIGN = -2,         /* a pointer is not 16-byte aligned; nothing launched */
+    ISOLOCO_ERR_NONFINITE = -3,     /* NaN/Inf in the pseudo-gradient: theta, B untouched */
+    ISOLOCO_ERR_NOT_CONVERGED = -4, /* a polar iteration hit max_iter (update still applied) */
+    ISOLOCO_ERR_CUDA = -5,          /* a CUDA runtime call failed */
+    ISOLOCO_ERR_OOM = -6,           /* workspace allocation failed */
+    ISOLOCO_ERR_TIMEOUT = -7        /* a device-side wait gave up (kernel returned early) */
+} isoloco_status_t;
+
+/* Options of one outer step (Alg. 2's hyperparameters plus solver controls). */
+typedef struct {
+    float alpha;      /* Iso-C scale (Eq. 1's lambda); multiplies the 2-D output only. */
+    float outer_lr;   /* eta_out of Alg. 2. */
+    float momentum;   /* mu of Alg. 2 (0 = plain SGD outer step, Eq. 2). */
+    int reduce_mean;  /* 1: Delta is the mean over workers (Alg. 1/2); 0: the sum. */
+    int max_iter;     /* cap on polar iterations per matrix; <= 0 selects 29. */
+    float tol;        /* convergence test ||X^T X - I||_F / sqrt(n) < tol; <= 0 selects 4e-3. */
+    int sync;         /* 1: synchronize `stream` and return the step's device status. */
+} isoloco_opts_t;
+
+/* Fills *opts with alpha = 1, outer_lr = 0.7, momentum = 0.9 (the paper's DiLoCo
+ * optimum at R = 8, App. A Table 6), reduce_mean = 1, default solver controls. */
+int isoloco_opts_default(isoloco_opts_t* opts);
+
+/* Creates a plan for a parameter table.
+ *   table[n_params]: copied; tensors must lie inside [0, n_total) and not overlap.
+ *   K: number of worker replicas (1..64).  replica_dtype: their element type.
+ * Allocates the device workspace (Delta, polar iterates, Gram and polynomial
+ * buffers, per-matrix state) on the current device, and builds the TMA
+ * descriptors.  Returns OK, INVALID, OOM or CUDA; *plan is NULL on failure. */
+int isoloco_plan_create(isoloco_plan_t* plan, const isoloco_param_t* table, int n_params,
+                        int64_t n_total, int K, isoloco_dtype_t replica_dtype);
+
+/* Frees the plan and its workspace (synchronizes the device first). */
+void isoloco_plan_destroy(isoloco_plan_t plan);
+
+/* Device bytes held by the plan's workspace. */
+int64_t isoloco_plan_workspace_bytes(isoloco_plan_t plan);
+
+/* IsoLoCo outer step, Alg. 2.
+ *   theta[n_total], momentum[n_total]: fp32, read and overwritten in place.
+ *   replicas: host array of K device pointers (the plan's dtype), read only.
+ *   update_out: nullable fp32 [n_total]; if given, receives the update direction
+ *     U (alpha * sigma_bar * Q for 2-D tensors, the mean Delta for 1-D ones).
+ * On a non-finite pseudo-gradient nothing is written and the step's status is
+ * NONFINITE.  Asynchronous unless opts->sync. */
+int isoloco_outer_step(isoloco_plan_t plan, float* theta, float* momentum,
+                       const void* const* replicas, const isoloco_opts_t* opts, void* stream,
+                       float* update_out);
+
+/* Same step with every buffer in HOST memory (pinned memory is fastest): the
+ * call copies theta, momentum and the replicas to plan-owned device buffers,
+ * runs the step and copies theta and momentum back, all on `stream`, and
+ * synchronizes before returning the step's status. */
+int isoloco_outer_step_host(isoloco_plan_t plan, float* theta_host, float* momentum_host,
+                            const void* const* replicas_host, const isoloco_opts_t* opts,
+                            void* stream);
+
+/* DiLoCo outer step, Alg. 1 with Nesterov SGD: one streaming pass over every
+ * parameter (no Iso-C).  Elementwise, so a non-finite input only affects its own
+ * element; the step's status reports it. */
+int diloco_outer_step(isoloco_plan_t plan, float* theta, float* momentum,
+                      const void* const* replicas, const isoloco_opts_t* opts, void* stream);
+
+/* Iso-C model merging (Sec. 2.2, Eq. 1 form): tau_k = experts_k - theta_base,
+ * T = sum_k tau_k;  out = theta_base + alpha * IsoC(T) for 2-D tensors and
+ * out = theta_base + alpha * T for 1-D tensors.  out[n_total] fp32 may alias
+ * nothing else.  The plan's K is the number of experts. */
+int iso_c_merge(isoloco_plan_t plan, const float* theta_base, const void* const* experts,
+                float alpha, float* out, void* stream);
+
+/* Synchronizes `stream` and returns the device status of the plan's last call. */
+int isoloco_last_status(isoloco_plan_t plan, void* stream);
+
+/* Per-matrix diagnostics of the last call, in table order over the 2-D tensors
+ * only (n_matrices entries each; any pointer may be NULL).  Synchronizes `stream`.
+ *   sigma_bar: tr(Q^T Delta) / min(m, n);  iters: polar iterations used;
+ *   status: 0 or NOT_CONVERGED;  residual: last ||X^T X - I||_F / sqrt(n). */
+int isoloco_read_diag(isoloco_plan_t plan, void* stream, float* sigma_bar_host,
+                      int32_t* iters_host, int32_t* status_host, float* residual_host);
+
+/* Number of 2-D tensors in the plan's table. */
+int isoloco_plan_num_matrices(isoloco_plan_t plan);
+
+/* Batched split-precision GEMM of the polar iteration, exposed for testing:
+ *   D[b] = op(A[b]) op(B[b])^T-free product with fp32 inputs split into bf16
+ *   hi + lo parts and three tcgen05 passes (hi*hi + hi*lo + lo*hi), fp32
+ *   accumulation in tensor memory.
+ *   a_mn_major = 0: A[b] is row-major M x K;  1: A[b] is row-major K x M.
+ *   b_mn_major = 0: B[b] is row-major N x K;  1: B[b] is row-major K x N.
+ *   D[b] is row-major M x N fp32:  D[b][i][j] = sum_k A(i,k) B(j,k).
+ * All pointers are device fp32, contiguous per batch.  Allocates scratch with
+ * cudaMalloc and synchronizes `stream` before returning. */
+int isoloco_debug_gemm(int a_mn_major, int b_mn_major, int batch, int M, int N, int K,
+                       const float* A, const float* B, float* D, void* stream);
+
+/* Thread-local message describing the last error returned on this thread. */
+const char* isoloco_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ISOLOCO_H_ */

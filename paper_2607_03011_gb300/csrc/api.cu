@@ -1,0 +1,814 @@
+// api.cu -- plan (bucketing, workspace, TMA descriptors), launch sequencing and the
+// C ABI declared in include/isoloco.h.
+//
+// One IsoLoCo outer step (Alg. 2) on a stream:
+//   k_reset_state -> k_reduce (Delta, all tensors)
+//   for t = 0..max_iter:   Gram X^T X (tcgen05) -> k_gram_finalize -> k_control
+//                          -> G^2 with P = a I + b G + c G^2 epilogue (tcgen05)
+//                          -> X P (tcgen05)  [matrices that finished exit at once]
+//   k_trace_partial -> k_trace_final (sigma_bar) -> k_apply (Nesterov) -> status copy
+// Every kernel reads its per-matrix decisions from device memory: the host never
+// waits inside a step.
+#include <algorithm>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <map>
+#include <string>
+#include <vector>
+
+#include "common.cuh"
+#include "isoloco.h"
+#include "types.h"
+
+namespace isoloco {
+
+// kernels defined in the other translation units
+cudaError_t launch_gemm(const GemmParams& p, bool a_mn, bool b_mn, cudaStream_t stream);
+__global__ void k_gram_finalize(const MatDesc*, const int2*, const MatState*, const float*, const int64_t*,
+                                const int64_t*, const int*, float*, __nv_bfloat16*, __nv_bfloat16*, float*);
+__global__ void k_control(const MatDesc*, int, MatState*, const float*, int, int, float, uint32_t*);
+__global__ void k_trace_partial(const MatDesc*, const int4*, const MatState*, const __nv_bfloat16*,
+                                const __nv_bfloat16*, const __nv_bfloat16*, const __nv_bfloat16*,
+                                const __nv_bfloat16*, const __nv_bfloat16*, double*);
+__global__ void k_trace_final(const MatDesc*, int, MatState*, const double*);
+__global__ void k_reset_state(MatState*, int, uint32_t*);
+__global__ void k_reduce(const Chunk*, const MatDesc*, ReplicaPtrs, int, int, const float*, float,
+                         __nv_bfloat16*, __nv_bfloat16*, float*, uint32_t*);
+__global__ void k_apply(const Chunk*, const MatDesc*, const MatState*, UpdateSrc, int, float, float, float,
+                        float*, float*, const float*, float*, float*, const uint32_t*);
+__global__ void k_diloco(ReplicaPtrs, int, int, float*, float*, int64_t, float, float, float, uint32_t*);
+__global__ void k_split_planes(const float*, int64_t, int, int, int, __nv_bfloat16*, __nv_bfloat16*);
+
+constexpr int kChunkElems = 16384;
+constexpr int kTraceChunkElems = 16384;
+constexpr int kFinTileEdge = 64;
+constexpr int kDefaultMaxIter = 28;
+constexpr float kDefaultTol = 4e-3f;
+
+// Roles of the tensor maps of one bucket.
+enum MapRole { kRoleKA = 0, kRoleKB = 1, kRoleMN = 2 };
+constexpr int kMapsPerBucket = 26;  // 3 sources x 3 roles x 2 planes + G (2x2) + P (2x2)
+inline int src_map(int src, int role, int plane) { return (src * 3 + role) * 2 + plane; }
+inline int g_map(int role, int plane) { return 18 + role * 2 + plane; }
+inline int p_map(int role, int plane) { return 22 + role * 2 + plane; }
+
+struct Bucket {
+    int rows, cols, ld, n, ld_n, count;
+    bool tall;
+    int mat_base;
+    int64_t plane_off, gplane_off, gpart_off;
+    int splits;
+};
+
+}  // namespace isoloco
+
+using namespace isoloco;
+
+struct isoloco_plan {
+    int device = 0;
+    int num_sms = 148;
+    int K = 0;
+    int dtype = 0;
+    int64_t N = 0;
+    std::vector<isoloco_param_t> table;
+    std::vector<int> mat_param;
+    std::vector<MatDesc> mats_h;
+    std::vector<Bucket> buckets;
+    int nmat = 0, nchunks = 0, nftiles = 0, ntchunks = 0;
+    int64_t plane_elems = 0, gplane_elems = 0, gpart_elems = 0, n1d = 0;
+    // device workspace
+    std::vector<void*> allocs;
+    int64_t ws_bytes = 0;
+    __nv_bfloat16 *dhi = nullptr, *dlo = nullptr, *xhi[2] = {nullptr, nullptr}, *xlo[2] = {nullptr, nullptr};
+    float* gf32 = nullptr;
+    __nv_bfloat16 *ghi = nullptr, *glo = nullptr, *phi = nullptr, *plo = nullptr;
+    float* gpart = nullptr;
+    float* d1d = nullptr;
+    float* fin_part = nullptr;
+    int2* ftiles = nullptr;
+    double* tpart = nullptr;
+    int4* tchunks = nullptr;
+    MatState* state = nullptr;
+    MatDesc* mats_d = nullptr;
+    int64_t* gpart_off_d = nullptr;
+    int64_t* gpart_sstride_d = nullptr;
+    int* nsplit_d = nullptr;
+    Chunk* chunks_d = nullptr;
+    uint32_t* err_d = nullptr;
+    uint32_t* err_h = nullptr;  // pinned
+    CUtensorMap* tmaps_d = nullptr;
+    cudaEvent_t done_ev = nullptr;
+    // staging for the host-buffer entry point (allocated on first use)
+    float* st_theta = nullptr;
+    float* st_mom = nullptr;
+    void* st_reps = nullptr;
+};
+
+// ------------------------------------------------------------------ errors
+static thread_local std::string g_last_error;
+
+static int fail(int code, const std::string& msg) {
+    g_last_error = msg;
+    return code;
+}
+
+#define CUDA_TRY(expr)                                                                        \
+    do {                                                                                      \
+        cudaError_t _e = (expr);                                                              \
+        if (_e != cudaSuccess)                                                                \
+            return fail(ISOLOCO_ERR_CUDA, std::string(#expr) + ": " + cudaGetErrorString(_e)); \
+    } while (0)
+
+// ------------------------------------------------------------------ tensor maps
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
+    return fn;
+}
+
+// 3-D bf16 map over [count][rows][ld] with logical extent cols x rows x count.
+static bool make_map(CUtensorMap* m, const void* base, int cols, int rows, int count, int ld, int role) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)cols, (cuuint64_t)rows, (cuuint64_t)count};
+    cuuint64_t strides[2] = {(cuuint64_t)ld * 2, (cuuint64_t)rows * ld * 2};
+    cuuint32_t box[3];
+    CUtensorMapSwizzle sw;
+    if (role == kRoleMN) {
+        box[0] = 64; box[1] = BK; sw = CU_TENSOR_MAP_SWIZZLE_128B;
+    } else {
+        box[0] = BK; box[1] = (role == kRoleKA) ? BM : BN; sw = CU_TENSOR_MAP_SWIZZLE_64B;
+    }
+    box[2] = 1;
+    cuuint32_t es[3] = {1, 1, 1};
+    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+static inline int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
+
+template <typename T>
+static int dalloc(isoloco_plan* p, T** ptr, int64_t count) {
+    *ptr = nullptr;
+    if (count <= 0) count = 1;
+    const size_t bytes = static_cast<size_t>(count) * sizeof(T);
+    cudaError_t e = cudaMalloc(reinterpret_cast<void**>(ptr), bytes);
+    if (e != cudaSuccess) {
+        (void)cudaGetLastError();
+        return fail(ISOLOCO_ERR_OOM, std::string("cudaMalloc of ") + std::to_string(bytes) + " bytes failed");
+    }
+    p->allocs.push_back(*ptr);
+    p->ws_bytes += static_cast<int64_t>(bytes);
+    return ISOLOCO_OK;
+}
+
+static void free_plan(isoloco_plan* p) {
+    if (!p) return;
+    for (void* a : p->allocs) cudaFree(a);
+    if (p->err_h) cudaFreeHost(p->err_h);
+    if (p->done_ev) cudaEventDestroy(p->done_ev);
+    delete p;
+}
+
+static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// ------------------------------------------------------------------ plan creation
+static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_params) {
+    // --- matrices and buckets
+    std::map<std::pair<int, int>, int> bucket_of;
+    std::vector<std::vector<int>> members;
+    for (int i = 0; i < n_params; ++i) {
+        const isoloco_param_t& t = table[i];
+        if (t.cols > 0) {
+            auto key = std::make_pair((int)t.rows, (int)t.cols);
+            auto it = bucket_of.find(key);
+            int b;
+            if (it == bucket_of.end()) {
+                b = (int)p->buckets.size();
+                bucket_of[key] = b;
+                Bucket bk{};
+                bk.rows = t.rows;
+                bk.cols = t.cols;
+                bk.ld = (int)round_up(t.cols, 8);
+                bk.n = std::min(t.rows, t.cols);
+                bk.ld_n = (int)round_up(bk.n, 8);
+                bk.tall = t.rows >= t.cols;
+                p->buckets.push_back(bk);
+                members.emplace_back();
+            } else {
+                b = it->second;
+            }
+            members[b].push_back(i);
+        }
+    }
+    // matrices ordered bucket by bucket so each bucket's slots are contiguous
+    std::vector<int> mat_of_param(n_params, -1);
+    int64_t plane = 0, gplane = 0, gpart = 0, fin = 0, tr = 0;
+    std::vector<int2> ftiles;
+    std::vector<int4> tchunks;
+    std::vector<int64_t> gpoff, gpss;
+    std::vector<int> nsp;
+    for (size_t b = 0; b < p->buckets.size(); ++b) {
+        Bucket& bk = p->buckets[b];
+        bk.count = (int)members[b].size();
+        bk.mat_base = (int)p->mats_h.size();
+        bk.plane_off = plane;
+        bk.gplane_off = gplane;
+        bk.gpart_off = gpart;
+        // split-K for the Gram when the bucket has few output tiles
+        const int tiles = ((bk.n + BM - 1) / BM) * ((bk.n + BN - 1) / BN) * bk.count;
+        const int kdim = bk.tall ? bk.rows : bk.cols;
+        const int kblocks = (kdim + BK - 1) / BK;
+        int splits = std::max(1, (2 * p->num_sms) / std::max(1, tiles));
+        splits = std::min(splits, std::max(1, kblocks / 8));
+        int kper = (kblocks + splits - 1) / splits;
+        splits = (kblocks + kper - 1) / kper;  // no empty split
+        bk.splits = splits;
+        const int64_t mat_elems = (int64_t)bk.rows * bk.ld;
+        const int64_t g_elems = (int64_t)bk.n * bk.ld_n;
+        const int ftc = (bk.n + kFinTileEdge - 1) / kFinTileEdge;
+        for (int j = 0; j < bk.count; ++j) {
+            const int pi = members[b][j];
+            MatDesc md{};
+            md.param_offset = table[pi].offset;
+            md.slot = plane + j * mat_elems;
+            md.rows = bk.rows;
+            md.cols = bk.cols;
+            md.ld = bk.ld;
+            md.n = bk.n;
+            md.ld_n = bk.ld_n;
+            md.bucket = (int)b;
+            md.gslot = gplane + j * g_elems;
+            md.gpart_slot = fin;
+            md.n_gtiles = ftc * ftc;
+            md.trace_part = tr;
+            const int rows_per = std::max(1, kTraceChunkElems / bk.cols);
+            md.n_tchunks = (bk.rows + rows_per - 1) / rows_per;
+            const int mi = (int)p->mats_h.size();
+            for (int t = 0; t < md.n_gtiles; ++t) ftiles.push_back(make_int2(mi, t));
+            for (int c = 0; c < md.n_tchunks; ++c) {
+                const int r0 = c * rows_per;
+                tchunks.push_back(make_int4(mi, r0, std::min(rows_per, bk.rows - r0), c));
+            }
+            fin += md.n_gtiles;
+            tr += md.n_tchunks;
+            gpoff.push_back(gpart + j * g_elems);
+            gpss.push_back((int64_t)bk.count * g_elems);
+            nsp.push_back(splits);
+            mat_of_param[pi] = mi;
+            p->mat_param.push_back(pi);
+            p->mats_h.push_back(md);
+        }
+        plane += round_up((int64_t)bk.count * mat_elems, 128);
+        gplane += round_up((int64_t)bk.count * g_elems, 128);
+        gpart += round_up((int64_t)splits * bk.count * g_elems, 128);
+    }
+    p->nmat = (int)p->mats_h.size();
+    p->plane_elems = plane;
+    p->gplane_elems = gplane;
+    p->gpart_elems = gpart;
+    p->nftiles = (int)ftiles.size();
+    p->ntchunks = (int)tchunks.size();
+
+    // --- streaming chunks (table order) and the 1-D workspace
+    std::vector<Chunk> chunks;
+    int64_t d1 = 0;
+    for (int i = 0; i < n_params; ++i) {
+        const isoloco_param_t& t = table[i];
+        const int64_t len = (int64_t)t.rows * (t.cols > 0 ? t.cols : 1);
+        int64_t dst = 0;
+        if (t.cols == 0) {
+            dst = d1;
+            d1 += round_up(len, 4);
+        }
+        for (int64_t e = 0; e < len; e += kChunkElems) {
+            Chunk c{};
+            c.flat_begin = t.offset + e;
+            c.count = (int32_t)std::min<int64_t>(kChunkElems, len - e);
+            c.param = i;
+            c.matrix = mat_of_param[i];
+            c.elem_begin = (int32_t)e;
+            c.dst = dst + e;
+            chunks.push_back(c);
+        }
+    }
+    p->n1d = d1;
+    p->nchunks = (int)chunks.size();
+
+    // --- allocations
+    int rc;
+    if ((rc = dalloc(p, &p->dhi, plane)) || (rc = dalloc(p, &p->dlo, plane)) || (rc = dalloc(p, &p->xhi[0], plane)) ||
+        (rc = dalloc(p, &p->xlo[0], plane)) || (rc = dalloc(p, &p->xhi[1], plane)) ||
+        (rc = dalloc(p, &p->xlo[1], plane)) || (rc = dalloc(p, &p->gf32, gplane)) ||
+        (rc = dalloc(p, &p->ghi, gplane)) || (rc = dalloc(p, &p->glo, gplane)) || (rc = dalloc(p, &p->phi, gplane)) ||
+        (rc = dalloc(p, &p->plo, gplane)) || (rc = dalloc(p, &p->gpart, gpart)) || (rc = dalloc(p, &p->d1d, d1)) ||
+        (rc = dalloc(p, &p->fin_part, 3 * fin)) || (rc = dalloc(p, &p->ftiles, fin)) ||
+        (rc = dalloc(p, &p->tpart, tr)) || (rc = dalloc(p, &p->tchunks, tr)) ||
+        (rc = dalloc(p, &p->state, p->nmat)) || (rc = dalloc(p, &p->mats_d, p->nmat)) ||
+        (rc = dalloc(p, &p->gpart_off_d, p->nmat)) || (rc = dalloc(p, &p->gpart_sstride_d, p->nmat)) ||
+        (rc = dalloc(p, &p->nsplit_d, p->nmat)) || (rc = dalloc(p, &p->chunks_d, p->nchunks)) ||
+        (rc = dalloc(p, &p->err_d, 1)) ||
+        (rc = dalloc(p, &p->tmaps_d, (int64_t)kMapsPerBucket * std::max<size_t>(1, p->buckets.size()))))
+        return rc;
+    CUDA_TRY(cudaHostAlloc(reinterpret_cast<void**>(&p->err_h), sizeof(uint32_t), cudaHostAllocDefault));
+    *p->err_h = 0;
+    CUDA_TRY(cudaEventCreateWithFlags(&p->done_ev, cudaEventDisableTiming));
+    // zero the planes once so that padding columns hold zeros
+    for (void* a : {(void*)p->dhi, (void*)p->dlo, (void*)p->xhi[0], (void*)p->xlo[0], (void*)p->xhi[1],
+                    (void*)p->xlo[1]})
+        CUDA_TRY(cudaMemset(a, 0, std::max<int64_t>(1, plane) * 2));
+    for (void* a : {(void*)p->ghi, (void*)p->glo, (void*)p->phi, (void*)p->plo})
+        CUDA_TRY(cudaMemset(a, 0, std::max<int64_t>(1, gplane) * 2));
+    CUDA_TRY(cudaMemset(p->gf32, 0, std::max<int64_t>(1, gplane) * 4));
+    CUDA_TRY(cudaMemset(p->err_d, 0, 4));
+    if (p->nmat) {
+        CUDA_TRY(cudaMemcpy(p->mats_d, p->mats_h.data(), sizeof(MatDesc) * p->nmat, cudaMemcpyHostToDevice));
+        CUDA_TRY(cudaMemcpy(p->gpart_off_d, gpoff.data(), sizeof(int64_t) * p->nmat, cudaMemcpyHostToDevice));
+        CUDA_TRY(cudaMemcpy(p->gpart_sstride_d, gpss.data(), sizeof(int64_t) * p->nmat, cudaMemcpyHostToDevice));
+        CUDA_TRY(cudaMemcpy(p->nsplit_d, nsp.data(), sizeof(int) * p->nmat, cudaMemcpyHostToDevice));
+        CUDA_TRY(cudaMemcpy(p->ftiles, ftiles.data(), sizeof(int2) * fin, cudaMemcpyHostToDevice));
+        CUDA_TRY(cudaMemcpy(p->tchunks, tchunks.data(), sizeof(int4) * tr, cudaMemcpyHostToDevice));
+    }
+    if (p->nchunks)
+        CUDA_TRY(cudaMemcpy(p->chunks_d, chunks.data(), sizeof(Chunk) * p->nchunks, cudaMemcpyHostToDevice));
+
+    // --- tensor maps
+    if (!p->buckets.empty()) {
+        std::vector<CUtensorMap> maps(kMapsPerBucket * p->buckets.size());
+        for (size_t b = 0; b < p->buckets.size(); ++b) {
+            const Bucket& bk = p->buckets[b];
+            CUtensorMap* m = &maps[b * kMapsPerBucket];
+            const __nv_bfloat16* src_hi[3] = {p->dhi, p->xhi[0], p->xhi[1]};
+            const __nv_bfloat16* src_lo[3] = {p->dlo, p->xlo[0], p->xlo[1]};
+            for (int s = 0; s < 3; ++s)
+                for (int role = 0; role < 3; ++role)
+                    for (int pl = 0; pl < 2; ++pl) {
+                        const __nv_bfloat16* base = (pl == 0 ? src_hi[s] : src_lo[s]) + bk.plane_off;
+                        if (!make_map(&m[src_map(s, role, pl)], base, bk.cols, bk.rows, bk.count, bk.ld, role))
+                            return fail(ISOLOCO_ERR_CUDA, "cuTensorMapEncodeTiled failed (iterate planes)");
+                    }
+            for (int role = 0; role < 2; ++role)
+                for (int pl = 0; pl < 2; ++pl) {
+                    if (!make_map(&m[g_map(role, pl)], (pl == 0 ? p->ghi : p->glo) + bk.gplane_off, bk.n, bk.n,
+                                  bk.count, bk.ld_n, role) ||
+                        !make_map(&m[p_map(role, pl)], (pl == 0 ? p->phi : p->plo) + bk.gplane_off, bk.n, bk.n,
+                                  bk.count, bk.ld_n, role))
+                        return fail(ISOLOCO_ERR_CUDA, "cuTensorMapEncodeTiled failed (Gram planes)");
+                }
+        }
+        CUDA_TRY(cudaMemcpy(p->tmaps_d, maps.data(), sizeof(CUtensorMap) * maps.size(), cudaMemcpyHostToDevice));
+    }
+    CUDA_TRY(cudaDeviceSynchronize());
+    return ISOLOCO_OK;
+}
+
+// ------------------------------------------------------------------ launch helpers
+static void set_group_common(GemmGroup& g, int M, int N, int K, int batch, int splits, int mat_base) {
+    g.M = M;
+    g.N = N;
+    g.K = K;
+    g.batch = batch;
+    g.tiles_m = (M + BM - 1) / BM;
+    g.tiles_n = (N + BN - 1) / BN;
+    const int kblocks = (K + BK - 1) / BK;
+    g.kblocks_per_split = (kblocks + splits - 1) / splits;
+    g.splits = splits;
+    g.mat_base = mat_base;
+}
+
+struct LaunchSet {
+    GemmParams p;
+    int cta = 0;
+    void add(const GemmGroup& g) {
+        p.g[p.num_groups] = g;
+        p.g[p.num_groups].cta_begin = cta;
+        cta += g.batch * g.tiles_m * g.tiles_n * g.splits;
+        p.num_groups++;
+    }
+};
+
+static void init_set(LaunchSet& s, int epi, int gate, isoloco_plan* pl) {
+    memset(&s.p, 0, sizeof(s.p));
+    s.cta = 0;
+    s.p.epi = epi;
+    s.p.gate = gate;
+    s.p.state = pl->state;
+    s.p.err = pl->err_d;
+}
+
+static int flush_set(LaunchSet& s, bool a_mn, bool b_mn, cudaStream_t st) {
+    if (s.p.num_groups == 0) return ISOLOCO_OK;
+    CUDA_TRY(launch_gemm(s.p, a_mn, b_mn, st));
+    return ISOLOCO_OK;
+}
+
+// The polar iteration for every matrix, from Delta (planes dhi/dlo) to Q and sigma_bar.
+static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) {
+    if (p->nmat == 0) return ISOLOCO_OK;
+    const CUtensorMap* maps = p->tmaps_d;
+    for (int t = 0; t <= max_iter; ++t) {
+        const int src = (t == 0) ? 0 : 1 + (t & 1);  // Delta, X0 or X1 as the current iterate
+        const int dst = (t + 1) & 1;
+        // ---- Gram G = X^T X (tall, MN-major operands) or X X^T (wide, K-major)
+        LaunchSet tall, wide;
+        init_set(tall, kEpiF32, kGateActive, p);
+        init_set(wide, kEpiF32, kGateActive, p);
+        for (size_t b = 0; b < p->buckets.size(); ++b) {
+            const Bucket& bk = p->buckets[b];
+            const CUtensorMap* m = maps + b * kMapsPerBucket;
+            GemmGroup g{};
+            const int role_a = bk.tall ? kRoleMN : kRoleKA;
+            const int role_b = bk.tall ? kRoleMN : kRoleKB;
+            g.a_hi = m + src_map(src, role_a, 0);
+            g.a_lo = m + src_map(src, role_a, 1);
+            g.b_hi = m + src_map(src, role_b, 0);
+            g.b_lo = m + src_map(src, role_b, 1);
+            set_group_common(g, bk.n, bk.n, bk.tall ? bk.rows : bk.cols, bk.count, bk.splits, bk.mat_base);
+            g.out_f32 = p->gpart + bk.gpart_off;
+            g.f32_batch_stride = (int64_t)bk.n * bk.ld_n;
+            g.f32_split_stride = (int64_t)bk.count * bk.n * bk.ld_n;
+            g.ld_f32 = bk.ld_n;
+            (bk.tall ? tall : wide).add(g);
+        }
+        int rc;
+        if ((rc = flush_set(tall, true, true, st)) || (rc = flush_set(wide, false, false, st))) return rc;
+        k_gram_finalize<<<p->nftiles, 256, 0, st>>>(p->mats_d, p->ftiles, p->state, p->gpart, p->gpart_off_d,
+                                                    p->gpart_sstride_d, p->nsplit_d, p->gf32, p->ghi, p->glo,
+                                                    p->fin_part);
+        CUDA_TRY(cudaGetLastError());
+        k_control<<<(p->nmat + 7) / 8, 256, 0, st>>>(p->mats_d, p->nmat, p->state, p->fin_part, t, max_iter, tol,
+                                                     p->err_d);
+        CUDA_TRY(cudaGetLastError());
+        // ---- P = a I + b G + c G^2
+        LaunchSet poly;
+        init_set(poly, kEpiPoly, kGateStep, p);
+        for (size_t b = 0; b < p->buckets.size(); ++b) {
+            const Bucket& bk = p->buckets[b];
+            const CUtensorMap* m = maps + b * kMapsPerBucket;
+            GemmGroup g{};
+            g.a_hi = m + g_map(kRoleKA, 0);
+            g.a_lo = m + g_map(kRoleKA, 1);
+            g.b_hi = m + g_map(kRoleKB, 0);
+            g.b_lo = m + g_map(kRoleKB, 1);
+            set_group_common(g, bk.n, bk.n, bk.n, bk.count, 1, bk.mat_base);
+            g.out_hi = p->phi + bk.gplane_off;
+            g.out_lo = p->plo + bk.gplane_off;
+            g.bf_batch_stride = (int64_t)bk.n * bk.ld_n;
+            g.ld_bf = bk.ld_n;
+            g.g_f32 = p->gf32 + bk.gplane_off;
+            g.g_batch_stride = (int64_t)bk.n * bk.ld_n;
+            g.ld_g = bk.ld_n;
+            poly.add(g);
+        }
+        if ((rc = flush_set(poly, false, false, st))) return rc;
+        // ---- X_{t+1} = xscale * X_t P (tall) or P X_t (wide)
+        LaunchSet utall, uwide;
+        init_set(utall, kEpiXSplit, kGateStep, p);
+        init_set(uwide, kEpiXSplit, kGateStep, p);
+        for (size_t b = 0; b < p->buckets.size(); ++b) {
+            const Bucket& bk = p->buckets[b];
+            const CUtensorMap* m = maps + b * kMapsPerBucket;
+            GemmGroup g{};
+            if (bk.tall) {
+                g.a_hi = m + src_map(src, kRoleKA, 0);
+                g.a_lo = m + src_map(src, kRoleKA, 1);
+                g.b_hi = m + p_map(kRoleKB, 0);
+                g.b_lo = m + p_map(kRoleKB, 1);
+            } else {
+                g.a_hi = m + p_map(kRoleKA, 0);
+                g.a_lo = m + p_map(kRoleKA, 1);
+                g.b_hi = m + src_map(src, kRoleMN, 0);
+                g.b_lo = m + src_map(src, kRoleMN, 1);
+            }
+            set_group_common(g, bk.rows, bk.cols, bk.n, bk.count, 1, bk.mat_base);
+            g.out_hi = p->xhi[dst] + bk.plane_off;
+            g.out_lo = p->xlo[dst] + bk.plane_off;
+            g.bf_batch_stride = (int64_t)bk.rows * bk.ld;
+            g.ld_bf = bk.ld;
+            (bk.tall ? utall : uwide).add(g);
+        }
+        if ((rc = flush_set(utall, false, false, st)) || (rc = flush_set(uwide, false, true, st))) return rc;
+    }
+    k_trace_partial<<<p->ntchunks, 256, 0, st>>>(p->mats_d, p->tchunks, p->state, p->dhi, p->dlo, p->xhi[0],
+                                                 p->xlo[0], p->xhi[1], p->xlo[1], p->tpart);
+    CUDA_TRY(cudaGetLastError());
+    k_trace_final<<<(p->nmat + 7) / 8, 256, 0, st>>>(p->mats_d, p->nmat, p->state, p->tpart);
+    CUDA_TRY(cudaGetLastError());
+    return ISOLOCO_OK;
+}
+
+static int finish_call(isoloco_plan* p, cudaStream_t st, int sync) {
+    CUDA_TRY(cudaMemcpyAsync(p->err_h, p->err_d, sizeof(uint32_t), cudaMemcpyDeviceToHost, st));
+    CUDA_TRY(cudaEventRecord(p->done_ev, st));
+    if (!sync) return ISOLOCO_OK;
+    return isoloco_last_status(p, st);
+}
+
+static int check_opts(const isoloco_opts_t* o, isoloco_opts_t* out) {
+    isoloco_opts_default(out);
+    if (o) *out = *o;
+    if (out->max_iter <= 0) out->max_iter = kDefaultMaxIter;
+    if (out->max_iter > 200) return fail(ISOLOCO_ERR_INVALID, "max_iter must be <= 200");
+    if (!(out->tol > 0.f)) out->tol = kDefaultTol;
+    return ISOLOCO_OK;
+}
+
+static int check_replicas(isoloco_plan* p, const void* const* reps, ReplicaPtrs& rp) {
+    if (!reps) return fail(ISOLOCO_ERR_INVALID, "replicas array is NULL");
+    memset(&rp, 0, sizeof(rp));
+    for (int k = 0; k < p->K; ++k) {
+        if (!reps[k]) return fail(ISOLOCO_ERR_INVALID, "replica pointer is NULL");
+        if (!aligned16(reps[k])) return fail(ISOLOCO_ERR_ALIGN, "replica pointer is not 16-byte aligned");
+        rp.p[k] = reps[k];
+    }
+    return ISOLOCO_OK;
+}
+
+static int run_isoc_step(isoloco_plan* p, int merge, float* theta, float* mom, const void* const* reps,
+                         const isoloco_opts_t* opts_in, cudaStream_t st, float* upd_out, const float* base,
+                         float* out, float alpha_merge) {
+    isoloco_opts_t o;
+    int rc;
+    if ((rc = check_opts(opts_in, &o))) return rc;
+    ReplicaPtrs rp;
+    if ((rc = check_replicas(p, reps, rp))) return rc;
+    CUDA_TRY(cudaSetDevice(p->device));
+    const float* th_src = merge ? base : theta;
+    const float scale = merge ? -1.f : (o.reduce_mean ? 1.f / (float)p->K : 1.f);
+    k_reset_state<<<(std::max(1, p->nmat) + 255) / 256, 256, 0, st>>>(p->state, p->nmat, p->err_d);
+    CUDA_TRY(cudaGetLastError());
+    if (p->nchunks) {
+        k_reduce<<<p->nchunks, 256, 0, st>>>(p->chunks_d, p->mats_d, rp, p->K, p->dtype, th_src, scale, p->dhi,
+                                             p->dlo, p->d1d, p->err_d);
+        CUDA_TRY(cudaGetLastError());
+    }
+    if ((rc = run_polar(p, o.max_iter, o.tol, st))) return rc;
+    UpdateSrc us;
+    us.qh[0] = p->xhi[0];
+    us.qh[1] = p->xhi[1];
+    us.ql[0] = p->xlo[0];
+    us.ql[1] = p->xlo[1];
+    us.d1d = p->d1d;
+    if (p->nchunks) {
+        if (merge)
+            k_apply<<<p->nchunks, 256, 0, st>>>(p->chunks_d, p->mats_d, p->state, us, 1, alpha_merge, 0.f, 0.f,
+                                                nullptr, nullptr, base, out, nullptr, p->err_d);
+        else
+            k_apply<<<p->nchunks, 256, 0, st>>>(p->chunks_d, p->mats_d, p->state, us, 0, o.alpha, o.outer_lr,
+                                                o.momentum, theta, mom, nullptr, nullptr, upd_out, p->err_d);
+        CUDA_TRY(cudaGetLastError());
+    }
+    return finish_call(p, st, o.sync);
+}
+
+// ================================================================== C ABI
+extern "C" {
+
+const char* isoloco_last_error(void) { return g_last_error.c_str(); }
+
+int isoloco_opts_default(isoloco_opts_t* o) {
+    if (!o) return fail(ISOLOCO_ERR_INVALID, "opts is NULL");
+    o->alpha = 1.f;
+    o->outer_lr = 0.7f;
+    o->momentum = 0.9f;
+    o->reduce_mean = 1;
+    o->max_iter = kDefaultMaxIter;
+    o->tol = kDefaultTol;
+    o->sync = 0;
+    return ISOLOCO_OK;
+}
+
+int isoloco_plan_create(isoloco_plan_t* out, const isoloco_param_t* table, int n_params, int64_t n_total, int K,
+                        isoloco_dtype_t replica_dtype) {
+    if (!out) return fail(ISOLOCO_ERR_INVALID, "plan out-pointer is NULL");
+    *out = nullptr;
+    if (n_params < 0 || (n_params > 0 && !table)) return fail(ISOLOCO_ERR_INVALID, "bad table");
+    if (n_total <= 0) return fail(ISOLOCO_ERR_INVALID, "n_total must be positive");
+    if (K < 1 || K > kMaxK) return fail(ISOLOCO_ERR_INVALID, "K must be in 1..64");
+    if (replica_dtype != ISOLOCO_F32 && replica_dtype != ISOLOCO_BF16)
+        return fail(ISOLOCO_ERR_INVALID, "bad replica dtype");
+    std::vector<std::pair<int64_t, int64_t>> spans;
+    for (int i = 0; i < n_params; ++i) {
+        const isoloco_param_t& t = table[i];
+        if (t.rows <= 0 || t.cols < 0 || t.offset < 0) return fail(ISOLOCO_ERR_INVALID, "bad table entry");
+        const int64_t len = (int64_t)t.rows * (t.cols > 0 ? t.cols : 1);
+        if (len > 2147483647LL || t.offset + len > n_total)
+            return fail(ISOLOCO_ERR_INVALID, "table entry outside [0, n_total)");
+        spans.emplace_back(t.offset, t.offset + len);
+    }
+    std::sort(spans.begin(), spans.end());
+    for (size_t i = 1; i < spans.size(); ++i)
+        if (spans[i].first < spans[i - 1].second) return fail(ISOLOCO_ERR_INVALID, "table entries overlap");
+    isoloco_plan* p = new isoloco_plan();
+    cudaError_t e = cudaGetDevice(&p->device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount, p->device);
+    if (e != cudaSuccess) {
+        delete p;
+        return fail(ISOLOCO_ERR_CUDA, std::string("no CUDA device: ") + cudaGetErrorString(e));
+    }
+    p->K = K;
+    p->dtype = (int)replica_dtype;
+    p->N = n_total;
+    p->table.assign(table, table + n_params);
+    int rc = build_plan(p, table, n_params);
+    if (rc != ISOLOCO_OK) {
+        free_plan(p);
+        return rc;
+    }
+    *out = p;
+    return ISOLOCO_OK;
+}
+
+void isoloco_plan_destroy(isoloco_plan_t p) {
+    if (!p) return;
+    cudaSetDevice(p->device);
+    cudaDeviceSynchronize();
+    free_plan(p);
+}
+
+int64_t isoloco_plan_workspace_bytes(isoloco_plan_t p) { return p ? p->ws_bytes : 0; }
+
+int isoloco_plan_num_matrices(isoloco_plan_t p) { return p ? p->nmat : 0; }
+
+int isoloco_outer_step(isoloco_plan_t p, float* theta, float* momentum, const void* const* replicas,
+                       const isoloco_opts_t* opts, void* stream, float* update_out) {
+    if (!p) return fail(ISOLOCO_ERR_INVALID, "plan is NULL");
+    if (!theta || !momentum) return fail(ISOLOCO_ERR_INVALID, "theta or momentum is NULL");
+    if (!aligned16(theta) || !aligned16(momentum) || (update_out && !aligned16(update_out)))
+        return fail(ISOLOCO_ERR_ALIGN, "theta, momentum and update_out must be 16-byte aligned");
+    return run_isoc_step(p, 0, theta, momentum, replicas, opts, static_cast<cudaStream_t>(stream), update_out,
+                         nullptr, nullptr, 0.f);
+}
+
+int iso_c_merge(isoloco_plan_t p, const float* base, const void* const* experts, float alpha, float* out,
+                void* stream) {
+    if (!p) return fail(ISOLOCO_ERR_INVALID, "plan is NULL");
+    if (!base || !out) return fail(ISOLOCO_ERR_INVALID, "base or out is NULL");
+    if (!aligned16(base) || !aligned16(out)) return fail(ISOLOCO_ERR_ALIGN, "base and out must be 16-byte aligned");
+    isoloco_opts_t o;
+    isoloco_opts_default(&o);
+    return run_isoc_step(p, 1, nullptr, nullptr, experts, &o, static_cast<cudaStream_t>(stream), nullptr, base,
+                         out, alpha);
+}
+
+int diloco_outer_step(isoloco_plan_t p, float* theta, float* momentum, const void* const* replicas,
+                      const isoloco_opts_t* opts_in, void* stream) {
+    if (!p) return fail(ISOLOCO_ERR_INVALID, "plan is NULL");
+    if (!theta || !momentum) return fail(ISOLOCO_ERR_INVALID, "theta or momentum is NULL");
+    if (!aligned16(theta) || !aligned16(momentum)) return fail(ISOLOCO_ERR_ALIGN, "theta/momentum not aligned");
+    isoloco_opts_t o;
+    int rc;
+    if ((rc = check_opts(opts_in, &o))) return rc;
+    ReplicaPtrs rp;
+    if ((rc = check_replicas(p, replicas, rp))) return rc;
+    CUDA_TRY(cudaSetDevice(p->device));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    CUDA_TRY(cudaMemsetAsync(p->err_d, 0, 4, st));
+    const float scale = o.reduce_mean ? 1.f / (float)p->K : 1.f;
+    const int grid = p->num_sms * 8;
+    k_diloco<<<grid, 256, 0, st>>>(rp, p->K, p->dtype, theta, momentum, p->N, scale, o.outer_lr, o.momentum,
+                                   p->err_d);
+    CUDA_TRY(cudaGetLastError());
+    return finish_call(p, st, o.sync);
+}
+
+int isoloco_outer_step_host(isoloco_plan_t p, float* theta_h, float* mom_h, const void* const* reps_h,
+                            const isoloco_opts_t* opts, void* stream) {
+    if (!p) return fail(ISOLOCO_ERR_INVALID, "plan is NULL");
+    if (!theta_h || !mom_h || !reps_h) return fail(ISOLOCO_ERR_INVALID, "NULL host buffer");
+    for (int k = 0; k < p->K; ++k)
+        if (!reps_h[k]) return fail(ISOLOCO_ERR_INVALID, "NULL host replica");
+    CUDA_TRY(cudaSetDevice(p->device));
+    const size_t eb = p->dtype == ISOLOCO_F32 ? 4 : 2;
+    const size_t rep_bytes = round_up((int64_t)(p->N * eb), 256);
+    int rc;
+    if (!p->st_theta) {
+        if ((rc = dalloc(p, &p->st_theta, p->N)) || (rc = dalloc(p, &p->st_mom, p->N))) return rc;
+        uint8_t* r = nullptr;
+        if ((rc = dalloc(p, &r, (int64_t)rep_bytes * p->K))) return rc;
+        p->st_reps = r;
+    }
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    CUDA_TRY(cudaMemcpyAsync(p->st_theta, theta_h, p->N * 4, cudaMemcpyHostToDevice, st));
+    CUDA_TRY(cudaMemcpyAsync(p->st_mom, mom_h, p->N * 4, cudaMemcpyHostToDevice, st));
+    std::vector<const void*> dr(p->K);
+    for (int k = 0; k < p->K; ++k) {
+        void* d = static_cast<uint8_t*>(p->st_reps) + k * rep_bytes;
+        CUDA_TRY(cudaMemcpyAsync(d, reps_h[k], p->N * eb, cudaMemcpyHostToDevice, st));
+        dr[k] = d;
+    }
+    isoloco_opts_t o;
+    if ((rc = check_opts(opts, &o))) return rc;
+    o.sync = 0;
+    if ((rc = run_isoc_step(p, 0, p->st_theta, p->st_mom, dr.data(), &o, st, nullptr, nullptr, nullptr, 0.f)))
+        return rc;
+    CUDA_TRY(cudaMemcpyAsync(theta_h, p->st_theta, p->N * 4, cudaMemcpyDeviceToHost, st));
+    CUDA_TRY(cudaMemcpyAsync(mom_h, p->st_mom, p->N * 4, cudaMemcpyDeviceToHost, st));
+    return isoloco_last_status(p, st);
+}
+
+int isoloco_last_status(isoloco_plan_t p, void* stream) {
+    if (!p) return fail(ISOLOCO_ERR_INVALID, "plan is NULL");
+    CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+    CUDA_TRY(cudaEventSynchronize(p->done_ev));
+    const uint32_t e = *p->err_h;
+    if (e & kErrTimeout) return fail(ISOLOCO_ERR_TIMEOUT, "a device-side wait timed out");
+    if (e & kErrNonFinite) return fail(ISOLOCO_ERR_NONFINITE, "non-finite pseudo-gradient");
+    if (e & kErrNotConverged) return fail(ISOLOCO_ERR_NOT_CONVERGED, "polar iteration hit max_iter");
+    return ISOLOCO_OK;
+}
+
+int isoloco_read_diag(isoloco_plan_t p, void* stream, float* sigma_bar, int32_t* iters, int32_t* status,
+                      float* resid) {
+    if (!p) return fail(ISOLOCO_ERR_INVALID, "plan is NULL");
+    CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+    if (p->nmat == 0) return ISOLOCO_OK;
+    std::vector<MatState> s(p->nmat);
+    CUDA_TRY(cudaMemcpy(s.data(), p->state, sizeof(MatState) * p->nmat, cudaMemcpyDeviceToHost));
+    // report in table order of the 2-D tensors
+    std::vector<int> order(p->nmat);
+    for (int i = 0; i < p->nmat; ++i) order[i] = i;
+    std::sort(order.begin(), order.end(), [&](int a, int b) { return p->mat_param[a] < p->mat_param[b]; });
+    for (int j = 0; j < p->nmat; ++j) {
+        const MatState& m = s[order[j]];
+        if (sigma_bar) sigma_bar[j] = m.sigma_bar;
+        if (iters) iters[j] = m.iters;
+        if (status) status[j] = m.status ? ISOLOCO_ERR_NOT_CONVERGED : ISOLOCO_OK;
+        if (resid) resid[j] = m.resid;
+    }
+    return ISOLOCO_OK;
+}
+
+int isoloco_debug_gemm(int a_mn, int b_mn, int batch, int M, int N, int K, const float* A, const float* B,
+                       float* D, void* stream) {
+    if (batch <= 0 || M <= 0 || N <= 0 || K <= 0 || !A || !B || !D)
+        return fail(ISOLOCO_ERR_INVALID, "bad debug_gemm arguments");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int a_rows = a_mn ? K : M, a_cols = a_mn ? M : K;
+    const int b_rows = b_mn ? K : N, b_cols = b_mn ? N : K;
+    const int lda = (int)round_up(a_cols, 8), ldb = (int)round_up(b_cols, 8);
+    const int64_t asz = (int64_t)batch * a_rows * lda, bsz = (int64_t)batch * b_rows * ldb;
+    __nv_bfloat16 *ah = nullptr, *al = nullptr, *bh = nullptr, *bl = nullptr;
+    CUtensorMap* maps_d = nullptr;
+    MatState* dummy_state = nullptr;
+    uint32_t* err = nullptr;
+    auto cleanup = [&]() {
+        cudaFree(ah); cudaFree(al); cudaFree(bh); cudaFree(bl); cudaFree(maps_d); cudaFree(dummy_state); cudaFree(err);
+    };
+    if (cudaMalloc(&ah, asz * 2) || cudaMalloc(&al, asz * 2) || cudaMalloc(&bh, bsz * 2) || cudaMalloc(&bl, bsz * 2) ||
+        cudaMalloc(&maps_d, 4 * sizeof(CUtensorMap)) || cudaMalloc(&err, 4)) {
+        cleanup();
+        return fail(ISOLOCO_ERR_OOM, "debug_gemm scratch allocation failed");
+    }
+    cudaMemsetAsync(ah, 0, asz * 2, st); cudaMemsetAsync(al, 0, asz * 2, st);
+    cudaMemsetAsync(bh, 0, bsz * 2, st); cudaMemsetAsync(bl, 0, bsz * 2, st);
+    cudaMemsetAsync(err, 0, 4, st);
+    k_split_planes<<<1024, 256, 0, st>>>(A, (int64_t)batch * a_rows * a_cols, a_rows, a_cols, lda, ah, al);
+    k_split_planes<<<1024, 256, 0, st>>>(B, (int64_t)batch * b_rows * b_cols, b_rows, b_cols, ldb, bh, bl);
+    CUtensorMap maps[4];
+    const int ra = a_mn ? kRoleMN : kRoleKA, rb = b_mn ? kRoleMN : kRoleKB;
+    if (!make_map(&maps[0], ah, a_cols, a_rows, batch, lda, ra) || !make_map(&maps[1], al, a_cols, a_rows, batch, lda, ra) ||
+        !make_map(&maps[2], bh, b_cols, b_rows, batch, ldb, rb) || !make_map(&maps[3], bl, b_cols, b_rows, batch, ldb, rb)) {
+        cleanup();
+        return fail(ISOLOCO_ERR_CUDA, "cuTensorMapEncodeTiled failed");
+    }
+    cudaMemcpyAsync(maps_d, maps, sizeof(maps), cudaMemcpyHostToDevice, st);
+    GemmParams gp;
+    memset(&gp, 0, sizeof(gp));
+    gp.epi = kEpiF32;
+    gp.gate = kGateNone;
+    gp.err = err;
+    GemmGroup& g = gp.g[0];
+    g.a_hi = maps_d; g.a_lo = maps_d + 1; g.b_hi = maps_d + 2; g.b_lo = maps_d + 3;
+    set_group_common(g, M, N, K, batch, 1, 0);
+    g.cta_begin = 0;
+    g.out_f32 = D;
+    g.f32_batch_stride = (int64_t)M * N;
+    g.f32_split_stride = 0;
+    g.ld_f32 = N;
+    gp.num_groups = 1;
+    cudaError_t e = launch_gemm(gp, a_mn != 0, b_mn != 0, st);
+    uint32_t herr = 0;
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&herr, err, 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    cleanup();
+    if (e != cudaSuccess) return fail(ISOLOCO_ERR_CUDA, std::string("debug_gemm: ") + cudaGetErrorString(e));
+    if (herr & kErrTimeout) return fail(ISOLOCO_ERR_TIMEOUT, "debug_gemm: device wait timed out");
+    return ISOLOCO_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,254 @@
+// polar.cu -- per-iteration bookkeeping of the batched polar iteration, and sigma_bar.
+//
+//  k_gram_finalize : G = sum of the split-K Gram partials; writes G (fp32 and bf16
+//                    hi/lo planes) and per-tile partial sums of G^2, diag(G) and
+//                    (G - I)^2 for the convergence test.
+//  k_control       : one warp per matrix; sums the partials in a fixed order (fp64),
+//                    normalises at t = 0 (s^2 = ||Delta^T Delta||_F >= sigma_max^2),
+//                    tests ||X^T X - I||_F / sqrt(n) < tol and picks this
+//                    iteration's polynomial: the next quintic of the schedule, the
+//                    final cubic polish, or stop.
+//  k_trace_partial / k_trace_final : sigma_bar = tr(Q^T Delta) / n (Alg. 2's mean
+//                    singular value: for the polar factor Q, Q^T Delta = V S V^T).
+//
+// All reductions use fixed assignments and fixed shuffle trees: two runs on the same
+// inputs give bitwise-identical results.
+#include "common.cuh"
+#include "ns_schedule.h"
+#include "types.h"
+
+namespace isoloco {
+
+constexpr int kFinTile = 64;  // finalize tile edge
+
+__device__ __forceinline__ float warp_sum_f(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+__device__ __forceinline__ double warp_sum_d(double v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// grid: one block (256 threads) per (matrix, 64 x 64 tile) listed in `ftiles`.
+__global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict__ mats,
+                                                       const int2* __restrict__ ftiles,
+                                                       const MatState* __restrict__ state,
+                                                       const float* __restrict__ gpart,
+                                                       const int64_t* __restrict__ gpart_off,
+                                                       const int64_t* __restrict__ gpart_split_stride,
+                                                       const int* __restrict__ nsplit,
+                                                       float* __restrict__ gf32,
+                                                       __nv_bfloat16* __restrict__ ghi,
+                                                       __nv_bfloat16* __restrict__ glo,
+                                                       float* __restrict__ fin_part) {
+    const int2 ft = ftiles[blockIdx.x];
+    const int mi = ft.x;
+    if (state[mi].done) return;
+    const MatDesc md = mats[mi];
+    const int n = md.n, ld = md.ld_n;
+    const int tiles_c = (n + kFinTile - 1) / kFinTile;
+    const int r0 = (ft.y / tiles_c) * kFinTile, c0 = (ft.y % tiles_c) * kFinTile;
+    const int64_t poff = gpart_off[mi];
+    const int64_t sstride = gpart_split_stride[mi];
+    const int splits = nsplit[mi];
+
+    float sq = 0.f, tr = 0.f, dev = 0.f;
+    for (int e = threadIdx.x; e < kFinTile * kFinTile; e += blockDim.x) {
+        const int r = r0 + e / kFinTile, c = c0 + e % kFinTile;
+        if (r >= n || c >= n) continue;
+        const int64_t idx = static_cast<int64_t>(r) * ld + c;
+        float v = 0.f;
+        for (int s = 0; s < splits; ++s) v += gpart[poff + s * sstride + idx];
+        gf32[md.gslot + idx] = v;
+        __nv_bfloat16 h, l;
+        split_bf16(v, h, l);
+        ghi[md.gslot + idx] = h;
+        glo[md.gslot + idx] = l;
+        sq += v * v;
+        const float dlt = (r == c) ? 1.f : 0.f;
+        tr += (r == c) ? v : 0.f;
+        dev += (v - dlt) * (v - dlt);
+    }
+    __shared__ float red[3][8];
+    sq = warp_sum_f(sq);
+    tr = warp_sum_f(tr);
+    dev = warp_sum_f(dev);
+    const int w = threadIdx.x >> 5;
+    if ((threadIdx.x & 31) == 0) {
+        red[0][w] = sq;
+        red[1][w] = tr;
+        red[2][w] = dev;
+    }
+    __syncthreads();
+    if (threadIdx.x < 3) {
+        float s = 0.f;
+        for (int i = 0; i < (int)(blockDim.x >> 5); ++i) s += red[threadIdx.x][i];
+        fin_part[(md.gpart_slot + ft.y) * 3 + threadIdx.x] = s;
+    }
+}
+
+// One warp per matrix.  t: iteration index (0 = first Gram of Delta itself).
+__global__ void k_control(const MatDesc* __restrict__ mats, int nmat, MatState* __restrict__ state,
+                          const float* __restrict__ fin_part, int t, int max_iter, float tol,
+                          uint32_t* __restrict__ err) {
+    const int mi = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (mi >= nmat) return;
+    MatState& st = state[mi];
+    if (st.done) {
+        if (lane == 0) st.mode = 0;
+        return;
+    }
+    const MatDesc md = mats[mi];
+    double sq = 0.0, tr = 0.0, dev = 0.0;
+    for (int i = lane; i < md.n_gtiles; i += 32) {
+        const float* pp = fin_part + (md.gpart_slot + i) * 3;
+        sq += pp[0];
+        tr += pp[1];
+        dev += pp[2];
+    }
+    sq = warp_sum_d(sq);
+    tr = warp_sum_d(tr);
+    dev = warp_sum_d(dev);
+    if (lane != 0) return;
+
+    const double n = static_cast<double>(md.n);
+    double d, gscale = 1.0, xscale = 1.0;
+    if (t == 0) {
+        const double s2 = sqrt(sq);  // ||Delta^T Delta||_F >= sigma_max(Delta)^2
+        if (!(s2 > 0.0) || !isfinite(s2)) {
+            // Delta = 0 (or unusable): Q = 0, sigma_bar = 0, zero update.
+            if (!isfinite(s2)) atomicOr(err, kErrNonFinite);
+            st.mode = 0;
+            st.done = 1;
+            st.final_buf = 2;
+            st.resid = 0.f;
+            return;
+        }
+        gscale = 1.0 / s2;
+        xscale = 1.0 / sqrt(s2);
+        // ||G/s2 - I||_F^2 = ||G||^2/s2^2 - 2 tr(G)/s2 + n, with ||G||^2/s2^2 = 1
+        d = sqrt(fmax(0.0, 1.0 - 2.0 * tr * gscale + n) / n);
+    } else {
+        d = sqrt(fmax(0.0, dev) / n);
+    }
+    st.resid = static_cast<float>(d);
+    st.xscale = static_cast<float>(xscale);
+    if (!isfinite(d)) {
+        atomicOr(err, kErrNonFinite);
+        st.mode = 0;
+        st.done = 1;
+        st.final_buf = 2;
+        return;
+    }
+    if (d < tol) {
+        // Cubic polish p(x) = 1.5 x - 0.5 x^3 on singular values already near 1.
+        st.mode = 2;
+        st.a = 1.5f;
+        st.b = static_cast<float>(-0.5 * gscale);
+        st.c = 0.f;
+        st.iters += 1;
+        st.done = 1;
+        st.final_buf = (t + 1) & 1;
+    } else if (st.iters >= max_iter) {
+        st.mode = 0;
+        st.done = 1;
+        st.final_buf = t & 1;
+        st.status = kErrNotConverged;
+        atomicOr(err, kErrNotConverged);
+    } else {
+        const int k = st.step % kSchedSteps;
+        st.mode = 1;
+        st.a = kSched[k][0];
+        st.b = static_cast<float>(kSched[k][1] * gscale);
+        st.c = static_cast<float>(kSched[k][2] * gscale * gscale);
+        st.step += 1;
+        st.iters += 1;
+    }
+}
+
+// grid: one block (256 threads) per (matrix, row chunk) listed in `tchunks`
+// (x = matrix, y = first row, z = rows, w = chunk index within the matrix).  Q comes from the final ping-pong buffer.
+__global__ void __launch_bounds__(256) k_trace_partial(const MatDesc* __restrict__ mats,
+                                                       const int4* __restrict__ tchunks,
+                                                       const MatState* __restrict__ state,
+                                                       const __nv_bfloat16* __restrict__ dhi,
+                                                       const __nv_bfloat16* __restrict__ dlo,
+                                                       const __nv_bfloat16* __restrict__ x0hi,
+                                                       const __nv_bfloat16* __restrict__ x0lo,
+                                                       const __nv_bfloat16* __restrict__ x1hi,
+                                                       const __nv_bfloat16* __restrict__ x1lo,
+                                                       double* __restrict__ tpart) {
+    const int4 tc = tchunks[blockIdx.x];
+    const MatDesc md = mats[tc.x];
+    const int fb = state[tc.x].final_buf;
+    double acc = 0.0;
+    if (fb == 0 || fb == 1) {
+        const __nv_bfloat16* qh = (fb == 0 ? x0hi : x1hi) + md.slot;
+        const __nv_bfloat16* ql = (fb == 0 ? x0lo : x1lo) + md.slot;
+        const __nv_bfloat16* dh = dhi + md.slot;
+        const __nv_bfloat16* dl = dlo + md.slot;
+        float part = 0.f;
+        const int total = tc.z * md.cols;
+        for (int e = threadIdx.x; e < total; e += blockDim.x) {
+            const int r = tc.y + e / md.cols, c = e % md.cols;
+            const int64_t idx = static_cast<int64_t>(r) * md.ld + c;
+            const float q = __bfloat162float(qh[idx]) + __bfloat162float(ql[idx]);
+            const float dv = __bfloat162float(dh[idx]) + __bfloat162float(dl[idx]);
+            part = fmaf(q, dv, part);
+        }
+        acc = static_cast<double>(part);
+    }
+    __shared__ double red[8];
+    acc = warp_sum_d(acc);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double s = 0.0;
+        for (int i = 0; i < (int)(blockDim.x >> 5); ++i) s += red[i];
+        tpart[md.trace_part + tc.w] = s;
+    }
+}
+
+// One warp per matrix: sigma_bar = (sum of the trace partials) / n.
+__global__ void k_trace_final(const MatDesc* __restrict__ mats, int nmat, MatState* __restrict__ state,
+                              const double* __restrict__ tpart) {
+    const int mi = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (mi >= nmat) return;
+    const MatDesc md = mats[mi];
+    double s = 0.0;
+    for (int i = lane; i < md.n_tchunks; i += 32) s += tpart[md.trace_part + i];
+    s = warp_sum_d(s);
+    if (lane == 0) {
+        MatState& st = state[mi];
+        st.trace = s;
+        st.sigma_bar = (st.final_buf == 2) ? 0.f : static_cast<float>(s / md.n);
+    }
+}
+
+// Resets the per-matrix state before a step.
+__global__ void k_reset_state(MatState* state, int nmat, uint32_t* err) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i == 0) *err = 0u;
+    if (i >= nmat) return;
+    MatState s;
+    s.a = s.b = s.c = 0.f;
+    s.xscale = 1.f;
+    s.resid = 0.f;
+    s.sigma_bar = 0.f;
+    s.mode = 0;
+    s.step = 0;
+    s.iters = 0;
+    s.done = 0;
+    s.final_buf = 2;
+    s.status = 0;
+    s.trace = 0.0;
+    state[i] = s;
+}
+
+}  // namespace isoloco

@@ -1,0 +1,268 @@
+// stream.cu -- HBM-bound streaming kernels of the outer step.
+//
+//  k_reduce       : pseudo-gradient reduction (Alg. 1/2 "average pseudo-gradients"):
+//                   d = scale * sum_k (theta - theta_k), every replica read once with
+//                   16-byte loads; each difference is taken before the sum (exact for
+//                   nearby values).  2-D tensors -> bf16 hi/lo planes of the polar
+//                   workspace; 1-D tensors -> fp32.  Raises kErrNonFinite.
+//  k_nesterov     : Alg. 2's update B <- mu B + U, theta <- theta - eta (U + mu B) with
+//                   U = alpha sigma_bar Q (2-D) or the mean pseudo-gradient (1-D).
+//  k_diloco       : Alg. 1 with Nesterov SGD fused into a single pass over all
+//                   parameters (reduction + update, no workspace).
+//  k_merge_out    : Iso-C merge output base + alpha IsoC(T) / base + alpha T (Eq. 1).
+//  k_split_planes : fp32 -> bf16 hi/lo planes (tests of the split-precision GEMM).
+#include "common.cuh"
+#include "types.h"
+
+namespace isoloco {
+
+constexpr int kStreamThreads = 256;
+
+__device__ __forceinline__ float4 ld_rep4(const void* base, int dtype, int64_t i) {
+    if (dtype == 0) return __ldg(reinterpret_cast<const float4*>(static_cast<const float*>(base) + i));
+    const uint2 u = __ldg(reinterpret_cast<const uint2*>(static_cast<const uint16_t*>(base) + i));
+    return make_float4(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xFFFF0000u),
+                       __uint_as_float(u.y << 16), __uint_as_float(u.y & 0xFFFF0000u));
+}
+
+__device__ __forceinline__ float ld_rep1(const void* base, int dtype, int64_t i) {
+    if (dtype == 0) return __ldg(static_cast<const float*>(base) + i);
+    return bf16_bits_to_float(__ldg(static_cast<const uint16_t*>(base) + i));
+}
+
+__device__ __forceinline__ void raise_nonfinite(bool bad, uint32_t* err) {
+    if (__any_sync(0xffffffffu, bad) && (threadIdx.x & 31) == 0) atomicOr(err, kErrNonFinite);
+}
+
+// grid: one CTA per chunk.
+__global__ void __launch_bounds__(kStreamThreads) k_reduce(const Chunk* __restrict__ chunks,
+                                                           const MatDesc* __restrict__ mats,
+                                                           ReplicaPtrs reps, int K, int dtype,
+                                                           const float* __restrict__ theta, float scale,
+                                                           __nv_bfloat16* __restrict__ dhi,
+                                                           __nv_bfloat16* __restrict__ dlo,
+                                                           float* __restrict__ d1d,
+                                                           uint32_t* __restrict__ err) {
+    const Chunk ch = chunks[blockIdx.x];
+    bool bad = false;
+    const int64_t f0 = ch.flat_begin;
+    if (ch.matrix < 0) {
+        for (int e = threadIdx.x; e < ch.count; e += blockDim.x) {
+            const float th = __ldg(theta + f0 + e);
+            float s = 0.f;
+            for (int k = 0; k < K; ++k) s += th - ld_rep1(reps.p[k], dtype, f0 + e);
+            const float d = s * scale;
+            bad |= !isfinite(d);
+            d1d[ch.dst + e] = d;
+        }
+    } else {
+        const MatDesc md = mats[ch.matrix];
+        const bool contiguous = (md.ld == md.cols);
+        if (contiguous && (f0 & 3) == 0 && (ch.count & 3) == 0) {
+            __nv_bfloat16* oh = dhi + md.slot + ch.elem_begin;
+            __nv_bfloat16* ol = dlo + md.slot + ch.elem_begin;
+            const int nv = ch.count >> 2;
+            for (int v = threadIdx.x; v < nv; v += blockDim.x) {
+                const int64_t i = f0 + 4 * static_cast<int64_t>(v);
+                const float4 th = __ldg(reinterpret_cast<const float4*>(theta + i));
+                float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+                for (int k = 0; k < K; ++k) {
+                    const float4 r = ld_rep4(reps.p[k], dtype, i);
+                    s.x += th.x - r.x;
+                    s.y += th.y - r.y;
+                    s.z += th.z - r.z;
+                    s.w += th.w - r.w;
+                }
+                const float d[4] = {s.x * scale, s.y * scale, s.z * scale, s.w * scale};
+                __nv_bfloat16 h[4], l[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    bad |= !isfinite(d[j]);
+                    split_bf16(d[j], h[j], l[j]);
+                }
+                reinterpret_cast<uint2*>(oh)[v] = make_uint2(pack_bf16x2(h[0], h[1]), pack_bf16x2(h[2], h[3]));
+                reinterpret_cast<uint2*>(ol)[v] = make_uint2(pack_bf16x2(l[0], l[1]), pack_bf16x2(l[2], l[3]));
+            }
+        } else {
+            for (int e = threadIdx.x; e < ch.count; e += blockDim.x) {
+                const int64_t i = f0 + e;
+                const float th = __ldg(theta + i);
+                float s = 0.f;
+                for (int k = 0; k < K; ++k) s += th - ld_rep1(reps.p[k], dtype, i);
+                const float d = s * scale;
+                bad |= !isfinite(d);
+                const int pe = ch.elem_begin + e;
+                const int64_t o = md.slot + static_cast<int64_t>(pe / md.cols) * md.ld + pe % md.cols;
+                __nv_bfloat16 h, l;
+                split_bf16(d, h, l);
+                dhi[o] = h;
+                dlo[o] = l;
+            }
+        }
+    }
+    raise_nonfinite(bad, err);
+}
+
+
+// grid: one CTA per chunk.  mode 0: Nesterov (theta, B in place); mode 1: merge output.
+__global__ void __launch_bounds__(kStreamThreads) k_apply(const Chunk* __restrict__ chunks,
+                                                          const MatDesc* __restrict__ mats,
+                                                          const MatState* __restrict__ state,
+                                                          UpdateSrc src, int mode, float alpha,
+                                                          float eta, float mu,
+                                                          float* __restrict__ theta,
+                                                          float* __restrict__ mom,
+                                                          const float* __restrict__ base,
+                                                          float* __restrict__ out,
+                                                          float* __restrict__ upd_out,
+                                                          const uint32_t* __restrict__ err) {
+    if (*err & kErrNonFinite) return;  // leave theta and B untouched
+    const Chunk ch = chunks[blockIdx.x];
+    const int64_t f0 = ch.flat_begin;
+    // U = ucoef * q where q is read from the Q planes (2-D) or Delta (1-D)
+    float ucoef = 1.f;
+    const __nv_bfloat16* qh = nullptr;
+    const __nv_bfloat16* ql = nullptr;
+    MatDesc md;
+    bool zero = false, contiguous = true;
+    if (ch.matrix >= 0) {
+        md = mats[ch.matrix];
+        const MatState st = state[ch.matrix];
+        if (st.final_buf == 2) {
+            zero = true;
+        } else {
+            qh = src.qh[st.final_buf] + md.slot;
+            ql = src.ql[st.final_buf] + md.slot;
+        }
+        ucoef = alpha * st.sigma_bar;
+        contiguous = (md.ld == md.cols);
+    } else if (mode == 1) {
+        ucoef = alpha;  // Eq. 1: base + lambda * sum tau for non-matrix tensors
+    }
+    auto uval = [&](int e) -> float {
+        if (ch.matrix < 0) return ucoef * src.d1d[ch.dst + e];
+        if (zero) return 0.f;
+        const int pe = ch.elem_begin + e;
+        const int64_t o = contiguous ? pe : static_cast<int64_t>(pe / md.cols) * md.ld + pe % md.cols;
+        return ucoef * (__bfloat162float(qh[o]) + __bfloat162float(ql[o]));
+    };
+    const bool vec = (f0 & 3) == 0 && (ch.count & 3) == 0 && (ch.matrix < 0 || contiguous) &&
+                     ((ch.matrix < 0 ? (ch.dst & 3) : (ch.elem_begin & 3)) == 0);
+    if (vec) {
+        const int nv = ch.count >> 2;
+        for (int v = threadIdx.x; v < nv; v += blockDim.x) {
+            const int64_t i = f0 + 4 * static_cast<int64_t>(v);
+            float u[4];
+            if (ch.matrix < 0) {
+                const float4 d = *reinterpret_cast<const float4*>(src.d1d + ch.dst + 4 * v);
+                u[0] = ucoef * d.x; u[1] = ucoef * d.y; u[2] = ucoef * d.z; u[3] = ucoef * d.w;
+            } else if (zero) {
+                u[0] = u[1] = u[2] = u[3] = 0.f;
+            } else {
+                const uint2 hh = *reinterpret_cast<const uint2*>(qh + ch.elem_begin + 4 * v);
+                const uint2 ll = *reinterpret_cast<const uint2*>(ql + ch.elem_begin + 4 * v);
+                u[0] = ucoef * (__uint_as_float(hh.x << 16) + __uint_as_float(ll.x << 16));
+                u[1] = ucoef * (__uint_as_float(hh.x & 0xFFFF0000u) + __uint_as_float(ll.x & 0xFFFF0000u));
+                u[2] = ucoef * (__uint_as_float(hh.y << 16) + __uint_as_float(ll.y << 16));
+                u[3] = ucoef * (__uint_as_float(hh.y & 0xFFFF0000u) + __uint_as_float(ll.y & 0xFFFF0000u));
+            }
+            if (mode == 0) {
+                const float4 th = *reinterpret_cast<const float4*>(theta + i);
+                const float4 bb = *reinterpret_cast<const float4*>(mom + i);
+                float4 nb, nt;
+                nb.x = fmaf(mu, bb.x, u[0]); nt.x = th.x - eta * fmaf(mu, nb.x, u[0]);
+                nb.y = fmaf(mu, bb.y, u[1]); nt.y = th.y - eta * fmaf(mu, nb.y, u[1]);
+                nb.z = fmaf(mu, bb.z, u[2]); nt.z = th.z - eta * fmaf(mu, nb.z, u[2]);
+                nb.w = fmaf(mu, bb.w, u[3]); nt.w = th.w - eta * fmaf(mu, nb.w, u[3]);
+                *reinterpret_cast<float4*>(mom + i) = nb;
+                *reinterpret_cast<float4*>(theta + i) = nt;
+            } else {
+                const float4 bs = *reinterpret_cast<const float4*>(base + i);
+                *reinterpret_cast<float4*>(out + i) = make_float4(bs.x + u[0], bs.y + u[1], bs.z + u[2], bs.w + u[3]);
+            }
+            if (upd_out) *reinterpret_cast<float4*>(upd_out + i) = make_float4(u[0], u[1], u[2], u[3]);
+        }
+    } else {
+        for (int e = threadIdx.x; e < ch.count; e += blockDim.x) {
+            const int64_t i = f0 + e;
+            const float u = uval(e);
+            if (mode == 0) {
+                const float nb = fmaf(mu, mom[i], u);
+                theta[i] = theta[i] - eta * fmaf(mu, nb, u);
+                mom[i] = nb;
+            } else {
+                out[i] = base[i] + u;
+            }
+            if (upd_out) upd_out[i] = u;
+        }
+    }
+}
+
+// Alg. 1 outer step fused: d = scale * sum_k (theta - theta_k); B <- mu B + d;
+// theta <- theta - eta (d + mu B).  Grid-stride over float4 vectors of all N params.
+__global__ void __launch_bounds__(kStreamThreads) k_diloco(ReplicaPtrs reps, int K, int dtype,
+                                                           float* __restrict__ theta,
+                                                           float* __restrict__ mom, int64_t N,
+                                                           float scale, float eta, float mu,
+                                                           uint32_t* __restrict__ err) {
+    bool bad = false;
+    const int64_t nv = N >> 2;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t v = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; v < nv; v += stride) {
+        const int64_t i = 4 * v;
+        const float4 th = *reinterpret_cast<const float4*>(theta + i);
+        const float4 bb = *reinterpret_cast<const float4*>(mom + i);
+        float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 8
+        for (int k = 0; k < K; ++k) {
+            const float4 r = ld_rep4(reps.p[k], dtype, i);
+            s.x += th.x - r.x;
+            s.y += th.y - r.y;
+            s.z += th.z - r.z;
+            s.w += th.w - r.w;
+        }
+        const float d0 = s.x * scale, d1 = s.y * scale, d2 = s.z * scale, d3 = s.w * scale;
+        bad |= !(isfinite(d0) && isfinite(d1) && isfinite(d2) && isfinite(d3));
+        float4 nb, nt;
+        nb.x = fmaf(mu, bb.x, d0); nt.x = th.x - eta * fmaf(mu, nb.x, d0);
+        nb.y = fmaf(mu, bb.y, d1); nt.y = th.y - eta * fmaf(mu, nb.y, d1);
+        nb.z = fmaf(mu, bb.z, d2); nt.z = th.z - eta * fmaf(mu, nb.z, d2);
+        nb.w = fmaf(mu, bb.w, d3); nt.w = th.w - eta * fmaf(mu, nb.w, d3);
+        *reinterpret_cast<float4*>(mom + i) = nb;
+        *reinterpret_cast<float4*>(theta + i) = nt;
+    }
+    // scalar tail
+    if (blockIdx.x == 0) {
+        for (int64_t i = 4 * nv + threadIdx.x; i < N; i += blockDim.x) {
+            const float th = theta[i];
+            float s = 0.f;
+            for (int k = 0; k < K; ++k) s += th - ld_rep1(reps.p[k], dtype, i);
+            const float d = s * scale;
+            bad |= !isfinite(d);
+            const float nb = fmaf(mu, mom[i], d);
+            theta[i] = th - eta * fmaf(mu, nb, d);
+            mom[i] = nb;
+        }
+    }
+    raise_nonfinite(bad, err);
+}
+
+// fp32 [batch][rows][cols] -> bf16 hi/lo planes with leading dimension ld.
+__global__ void k_split_planes(const float* __restrict__ x, int64_t total, int rows, int cols, int ld,
+                               __nv_bfloat16* __restrict__ hi, __nv_bfloat16* __restrict__ lo) {
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total; i += stride) {
+        const int64_t bm = i / cols;
+        const int c = static_cast<int>(i - bm * cols);
+        const int64_t b = bm / rows;
+        const int r = static_cast<int>(bm - b * rows);
+        const int64_t o = (b * rows + r) * ld + c;
+        __nv_bfloat16 h, l;
+        split_bf16(x[i], h, l);
+        hi[o] = h;
+        lo[o] = l;
+    }
+}
+
+}  // namespace isoloco

@@ -1,0 +1,125 @@
+// types.h -- structures shared by the host plan code and the kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+namespace isoloco {
+
+// ------------------------------------------------------------------ GEMM tiles
+// One CTA computes a BM x BN fp32 tile in tensor memory from bf16 hi/lo operand
+// planes staged BK deep per pipeline stage.
+constexpr int BM = 128;
+constexpr int BN = 256;
+constexpr int BK = 32;
+constexpr int kStages = 4;
+constexpr int kTileABytes = BM * BK * 2;                       // one bf16 plane of A
+constexpr int kTileBBytes = BN * BK * 2;                       // one bf16 plane of B
+constexpr int kStageBytes = 2 * kTileABytes + 2 * kTileBBytes;  // hi + lo of A and B
+constexpr int kGemmThreads = 192;  // warp 0 TMA, warp 1 MMA, warps 2..5 epilogue
+constexpr int kTmemCols = 256;
+constexpr int kMaxGroups = 8;
+constexpr int kGemmSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+
+// Epilogue of the split-precision GEMM.
+enum EpiMode : int {
+    kEpiF32 = 0,     // store the fp32 accumulator (Gram partial products)
+    kEpiPoly = 1,    // P = a I + b G + c acc  -> bf16 hi/lo planes
+    kEpiXSplit = 2,  // X = xscale * acc       -> bf16 hi/lo planes
+};
+
+// Which matrices a GEMM launch works on, read from the per-matrix state.
+enum GateMode : int {
+    kGateNone = 0,    // all (debug GEMM)
+    kGateActive = 1,  // matrices not yet done (Gram)
+    kGateStep = 2,    // matrices whose mode this iteration is quintic or polish
+};
+
+struct GemmGroup {
+    const CUtensorMap* a_hi;
+    const CUtensorMap* a_lo;
+    const CUtensorMap* b_hi;
+    const CUtensorMap* b_lo;
+    int M, N, K;  // output tile space M x N, reduction length K
+    int batch;    // matrices in this group
+    int tiles_m, tiles_n, splits, kblocks_per_split;
+    int cta_begin;  // first blockIdx.x of the group
+    int mat_base;   // index of the group's first matrix in the state array
+    // fp32 output (kEpiF32): out_f32 + split*split_stride + b*batch_stride + row*ld + col
+    float* out_f32;
+    int64_t f32_split_stride, f32_batch_stride;
+    int ld_f32;
+    // bf16 hi/lo output (kEpiPoly, kEpiXSplit)
+    __nv_bfloat16* out_hi;
+    __nv_bfloat16* out_lo;
+    int64_t bf_batch_stride;
+    int ld_bf;
+    // kEpiPoly: the fp32 Gram matrix G (same indexing as the output)
+    const float* g_f32;
+    int64_t g_batch_stride;
+    int ld_g;
+};
+
+// Per-matrix state of the polar iteration (device memory, one per 2-D tensor).
+struct MatState {
+    float a, b, c;    // P = a I + b G + c G^2 for this iteration
+    float xscale;     // X_{t+1} = xscale * X_t P
+    float resid;      // last ||X^T X - I||_F / sqrt(n)
+    float sigma_bar;  // tr(Q^T Delta) / n
+    int mode;         // 0 none, 1 quintic step, 2 final cubic polish
+    int step;         // quintic steps taken
+    int iters;        // GEMM iterations used
+    int done;         // 1 once finished
+    int final_buf;    // ping-pong buffer holding Q (0/1), or 2 when Q = 0
+    int status;       // 0, or kErrNotConverged
+    double trace;     // tr(Q^T Delta)
+};
+
+struct GemmParams {
+    GemmGroup g[kMaxGroups];
+    int num_groups;
+    int epi;
+    int gate;
+    MatState* state;
+    uint32_t* err;
+};
+
+// Description of one 2-D tensor in the workspace (device array, one per matrix).
+struct MatDesc {
+    int64_t param_offset;  // offset in the flat parameter buffers
+    int64_t slot;          // element offset of the matrix in the bucket's planes
+    int rows, cols, ld;    // row-major, leading dimension ld (multiple of 8)
+    int n;                 // min(rows, cols): size of the Gram matrix
+    int ld_n;              // leading dimension of the n x n planes
+    int bucket;
+    int64_t gslot;         // element offset of the matrix in the n x n planes
+    int64_t gpart_slot;    // first partial (3 floats each) of the finalize pass
+    int64_t trace_part;    // first partial of the trace pass
+    int n_gtiles;          // finalize tiles of this matrix
+    int n_tchunks;         // trace chunks of this matrix
+};
+
+// A contiguous range of one parameter handled by one streaming CTA.
+struct Chunk {
+    int64_t flat_begin;  // first element in the flat buffers
+    int32_t count;       // elements
+    int32_t param;       // index in the parameter table
+    int32_t matrix;      // index of the 2-D tensor, or -1 for 1-D
+    int32_t elem_begin;  // first element within the parameter
+    int64_t dst;         // 1-D: offset in the 1-D workspace; 2-D: unused
+};
+
+// Sources of the update direction U read by the apply pass.
+struct UpdateSrc {
+    const __nv_bfloat16* qh[2];  // hi planes of the two ping-pong iterate buffers
+    const __nv_bfloat16* ql[2];  // lo planes
+    const float* d1d;            // mean pseudo-gradient of the 1-D tensors
+};
+
+constexpr int kMaxK = 64;
+struct ReplicaPtrs {
+    const void* p[kMaxK];
+};
+
+}  // namespace isoloco

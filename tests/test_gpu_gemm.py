@@ -1,0 +1,59 @@
+"""Split-precision tcgen05 GEMM (the building block of the polar iteration) vs fp64.
+
+Covers the three operand-layout pairs the polar iteration uses (K/K for G^2 and
+the tall update, MN/MN for the tall Gram, K/MN for the wide update) on tiles that
+are full, ragged, and smaller than one tile, with several batch entries.
+Tolerance: ~2^-16 per operand from the bf16 hi+lo split -> relative Frobenius
+error <= 3e-5 against fp64; a single bf16 pass would be ~2e-3.
+"""
+import pytest
+import torch
+
+pytestmark = pytest.mark.gpu
+
+CASES = [
+    (2, 128, 256, 64),
+    (3, 256, 512, 1024),
+    (2, 65, 130, 70),
+    (1, 1, 1, 1),
+    (2, 300, 40, 999),
+    (1, 1024, 1024, 2816),
+]
+
+
+@pytest.fixture(scope="module")
+def iso():
+    from paper_2607_03011_gb300 import isoloco
+    isoloco.lib()
+    return isoloco
+
+
+def _ref(A, B, a_mn, b_mn):
+    Ad = A.double().transpose(1, 2) if a_mn else A.double()     # [b, M, K]
+    Bd = B.double().transpose(1, 2) if b_mn else B.double()     # [b, N, K]
+    return Ad @ Bd.transpose(1, 2)
+
+
+@pytest.mark.parametrize("a_mn,b_mn", [(0, 0), (1, 1), (0, 1), (1, 0)])
+@pytest.mark.parametrize("batch,M,N,K", CASES)
+def test_debug_gemm_layouts(iso, a_mn, b_mn, batch, M, N, K):
+    g = torch.Generator(device="cuda").manual_seed(M * 7 + N * 3 + K)
+    A = torch.randn((batch, K, M) if a_mn else (batch, M, K), device="cuda", generator=g)
+    B = torch.randn((batch, K, N) if b_mn else (batch, N, K), device="cuda", generator=g)
+    D = iso.debug_gemm(A, B, a_mn, b_mn, M, N, K)
+    R = _ref(A, B, a_mn, b_mn)
+    err = (D.double() - R).norm() / R.norm()
+    assert err < 3e-5, float(err)
+    # the split is what buys the accuracy: one bf16 pass is ~100x worse
+    one_pass = _ref(A.bfloat16().float(), B.bfloat16().float(), a_mn, b_mn)
+    if K >= 16:
+        assert (one_pass - R).norm() / R.norm() > 10 * err
+
+
+def test_debug_gemm_deterministic(iso):
+    g = torch.Generator(device="cuda").manual_seed(5)
+    A = torch.randn((2, 256, 512), device="cuda", generator=g)
+    B = torch.randn((2, 512, 512), device="cuda", generator=g)
+    D1 = iso.debug_gemm(A, B, 0, 1, 256, 512, 512)
+    D2 = iso.debug_gemm(A, B, 0, 1, 256, 512, 512)
+    assert torch.equal(D1, D2)

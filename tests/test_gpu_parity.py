@@ -1,0 +1,228 @@
+"""CUDA path vs the fp64 oracle on the same seeded inputs, through the C ABI.
+
+Tolerances (the method's targets): relative Frobenius error of every Iso-C
+update alpha*sigma_bar*Q <= 2e-3, sigma_bar relative error <= 1e-4, elementwise
+relative error <= 1e-5 on theta and momentum of the non-matrix tensors (with a
+floor at the rms of the reference for entries that cancel).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_03011_gb300 import workloads as W
+from parity import check_step, elementwise_rel, oracle_step, rel_fro
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def iso():
+    from paper_2607_03011_gb300 import isoloco
+    isoloco.lib()
+    return isoloco
+
+
+def run_gpu(iso, wl, alpha, eta, mu, reps=None, theta=None, mom=None, max_iter=0, reduce_mean=True,
+            plan=None):
+    plan = plan or iso.Plan(wl.table, wl.N, wl.K, wl.replicas.dtype)
+    th = (wl.theta if theta is None else theta).clone()
+    b = (wl.momentum if mom is None else mom).clone()
+    upd = torch.empty_like(th)
+    rc = plan.outer_step(th, b, wl.replicas if reps is None else reps,
+                         iso.make_opts(alpha, eta, mu, reduce_mean=reduce_mean, max_iter=max_iter, sync=True),
+                         update_out=upd)
+    diag = plan.read_diag()
+    return rc, th, b, upd, diag, plan
+
+
+def compare(wl, rc, th, b, upd, diag, alpha, eta, mu, theta_in=None, mom_in=None, reps=None, only=None):
+    assert rc == 0
+    ref = oracle_step(wl.table, wl.theta if theta_in is None else theta_in,
+                      wl.momentum if mom_in is None else mom_in, wl.replicas if reps is None else reps,
+                      alpha, eta, mu, only=only)
+    ref["theta_in"] = (wl.theta if theta_in is None else theta_in).double().cpu().numpy()
+    mats = [i for i, t in enumerate(wl.table) if t[2] > 0]
+    sig = diag["sigma_bar"]
+    return check_step(wl.table, th.double().cpu().numpy(), b.double().cpu().numpy(),
+                      upd.double().cpu().numpy(), sig, ref, only=only), ref
+
+
+def test_tiny_two_steps(iso):
+    """Tiny config: one outer step, then a second one reusing the momentum."""
+    wl = W.make_workload("tiny", seed=0, device="cuda")
+    sp = wl.spec
+    rc, th, b, upd, diag, plan = run_gpu(iso, wl, sp.alpha, sp.outer_lr, sp.momentum)
+    worst, ref = compare(wl, rc, th, b, upd, diag, sp.alpha, sp.outer_lr, sp.momentum)
+    assert all(s == 0 for s in diag["status"])
+    # step 2: each side regenerates replicas (seed 1) from its own theta and keeps its B
+    th_o = torch.from_numpy(ref["theta"].astype(np.float32))
+    b_o = torch.from_numpy(ref["momentum"].astype(np.float32))
+    reps_g = W.make_replicas(sp, wl.table, th, seed=1)
+    reps_o = W.make_replicas(sp, wl.table, th_o, seed=1)
+    th2, b2 = th.clone(), b.clone()
+    upd2 = torch.empty_like(th2)
+    rc = plan.outer_step(th2, b2, reps_g, iso.make_opts(sp.alpha, sp.outer_lr, sp.momentum, sync=True),
+                         update_out=upd2)
+    assert rc == 0
+    ref2 = oracle.isoloco_outer_step(wl.table, th_o.numpy(), b_o.numpy(), W.replicas_as_numpy(reps_o),
+                                     alpha=sp.alpha, eta=sp.outer_lr, mu=sp.momentum)
+    ref2["theta_in"] = th_o.double().numpy()
+    check_step(wl.table, th2.double().cpu().numpy(), b2.double().cpu().numpy(), upd2.double().cpu().numpy(),
+               plan.read_diag()["sigma_bar"], ref2)
+
+
+@pytest.mark.parametrize("alpha,eta,mu", [(1.0, 1.8, 0.8), (0.5, 0.7, 0.0)])
+def test_tiny_hyperparameters(iso, alpha, eta, mu):
+    wl = W.make_workload("tiny", seed=3, device="cuda")
+    rc, th, b, upd, diag, _ = run_gpu(iso, wl, alpha, eta, mu)
+    compare(wl, rc, th, b, upd, diag, alpha, eta, mu)
+
+
+RAGGED = [("a", 65, 130), ("b", 130, 65), ("c", 1, 9), ("d", 9, 1), ("e", 200, 3), ("f", 3, 200),
+          ("g", 1, 1), ("v", 7, 0), ("h", 300, 257), ("w", 5, 0), ("i", 257, 300), ("j", 129, 129)]
+
+
+def test_ragged_shapes_and_tails(iso):
+    spec = W.custom_spec(RAGGED, K=3, rank=2, momentum_std=1e-4)
+    wl = W.make_workload(spec, seed=11, device="cuda")
+    rc, th, b, upd, diag, _ = run_gpu(iso, wl, 1.0, 0.7, 0.9)
+    compare(wl, rc, th, b, upd, diag, 1.0, 0.7, 0.9)
+
+
+def test_split_k_gram(iso):
+    """Tall-skinny matrices whose Gram takes several split-K passes."""
+    spec = W.custom_spec([("t", 6000, 64), ("u", 64, 5000), ("v", 100, 0)], K=2, rank=3)
+    wl = W.make_workload(spec, seed=2, device="cuda")
+    rc, th, b, upd, diag, _ = run_gpu(iso, wl, 1.0, 0.7, 0.9)
+    compare(wl, rc, th, b, upd, diag, 1.0, 0.7, 0.9)
+
+
+def test_single_worker_and_sum_reduction(iso):
+    spec = W.custom_spec([("m", 96, 64), ("v", 64, 0)], K=1, rank=2)
+    wl = W.make_workload(spec, seed=4, device="cuda")
+    rc, th, b, upd, diag, _ = run_gpu(iso, wl, 1.0, 0.7, 0.9)
+    compare(wl, rc, th, b, upd, diag, 1.0, 0.7, 0.9)
+    spec = W.custom_spec([("m", 96, 64), ("v", 64, 0)], K=4, rank=2)
+    wl = W.make_workload(spec, seed=4, device="cuda")
+    rc, th, b, upd, diag, _ = run_gpu(iso, wl, 1.0, 0.7, 0.9, reduce_mean=False)
+    assert rc == 0
+    ref = oracle_step(wl.table, wl.theta, wl.momentum, wl.replicas, 1.0, 0.7, 0.9, reduce_mean=False)
+    o, r, c = wl.table[0]
+    assert rel_fro(upd[o:o + r * c].cpu().numpy(), ref["update"][o:o + r * c]) < 2e-3
+
+
+def test_bf16_replicas(iso):
+    spec = W.custom_spec([("m", 192, 128), ("n", 128, 320), ("v", 128, 0)], K=4, rank=3,
+                         replica_dtype="bf16", shared_std=2e-3, noise_std=1e-3)
+    wl = W.make_workload(spec, seed=8, device="cuda")
+    assert wl.replicas.dtype == torch.bfloat16
+    rc, th, b, upd, diag, _ = run_gpu(iso, wl, 1.0, 0.7, 0.9)
+    compare(wl, rc, th, b, upd, diag, 1.0, 0.7, 0.9)
+
+
+def test_zero_pseudo_gradient(iso):
+    spec = W.custom_spec([("m", 64, 48), ("v", 16, 0)], K=2, momentum_std=1e-3)
+    wl = W.make_workload(spec, seed=1, device="cuda")
+    reps = wl.theta.unsqueeze(0).repeat(2, 1)
+    rc, th, b, upd, diag, _ = run_gpu(iso, wl, 1.0, 0.7, 0.9, reps=reps)
+    assert rc == 0
+    assert torch.count_nonzero(upd) == 0
+    torch.testing.assert_close(b, 0.9 * wl.momentum, rtol=1e-6, atol=0)
+    torch.testing.assert_close(th, wl.theta - 0.7 * 0.9 * (0.9 * wl.momentum), rtol=1e-6, atol=1e-9)
+    assert diag["sigma_bar"] == [0.0]
+
+
+def test_nonfinite_leaves_state_untouched(iso):
+    spec = W.custom_spec([("m", 64, 48), ("v", 16, 0)], K=2, momentum_std=1e-3)
+    wl = W.make_workload(spec, seed=1, device="cuda")
+    reps = wl.replicas.clone()
+    reps[1, 100] = float("nan")
+    rc, th, b, upd, diag, _ = run_gpu(iso, wl, 1.0, 0.7, 0.9, reps=reps)
+    assert rc == iso.ERR_NONFINITE
+    assert torch.equal(th, wl.theta) and torch.equal(b, wl.momentum)
+
+
+def test_max_iter_reports_not_converged(iso):
+    wl = W.make_workload("tiny", seed=0, device="cuda")
+    rc, th, b, upd, diag, _ = run_gpu(iso, wl, 1.0, 0.7, 0.9, max_iter=1)
+    assert rc == iso.ERR_NOT_CONVERGED
+    assert any(s == iso.ERR_NOT_CONVERGED for s in diag["status"])
+
+
+def test_deterministic(iso):
+    wl = W.make_workload("tiny", seed=5, device="cuda")
+    plan = iso.Plan(wl.table, wl.N, wl.K)
+    r1 = run_gpu(iso, wl, 1.0, 0.7, 0.9, plan=plan)
+    r2 = run_gpu(iso, wl, 1.0, 0.7, 0.9, plan=plan)
+    assert torch.equal(r1[1], r2[1]) and torch.equal(r1[2], r2[2]) and torch.equal(r1[3], r2[3])
+
+
+def test_diloco_outer_step(iso):
+    spec = W.custom_spec(RAGGED, K=3, rank=2, momentum_std=1e-4)
+    wl = W.make_workload(spec, seed=6, device="cuda")
+    plan = iso.Plan(wl.table, wl.N, wl.K)
+    th, b = wl.theta.clone(), wl.momentum.clone()
+    assert plan.diloco_outer_step(th, b, wl.replicas, iso.make_opts(outer_lr=0.7, momentum=0.9, sync=True)) == 0
+    ref = oracle.diloco_outer_step(wl.theta.cpu().numpy(), wl.momentum.cpu().numpy(),
+                                   W.replicas_as_numpy(wl.replicas), eta=0.7, mu=0.9)
+    assert elementwise_rel(th.cpu().numpy(), ref["theta"]) < 1e-5
+    assert elementwise_rel(b.cpu().numpy(), ref["momentum"]) < 1e-5
+
+
+def test_iso_c_merge(iso):
+    spec = W.custom_spec([("m", 96, 64), ("n", 64, 160), ("v", 33, 0)], K=3, rank=2)
+    wl = W.make_workload(spec, seed=9, device="cuda")
+    plan = iso.Plan(wl.table, wl.N, wl.K)
+    out = torch.empty_like(wl.theta)
+    assert plan.iso_c_merge(wl.theta, wl.replicas, 0.8, out) == 0
+    assert plan.last_status() == 0
+    ref = oracle.iso_c_merge(wl.table, wl.theta.cpu().numpy(), W.replicas_as_numpy(wl.replicas), alpha=0.8)
+    for (o, r, c) in wl.table:
+        sl = slice(o, o + r * (c or 1))
+        got = out[sl].double().cpu().numpy() - wl.theta[sl].double().cpu().numpy()
+        want = ref["out"][sl] - wl.theta[sl].double().cpu().numpy()
+        assert rel_fro(got, want) < (2e-3 if c else 1e-5)
+
+
+def test_host_buffer_entry_point(iso):
+    wl = W.make_workload("tiny", seed=2, device="cuda")
+    plan = iso.Plan(wl.table, wl.N, wl.K)
+    th, b = wl.theta.clone(), wl.momentum.clone()
+    assert plan.outer_step(th, b, wl.replicas, iso.make_opts(sync=True)) == 0
+    th_h = wl.theta.cpu().pin_memory()
+    b_h = wl.momentum.cpu().pin_memory()
+    reps_h = [wl.replicas[k].cpu().pin_memory() for k in range(wl.K)]
+    assert plan.outer_step_host(th_h, b_h, reps_h, iso.make_opts()) == 0
+    assert torch.equal(th_h, th.cpu()) and torch.equal(b_h, b.cpu())
+
+
+def test_llama_180m_k8_sampled(iso):
+    """The benchmarked configuration (180M shapes, K = 8), full size on the GPU,
+    checked on one matrix of each shape bucket plus every 1-D tensor."""
+    wl = W.make_workload("llama_180m_k8", seed=0, device="cuda")
+    sp = wl.spec
+    rc, th, b, upd, diag, plan = run_gpu(iso, wl, sp.alpha, sp.outer_lr, sp.momentum)
+    assert rc == 0
+    names = [s[0] for s in sp.shapes]
+    pick = [names.index(n) for n in ("layers.0.wq", "layers.5.w_gate", "layers.11.w_down", "head")]
+    pick += [i for i, s in enumerate(sp.shapes) if s[2] == 0]
+    # the oracle gets only the sampled tensors, re-packed densely (host copies of the inputs)
+    sub_table, parts, off = [], [], 0
+    for i in pick:
+        o, r, c = wl.table[i]
+        n = r * (c or 1)
+        sub_table.append((off, r, c))
+        parts.append((o, n))
+        off += n
+    idx = torch.cat([torch.arange(o, o + n, device="cuda") for o, n in parts])
+    ref = oracle.isoloco_outer_step(sub_table, wl.theta[idx].cpu().numpy(), wl.momentum[idx].cpu().numpy(),
+                                    W.replicas_as_numpy(wl.replicas[:, idx]), alpha=sp.alpha,
+                                    eta=sp.outer_lr, mu=sp.momentum)
+    ref["theta_in"] = wl.theta[idx].double().cpu().numpy()
+    mat_index = {p: j for j, p in enumerate([i for i, s in enumerate(sp.shapes) if s[2] > 0])}
+    sig = [diag["sigma_bar"][mat_index[i]] for i in pick if sp.shapes[i][2] > 0]
+    worst = check_step(sub_table, th[idx].double().cpu().numpy(), b[idx].double().cpu().numpy(),
+                       upd[idx].double().cpu().numpy(), sig, ref)
+    assert all(s == 0 for s in diag["status"])
+    print("worst errors", worst, "iterations", sorted(set(diag["iters"])))
