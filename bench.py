@@ -1,0 +1,355 @@
+#!/usr/bin/env python
+"""Benchmark of the IsoLoCo outer step (Alg. 2) on GB300.
+
+Default workload: the ~180M LLaMA-style shape set with K = 8 fp32 worker
+replicas resident in HBM (219,701,248 parameters, 86 matrices), synthetic
+seeded inputs.  One step = one full outer step through the C ABI: K-way
+pseudo-gradient reduction, Iso-C on every matrix (batched polar iteration on
+tcgen05 tensor cores, sigma_bar by trace), Nesterov update of theta and B.
+
+Prints ONE JSON line (rank 0).  Under torchrun every rank runs its own replica
+of the workload on its own GPU (the outer step has no cross-GPU exchange when
+all workers share one GPU): weak scaling, value = all ranks' parameters / time.
+
+--impl reference times the fp64 CPU oracle on the host cores instead, on a
+bounded sample of the same workload (the reference arm of this benchmark).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "IsoLoCo outer-step ms & params/s at ~180M shapes, K=8; % HBM / TC roofline"
+UNIT = "params/s"
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return d, "measured"
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+# --------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """Samples nvidia-smi clocks and throttle reasons while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        smax = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if "Active" in r[5 + i]})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# --------------------------------------------------------------------------- accounting
+def gemm_flops(table, diag):
+    """Algorithmic (single-pass) FLOPs of the polar GEMMs of one step, from the
+    per-matrix iteration counts: a full Gram 2*r*n^2 and an update 2*r*n^2 per
+    iteration, G^2 = 2*n^3 per quintic step (r = long side, n = short side)."""
+    total = 0.0
+    mats = [(r, c) for (_, r, c) in table if c > 0]
+    for (r, c), it, st, sb in zip(mats, diag["iters"], diag["status"], diag["sigma_bar"]):
+        big, small = max(r, c), min(r, c)
+        if it == 0:
+            total += 2.0 * big * small * small  # one Gram, then found zero
+            continue
+        converged = (st == 0)
+        grams = it + (0 if converged else 1)
+        quintic = it - (1 if converged else 0)
+        total += grams * 2.0 * big * small ** 2 + it * 2.0 * big * small ** 2 + quintic * 2.0 * small ** 3
+    return total
+
+
+def stream_bytes(table, K, replica_bytes):
+    n = sum(r * (c or 1) for (_, r, c) in table)
+    n2 = sum(r * c for (_, r, c) in table if c > 0)
+    return {
+        "reduce": (K * replica_bytes + 4) * n + 4 * n,   # replicas + theta in; Delta (hi/lo or fp32) out
+        "apply": 8 * n + 4 * n + 8 * n,                   # theta, B, U-source in; theta, B out
+        "trace": 8 * n2,                                  # Q and Delta hi/lo
+        "algorithmic_step": (K * replica_bytes + 16) * n + 8 * n2,
+    }
+
+
+# --------------------------------------------------------------------------- CPU oracle arm
+CPU_SAMPLE = ["layers.0.attn_norm", "layers.0.wq", "layers.0.ffn_norm", "layers.0.w_gate", "layers.0.w_down"]
+REF_SAMPLE = ["layers.0.attn_norm", "layers.0.wq", "layers.0.ffn_norm"]
+
+
+def oracle_sample_run(workload: str, names, seed: int = 0):
+    """Runs the oracle's outer step on a sample of the workload's tensors, with the
+    workload's generator recipe (CPU generator).  Returns (params, seconds)."""
+    import oracle
+    from paper_2607_03011_gb300 import workloads as W
+    base = W.SPECS[workload]
+    shapes = [s for s in base.shapes if s[0] in names]
+    spec = W.custom_spec(shapes, K=base.K, rank=base.rank, shared_std=base.shared_std,
+                         noise_std=base.noise_std, momentum_std=base.momentum_std,
+                         replica_dtype=base.replica_dtype, name=base.name + "_sample")
+    wl = W.make_workload(spec, seed=seed, device="cpu")
+    reps = W.replicas_as_numpy(wl.replicas)
+    th, b = wl.theta.numpy(), wl.momentum.numpy()
+    t0 = time.perf_counter()
+    oracle.isoloco_outer_step(wl.table, th, b, reps, alpha=base.alpha, eta=base.outer_lr, mu=base.momentum)
+    dt = time.perf_counter() - t0
+    return wl.N, dt, "+".join(f"{n}:{r}x{c}" if c else f"{n}:{r}" for (n, r, c) in shapes)
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    import oracle
+    oracle.build()
+    cores = oracle.num_threads()
+    times, nparams, desc = [], 0, ""
+    for i in range(args.warmup + args.steps):
+        nparams, dt, desc = oracle_sample_run(args.workload, REF_SAMPLE, seed=i)
+        if i >= args.warmup:
+            times.append(dt)
+    ms = 1000.0 * sum(times) / len(times)
+    value = nparams / (ms / 1000.0)
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": args.workload, "sample": desc, "sample_params": nparams},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": f"oracle outer step on {desc} ({nparams} params) per step"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+# --------------------------------------------------------------------------- GPU arm
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="llama_180m_k8")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(3, args.warmup)
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+
+    from paper_2607_03011_gb300 import isoloco
+    from paper_2607_03011_gb300 import workloads as W
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    spec = W.SPECS[args.workload]
+    wl = W.make_workload(spec, seed=rank, device="cuda")
+    plan = isoloco.Plan(wl.table, wl.N, wl.K, wl.replicas.dtype)
+    opts = isoloco.make_opts(spec.alpha, spec.outer_lr, spec.momentum)
+    theta0, mom0 = wl.theta.clone(), wl.momentum.clone()
+    th, b = wl.theta, wl.momentum
+    stream = torch.cuda.current_stream()
+
+    def restore():
+        th.copy_(theta0)
+        b.copy_(mom0)
+
+    for _ in range(args.warmup):
+        restore()
+        rc = plan.outer_step(th, b, wl.replicas, opts)
+    if plan.last_status() not in (0,):
+        raise RuntimeError(f"warm-up step status {isoloco.STATUS_NAMES.get(plan.last_status())}")
+
+    # ---- timed region: K outer steps, each bracketed by CUDA events on the stream.
+    plan.profile(True)
+    launches0 = plan.launches
+    clocks = ClockSampler(local)
+    torch.cuda.synchronize()
+    barrier()
+    clocks.start()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    for i in range(args.steps):
+        restore()                       # outside the event pair: theta/B back to the step's inputs
+        ev[i][0].record(stream)
+        plan.outer_step(th, b, wl.replicas, opts)
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop()
+    status = plan.last_status()
+    step_ms = [a.elapsed_time(z) for a, z in ev]
+    total_ms = sum(step_ms)
+    launches = plan.launches - launches0
+    prof = plan.profile_read()
+    plan.profile(False)
+    diag = plan.read_diag()
+    if dist is not None:
+        t = torch.tensor([total_ms], device="cuda", dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+    value = world * wl.N * args.steps / (total_ms / 1000.0)
+
+    # ---- end-to-end through the host-buffer entry point (pinned host memory)
+    e2e = None
+    if not args.no_e2e and rank == 0:
+        th_h = theta0.cpu().pin_memory()
+        b_h = mom0.cpu().pin_memory()
+        th0_h, b0_h = th_h.clone(), b_h.clone()
+        reps_h = [wl.replicas[k].cpu().pin_memory() for k in range(wl.K)]
+        plan.outer_step_host(th_h, b_h, reps_h, opts)    # first call allocates the staging buffers
+        e_ms = []
+        for _ in range(args.e2e_steps):
+            th_h.copy_(th0_h)
+            b_h.copy_(b0_h)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            rc = plan.outer_step_host(th_h, b_h, reps_h, opts)
+            e1.record(stream)
+            e1.synchronize()
+            e_ms.append(e0.elapsed_time(e1))
+        rep_bytes = wl.replicas.element_size()
+        e2e = {"value": wl.N / (statistics.median(e_ms) / 1000.0), "unit": UNIT,
+               "h2d_bytes_per_step": int(wl.N * (4 + 4 + wl.K * rep_bytes)),
+               "d2h_bytes_per_step": int(wl.N * 8), "ms_per_step": statistics.median(e_ms),
+               "api": "isoloco_outer_step_host"}
+        del reps_h
+
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return 0
+
+    peaks, peak_src = load_peaks()
+    flops = gemm_flops(wl.table, diag) * args.steps
+    gemm_ms = prof["gram"][0] + prof["poly"][0] + prof["update"][0]
+    gemm_launches = prof["gram"][1] + prof["poly"][1] + prof["update"][1]
+    tc_peak = peaks["bf16_tflops_sustained"] / 3.0   # three bf16 tensor passes per fp32-accurate product
+    achieved_tf = flops / (gemm_ms / 1000.0) / 1e12 if gemm_ms > 0 else 0.0
+    sb = stream_bytes(wl.table, wl.K, wl.replicas.element_size())
+    hbm = peaks["hbm_gbs"]
+
+    def gbs(phase, nbytes):
+        ms, n = prof[phase]
+        return nbytes * args.steps / (ms / 1000.0) / 1e9 if ms > 0 else 0.0
+
+    roofline = {"bound": "tensor", "kernel": "k_gemm_bf16x3 (Gram, G^2 and update GEMMs)",
+                "achieved": achieved_tf, "peak": tc_peak, "unit": "TFLOP/s",
+                "frac": achieved_tf / tc_peak if tc_peak else None, "traffic": None,
+                "peak_source": f"{peak_src} bf16_tflops_sustained {peaks['bf16_tflops_sustained']} / 3 "
+                               "(bf16 hi/lo split: 3 tensor passes per product)",
+                "algorithmic_tflop_per_step": flops / args.steps / 1e12,
+                "executed_tensor_tflop_per_step": 3 * flops / args.steps / 1e12,
+                "gemm_ms_per_step": gemm_ms / args.steps, "gemm_launches_per_step": gemm_launches / args.steps}
+    roofline_hbm = {
+        "reduce": {"achieved": gbs("reduce", sb["reduce"]), "peak": hbm, "unit": "GB/s",
+                   "frac": gbs("reduce", sb["reduce"]) / hbm, "bytes_per_launch": sb["reduce"],
+                   "ms_per_step": prof["reduce"][0] / args.steps},
+        "apply": {"achieved": gbs("apply", sb["apply"]), "peak": hbm, "unit": "GB/s",
+                  "frac": gbs("apply", sb["apply"]) / hbm, "bytes_per_launch": sb["apply"],
+                  "ms_per_step": prof["apply"][0] / args.steps},
+        "trace": {"achieved": gbs("trace", sb["trace"]), "peak": hbm, "unit": "GB/s",
+                  "frac": gbs("trace", sb["trace"]) / hbm, "bytes_per_launch": sb["trace"],
+                  "ms_per_step": prof["trace"][0] / args.steps},
+        "peak_source": f"{peak_src} hbm_gbs",
+    }
+    phases_ms = {k: round(v[0] / args.steps, 4) for k, v in prof.items() if v[1]}
+
+    cpu = None
+    if not args.no_cpu_baseline and world == 1:
+        import oracle
+        oracle.build()
+        nparams, dt, desc = oracle_sample_run(args.workload, CPU_SAMPLE)
+        cpu = {"value": nparams / dt, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+               "sample": f"fp64 oracle outer step on {desc} ({nparams} params, {dt:.1f} s), "
+                         "same generator recipe"}
+
+    iters = diag["iters"]
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": args.workload, "params": wl.N, "K": wl.K, "matrices": plan.num_matrices,
+                   "replica_dtype": str(wl.replicas.dtype).replace("torch.", ""),
+                   "alpha": spec.alpha, "outer_lr": spec.outer_lr, "momentum": spec.momentum,
+                   "l2": "inputs larger than L2 (K replicas = %.1f GB)" % (wl.replicas.numel() *
+                                                                      wl.replicas.element_size() / 1e9),
+                   "timing": "sum of per-step CUDA-event intervals on the launch stream; theta/B "
+                             "restored between steps outside the intervals",
+                   "parallelism": f"replicas x{world}"},
+        "status": isoloco.STATUS_NAMES.get(status, status),
+        "polar_iters": {"min": min(iters), "max": max(iters), "mean": sum(iters) / len(iters)},
+        "phases_ms_per_step": phases_ms,
+        "roofline": roofline, "roofline_hbm": roofline_hbm,
+        "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
+        "clocks": clk, "step_ms": [round(x, 3) for x in step_ms],
+    }
+    print(json.dumps(line))
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

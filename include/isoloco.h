@@ -73,7 +73,7 @@ typedef struct {
     float outer_lr;   /* eta_out of Alg. 2. */
     float momentum;   /* mu of Alg. 2 (0 = plain SGD outer step, Eq. 2). */
     int reduce_mean;  /* 1: Delta is the mean over workers (Alg. 1/2); 0: the sum. */
-    int max_iter;     /* cap on polar iterations per matrix; <= 0 selects 29. */
+    int max_iter;     /* cap on quintic polar steps per matrix; <= 0 selects 28. */
     float tol;        /* convergence test ||X^T X - I||_F / sqrt(n) < tol; <= 0 selects 4e-3. */
     int sync;         /* 1: synchronize `stream` and return the step's device status. */
 } isoloco_opts_t;
@@ -153,6 +153,35 @@ int isoloco_plan_num_matrices(isoloco_plan_t plan);
  * cudaMalloc and synchronizes `stream` before returning. */
 int isoloco_debug_gemm(int a_mn_major, int b_mn_major, int batch, int M, int N, int K,
                        const float* A, const float* B, float* D, void* stream);
+
+/* Phases of the launch sequence, for isoloco_profile_read. */
+enum {
+    ISOLOCO_PHASE_REDUCE = 0,   /* pseudo-gradient reduction (HBM stream) */
+    ISOLOCO_PHASE_GRAM = 1,     /* X^T X (or X X^T) split-precision tcgen05 GEMMs */
+    ISOLOCO_PHASE_FINALIZE = 2, /* split-K sum of the Gram, convergence partials */
+    ISOLOCO_PHASE_CONTROL = 3,  /* per-matrix schedule / convergence decisions */
+    ISOLOCO_PHASE_POLY = 4,     /* G^2 GEMMs with the P = a I + b G + c G^2 epilogue */
+    ISOLOCO_PHASE_UPDATE = 5,   /* X P (or P X) GEMMs */
+    ISOLOCO_PHASE_TRACE = 6,    /* sigma_bar = tr(Q^T Delta) / n */
+    ISOLOCO_PHASE_APPLY = 7,    /* Nesterov update / merge output (HBM stream) */
+    ISOLOCO_PHASE_DILOCO = 8,   /* fused DiLoCo pass */
+    ISOLOCO_PHASE_OTHER = 9,
+    ISOLOCO_NUM_PHASES = 10
+};
+
+/* Per-phase timing.  enable != 0 makes every later call record a CUDA event pair
+ * around each phase's launches on the call's stream (a few microseconds of
+ * overhead per launch); enabling or disabling resets the accumulators and
+ * synchronizes the device.  Launch counts accumulate whether or not timing is on. */
+int isoloco_profile_enable(isoloco_plan_t plan, int enable);
+
+/* Synchronizes `stream`, then writes the accumulated milliseconds and launch
+ * counts of the first `nphases` phases (either array may be NULL). */
+int isoloco_profile_read(isoloco_plan_t plan, void* stream, double* ms_host, int64_t* launches_host,
+                         int nphases);
+
+/* Kernels launched by the plan since its creation. */
+int64_t isoloco_plan_launches(isoloco_plan_t plan);
 
 /* Thread-local message describing the last error returned on this thread. */
 const char* isoloco_last_error(void);

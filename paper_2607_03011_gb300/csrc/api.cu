@@ -99,6 +99,13 @@ struct isoloco_plan {
     uint32_t* err_h = nullptr;  // pinned
     CUtensorMap* tmaps_d = nullptr;
     cudaEvent_t done_ev = nullptr;
+    // phase timing (isoloco_profile_enable) and launch counting
+    bool prof = false;
+    std::vector<std::pair<cudaEvent_t, cudaEvent_t>> pend[ISOLOCO_NUM_PHASES];
+    std::vector<cudaEvent_t> ev_pool;
+    double prof_ms[ISOLOCO_NUM_PHASES] = {0};
+    int64_t prof_n[ISOLOCO_NUM_PHASES] = {0};
+    int64_t launches = 0;
     // staging for the host-buffer entry point (allocated on first use)
     float* st_theta = nullptr;
     float* st_mom = nullptr;
@@ -179,12 +186,52 @@ static int dalloc(isoloco_plan* p, T** ptr, int64_t count) {
 static void free_plan(isoloco_plan* p) {
     if (!p) return;
     for (void* a : p->allocs) cudaFree(a);
+    for (int ph = 0; ph < ISOLOCO_NUM_PHASES; ++ph)
+        for (auto& pr : p->pend[ph]) {
+            cudaEventDestroy(pr.first);
+            cudaEventDestroy(pr.second);
+        }
+    for (cudaEvent_t e : p->ev_pool) cudaEventDestroy(e);
     if (p->err_h) cudaFreeHost(p->err_h);
     if (p->done_ev) cudaEventDestroy(p->done_ev);
     delete p;
 }
 
 static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Records CUDA events around the launches of one phase when profiling is on, and
+// counts the launches either way.
+struct PhaseTimer {
+    isoloco_plan* p;
+    int phase;
+    cudaStream_t st;
+    cudaEvent_t e0 = nullptr;
+    static cudaEvent_t get(isoloco_plan* p) {
+        if (!p->ev_pool.empty()) {
+            cudaEvent_t e = p->ev_pool.back();
+            p->ev_pool.pop_back();
+            return e;
+        }
+        cudaEvent_t e = nullptr;
+        cudaEventCreate(&e);
+        return e;
+    }
+    PhaseTimer(isoloco_plan* p_, int ph, cudaStream_t s, int nlaunch = 1) : p(p_), phase(ph), st(s) {
+        p->launches += nlaunch;
+        p->prof_n[phase] += nlaunch;
+        if (p->prof) {
+            e0 = get(p);
+            cudaEventRecord(e0, st);
+        }
+    }
+    ~PhaseTimer() {
+        if (e0) {
+            cudaEvent_t e1 = get(p);
+            cudaEventRecord(e1, st);
+            p->pend[phase].emplace_back(e0, e1);
+        }
+    }
+};
 
 // ------------------------------------------------------------------ plan creation
 static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_params) {
@@ -390,29 +437,37 @@ static void set_group_common(GemmGroup& g, int M, int N, int K, int batch, int s
     g.mat_base = mat_base;
 }
 
+// Groups (one per shape bucket) of one GEMM phase; launched kMaxGroups at a time.
 struct LaunchSet {
     GemmParams p;
-    int cta = 0;
-    void add(const GemmGroup& g) {
-        p.g[p.num_groups] = g;
-        p.g[p.num_groups].cta_begin = cta;
-        cta += g.batch * g.tiles_m * g.tiles_n * g.splits;
-        p.num_groups++;
-    }
+    std::vector<GemmGroup> groups;
+    void add(const GemmGroup& g) { groups.push_back(g); }
 };
 
 static void init_set(LaunchSet& s, int epi, int gate, isoloco_plan* pl) {
     memset(&s.p, 0, sizeof(s.p));
-    s.cta = 0;
+    s.groups.clear();
     s.p.epi = epi;
     s.p.gate = gate;
     s.p.state = pl->state;
     s.p.err = pl->err_d;
 }
 
-static int flush_set(LaunchSet& s, bool a_mn, bool b_mn, cudaStream_t st) {
-    if (s.p.num_groups == 0) return ISOLOCO_OK;
-    CUDA_TRY(launch_gemm(s.p, a_mn, b_mn, st));
+static int flush_set(isoloco_plan* pl, int phase, LaunchSet& s, bool a_mn, bool b_mn, cudaStream_t st) {
+    if (s.groups.empty()) return ISOLOCO_OK;
+    PhaseTimer timer(pl, phase, st, (int)((s.groups.size() + kMaxGroups - 1) / kMaxGroups));
+    for (size_t first = 0; first < s.groups.size(); first += kMaxGroups) {
+        GemmParams p = s.p;
+        p.num_groups = 0;
+        int cta = 0;
+        for (size_t i = first; i < s.groups.size() && p.num_groups < kMaxGroups; ++i) {
+            GemmGroup g = s.groups[i];
+            g.cta_begin = cta;
+            cta += g.batch * g.tiles_m * g.tiles_n * g.splits;
+            p.g[p.num_groups++] = g;
+        }
+        CUDA_TRY(launch_gemm(p, a_mn, b_mn, st));
+    }
     return ISOLOCO_OK;
 }
 
@@ -445,13 +500,17 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             (bk.tall ? tall : wide).add(g);
         }
         int rc;
-        if ((rc = flush_set(tall, true, true, st)) || (rc = flush_set(wide, false, false, st))) return rc;
+        if ((rc = flush_set(p, ISOLOCO_PHASE_GRAM, tall, true, true, st)) ||
+            (rc = flush_set(p, ISOLOCO_PHASE_GRAM, wide, false, false, st)))
+            return rc;
+        { PhaseTimer tm(p, ISOLOCO_PHASE_FINALIZE, st);
         k_gram_finalize<<<p->nftiles, 256, 0, st>>>(p->mats_d, p->ftiles, p->state, p->gpart, p->gpart_off_d,
                                                     p->gpart_sstride_d, p->nsplit_d, p->gf32, p->ghi, p->glo,
-                                                    p->fin_part);
+                                                    p->fin_part); }
         CUDA_TRY(cudaGetLastError());
+        { PhaseTimer tm(p, ISOLOCO_PHASE_CONTROL, st);
         k_control<<<(p->nmat + 7) / 8, 256, 0, st>>>(p->mats_d, p->nmat, p->state, p->fin_part, t, max_iter, tol,
-                                                     p->err_d);
+                                                     p->err_d); }
         CUDA_TRY(cudaGetLastError());
         // ---- P = a I + b G + c G^2
         LaunchSet poly;
@@ -474,7 +533,7 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             g.ld_g = bk.ld_n;
             poly.add(g);
         }
-        if ((rc = flush_set(poly, false, false, st))) return rc;
+        if ((rc = flush_set(p, ISOLOCO_PHASE_POLY, poly, false, false, st))) return rc;
         // ---- X_{t+1} = xscale * X_t P (tall) or P X_t (wide)
         LaunchSet utall, uwide;
         init_set(utall, kEpiXSplit, kGateStep, p);
@@ -501,12 +560,15 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             g.ld_bf = bk.ld;
             (bk.tall ? utall : uwide).add(g);
         }
-        if ((rc = flush_set(utall, false, false, st)) || (rc = flush_set(uwide, false, true, st))) return rc;
+        if ((rc = flush_set(p, ISOLOCO_PHASE_UPDATE, utall, false, false, st)) ||
+            (rc = flush_set(p, ISOLOCO_PHASE_UPDATE, uwide, false, true, st)))
+            return rc;
     }
+    { PhaseTimer tm(p, ISOLOCO_PHASE_TRACE, st, 2);
     k_trace_partial<<<p->ntchunks, 256, 0, st>>>(p->mats_d, p->tchunks, p->state, p->dhi, p->dlo, p->xhi[0],
                                                  p->xlo[0], p->xhi[1], p->xlo[1], p->tpart);
     CUDA_TRY(cudaGetLastError());
-    k_trace_final<<<(p->nmat + 7) / 8, 256, 0, st>>>(p->mats_d, p->nmat, p->state, p->tpart);
+    k_trace_final<<<(p->nmat + 7) / 8, 256, 0, st>>>(p->mats_d, p->nmat, p->state, p->tpart); }
     CUDA_TRY(cudaGetLastError());
     return ISOLOCO_OK;
 }
@@ -549,9 +611,11 @@ static int run_isoc_step(isoloco_plan* p, int merge, float* theta, float* mom, c
     CUDA_TRY(cudaSetDevice(p->device));
     const float* th_src = merge ? base : theta;
     const float scale = merge ? -1.f : (o.reduce_mean ? 1.f / (float)p->K : 1.f);
-    k_reset_state<<<(std::max(1, p->nmat) + 255) / 256, 256, 0, st>>>(p->state, p->nmat, p->err_d);
+    { PhaseTimer tm(p, ISOLOCO_PHASE_OTHER, st);
+    k_reset_state<<<(std::max(1, p->nmat) + 255) / 256, 256, 0, st>>>(p->state, p->nmat, p->err_d); }
     CUDA_TRY(cudaGetLastError());
     if (p->nchunks) {
+        PhaseTimer tm(p, ISOLOCO_PHASE_REDUCE, st);
         k_reduce<<<p->nchunks, 256, 0, st>>>(p->chunks_d, p->mats_d, rp, p->K, p->dtype, th_src, scale, p->dhi,
                                              p->dlo, p->d1d, p->err_d);
         CUDA_TRY(cudaGetLastError());
@@ -564,6 +628,7 @@ static int run_isoc_step(isoloco_plan* p, int merge, float* theta, float* mom, c
     us.ql[1] = p->xlo[1];
     us.d1d = p->d1d;
     if (p->nchunks) {
+        PhaseTimer tm(p, ISOLOCO_PHASE_APPLY, st);
         if (merge)
             k_apply<<<p->nchunks, 256, 0, st>>>(p->chunks_d, p->mats_d, p->state, us, 1, alpha_merge, 0.f, 0.f,
                                                 nullptr, nullptr, base, out, nullptr, p->err_d);
@@ -680,8 +745,9 @@ int diloco_outer_step(isoloco_plan_t p, float* theta, float* momentum, const voi
     CUDA_TRY(cudaMemsetAsync(p->err_d, 0, 4, st));
     const float scale = o.reduce_mean ? 1.f / (float)p->K : 1.f;
     const int grid = p->num_sms * 8;
+    { PhaseTimer tm(p, ISOLOCO_PHASE_DILOCO, st);
     k_diloco<<<grid, 256, 0, st>>>(rp, p->K, p->dtype, theta, momentum, p->N, scale, o.outer_lr, o.momentum,
-                                   p->err_d);
+                                   p->err_d); }
     CUDA_TRY(cudaGetLastError());
     return finish_call(p, st, o.sync);
 }
@@ -731,6 +797,44 @@ int isoloco_last_status(isoloco_plan_t p, void* stream) {
     if (e & kErrNotConverged) return fail(ISOLOCO_ERR_NOT_CONVERGED, "polar iteration hit max_iter");
     return ISOLOCO_OK;
 }
+
+int isoloco_profile_enable(isoloco_plan_t p, int enable) {
+    if (!p) return fail(ISOLOCO_ERR_INVALID, "plan is NULL");
+    CUDA_TRY(cudaDeviceSynchronize());
+    for (int ph = 0; ph < ISOLOCO_NUM_PHASES; ++ph) {
+        for (auto& pr : p->pend[ph]) {
+            p->ev_pool.push_back(pr.first);
+            p->ev_pool.push_back(pr.second);
+        }
+        p->pend[ph].clear();
+        p->prof_ms[ph] = 0.0;
+        p->prof_n[ph] = 0;
+    }
+    p->prof = enable != 0;
+    return ISOLOCO_OK;
+}
+
+int isoloco_profile_read(isoloco_plan_t p, void* stream, double* ms, int64_t* launches, int nphases) {
+    if (!p) return fail(ISOLOCO_ERR_INVALID, "plan is NULL");
+    CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+    for (int ph = 0; ph < ISOLOCO_NUM_PHASES; ++ph) {
+        for (auto& pr : p->pend[ph]) {
+            float t = 0.f;
+            CUDA_TRY(cudaEventElapsedTime(&t, pr.first, pr.second));
+            p->prof_ms[ph] += t;
+            p->ev_pool.push_back(pr.first);
+            p->ev_pool.push_back(pr.second);
+        }
+        p->pend[ph].clear();
+    }
+    for (int ph = 0; ph < nphases && ph < ISOLOCO_NUM_PHASES; ++ph) {
+        if (ms) ms[ph] = p->prof_ms[ph];
+        if (launches) launches[ph] = p->prof_n[ph];
+    }
+    return ISOLOCO_OK;
+}
+
+int64_t isoloco_plan_launches(isoloco_plan_t p) { return p ? p->launches : 0; }
 
 int isoloco_read_diag(isoloco_plan_t p, void* stream, float* sigma_bar, int32_t* iters, int32_t* status,
                       float* resid) {

@@ -17,6 +17,8 @@ import torch
 
 from . import _build
 
+PHASES = ["reduce", "gram", "finalize", "control", "poly", "update", "trace", "apply", "diloco", "other"]
+
 OK = 0
 ERR_INVALID = -1
 ERR_ALIGN = -2
@@ -73,6 +75,10 @@ def lib():
             L.iso_c_merge.argtypes = [_vp, _vp, ctypes.POINTER(_vp), ctypes.c_float, _vp, _vp]
             L.isoloco_last_status.argtypes = [_vp, _vp]
             L.isoloco_read_diag.argtypes = [_vp, _vp, _vp, _vp, _vp, _vp]
+            L.isoloco_profile_enable.argtypes = [_vp, ctypes.c_int]
+            L.isoloco_profile_read.argtypes = [_vp, _vp, _vp, _vp, ctypes.c_int]
+            L.isoloco_plan_launches.argtypes = [_vp]
+            L.isoloco_plan_launches.restype = ctypes.c_int64
             L.isoloco_debug_gemm.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                              ctypes.c_int, _vp, _vp, _vp, _vp]
             _lib = L
@@ -202,6 +208,23 @@ class Plan:
 
     def last_status(self, stream=None) -> int:
         return int(self._L.isoloco_last_status(self._h, _stream(stream)))
+
+    def profile(self, enable: bool = True):
+        """Turns per-phase CUDA-event timing on or off (resets the accumulators)."""
+        _check(self._L.isoloco_profile_enable(self._h, int(bool(enable))), "isoloco_profile_enable")
+
+    def profile_read(self, stream=None):
+        """{phase: (milliseconds, launches)} accumulated since profile() was called."""
+        n = len(PHASES)
+        ms = (ctypes.c_double * n)()
+        cnt = (ctypes.c_int64 * n)()
+        _check(self._L.isoloco_profile_read(self._h, _stream(stream), ms, cnt, n), "isoloco_profile_read")
+        return {ph: (ms[i], cnt[i]) for i, ph in enumerate(PHASES)}
+
+    @property
+    def launches(self) -> int:
+        """Kernels launched by this plan since its creation."""
+        return int(self._L.isoloco_plan_launches(self._h))
 
     def read_diag(self, stream=None):
         n = self.num_matrices

@@ -157,7 +157,9 @@ def make_replicas(spec: WorkloadSpec, table, theta: torch.Tensor, seed: int,
     g = _gen(device, seed * 7919 + 17)
     shared = _shared_part(spec, table, device, g)
     dt = torch.bfloat16 if spec.replica_dtype == "bf16" else torch.float32
-    reps = torch.empty((K, theta.numel()), dtype=dt, device=device)
+    # rows padded to 64 elements so every replica starts 16-byte aligned
+    n = theta.numel()
+    reps = torch.empty((K, (n + 63) // 64 * 64), dtype=dt, device=device)[:, :n]
     for k in range(K):
         gk = _gen(device, seed * 1_000_003 + 1000 + k)
         noise = torch.randn(theta.numel(), generator=gk, device=device) * spec.noise_std

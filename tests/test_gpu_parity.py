@@ -56,7 +56,7 @@ def test_tiny_two_steps(iso):
     worst, ref = compare(wl, rc, th, b, upd, diag, sp.alpha, sp.outer_lr, sp.momentum)
     assert all(s == 0 for s in diag["status"])
     # step 2: each side regenerates replicas (seed 1) from its own theta and keeps its B
-    th_o = torch.from_numpy(ref["theta"].astype(np.float32))
+    th_o = torch.from_numpy(ref["theta"].astype(np.float32)).cuda()   # the oracle's own step-1 result
     b_o = torch.from_numpy(ref["momentum"].astype(np.float32))
     reps_g = W.make_replicas(sp, wl.table, th, seed=1)
     reps_o = W.make_replicas(sp, wl.table, th_o, seed=1)
@@ -65,9 +65,9 @@ def test_tiny_two_steps(iso):
     rc = plan.outer_step(th2, b2, reps_g, iso.make_opts(sp.alpha, sp.outer_lr, sp.momentum, sync=True),
                          update_out=upd2)
     assert rc == 0
-    ref2 = oracle.isoloco_outer_step(wl.table, th_o.numpy(), b_o.numpy(), W.replicas_as_numpy(reps_o),
+    ref2 = oracle.isoloco_outer_step(wl.table, th_o.cpu().numpy(), b_o.numpy(), W.replicas_as_numpy(reps_o),
                                      alpha=sp.alpha, eta=sp.outer_lr, mu=sp.momentum)
-    ref2["theta_in"] = th_o.double().numpy()
+    ref2["theta_in"] = th_o.double().cpu().numpy()
     check_step(wl.table, th2.double().cpu().numpy(), b2.double().cpu().numpy(), upd2.double().cpu().numpy(),
                plan.read_diag()["sigma_bar"], ref2)
 
