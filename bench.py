@@ -92,21 +92,23 @@ class ClockSampler:
 
 # --------------------------------------------------------------------------- accounting
 def gemm_flops(table, diag):
-    """Algorithmic (single-pass) FLOPs of the polar GEMMs of one step, from the
-    per-matrix iteration counts: a full Gram 2*r*n^2 and an update 2*r*n^2 per
-    iteration, G^2 = 2*n^3 per quintic step (r = long side, n = short side)."""
-    total = 0.0
+    """Algorithmic (single-pass) FLOPs of the polar GEMMs of one step, per phase, from
+    the per-matrix iteration counts: a full Gram 2*r*n^2 per iteration (symmetry not
+    discounted), G^2 = 2*n^3 per quintic step, an update 2*r*n^2 per iteration
+    (r = long side, n = short side of the matrix)."""
+    out = {"gram": 0.0, "poly": 0.0, "update": 0.0}
     mats = [(r, c) for (_, r, c) in table if c > 0]
-    for (r, c), it, st, sb in zip(mats, diag["iters"], diag["status"], diag["sigma_bar"]):
+    for (r, c), it, st in zip(mats, diag["iters"], diag["status"]):
         big, small = max(r, c), min(r, c)
+        gram1, sq1 = 2.0 * big * small * small, 2.0 * small ** 3
         if it == 0:
-            total += 2.0 * big * small * small  # one Gram, then found zero
+            out["gram"] += gram1  # one Gram, then found zero
             continue
         converged = (st == 0)
-        grams = it + (0 if converged else 1)
-        quintic = it - (1 if converged else 0)
-        total += grams * 2.0 * big * small ** 2 + it * 2.0 * big * small ** 2 + quintic * 2.0 * small ** 3
-    return total
+        out["gram"] += (it + (0 if converged else 1)) * gram1
+        out["poly"] += (it - (1 if converged else 0)) * sq1
+        out["update"] += it * gram1
+    return out
 
 
 def stream_bytes(table, K, replica_bytes):
@@ -282,7 +284,8 @@ def main():
         return 0
 
     peaks, peak_src = load_peaks()
-    flops = gemm_flops(wl.table, diag) * args.steps
+    fl = gemm_flops(wl.table, diag)
+    flops = sum(fl.values()) * args.steps
     gemm_ms = prof["gram"][0] + prof["poly"][0] + prof["update"][0]
     gemm_launches = prof["gram"][1] + prof["poly"][1] + prof["update"][1]
     tc_peak = peaks["bf16_tflops_sustained"] / 3.0   # three bf16 tensor passes per fp32-accurate product
@@ -315,6 +318,8 @@ def main():
         "peak_source": f"{peak_src} hbm_gbs",
     }
     phases_ms = {k: round(v[0] / args.steps, 4) for k, v in prof.items() if v[1]}
+    phases_tflops = {k: round(fl[k] / (prof[k][0] / args.steps / 1000.0) / 1e12, 1)
+                     for k in fl if prof[k][0] > 0}
 
     cpu = None
     if not args.no_cpu_baseline and world == 1:
@@ -340,7 +345,7 @@ def main():
                    "parallelism": f"replicas x{world}"},
         "status": isoloco.STATUS_NAMES.get(status, status),
         "polar_iters": {"min": min(iters), "max": max(iters), "mean": sum(iters) / len(iters)},
-        "phases_ms_per_step": phases_ms,
+        "phases_ms_per_step": phases_ms, "phases_algorithmic_tflops": phases_tflops,
         "roofline": roofline, "roofline_hbm": roofline_hbm,
         "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
         "clocks": clk, "step_ms": [round(x, 3) for x in step_ms],

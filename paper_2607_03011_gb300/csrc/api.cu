@@ -26,7 +26,7 @@ namespace isoloco {
 // kernels defined in the other translation units
 cudaError_t launch_gemm(const GemmParams& p, bool a_mn, bool b_mn, cudaStream_t stream);
 __global__ void k_gram_finalize(const MatDesc*, const int2*, const MatState*, const float*, const int64_t*,
-                                const int64_t*, const int*, float*, __nv_bfloat16*, __nv_bfloat16*, float*);
+                                const int64_t*, const int*, __nv_bfloat16*, __nv_bfloat16*, float*);
 __global__ void k_control(const MatDesc*, int, MatState*, const float*, int, int, float, uint32_t*);
 __global__ void k_trace_partial(const MatDesc*, const int4*, const MatState*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, const __nv_bfloat16*,
@@ -42,7 +42,6 @@ __global__ void k_split_planes(const float*, int64_t, int, int, int, __nv_bfloat
 
 constexpr int kChunkElems = 16384;
 constexpr int kTraceChunkElems = 16384;
-constexpr int kFinTileEdge = 64;
 constexpr int kDefaultMaxIter = 28;
 constexpr float kDefaultTol = 4e-3f;
 
@@ -81,7 +80,6 @@ struct isoloco_plan {
     std::vector<void*> allocs;
     int64_t ws_bytes = 0;
     __nv_bfloat16 *dhi = nullptr, *dlo = nullptr, *xhi[2] = {nullptr, nullptr}, *xlo[2] = {nullptr, nullptr};
-    float* gf32 = nullptr;
     __nv_bfloat16 *ghi = nullptr, *glo = nullptr, *phi = nullptr, *plo = nullptr;
     float* gpart = nullptr;
     float* d1d = nullptr;
@@ -167,6 +165,15 @@ static bool make_map(CUtensorMap* m, const void* base, int cols, int rows, int c
 }
 
 static inline int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
+
+// Output tiles of an n x n symmetric product that touch the upper triangle.
+static int sym_tiles(int n) {
+    const int tm_n = (n + BM - 1) / BM, tn_n = (n + BN - 1) / BN;
+    int c = 0;
+    for (int tm = 0; tm < tm_n; ++tm) c += tn_n - sym_first_tile_n(tm);
+    return c;
+}
+
 
 template <typename T>
 static int dalloc(isoloco_plan* p, T** ptr, int64_t count) {
@@ -277,17 +284,19 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         bk.gplane_off = gplane;
         bk.gpart_off = gpart;
         // split-K for the Gram when the bucket has few output tiles
-        const int tiles = ((bk.n + BM - 1) / BM) * ((bk.n + BN - 1) / BN) * bk.count;
+        const int tiles = sym_tiles(bk.n) * bk.count;
         const int kdim = bk.tall ? bk.rows : bk.cols;
         const int kblocks = (kdim + BK - 1) / BK;
-        int splits = std::max(1, (2 * p->num_sms) / std::max(1, tiles));
+        int splits = std::max(1, (2 * kGemmCtasPerSm * p->num_sms) / std::max(1, tiles));
         splits = std::min(splits, std::max(1, kblocks / 8));
         int kper = (kblocks + splits - 1) / splits;
         splits = (kblocks + kper - 1) / kper;  // no empty split
         bk.splits = splits;
         const int64_t mat_elems = (int64_t)bk.rows * bk.ld;
         const int64_t g_elems = (int64_t)bk.n * bk.ld_n;
-        const int ftc = (bk.n + kFinTileEdge - 1) / kFinTileEdge;
+        // Gram partial-sum slots per matrix: one per computed Gram tile (upper-triangle
+        // tiles) when the Gram's epilogue produces them, one per finalize tile otherwise
+        const int gtiles = splits > 1 ? ((bk.n + BM - 1) / BM) * ((bk.n + BN - 1) / BN) : sym_tiles(bk.n);
         for (int j = 0; j < bk.count; ++j) {
             const int pi = members[b][j];
             MatDesc md{};
@@ -301,12 +310,13 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
             md.bucket = (int)b;
             md.gslot = gplane + j * g_elems;
             md.gpart_slot = fin;
-            md.n_gtiles = ftc * ftc;
+            md.n_gtiles = gtiles;
             md.trace_part = tr;
             const int rows_per = std::max(1, kTraceChunkElems / bk.cols);
             md.n_tchunks = (bk.rows + rows_per - 1) / rows_per;
             const int mi = (int)p->mats_h.size();
-            for (int t = 0; t < md.n_gtiles; ++t) ftiles.push_back(make_int2(mi, t));
+            if (splits > 1)
+                for (int t = 0; t < md.n_gtiles; ++t) ftiles.push_back(make_int2(mi, t));
             for (int c = 0; c < md.n_tchunks; ++c) {
                 const int r0 = c * rows_per;
                 tchunks.push_back(make_int4(mi, r0, std::min(rows_per, bk.rows - r0), c));
@@ -360,10 +370,10 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
     int rc;
     if ((rc = dalloc(p, &p->dhi, plane)) || (rc = dalloc(p, &p->dlo, plane)) || (rc = dalloc(p, &p->xhi[0], plane)) ||
         (rc = dalloc(p, &p->xlo[0], plane)) || (rc = dalloc(p, &p->xhi[1], plane)) ||
-        (rc = dalloc(p, &p->xlo[1], plane)) || (rc = dalloc(p, &p->gf32, gplane)) ||
+        (rc = dalloc(p, &p->xlo[1], plane)) ||
         (rc = dalloc(p, &p->ghi, gplane)) || (rc = dalloc(p, &p->glo, gplane)) || (rc = dalloc(p, &p->phi, gplane)) ||
         (rc = dalloc(p, &p->plo, gplane)) || (rc = dalloc(p, &p->gpart, gpart)) || (rc = dalloc(p, &p->d1d, d1)) ||
-        (rc = dalloc(p, &p->fin_part, 3 * fin)) || (rc = dalloc(p, &p->ftiles, fin)) ||
+        (rc = dalloc(p, &p->fin_part, 3 * fin)) || (rc = dalloc(p, &p->ftiles, (int64_t)ftiles.size())) ||
         (rc = dalloc(p, &p->tpart, tr)) || (rc = dalloc(p, &p->tchunks, tr)) ||
         (rc = dalloc(p, &p->state, p->nmat)) || (rc = dalloc(p, &p->mats_d, p->nmat)) ||
         (rc = dalloc(p, &p->gpart_off_d, p->nmat)) || (rc = dalloc(p, &p->gpart_sstride_d, p->nmat)) ||
@@ -380,14 +390,14 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         CUDA_TRY(cudaMemset(a, 0, std::max<int64_t>(1, plane) * 2));
     for (void* a : {(void*)p->ghi, (void*)p->glo, (void*)p->phi, (void*)p->plo})
         CUDA_TRY(cudaMemset(a, 0, std::max<int64_t>(1, gplane) * 2));
-    CUDA_TRY(cudaMemset(p->gf32, 0, std::max<int64_t>(1, gplane) * 4));
     CUDA_TRY(cudaMemset(p->err_d, 0, 4));
     if (p->nmat) {
         CUDA_TRY(cudaMemcpy(p->mats_d, p->mats_h.data(), sizeof(MatDesc) * p->nmat, cudaMemcpyHostToDevice));
         CUDA_TRY(cudaMemcpy(p->gpart_off_d, gpoff.data(), sizeof(int64_t) * p->nmat, cudaMemcpyHostToDevice));
         CUDA_TRY(cudaMemcpy(p->gpart_sstride_d, gpss.data(), sizeof(int64_t) * p->nmat, cudaMemcpyHostToDevice));
         CUDA_TRY(cudaMemcpy(p->nsplit_d, nsp.data(), sizeof(int) * p->nmat, cudaMemcpyHostToDevice));
-        CUDA_TRY(cudaMemcpy(p->ftiles, ftiles.data(), sizeof(int2) * fin, cudaMemcpyHostToDevice));
+        if (!ftiles.empty())
+            CUDA_TRY(cudaMemcpy(p->ftiles, ftiles.data(), sizeof(int2) * ftiles.size(), cudaMemcpyHostToDevice));
         CUDA_TRY(cudaMemcpy(p->tchunks, tchunks.data(), sizeof(int4) * tr, cudaMemcpyHostToDevice));
     }
     if (p->nchunks)
@@ -438,6 +448,14 @@ static void set_group_common(GemmGroup& g, int M, int N, int K, int batch, int s
 }
 
 // Groups (one per shape bucket) of one GEMM phase; launched kMaxGroups at a time.
+static void set_sym(GemmGroup& g, int n) {
+    g.sym = 1;
+    g.tiles_sym = sym_tiles(n);
+}
+
+// Output tiles of one matrix of a group.
+static int group_tiles(const GemmGroup& g) { return g.sym ? g.tiles_sym : g.tiles_m * g.tiles_n; }
+
 struct LaunchSet {
     GemmParams p;
     std::vector<GemmGroup> groups;
@@ -463,7 +481,7 @@ static int flush_set(isoloco_plan* pl, int phase, LaunchSet& s, bool a_mn, bool 
         for (size_t i = first; i < s.groups.size() && p.num_groups < kMaxGroups; ++i) {
             GemmGroup g = s.groups[i];
             g.cta_begin = cta;
-            cta += g.batch * g.tiles_m * g.tiles_n * g.splits;
+            cta += g.batch * group_tiles(g) * g.splits;
             p.g[p.num_groups++] = g;
         }
         CUDA_TRY(launch_gemm(p, a_mn, b_mn, st));
@@ -480,8 +498,8 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
         const int dst = (t + 1) & 1;
         // ---- Gram G = X^T X (tall, MN-major operands) or X X^T (wide, K-major)
         LaunchSet tall, wide;
-        init_set(tall, kEpiF32, kGateActive, p);
-        init_set(wide, kEpiF32, kGateActive, p);
+        init_set(tall, kEpiGram, kGateActive, p);
+        init_set(wide, kEpiGram, kGateActive, p);
         for (size_t b = 0; b < p->buckets.size(); ++b) {
             const Bucket& bk = p->buckets[b];
             const CUtensorMap* m = maps + b * kMapsPerBucket;
@@ -497,17 +515,26 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             g.f32_batch_stride = (int64_t)bk.n * bk.ld_n;
             g.f32_split_stride = (int64_t)bk.count * bk.n * bk.ld_n;
             g.ld_f32 = bk.ld_n;
+            g.out_hi = p->ghi + bk.gplane_off;
+            g.out_lo = p->glo + bk.gplane_off;
+            g.bf_batch_stride = (int64_t)bk.n * bk.ld_n;
+            g.ld_bf = bk.ld_n;
+            g.part = p->fin_part;
+            g.part_base = p->mats_h[bk.mat_base].gpart_slot;
+            set_sym(g, bk.n);
             (bk.tall ? tall : wide).add(g);
         }
         int rc;
         if ((rc = flush_set(p, ISOLOCO_PHASE_GRAM, tall, true, true, st)) ||
             (rc = flush_set(p, ISOLOCO_PHASE_GRAM, wide, false, false, st)))
             return rc;
-        { PhaseTimer tm(p, ISOLOCO_PHASE_FINALIZE, st);
-        k_gram_finalize<<<p->nftiles, 256, 0, st>>>(p->mats_d, p->ftiles, p->state, p->gpart, p->gpart_off_d,
-                                                    p->gpart_sstride_d, p->nsplit_d, p->gf32, p->ghi, p->glo,
-                                                    p->fin_part); }
-        CUDA_TRY(cudaGetLastError());
+        if (p->nftiles) {
+            PhaseTimer tm(p, ISOLOCO_PHASE_FINALIZE, st);
+            k_gram_finalize<<<p->nftiles, 256, 0, st>>>(p->mats_d, p->ftiles, p->state, p->gpart, p->gpart_off_d,
+                                                        p->gpart_sstride_d, p->nsplit_d, p->ghi, p->glo,
+                                                        p->fin_part);
+            CUDA_TRY(cudaGetLastError());
+        }
         { PhaseTimer tm(p, ISOLOCO_PHASE_CONTROL, st);
         k_control<<<(p->nmat + 7) / 8, 256, 0, st>>>(p->mats_d, p->nmat, p->state, p->fin_part, t, max_iter, tol,
                                                      p->err_d); }
@@ -528,9 +555,9 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             g.out_lo = p->plo + bk.gplane_off;
             g.bf_batch_stride = (int64_t)bk.n * bk.ld_n;
             g.ld_bf = bk.ld_n;
-            g.g_f32 = p->gf32 + bk.gplane_off;
-            g.g_batch_stride = (int64_t)bk.n * bk.ld_n;
-            g.ld_g = bk.ld_n;
+            g.g_hi = p->ghi + bk.gplane_off;
+            g.g_lo = p->glo + bk.gplane_off;
+            set_sym(g, bk.n);
             poly.add(g);
         }
         if ((rc = flush_set(p, ISOLOCO_PHASE_POLY, poly, false, false, st))) return rc;

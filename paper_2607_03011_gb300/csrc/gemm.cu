@@ -76,10 +76,26 @@ __device__ __forceinline__ void store_bf16_row(__nv_bfloat16* hi_row, __nv_bfloa
     }
 }
 
+// Symmetric outputs: the t-th of the tiles that touch the upper triangle (col >= row),
+// in row-major order of tiles.
+__device__ __forceinline__ void sym_tile(int t, int tiles_m, int tiles_n, int& tm, int& tn) {
+    for (tm = 0; tm < tiles_m; ++tm) {
+        const int lo = sym_first_tile_n(tm);
+        const int cnt = tiles_n - lo;
+        if (t < cnt) {
+            tn = lo + t;
+            return;
+        }
+        t -= cnt;
+    }
+    tm = tiles_m - 1;
+    tn = tiles_n - 1;
+}
+
 }  // namespace
 
 template <bool A_MN, bool B_MN>
-__global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_bf16x3(const __grid_constant__ GemmParams p) {
+__global__ void __launch_bounds__(kGemmThreads, kGemmCtasPerSm) k_gemm_bf16x3(const __grid_constant__ GemmParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = align1024(smem_raw);
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
@@ -87,6 +103,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_bf16x3(const __grid_co
     uint64_t* accbar = empty + kStages;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accbar + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    float* red = reinterpret_cast<float*>(tmem_slot + 4);  // [4 warps][3] epilogue partial sums
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -98,12 +115,19 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_bf16x3(const __grid_co
     int local = static_cast<int>(blockIdx.x) - g.cta_begin;
     const int split = local % g.splits;
     local /= g.splits;
-    const int ntiles = g.tiles_m * g.tiles_n;
+    const int ntiles = g.sym ? g.tiles_sym : g.tiles_m * g.tiles_n;
     const int tile = local % ntiles;
     const int b = local / ntiles;
     if (b >= g.batch) return;
-    const int m0 = (tile / g.tiles_n) * BM;
-    const int n0 = (tile % g.tiles_n) * BN;
+    int tm, tn;
+    if (g.sym) {
+        sym_tile(tile, g.tiles_m, g.tiles_n, tm, tn);
+    } else {
+        tm = tile / g.tiles_n;
+        tn = tile % g.tiles_n;
+    }
+    const int m0 = tm * BM;
+    const int n0 = tn * BN;
     const int mat = g.mat_base + b;
 
     bool run_mma = true;
@@ -245,6 +269,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_bf16x3(const __grid_co
         }
     } else {
         // ================= epilogue (warps 2..5)
+        // Thread (eg, lane) owns output row `row` of the tile and walks its 256 columns
+        // in chunks of 32 (one tcgen05.ld each).  In symmetric mode (Gram, G^2) only
+        // entries with col >= row are produced from the accumulator; each entry with
+        // col > row is also written, bitwise identical, at (col, row).  Across a warp the
+        // mirrored stores hit 32 consecutive rows of one column: coalesced.
         const int eg = warp & 3;  // tensor-memory lane quarter this warp may access
         const bool ok = __all_sync(0xffffffffu, mbar_wait(accbar, 0));
         if (!ok && lane == 0) atomicOr(p.err, kErrTimeout);
@@ -252,6 +281,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_bf16x3(const __grid_co
         tc_fence_after();
         const int row = m0 + eg * 32 + lane;
         const bool row_ok = row < g.M;
+        const bool sym = g.sym != 0;
+        const bool f32_out = (p.epi == kEpiF32) || (p.epi == kEpiGram && g.splits > 1);
+        const bool gram_fused = (p.epi == kEpiGram && g.splits == 1);
+        float s_sq = 0.f, s_tr = 0.f, s_dev = 0.f;
         for (int c32 = 0; c32 < BN / 32; ++c32) {
             const int col0 = n0 + c32 * 32;
             if (col0 >= g.N) break;
@@ -267,12 +300,60 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_bf16x3(const __grid_co
 #pragma unroll
                 for (int j = 0; j < 32; ++j) v[j] = 0.f;
             }
-            if (row_ok) {
             const int nvalid = min(32, g.N - col0);
-            if (p.epi == kEpiF32) {
-                float* out = g.out_f32 + split * g.f32_split_stride + b * g.f32_batch_stride +
-                             static_cast<int64_t>(row) * g.ld_f32 + col0;
-                if (nvalid == 32 && (g.ld_f32 & 3) == 0) {
+            const int d = row - col0;  // column index of the diagonal inside this chunk
+            // chunk entirely below the diagonal: produced by a mirror elsewhere
+            if (!row_ok || (sym && d > nvalid - 1)) continue;
+            const bool upper_all = !sym || d < 0;  // every column of the chunk has col > row
+            const int64_t goff = b * g.bf_batch_stride + static_cast<int64_t>(row) * g.ld_bf + col0;
+            if (p.epi == kEpiPoly) {
+                const __nv_bfloat16* gh = g.g_hi + goff;
+                const __nv_bfloat16* gl = g.g_lo + goff;
+                if (nvalid == 32) {
+                    const uint4* h4 = reinterpret_cast<const uint4*>(gh);
+                    const uint4* l4 = reinterpret_cast<const uint4*>(gl);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const uint4 hh = h4[q], ll = l4[q];
+                        const uint32_t hw[4] = {hh.x, hh.y, hh.z, hh.w};
+                        const uint32_t lw[4] = {ll.x, ll.y, ll.z, ll.w};
+#pragma unroll
+                        for (int w = 0; w < 4; ++w) {
+                            const float g0 = __uint_as_float(hw[w] << 16) + __uint_as_float(lw[w] << 16);
+                            const float g1 = __uint_as_float(hw[w] & 0xFFFF0000u) + __uint_as_float(lw[w] & 0xFFFF0000u);
+                            v[8 * q + 2 * w] = cc * v[8 * q + 2 * w] + cb * g0;
+                            v[8 * q + 2 * w + 1] = cc * v[8 * q + 2 * w + 1] + cb * g1;
+                        }
+                    }
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        if (j < nvalid) v[j] = cc * v[j] + cb * (__bfloat162float(gh[j]) + __bfloat162float(gl[j]));
+                }
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                    if (j == d) v[j] += ca;
+            } else if (p.epi == kEpiXSplit) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) v[j] *= xs;
+            }
+            if (gram_fused) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+                    if (j < nvalid && (!sym || j >= d)) {
+                        const float x = v[j];
+                        const float e = (j == d) ? x - 1.f : x;
+                        const float w = (sym && j > d) ? 2.f : 1.f;  // mirrored entry counts twice
+                        s_sq = fmaf(w * x, x, s_sq);
+                        s_dev = fmaf(w * e, e, s_dev);
+                        if (j == d) s_tr += x;
+                    }
+                }
+            }
+            if (f32_out) {
+                float* base = g.out_f32 + split * g.f32_split_stride + b * g.f32_batch_stride;
+                float* out = base + static_cast<int64_t>(row) * g.ld_f32 + col0;
+                if (upper_all && nvalid == 32 && (g.ld_f32 & 3) == 0) {
                     float4* o4 = reinterpret_cast<float4*>(out);
 #pragma unroll
                     for (int q = 0; q < 8; ++q)
@@ -280,40 +361,60 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_bf16x3(const __grid_co
                 } else {
 #pragma unroll
                     for (int j = 0; j < 32; ++j)
-                        if (j < nvalid) out[j] = v[j];
+                        if (j < nvalid && (!sym || j >= d)) out[j] = v[j];
+                }
+                if (sym) {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        if (j < nvalid && j > d) base[static_cast<int64_t>(col0 + j) * g.ld_f32 + row] = v[j];
                 }
             } else {
-                if (p.epi == kEpiPoly) {
-                    const float* grow = g.g_f32 + b * g.g_batch_stride + static_cast<int64_t>(row) * g.ld_g + col0;
-                    if (nvalid == 32 && (g.ld_g & 3) == 0) {
-                        const float4* g4 = reinterpret_cast<const float4*>(grow);
-#pragma unroll
-                        for (int q = 0; q < 8; ++q) {
-                            const float4 t = g4[q];
-                            v[4 * q] = cc * v[4 * q] + cb * t.x;
-                            v[4 * q + 1] = cc * v[4 * q + 1] + cb * t.y;
-                            v[4 * q + 2] = cc * v[4 * q + 2] + cb * t.z;
-                            v[4 * q + 3] = cc * v[4 * q + 3] + cb * t.w;
-                        }
-                    } else {
-#pragma unroll
-                        for (int j = 0; j < 32; ++j)
-                            if (j < nvalid) v[j] = cc * v[j] + cb * grow[j];
-                    }
-                    const int d = row - col0;
-                    if (d >= 0 && d < 32) {
-#pragma unroll
-                        for (int j = 0; j < 32; ++j)
-                            if (j == d) v[j] += ca;
-                    }
+                if (upper_all) {
+                    store_bf16_row(g.out_hi + goff, g.out_lo + goff, v, nvalid);
                 } else {
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) v[j] *= xs;
+                    for (int j = 0; j < 32; ++j) {
+                        if (j < nvalid && j >= d) {
+                            __nv_bfloat16 h, l;
+                            split_bf16(v[j], h, l);
+                            g.out_hi[goff + j] = h;
+                            g.out_lo[goff + j] = l;
+                        }
+                    }
                 }
-                const int64_t off = b * g.bf_batch_stride + static_cast<int64_t>(row) * g.ld_bf + col0;
-                store_bf16_row(g.out_hi + off, g.out_lo + off, v, nvalid);
+                if (sym) {
+                    const int64_t mbase = b * g.bf_batch_stride + row;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        if (j < nvalid && j > d) {
+                            __nv_bfloat16 h, l;
+                            split_bf16(v[j], h, l);
+                            const int64_t o = mbase + static_cast<int64_t>(col0 + j) * g.ld_bf;
+                            g.out_hi[o] = h;
+                            g.out_lo[o] = l;
+                        }
+                    }
+                }
             }
-            }  // row_ok
+        }
+        if (gram_fused) {
+            // fixed-order reduction of the tile's sums over the 128 epilogue threads
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                s_sq += __shfl_xor_sync(0xffffffffu, s_sq, o);
+                s_tr += __shfl_xor_sync(0xffffffffu, s_tr, o);
+                s_dev += __shfl_xor_sync(0xffffffffu, s_dev, o);
+            }
+            if (lane == 0) {
+                red[eg * 3 + 0] = s_sq;
+                red[eg * 3 + 1] = s_tr;
+                red[eg * 3 + 2] = s_dev;
+            }
+            asm volatile("bar.sync 1, 128;" ::: "memory");
+            if (warp == 2 && lane < 3) {
+                const float t = red[lane] + red[3 + lane] + red[6 + lane] + red[9 + lane];
+                g.part[(g.part_base + static_cast<int64_t>(b) * ntiles + tile) * 3 + lane] = t;
+            }
         }
     }
 
@@ -346,7 +447,7 @@ cudaError_t launch_gemm(const GemmParams& p, bool a_mn, bool b_mn, cudaStream_t 
     int grid = 0;
     for (int i = 0; i < p.num_groups; ++i) {
         const GemmGroup& g = p.g[i];
-        grid = g.cta_begin + g.batch * g.tiles_m * g.tiles_n * g.splits;
+        grid = g.cta_begin + g.batch * (g.sym ? g.tiles_sym : g.tiles_m * g.tiles_n) * g.splits;
     }
     if (grid <= 0) return cudaSuccess;
     if (!a_mn && !b_mn) return launch_gemm_t<false, false>(p, grid, stream);

@@ -1,8 +1,8 @@
 // polar.cu -- per-iteration bookkeeping of the batched polar iteration, and sigma_bar.
 //
-//  k_gram_finalize : G = sum of the split-K Gram partials; writes G (fp32 and bf16
-//                    hi/lo planes) and per-tile partial sums of G^2, diag(G) and
-//                    (G - I)^2 for the convergence test.
+//  k_gram_finalize : split-K buckets only: G = sum of the Gram partials as bf16 hi/lo
+//                    planes, and per-tile sums of G^2, diag(G) and (G - I)^2 for the
+//                    convergence test (the Gram GEMM's epilogue does this otherwise).
 //  k_control       : one warp per matrix; sums the partials in a fixed order (fp64),
 //                    normalises at t = 0 (s^2 = ||Delta^T Delta||_F >= sigma_max^2),
 //                    tests ||X^T X - I||_F / sqrt(n) < tol and picks this
@@ -19,8 +19,6 @@
 
 namespace isoloco {
 
-constexpr int kFinTile = 64;  // finalize tile edge
-
 __device__ __forceinline__ float warp_sum_f(float v) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -33,7 +31,10 @@ __device__ __forceinline__ double warp_sum_d(double v) {
     return v;
 }
 
-// grid: one block (256 threads) per (matrix, 64 x 64 tile) listed in `ftiles`.
+// Split-K buckets only: grid = one block (256 threads) per (matrix, 128 x 256 tile of
+// the n x n Gram) listed in `ftiles`.  Sums the split partials, writes G as bf16 hi/lo
+// and the tile's sums of G^2, diag(G) and (G - I)^2 (unsplit buckets do all of this
+// in the Gram GEMM's epilogue).
 __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict__ mats,
                                                        const int2* __restrict__ ftiles,
                                                        const MatState* __restrict__ state,
@@ -41,7 +42,6 @@ __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict
                                                        const int64_t* __restrict__ gpart_off,
                                                        const int64_t* __restrict__ gpart_split_stride,
                                                        const int* __restrict__ nsplit,
-                                                       float* __restrict__ gf32,
                                                        __nv_bfloat16* __restrict__ ghi,
                                                        __nv_bfloat16* __restrict__ glo,
                                                        float* __restrict__ fin_part) {
@@ -50,20 +50,19 @@ __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict
     if (state[mi].done) return;
     const MatDesc md = mats[mi];
     const int n = md.n, ld = md.ld_n;
-    const int tiles_c = (n + kFinTile - 1) / kFinTile;
-    const int r0 = (ft.y / tiles_c) * kFinTile, c0 = (ft.y % tiles_c) * kFinTile;
+    const int tiles_c = (n + BN - 1) / BN;
+    const int r0 = (ft.y / tiles_c) * BM, c0 = (ft.y % tiles_c) * BN;
     const int64_t poff = gpart_off[mi];
     const int64_t sstride = gpart_split_stride[mi];
     const int splits = nsplit[mi];
 
     float sq = 0.f, tr = 0.f, dev = 0.f;
-    for (int e = threadIdx.x; e < kFinTile * kFinTile; e += blockDim.x) {
-        const int r = r0 + e / kFinTile, c = c0 + e % kFinTile;
+    for (int e = threadIdx.x; e < BM * BN; e += blockDim.x) {
+        const int r = r0 + e / BN, c = c0 + e % BN;
         if (r >= n || c >= n) continue;
         const int64_t idx = static_cast<int64_t>(r) * ld + c;
         float v = 0.f;
         for (int s = 0; s < splits; ++s) v += gpart[poff + s * sstride + idx];
-        gf32[md.gslot + idx] = v;
         __nv_bfloat16 h, l;
         split_bf16(v, h, l);
         ghi[md.gslot + idx] = h;
@@ -193,13 +192,37 @@ __global__ void __launch_bounds__(256) k_trace_partial(const MatDesc* __restrict
         const __nv_bfloat16* dh = dhi + md.slot;
         const __nv_bfloat16* dl = dlo + md.slot;
         float part = 0.f;
-        const int total = tc.z * md.cols;
-        for (int e = threadIdx.x; e < total; e += blockDim.x) {
-            const int r = tc.y + e / md.cols, c = e % md.cols;
-            const int64_t idx = static_cast<int64_t>(r) * md.ld + c;
-            const float q = __bfloat162float(qh[idx]) + __bfloat162float(ql[idx]);
-            const float dv = __bfloat162float(dh[idx]) + __bfloat162float(dl[idx]);
-            part = fmaf(q, dv, part);
+        if (md.ld == md.cols && (md.cols & 7) == 0) {
+            // contiguous rows: 8 elements per 16-byte load of each plane
+            const int64_t base = static_cast<int64_t>(tc.y) * md.cols;
+            const int nv = tc.z * md.cols / 8;
+            const uint4* a4 = reinterpret_cast<const uint4*>(qh + base);
+            const uint4* b4 = reinterpret_cast<const uint4*>(ql + base);
+            const uint4* c4 = reinterpret_cast<const uint4*>(dh + base);
+            const uint4* d4 = reinterpret_cast<const uint4*>(dl + base);
+            for (int v = threadIdx.x; v < nv; v += blockDim.x) {
+                const uint4 a = a4[v], bq = b4[v], c = c4[v], d = d4[v];
+                const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, bw[4] = {bq.x, bq.y, bq.z, bq.w};
+                const uint32_t cw[4] = {c.x, c.y, c.z, c.w}, dw[4] = {d.x, d.y, d.z, d.w};
+#pragma unroll
+                for (int w = 0; w < 4; ++w) {
+                    const float q0 = __uint_as_float(aw[w] << 16) + __uint_as_float(bw[w] << 16);
+                    const float q1 = __uint_as_float(aw[w] & 0xFFFF0000u) + __uint_as_float(bw[w] & 0xFFFF0000u);
+                    const float d0 = __uint_as_float(cw[w] << 16) + __uint_as_float(dw[w] << 16);
+                    const float d1 = __uint_as_float(cw[w] & 0xFFFF0000u) + __uint_as_float(dw[w] & 0xFFFF0000u);
+                    part = fmaf(q0, d0, part);
+                    part = fmaf(q1, d1, part);
+                }
+            }
+        } else {
+            for (int r = tc.y; r < tc.y + tc.z; ++r) {
+                for (int c = threadIdx.x; c < md.cols; c += blockDim.x) {
+                    const int64_t idx = static_cast<int64_t>(r) * md.ld + c;
+                    const float q = __bfloat162float(qh[idx]) + __bfloat162float(ql[idx]);
+                    const float dv = __bfloat162float(dh[idx]) + __bfloat162float(dl[idx]);
+                    part = fmaf(q, dv, part);
+                }
+            }
         }
         acc = static_cast<double>(part);
     }

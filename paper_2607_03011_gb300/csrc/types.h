@@ -13,7 +13,8 @@ namespace isoloco {
 constexpr int BM = 128;
 constexpr int BN = 256;
 constexpr int BK = 32;
-constexpr int kStages = 4;
+constexpr int kStages = 2;          // per CTA; two CTAs share an SM (measured best on GB300)
+constexpr int kGemmCtasPerSm = 2;
 constexpr int kTileABytes = BM * BK * 2;                       // one bf16 plane of A
 constexpr int kTileBBytes = BN * BK * 2;                       // one bf16 plane of B
 constexpr int kStageBytes = 2 * kTileABytes + 2 * kTileBBytes;  // hi + lo of A and B
@@ -24,9 +25,11 @@ constexpr int kGemmSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*ba
 
 // Epilogue of the split-precision GEMM.
 enum EpiMode : int {
-    kEpiF32 = 0,     // store the fp32 accumulator (Gram partial products)
+    kEpiF32 = 0,     // store the fp32 accumulator (tests; split-K Gram partial products)
     kEpiPoly = 1,    // P = a I + b G + c acc  -> bf16 hi/lo planes
     kEpiXSplit = 2,  // X = xscale * acc       -> bf16 hi/lo planes
+    kEpiGram = 3,    // G = acc -> bf16 hi/lo planes + per-tile sums of G^2, diag G, (G-I)^2;
+                     // with split-K (splits > 1) behaves as kEpiF32 and k_gram_finalize follows
 };
 
 // Which matrices a GEMM launch works on, read from the per-matrix state.
@@ -36,6 +39,11 @@ enum GateMode : int {
     kGateStep = 2,    // matrices whose mode this iteration is quintic or polish
 };
 
+// First tile column of tile row tm that touches the upper triangle of a square output.
+__host__ __device__ constexpr int sym_first_tile_n(int tm) {
+    return (tm * BM - BN + 1) <= 0 ? 0 : (tm * BM - BN + 1 + BN - 1) / BN;
+}
+
 struct GemmGroup {
     const CUtensorMap* a_hi;
     const CUtensorMap* a_lo;
@@ -44,6 +52,8 @@ struct GemmGroup {
     int M, N, K;  // output tile space M x N, reduction length K
     int batch;    // matrices in this group
     int tiles_m, tiles_n, splits, kblocks_per_split;
+    int sym;        // square symmetric output: compute only tiles touching col >= row
+    int tiles_sym;  // number of such tiles per matrix
     int cta_begin;  // first blockIdx.x of the group
     int mat_base;   // index of the group's first matrix in the state array
     // fp32 output (kEpiF32): out_f32 + split*split_stride + b*batch_stride + row*ld + col
@@ -55,10 +65,12 @@ struct GemmGroup {
     __nv_bfloat16* out_lo;
     int64_t bf_batch_stride;
     int ld_bf;
-    // kEpiPoly: the fp32 Gram matrix G (same indexing as the output)
-    const float* g_f32;
-    int64_t g_batch_stride;
-    int ld_g;
+    // kEpiPoly: the Gram matrix G as bf16 hi/lo planes (same indexing as the output)
+    const __nv_bfloat16* g_hi;
+    const __nv_bfloat16* g_lo;
+    // kEpiGram: per-tile partial sums, 3 floats at part[(part_base + b * tiles + tile) * 3]
+    float* part;
+    int64_t part_base;
 };
 
 // Per-matrix state of the polar iteration (device memory, one per 2-D tensor).
