@@ -287,8 +287,11 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         const int tiles = sym_tiles(bk.n) * bk.count;
         const int kdim = bk.tall ? bk.rows : bk.cols;
         const int kblocks = (kdim + BK - 1) / BK;
-        int splits = std::max(1, (2 * kGemmCtasPerSm * p->num_sms) / std::max(1, tiles));
-        splits = std::min(splits, std::max(1, kblocks / 8));
+        // split-K for long reductions: at most 256 k-blocks per split, and more splits
+        // (down to 32 k-blocks each) only while the bucket alone would not fill the GPU
+        const int slots = kGemmCtasPerSm * p->num_sms;
+        int splits = std::max(1, (kblocks + 255) / 256);
+        if (tiles * splits < slots) splits = std::max(splits, std::min(slots / std::max(1, tiles), kblocks / 32));
         int kper = (kblocks + splits - 1) / splits;
         splits = (kblocks + kper - 1) / kper;  // no empty split
         bk.splits = splits;
@@ -296,7 +299,7 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         const int64_t g_elems = (int64_t)bk.n * bk.ld_n;
         // Gram partial-sum slots per matrix: one per computed Gram tile (upper-triangle
         // tiles) when the Gram's epilogue produces them, one per finalize tile otherwise
-        const int gtiles = splits > 1 ? ((bk.n + BM - 1) / BM) * ((bk.n + BN - 1) / BN) : sym_tiles(bk.n);
+        const int gtiles = splits > 1 ? ((bk.n + kFinRows - 1) / kFinRows) * ((bk.n + BN - 1) / BN) : sym_tiles(bk.n);
         for (int j = 0; j < bk.count; ++j) {
             const int pi = members[b][j];
             MatDesc md{};
@@ -473,6 +476,10 @@ static void init_set(LaunchSet& s, int epi, int gate, isoloco_plan* pl) {
 
 static int flush_set(isoloco_plan* pl, int phase, LaunchSet& s, bool a_mn, bool b_mn, cudaStream_t st) {
     if (s.groups.empty()) return ISOLOCO_OK;
+    // longest CTAs first, so that short tiles fill in behind them (less tail)
+    std::stable_sort(s.groups.begin(), s.groups.end(), [](const GemmGroup& x, const GemmGroup& y) {
+        return x.kblocks_per_split > y.kblocks_per_split;
+    });
     PhaseTimer timer(pl, phase, st, (int)((s.groups.size() + kMaxGroups - 1) / kMaxGroups));
     for (size_t first = 0; first < s.groups.size(); first += kMaxGroups) {
         GemmParams p = s.p;

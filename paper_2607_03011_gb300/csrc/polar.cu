@@ -31,8 +31,8 @@ __device__ __forceinline__ double warp_sum_d(double v) {
     return v;
 }
 
-// Split-K buckets only: grid = one block (256 threads) per (matrix, 128 x 256 tile of
-// the n x n Gram) listed in `ftiles`.  Sums the split partials, writes G as bf16 hi/lo
+// Split-K buckets only: grid = one block (256 threads) per (matrix, kFinRows x 256 tile
+// of the n x n Gram) listed in `ftiles`.  Sums the split partials, writes G as bf16 hi/lo
 // and the tile's sums of G^2, diag(G) and (G - I)^2 (unsplit buckets do all of this
 // in the Gram GEMM's epilogue).
 __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict__ mats,
@@ -51,13 +51,13 @@ __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict
     const MatDesc md = mats[mi];
     const int n = md.n, ld = md.ld_n;
     const int tiles_c = (n + BN - 1) / BN;
-    const int r0 = (ft.y / tiles_c) * BM, c0 = (ft.y % tiles_c) * BN;
+    const int r0 = (ft.y / tiles_c) * kFinRows, c0 = (ft.y % tiles_c) * BN;
     const int64_t poff = gpart_off[mi];
     const int64_t sstride = gpart_split_stride[mi];
     const int splits = nsplit[mi];
 
     float sq = 0.f, tr = 0.f, dev = 0.f;
-    for (int e = threadIdx.x; e < BM * BN; e += blockDim.x) {
+    for (int e = threadIdx.x; e < kFinRows * BN; e += blockDim.x) {
         const int r = r0 + e / BN, c = c0 + e % BN;
         if (r >= n || c >= n) continue;
         const int64_t idx = static_cast<int64_t>(r) * ld + c;

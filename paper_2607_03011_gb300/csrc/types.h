@@ -21,6 +21,7 @@ constexpr int kStageBytes = 2 * kTileABytes + 2 * kTileBBytes;  // hi + lo of A 
 constexpr int kGemmThreads = 192;  // warp 0 TMA, warp 1 MMA, warps 2..5 epilogue
 constexpr int kTmemCols = 256;
 constexpr int kMaxGroups = 8;
+constexpr int kFinRows = 32;  // rows of one k_gram_finalize tile (x BN columns)
 constexpr int kGemmSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
 
 // Epilogue of the split-precision GEMM.
