@@ -297,7 +297,7 @@ def main():
         ms, n = prof[phase]
         return nbytes * args.steps / (ms / 1000.0) / 1e9 if ms > 0 else 0.0
 
-    roofline = {"bound": "tensor", "kernel": "k_gemm_bf16x3 (Gram, G^2 and update GEMMs)",
+    roofline = {"bound": "tensor", "kernel": "k_gemm_split (Gram, G^2 and update GEMMs)",
                 "achieved": achieved_tf, "peak": tc_peak, "unit": "TFLOP/s",
                 "frac": achieved_tf / tc_peak if tc_peak else None, "traffic": None,
                 "peak_source": f"{peak_src} bf16_tflops_sustained {peaks['bf16_tflops_sustained']} / 3 "

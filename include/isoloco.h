@@ -143,16 +143,19 @@ int isoloco_read_diag(isoloco_plan_t plan, void* stream, float* sigma_bar_host,
 int isoloco_plan_num_matrices(isoloco_plan_t plan);
 
 /* Batched split-precision GEMM of the polar iteration, exposed for testing:
- *   D[b] = op(A[b]) op(B[b])^T-free product with fp32 inputs split into bf16
- *   hi + lo parts and three tcgen05 passes (hi*hi + hi*lo + lo*hi), fp32
- *   accumulation in tensor memory.
+ *   D[b] = op(A[b]) op(B[b]) with fp32 inputs rounded to 16-bit hi + lo planes and
+ *   tcgen05 passes accumulated in fp32 in tensor memory.
+ *   precision 0: bf16 planes, A and B split (hi*hi + hi*lo + lo*hi, 3 passes);
+ *             1: fp16 planes, A split, B single (hi*hi + lo*hi, 2 passes);
+ *             2: fp16 planes, A single, B split (2 passes);
+ *             3: fp16 planes, both split (3 passes).
  *   a_mn_major = 0: A[b] is row-major M x K;  1: A[b] is row-major K x M.
  *   b_mn_major = 0: B[b] is row-major N x K;  1: B[b] is row-major K x N.
  *   D[b] is row-major M x N fp32:  D[b][i][j] = sum_k A(i,k) B(j,k).
  * All pointers are device fp32, contiguous per batch.  Allocates scratch with
  * cudaMalloc and synchronizes `stream` before returning. */
-int isoloco_debug_gemm(int a_mn_major, int b_mn_major, int batch, int M, int N, int K,
-                       const float* A, const float* B, float* D, void* stream);
+int isoloco_debug_gemm(int a_mn_major, int b_mn_major, int precision, int batch, int M, int N,
+                       int K, const float* A, const float* B, float* D, void* stream);
 
 /* Phases of the launch sequence, for isoloco_profile_read. */
 enum {

@@ -26,7 +26,7 @@ namespace isoloco {
 // kernels defined in the other translation units
 cudaError_t launch_gemm(const GemmParams& p, bool a_mn, bool b_mn, cudaStream_t stream);
 __global__ void k_gram_finalize(const MatDesc*, const int2*, const MatState*, const float*, const int64_t*,
-                                const int64_t*, const int*, __nv_bfloat16*, __nv_bfloat16*, float*);
+                                const int64_t*, const int*, __nv_bfloat16*, __nv_bfloat16*, float*, int);
 __global__ void k_control(const MatDesc*, int, MatState*, const float*, int, int, float, uint32_t*);
 __global__ void k_trace_partial(const MatDesc*, const int4*, const MatState*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, const __nv_bfloat16*,
@@ -38,7 +38,7 @@ __global__ void k_reduce(const Chunk*, const MatDesc*, ReplicaPtrs, int, int, co
 __global__ void k_apply(const Chunk*, const MatDesc*, const MatState*, UpdateSrc, int, float, float, float,
                         float*, float*, const float*, float*, float*, const uint32_t*);
 __global__ void k_diloco(ReplicaPtrs, int, int, float*, float*, int64_t, float, float, float, uint32_t*);
-__global__ void k_split_planes(const float*, int64_t, int, int, int, __nv_bfloat16*, __nv_bfloat16*);
+__global__ void k_split_planes(const float*, int64_t, int, int, int, __nv_bfloat16*, __nv_bfloat16*, int);
 
 constexpr int kChunkElems = 16384;
 constexpr int kTraceChunkElems = 16384;
@@ -154,7 +154,8 @@ static bool make_map(CUtensorMap* m, const void* base, int cols, int rows, int c
     if (role == kRoleMN) {
         box[0] = 64; box[1] = BK; sw = CU_TENSOR_MAP_SWIZZLE_128B;
     } else {
-        box[0] = BK; box[1] = (role == kRoleKA) ? BM : BN; sw = CU_TENSOR_MAP_SWIZZLE_64B;
+        box[0] = BK; box[1] = (role == kRoleKA) ? BM : BN;
+        sw = (BK * 2 == 128) ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
     }
     box[2] = 1;
     cuuint32_t es[3] = {1, 1, 1};
@@ -465,9 +466,22 @@ struct LaunchSet {
     void add(const GemmGroup& g) { groups.push_back(g); }
 };
 
-static void init_set(LaunchSet& s, int epi, int gate, isoloco_plan* pl) {
+// Precision of a GEMM launch: operand and output plane types and which operands carry
+// a lo plane.  Iteration 0 multiplies the unnormalised Delta: three bf16 passes.  Later
+// iterates are normalised and use fp16 planes with two passes (A or B split); the update
+// of a matrix's final polish step uses three.
+struct Precision {
+    int in_f16, out_f16, a_split, b_split, split_on_polish;
+};
+
+static void init_set(LaunchSet& s, int epi, int gate, isoloco_plan* pl, Precision pr) {
     memset(&s.p, 0, sizeof(s.p));
     s.groups.clear();
+    s.p.in_f16 = pr.in_f16;
+    s.p.out_f16 = pr.out_f16;
+    s.p.a_split = pr.a_split;
+    s.p.b_split = pr.b_split;
+    s.p.split_on_polish = pr.split_on_polish;
     s.p.epi = epi;
     s.p.gate = gate;
     s.p.state = pl->state;
@@ -504,9 +518,11 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
         const int src = (t == 0) ? 0 : 1 + (t & 1);  // Delta, X0 or X1 as the current iterate
         const int dst = (t + 1) & 1;
         // ---- Gram G = X^T X (tall, MN-major operands) or X X^T (wide, K-major)
+        const bool first = (t == 0);
+        const Precision gram_pr = first ? Precision{0, 0, 1, 1, 0} : Precision{1, 1, 1, 0, 0};
         LaunchSet tall, wide;
-        init_set(tall, kEpiGram, kGateActive, p);
-        init_set(wide, kEpiGram, kGateActive, p);
+        init_set(tall, kEpiGram, kGateActive, p, gram_pr);
+        init_set(wide, kEpiGram, kGateActive, p, gram_pr);
         for (size_t b = 0; b < p->buckets.size(); ++b) {
             const Bucket& bk = p->buckets[b];
             const CUtensorMap* m = maps + b * kMapsPerBucket;
@@ -539,7 +555,7 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             PhaseTimer tm(p, ISOLOCO_PHASE_FINALIZE, st);
             k_gram_finalize<<<p->nftiles, 256, 0, st>>>(p->mats_d, p->ftiles, p->state, p->gpart, p->gpart_off_d,
                                                         p->gpart_sstride_d, p->nsplit_d, p->ghi, p->glo,
-                                                        p->fin_part);
+                                                        p->fin_part, first ? 0 : 1);
             CUDA_TRY(cudaGetLastError());
         }
         { PhaseTimer tm(p, ISOLOCO_PHASE_CONTROL, st);
@@ -548,7 +564,7 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
         CUDA_TRY(cudaGetLastError());
         // ---- P = a I + b G + c G^2
         LaunchSet poly;
-        init_set(poly, kEpiPoly, kGateStep, p);
+        init_set(poly, kEpiPoly, kGateStep, p, first ? Precision{0, 0, 1, 1, 0} : Precision{1, 1, 1, 0, 0});
         for (size_t b = 0; b < p->buckets.size(); ++b) {
             const Bucket& bk = p->buckets[b];
             const CUtensorMap* m = maps + b * kMapsPerBucket;
@@ -569,9 +585,11 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
         }
         if ((rc = flush_set(p, ISOLOCO_PHASE_POLY, poly, false, false, st))) return rc;
         // ---- X_{t+1} = xscale * X_t P (tall) or P X_t (wide)
+        // X_{t+1} is always written as fp16 planes; X is the split operand (A when tall,
+        // B when wide), P the single one except in the polish step
         LaunchSet utall, uwide;
-        init_set(utall, kEpiXSplit, kGateStep, p);
-        init_set(uwide, kEpiXSplit, kGateStep, p);
+        init_set(utall, kEpiXSplit, kGateStep, p, first ? Precision{0, 1, 1, 1, 0} : Precision{1, 1, 1, 0, 1});
+        init_set(uwide, kEpiXSplit, kGateStep, p, first ? Precision{0, 1, 1, 1, 0} : Precision{1, 1, 0, 1, 1});
         for (size_t b = 0; b < p->buckets.size(); ++b) {
             const Bucket& bk = p->buckets[b];
             const CUtensorMap* m = maps + b * kMapsPerBucket;
@@ -891,8 +909,9 @@ int isoloco_read_diag(isoloco_plan_t p, void* stream, float* sigma_bar, int32_t*
     return ISOLOCO_OK;
 }
 
-int isoloco_debug_gemm(int a_mn, int b_mn, int batch, int M, int N, int K, const float* A, const float* B,
-                       float* D, void* stream) {
+int isoloco_debug_gemm(int a_mn, int b_mn, int precision, int batch, int M, int N, int K, const float* A,
+                       const float* B, float* D, void* stream) {
+    if (precision < 0 || precision > 3) return fail(ISOLOCO_ERR_INVALID, "bad debug_gemm precision");
     if (batch <= 0 || M <= 0 || N <= 0 || K <= 0 || !A || !B || !D)
         return fail(ISOLOCO_ERR_INVALID, "bad debug_gemm arguments");
     cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -915,8 +934,9 @@ int isoloco_debug_gemm(int a_mn, int b_mn, int batch, int M, int N, int K, const
     cudaMemsetAsync(ah, 0, asz * 2, st); cudaMemsetAsync(al, 0, asz * 2, st);
     cudaMemsetAsync(bh, 0, bsz * 2, st); cudaMemsetAsync(bl, 0, bsz * 2, st);
     cudaMemsetAsync(err, 0, 4, st);
-    k_split_planes<<<1024, 256, 0, st>>>(A, (int64_t)batch * a_rows * a_cols, a_rows, a_cols, lda, ah, al);
-    k_split_planes<<<1024, 256, 0, st>>>(B, (int64_t)batch * b_rows * b_cols, b_rows, b_cols, ldb, bh, bl);
+    const int f16 = precision > 0 ? 1 : 0;
+    k_split_planes<<<1024, 256, 0, st>>>(A, (int64_t)batch * a_rows * a_cols, a_rows, a_cols, lda, ah, al, f16);
+    k_split_planes<<<1024, 256, 0, st>>>(B, (int64_t)batch * b_rows * b_cols, b_rows, b_cols, ldb, bh, bl, f16);
     CUtensorMap maps[4];
     const int ra = a_mn ? kRoleMN : kRoleKA, rb = b_mn ? kRoleMN : kRoleKB;
     if (!make_map(&maps[0], ah, a_cols, a_rows, batch, lda, ra) || !make_map(&maps[1], al, a_cols, a_rows, batch, lda, ra) ||
@@ -929,6 +949,9 @@ int isoloco_debug_gemm(int a_mn, int b_mn, int batch, int M, int N, int K, const
     memset(&gp, 0, sizeof(gp));
     gp.epi = kEpiF32;
     gp.gate = kGateNone;
+    gp.in_f16 = f16;
+    gp.a_split = (precision == 0 || precision == 1 || precision == 3) ? 1 : 0;
+    gp.b_split = (precision == 0 || precision == 2 || precision == 3) ? 1 : 0;
     gp.err = err;
     GemmGroup& g = gp.g[0];
     g.a_hi = maps_d; g.a_lo = maps_d + 1; g.b_hi = maps_d + 2; g.b_lo = maps_d + 3;

@@ -4,6 +4,7 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -116,8 +117,9 @@ __device__ __forceinline__ void tc_fence_after() {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
-// D(tmem) (+)= A(smem desc) * B(smem desc), kind::f16 (bf16 inputs, fp32 accumulate).
-__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+// D(tmem) (+)= A(smem desc) * B(smem desc), kind::f16 (bf16 or fp16 inputs as the
+// instruction descriptor says, fp32 accumulate).
+__device__ __forceinline__ void umma_16bit(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
                                           uint32_t idesc, uint32_t accumulate) {
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
@@ -169,12 +171,13 @@ __device__ __forceinline__ uint64_t make_sdesc(uint32_t saddr, uint32_t lbo_byte
     return d;
 }
 
-// Instruction descriptor for kind::f16 with bf16 A/B, fp32 D, M x N tile.
-__host__ __device__ constexpr uint32_t make_idesc_bf16(int M, int N, bool a_mn_major,
-                                                       bool b_mn_major) {
+// Instruction descriptor for kind::f16: A and B both bf16 (f16 = false) or both fp16,
+// fp32 D, M x N tile.
+__host__ __device__ constexpr uint32_t make_idesc_16bit(int M, int N, bool a_mn_major,
+                                                        bool b_mn_major, bool f16) {
     return (1u << 4)                                 // D format: f32
-           | (1u << 7)                               // A format: bf16
-           | (1u << 10)                              // B format: bf16
+           | ((f16 ? 0u : 1u) << 7)                  // A format: f16 = 0, bf16 = 1
+           | ((f16 ? 0u : 1u) << 10)                 // B format (same type as A)
            | (static_cast<uint32_t>(a_mn_major) << 15) | (static_cast<uint32_t>(b_mn_major) << 16)
            | (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);
 }
@@ -184,6 +187,25 @@ __host__ __device__ constexpr uint32_t make_idesc_bf16(int M, int N, bool a_mn_m
 __device__ __forceinline__ void split_bf16(float x, __nv_bfloat16& hi, __nv_bfloat16& lo) {
     hi = __float2bfloat16_rn(x);
     lo = __float2bfloat16_rn(x - __bfloat162float(hi));
+}
+
+// x ~= hi + lo as fp16 (f16 = true: ~22 significant bits in the normal range) or bf16
+// bit patterns.
+__device__ __forceinline__ void split16(float x, bool f16, uint16_t& hi, uint16_t& lo) {
+    if (f16) {
+        const __half h = __float2half_rn(x);
+        hi = __half_as_ushort(h);
+        lo = __half_as_ushort(__float2half_rn(x - __half2float(h)));
+    } else {
+        const __nv_bfloat16 h = __float2bfloat16_rn(x);
+        hi = __bfloat16_as_ushort(h);
+        lo = __bfloat16_as_ushort(__float2bfloat16_rn(x - __bfloat162float(h)));
+    }
+}
+
+__device__ __forceinline__ float dec16(uint32_t bits, bool f16) {
+    return f16 ? __half2float(__ushort_as_half(static_cast<unsigned short>(bits)))
+               : __uint_as_float(bits << 16);
 }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(__nv_bfloat16 a, __nv_bfloat16 b) {

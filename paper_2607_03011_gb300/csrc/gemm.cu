@@ -2,10 +2,14 @@
 //
 // Computes, for every matrix b of a group and every BM x BN output tile,
 //     D[b](i, j) = sum_k A[b](i, k) B[b](j, k)
-// where each fp32 operand is carried as two bf16 planes (hi = bf16(x),
-// lo = bf16(x - hi)) and the product is hi*hi + hi*lo + lo*hi, accumulated in fp32
-// in tensor memory: about 16 significant bits per operand, the precision the polar
-// iteration needs (a single bf16 pass would perturb the polar factor by ~1e-3).
+// where an fp32 operand is carried as 16-bit planes hi = round(x), lo = round(x - hi)
+// (bf16 or fp16, chosen per launch).  The tensor core sums hi*hi, plus hi*lo_B when B
+// carries a lo plane and lo_A*hi when A does, into an fp32 accumulator in tensor memory:
+// three passes give ~16 (bf16) or ~22 (fp16) significant bits per operand, two passes
+// keep one operand at 11 bits (fp16).  The polar iteration uses three bf16 passes on
+// the unnormalised pseudo-gradient (iteration 0) and on the final polish step, and two
+// fp16 passes elsewhere (the operand that is not split only perturbs the iterate's
+// spectrum, which later steps correct).
 //
 // Roles (192 threads): warp 0 issues TMA loads into a kStages-deep ring of shared
 // memory stages; warp 1 owns the tensor-memory accumulator and issues tcgen05.mma
@@ -13,10 +17,10 @@
 // epilogue.  Stage hand-off uses mbarriers: `full` (TMA bytes landed), `empty`
 // (the MMAs reading a stage finished, via tcgen05.commit), `acc` (all MMAs done).
 //
-// Operand layouts: K-major operands (K contiguous in global memory) use 64-byte
-// swizzled tiles BK = 32 deep; MN-major operands (M or N contiguous) use 128-byte
-// swizzled tiles of 64 MN-elements x BK rows, two (A) or four (B) boxes per stage.
-// This lets X^T X, X P and P X all read the row-major iterate without transposes.
+// Operand layouts: K-major operands (K contiguous in global memory) use swizzled
+// tiles BK deep; MN-major operands (M or N contiguous) use 128-byte swizzled tiles of
+// 64 MN-elements x BK rows, two (A) or four (B) boxes per stage.  This lets X^T X,
+// X P and P X all read the row-major iterate without transposes.
 #include <cstdio>
 
 #include "common.cuh"
@@ -38,23 +42,24 @@ __device__ __forceinline__ uint64_t operand_desc(uint32_t plane_addr, int ks) {
         // 8-row K groups are 1024 bytes apart (SBO); a 16-deep K slice is 2048 bytes.
         return make_sdesc(plane_addr + ks * 2048, BK * 128, 1024, 2);
     } else {
-        // 64B swizzle, K-major: 8-row groups are 512 bytes apart (SBO); a 16-deep
-        // K slice is 32 bytes into the 64-byte row.
-        return make_sdesc(plane_addr + ks * 32, 16, 512, 4);
+        // K-major, rows of BK bf16 (64 or 128 bytes) with the matching swizzle: 8-row
+        // groups are 8 * BK * 2 bytes apart (SBO); a 16-deep K slice is 32 bytes into the row.
+        return make_sdesc(plane_addr + ks * 32, 16, 8 * BK * 2, BK * 2 == 128 ? 2 : 4);
     }
 }
 
-__device__ __forceinline__ void store_bf16_row(__nv_bfloat16* hi_row, __nv_bfloat16* lo_row,
-                                               const float* v, int ncols_valid) {
+// Stores 32 values of one row as hi/lo planes (bf16 or fp16 bits).
+__device__ __forceinline__ void store_split_row(uint16_t* hi_row, uint16_t* lo_row, const float* v,
+                                                int ncols_valid, bool f16) {
     if (ncols_valid >= 32) {
         uint32_t h[16], l[16];
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
-            __nv_bfloat16 h0, l0, h1, l1;
-            split_bf16(v[2 * j], h0, l0);
-            split_bf16(v[2 * j + 1], h1, l1);
-            h[j] = pack_bf16x2(h0, h1);
-            l[j] = pack_bf16x2(l0, l1);
+            uint16_t h0, l0, h1, l1;
+            split16(v[2 * j], f16, h0, l0);
+            split16(v[2 * j + 1], f16, h1, l1);
+            h[j] = static_cast<uint32_t>(h0) | (static_cast<uint32_t>(h1) << 16);
+            l[j] = static_cast<uint32_t>(l0) | (static_cast<uint32_t>(l1) << 16);
         }
         uint4* hp = reinterpret_cast<uint4*>(hi_row);
         uint4* lp = reinterpret_cast<uint4*>(lo_row);
@@ -67,8 +72,8 @@ __device__ __forceinline__ void store_bf16_row(__nv_bfloat16* hi_row, __nv_bfloa
 #pragma unroll
         for (int j = 0; j < 32; ++j) {
             if (j < ncols_valid) {
-                __nv_bfloat16 h0, l0;
-                split_bf16(v[j], h0, l0);
+                uint16_t h0, l0;
+                split16(v[j], f16, h0, l0);
                 hi_row[j] = h0;
                 lo_row[j] = l0;
             }
@@ -95,7 +100,7 @@ __device__ __forceinline__ void sym_tile(int t, int tiles_m, int tiles_n, int& t
 }  // namespace
 
 template <bool A_MN, bool B_MN>
-__global__ void __launch_bounds__(kGemmThreads, kGemmCtasPerSm) k_gemm_bf16x3(const __grid_constant__ GemmParams p) {
+__global__ void __launch_bounds__(kGemmThreads, kGemmCtasPerSm) k_gemm_split(const __grid_constant__ GemmParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = align1024(smem_raw);
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
@@ -131,6 +136,7 @@ __global__ void __launch_bounds__(kGemmThreads, kGemmCtasPerSm) k_gemm_bf16x3(co
     const int mat = g.mat_base + b;
 
     bool run_mma = true;
+    bool a_split = p.a_split != 0, b_split = p.b_split != 0;
     float ca = 0.f, cb = 0.f, cc = 1.f, xs = 1.f;
     if (p.gate != kGateNone) {
         const MatState& st = p.state[mat];
@@ -139,6 +145,7 @@ __global__ void __launch_bounds__(kGemmThreads, kGemmCtasPerSm) k_gemm_bf16x3(co
         } else {
             if (st.mode == 0) return;
             if (p.epi == kEpiPoly && st.mode == 2) run_mma = false;  // cubic polish: no G^2
+            if (p.split_on_polish && st.mode == 2) a_split = b_split = true;  // final step: 3 passes
         }
         ca = st.a;
         cb = st.b;
@@ -146,6 +153,7 @@ __global__ void __launch_bounds__(kGemmThreads, kGemmCtasPerSm) k_gemm_bf16x3(co
         xs = st.xscale;
     }
 
+    const uint32_t stage_bytes = kTileABytes * (a_split ? 2u : 1u) + kTileBBytes * (b_split ? 2u : 1u);
     const int total_kb = (g.K + BK - 1) / BK;
     const int kb_begin = split * g.kblocks_per_split;
     const int kb_end = min(total_kb, kb_begin + g.kblocks_per_split);
@@ -193,27 +201,27 @@ __global__ void __launch_bounds__(kGemmThreads, kGemmCtasPerSm) k_gemm_bf16x3(co
                 uint8_t* sa_lo = sa_hi + kTileABytes;
                 uint8_t* sb_hi = sa_lo + kTileABytes;
                 uint8_t* sb_lo = sb_hi + kTileBBytes;
-                mbar_arrive_expect_tx(&full[stage], kStageBytes);
+                mbar_arrive_expect_tx(&full[stage], stage_bytes);
                 const int k0 = kb * BK;
                 if (A_MN) {
 #pragma unroll
                     for (int c = 0; c < BM / 64; ++c) {
                         tma_load_3d(sa_hi + c * (BK * 128), g.a_hi, &full[stage], m0 + 64 * c, k0, b);
-                        tma_load_3d(sa_lo + c * (BK * 128), g.a_lo, &full[stage], m0 + 64 * c, k0, b);
+                        if (a_split) tma_load_3d(sa_lo + c * (BK * 128), g.a_lo, &full[stage], m0 + 64 * c, k0, b);
                     }
                 } else {
                     tma_load_3d(sa_hi, g.a_hi, &full[stage], k0, m0, b);
-                    tma_load_3d(sa_lo, g.a_lo, &full[stage], k0, m0, b);
+                    if (a_split) tma_load_3d(sa_lo, g.a_lo, &full[stage], k0, m0, b);
                 }
                 if (B_MN) {
 #pragma unroll
                     for (int c = 0; c < BN / 64; ++c) {
                         tma_load_3d(sb_hi + c * (BK * 128), g.b_hi, &full[stage], n0 + 64 * c, k0, b);
-                        tma_load_3d(sb_lo + c * (BK * 128), g.b_lo, &full[stage], n0 + 64 * c, k0, b);
+                        if (b_split) tma_load_3d(sb_lo + c * (BK * 128), g.b_lo, &full[stage], n0 + 64 * c, k0, b);
                     }
                 } else {
                     tma_load_3d(sb_hi, g.b_hi, &full[stage], k0, n0, b);
-                    tma_load_3d(sb_lo, g.b_lo, &full[stage], k0, n0, b);
+                    if (b_split) tma_load_3d(sb_lo, g.b_lo, &full[stage], k0, n0, b);
                 }
                 issued_mask |= 1u << stage;
                 issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
@@ -232,7 +240,7 @@ __global__ void __launch_bounds__(kGemmThreads, kGemmCtasPerSm) k_gemm_bf16x3(co
         // ================= MMA issuer (one thread)
         if (lane == 0) {
             if (run_mma) {
-                constexpr uint32_t idesc = make_idesc_bf16(BM, BN, A_MN, B_MN);
+                const uint32_t idesc = make_idesc_16bit(BM, BN, A_MN, B_MN, p.in_f16 != 0);
                 int stage = 0;
                 uint32_t phase = 0;
                 for (int kb = kb_begin; kb < kb_end; ++kb) {
@@ -254,9 +262,9 @@ __global__ void __launch_bounds__(kGemmThreads, kGemmCtasPerSm) k_gemm_bf16x3(co
                         const uint64_t dbh = operand_desc<B_MN>(sb_hi, ks);
                         const uint64_t dbl = operand_desc<B_MN>(sb_lo, ks);
                         const uint32_t acc = (kb > kb_begin || ks > 0) ? 1u : 0u;
-                        umma_bf16(tmem_base, dah, dbh, idesc, acc);
-                        umma_bf16(tmem_base, dah, dbl, idesc, 1u);
-                        umma_bf16(tmem_base, dal, dbh, idesc, 1u);
+                        umma_16bit(tmem_base, dah, dbh, idesc, acc);
+                        if (b_split) umma_16bit(tmem_base, dah, dbl, idesc, 1u);
+                        if (a_split) umma_16bit(tmem_base, dal, dbh, idesc, 1u);
                     }
                     umma_commit(&empty[stage]);
                     if (++stage == kStages) {
@@ -309,6 +317,7 @@ __global__ void __launch_bounds__(kGemmThreads, kGemmCtasPerSm) k_gemm_bf16x3(co
             if (p.epi == kEpiPoly) {
                 const __nv_bfloat16* gh = g.g_hi + goff;
                 const __nv_bfloat16* gl = g.g_lo + goff;
+                const bool gf16 = p.in_f16 != 0;
                 if (nvalid == 32) {
                     const uint4* h4 = reinterpret_cast<const uint4*>(gh);
                     const uint4* l4 = reinterpret_cast<const uint4*>(gl);
@@ -319,16 +328,18 @@ __global__ void __launch_bounds__(kGemmThreads, kGemmCtasPerSm) k_gemm_bf16x3(co
                         const uint32_t lw[4] = {ll.x, ll.y, ll.z, ll.w};
 #pragma unroll
                         for (int w = 0; w < 4; ++w) {
-                            const float g0 = __uint_as_float(hw[w] << 16) + __uint_as_float(lw[w] << 16);
-                            const float g1 = __uint_as_float(hw[w] & 0xFFFF0000u) + __uint_as_float(lw[w] & 0xFFFF0000u);
+                            const float g0 = dec16(hw[w] & 0xFFFFu, gf16) + dec16(lw[w] & 0xFFFFu, gf16);
+                            const float g1 = dec16(hw[w] >> 16, gf16) + dec16(lw[w] >> 16, gf16);
                             v[8 * q + 2 * w] = cc * v[8 * q + 2 * w] + cb * g0;
                             v[8 * q + 2 * w + 1] = cc * v[8 * q + 2 * w + 1] + cb * g1;
                         }
                     }
                 } else {
+                    const uint16_t* gh16 = reinterpret_cast<const uint16_t*>(gh);
+                    const uint16_t* gl16 = reinterpret_cast<const uint16_t*>(gl);
 #pragma unroll
                     for (int j = 0; j < 32; ++j)
-                        if (j < nvalid) v[j] = cc * v[j] + cb * (__bfloat162float(gh[j]) + __bfloat162float(gl[j]));
+                        if (j < nvalid) v[j] = cc * v[j] + cb * (dec16(gh16[j], gf16) + dec16(gl16[j], gf16));
                 }
 #pragma unroll
                 for (int j = 0; j < 32; ++j)
@@ -369,16 +380,19 @@ __global__ void __launch_bounds__(kGemmThreads, kGemmCtasPerSm) k_gemm_bf16x3(co
                         if (j < nvalid && j > d) base[static_cast<int64_t>(col0 + j) * g.ld_f32 + row] = v[j];
                 }
             } else {
+                uint16_t* oh = reinterpret_cast<uint16_t*>(g.out_hi);
+                uint16_t* ol = reinterpret_cast<uint16_t*>(g.out_lo);
+                const bool of16 = p.out_f16 != 0;
                 if (upper_all) {
-                    store_bf16_row(g.out_hi + goff, g.out_lo + goff, v, nvalid);
+                    store_split_row(oh + goff, ol + goff, v, nvalid, of16);
                 } else {
 #pragma unroll
                     for (int j = 0; j < 32; ++j) {
                         if (j < nvalid && j >= d) {
-                            __nv_bfloat16 h, l;
-                            split_bf16(v[j], h, l);
-                            g.out_hi[goff + j] = h;
-                            g.out_lo[goff + j] = l;
+                            uint16_t h, l;
+                            split16(v[j], of16, h, l);
+                            oh[goff + j] = h;
+                            ol[goff + j] = l;
                         }
                     }
                 }
@@ -387,11 +401,11 @@ __global__ void __launch_bounds__(kGemmThreads, kGemmCtasPerSm) k_gemm_bf16x3(co
 #pragma unroll
                     for (int j = 0; j < 32; ++j) {
                         if (j < nvalid && j > d) {
-                            __nv_bfloat16 h, l;
-                            split_bf16(v[j], h, l);
+                            uint16_t h, l;
+                            split16(v[j], of16, h, l);
                             const int64_t o = mbase + static_cast<int64_t>(col0 + j) * g.ld_bf;
-                            g.out_hi[o] = h;
-                            g.out_lo[o] = l;
+                            oh[o] = h;
+                            ol[o] = l;
                         }
                     }
                 }
@@ -433,13 +447,13 @@ template <bool A_MN, bool B_MN>
 static cudaError_t launch_gemm_t(const GemmParams& p, int grid, cudaStream_t stream) {
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(k_gemm_bf16x3<A_MN, B_MN>,
+        cudaError_t e = cudaFuncSetAttribute(k_gemm_split<A_MN, B_MN>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              kGemmSmemBytes);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    k_gemm_bf16x3<A_MN, B_MN><<<grid, kGemmThreads, kGemmSmemBytes, stream>>>(p);
+    k_gemm_split<A_MN, B_MN><<<grid, kGemmThreads, kGemmSmemBytes, stream>>>(p);
     return cudaGetLastError();
 }
 

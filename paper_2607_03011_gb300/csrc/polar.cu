@@ -10,6 +10,7 @@
 //                    final cubic polish, or stop.
 //  k_trace_partial / k_trace_final : sigma_bar = tr(Q^T Delta) / n (Alg. 2's mean
 //                    singular value: for the polar factor Q, Q^T Delta = V S V^T).
+//                    Q planes hold fp16 hi/lo bits, Delta planes bf16 hi/lo.
 //
 // All reductions use fixed assignments and fixed shuffle trees: two runs on the same
 // inputs give bitwise-identical results.
@@ -44,7 +45,7 @@ __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict
                                                        const int* __restrict__ nsplit,
                                                        __nv_bfloat16* __restrict__ ghi,
                                                        __nv_bfloat16* __restrict__ glo,
-                                                       float* __restrict__ fin_part) {
+                                                       float* __restrict__ fin_part, int out_f16) {
     const int2 ft = ftiles[blockIdx.x];
     const int mi = ft.x;
     if (state[mi].done) return;
@@ -63,10 +64,10 @@ __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict
         const int64_t idx = static_cast<int64_t>(r) * ld + c;
         float v = 0.f;
         for (int s = 0; s < splits; ++s) v += gpart[poff + s * sstride + idx];
-        __nv_bfloat16 h, l;
-        split_bf16(v, h, l);
-        ghi[md.gslot + idx] = h;
-        glo[md.gslot + idx] = l;
+        uint16_t h, l;
+        split16(v, out_f16 != 0, h, l);
+        reinterpret_cast<uint16_t*>(ghi)[md.gslot + idx] = h;
+        reinterpret_cast<uint16_t*>(glo)[md.gslot + idx] = l;
         sq += v * v;
         const float dlt = (r == c) ? 1.f : 0.f;
         tr += (r == c) ? v : 0.f;
@@ -206,8 +207,8 @@ __global__ void __launch_bounds__(256) k_trace_partial(const MatDesc* __restrict
                 const uint32_t cw[4] = {c.x, c.y, c.z, c.w}, dw[4] = {d.x, d.y, d.z, d.w};
 #pragma unroll
                 for (int w = 0; w < 4; ++w) {
-                    const float q0 = __uint_as_float(aw[w] << 16) + __uint_as_float(bw[w] << 16);
-                    const float q1 = __uint_as_float(aw[w] & 0xFFFF0000u) + __uint_as_float(bw[w] & 0xFFFF0000u);
+                    const float q0 = dec16(aw[w] & 0xFFFFu, true) + dec16(bw[w] & 0xFFFFu, true);
+                    const float q1 = dec16(aw[w] >> 16, true) + dec16(bw[w] >> 16, true);
                     const float d0 = __uint_as_float(cw[w] << 16) + __uint_as_float(dw[w] << 16);
                     const float d1 = __uint_as_float(cw[w] & 0xFFFF0000u) + __uint_as_float(dw[w] & 0xFFFF0000u);
                     part = fmaf(q0, d0, part);
@@ -218,7 +219,8 @@ __global__ void __launch_bounds__(256) k_trace_partial(const MatDesc* __restrict
             for (int r = tc.y; r < tc.y + tc.z; ++r) {
                 for (int c = threadIdx.x; c < md.cols; c += blockDim.x) {
                     const int64_t idx = static_cast<int64_t>(r) * md.ld + c;
-                    const float q = __bfloat162float(qh[idx]) + __bfloat162float(ql[idx]);
+                    const float q = dec16(__bfloat16_as_ushort(qh[idx]), true) +
+                                    dec16(__bfloat16_as_ushort(ql[idx]), true);
                     const float dv = __bfloat162float(dh[idx]) + __bfloat162float(dl[idx]);
                     part = fmaf(q, dv, part);
                 }

@@ -5,11 +5,12 @@
 //                   16-byte loads; each difference is taken before the sum (exact for
 //                   nearby values).  2-D tensors -> bf16 hi/lo planes of the polar
 //                   workspace; 1-D tensors -> fp32.  Raises kErrNonFinite.
-//  k_nesterov     : Alg. 2's update B <- mu B + U, theta <- theta - eta (U + mu B) with
-//                   U = alpha sigma_bar Q (2-D) or the mean pseudo-gradient (1-D).
+//  k_apply        : Alg. 2's update B <- mu B + U, theta <- theta - eta (U + mu B) with
+//                   U = alpha sigma_bar Q (2-D; Q as fp16 hi/lo planes) or the mean
+//                   pseudo-gradient (1-D).
 //  k_diloco       : Alg. 1 with Nesterov SGD fused into a single pass over all
 //                   parameters (reduction + update, no workspace).
-//  k_merge_out    : Iso-C merge output base + alpha IsoC(T) / base + alpha T (Eq. 1).
+//                   Mode 1: Iso-C merge output base + alpha IsoC(T) / base + alpha T (Eq. 1).
 //  k_split_planes : fp32 -> bf16 hi/lo planes (tests of the split-precision GEMM).
 #include "common.cuh"
 #include "types.h"
@@ -145,7 +146,7 @@ __global__ void __launch_bounds__(kStreamThreads) k_apply(const Chunk* __restric
         if (zero) return 0.f;
         const int pe = ch.elem_begin + e;
         const int64_t o = contiguous ? pe : static_cast<int64_t>(pe / md.cols) * md.ld + pe % md.cols;
-        return ucoef * (__bfloat162float(qh[o]) + __bfloat162float(ql[o]));
+        return ucoef * (dec16(__bfloat16_as_ushort(qh[o]), true) + dec16(__bfloat16_as_ushort(ql[o]), true));
     };
     const bool vec = (f0 & 3) == 0 && (ch.count & 3) == 0 && (ch.matrix < 0 || contiguous) &&
                      ((ch.matrix < 0 ? (ch.dst & 3) : (ch.elem_begin & 3)) == 0);
@@ -162,10 +163,10 @@ __global__ void __launch_bounds__(kStreamThreads) k_apply(const Chunk* __restric
             } else {
                 const uint2 hh = *reinterpret_cast<const uint2*>(qh + ch.elem_begin + 4 * v);
                 const uint2 ll = *reinterpret_cast<const uint2*>(ql + ch.elem_begin + 4 * v);
-                u[0] = ucoef * (__uint_as_float(hh.x << 16) + __uint_as_float(ll.x << 16));
-                u[1] = ucoef * (__uint_as_float(hh.x & 0xFFFF0000u) + __uint_as_float(ll.x & 0xFFFF0000u));
-                u[2] = ucoef * (__uint_as_float(hh.y << 16) + __uint_as_float(ll.y << 16));
-                u[3] = ucoef * (__uint_as_float(hh.y & 0xFFFF0000u) + __uint_as_float(ll.y & 0xFFFF0000u));
+                u[0] = ucoef * (dec16(hh.x & 0xFFFFu, true) + dec16(ll.x & 0xFFFFu, true));
+                u[1] = ucoef * (dec16(hh.x >> 16, true) + dec16(ll.x >> 16, true));
+                u[2] = ucoef * (dec16(hh.y & 0xFFFFu, true) + dec16(ll.y & 0xFFFFu, true));
+                u[3] = ucoef * (dec16(hh.y >> 16, true) + dec16(ll.y >> 16, true));
             }
             if (mode == 0) {
                 const float4 th = *reinterpret_cast<const float4*>(theta + i);
@@ -248,9 +249,9 @@ __global__ void __launch_bounds__(kStreamThreads) k_diloco(ReplicaPtrs reps, int
     raise_nonfinite(bad, err);
 }
 
-// fp32 [batch][rows][cols] -> bf16 hi/lo planes with leading dimension ld.
+// fp32 [batch][rows][cols] -> bf16 (f16 = 0) or fp16 hi/lo planes with leading dimension ld.
 __global__ void k_split_planes(const float* __restrict__ x, int64_t total, int rows, int cols, int ld,
-                               __nv_bfloat16* __restrict__ hi, __nv_bfloat16* __restrict__ lo) {
+                               __nv_bfloat16* __restrict__ hi, __nv_bfloat16* __restrict__ lo, int f16) {
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
     for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total; i += stride) {
         const int64_t bm = i / cols;
@@ -258,10 +259,10 @@ __global__ void k_split_planes(const float* __restrict__ x, int64_t total, int r
         const int64_t b = bm / rows;
         const int r = static_cast<int>(bm - b * rows);
         const int64_t o = (b * rows + r) * ld + c;
-        __nv_bfloat16 h, l;
-        split_bf16(x[i], h, l);
-        hi[o] = h;
-        lo[o] = l;
+        uint16_t h, l;
+        split16(x[i], f16 != 0, h, l);
+        reinterpret_cast<uint16_t*>(hi)[o] = h;
+        reinterpret_cast<uint16_t*>(lo)[o] = l;
     }
 }
 

@@ -94,6 +94,10 @@ struct GemmParams {
     int num_groups;
     int epi;
     int gate;
+    int in_f16;           // operand planes are fp16 (else bf16); also the G planes of kEpiPoly
+    int out_f16;          // hi/lo output planes are fp16 (else bf16)
+    int a_split, b_split; // operand carries a lo plane (adds one tensor pass each)
+    int split_on_polish;  // matrices in the polish step use both lo planes
     MatState* state;
     uint32_t* err;
 };

@@ -80,7 +80,7 @@ def lib():
             L.isoloco_plan_launches.argtypes = [_vp]
             L.isoloco_plan_launches.restype = ctypes.c_int64
             L.isoloco_debug_gemm.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
-                                             ctypes.c_int, _vp, _vp, _vp, _vp]
+                                             ctypes.c_int, ctypes.c_int, _vp, _vp, _vp, _vp]
             _lib = L
     return _lib
 
@@ -238,11 +238,11 @@ class Plan:
 
 
 def debug_gemm(A: torch.Tensor, B: torch.Tensor, a_mn_major: bool, b_mn_major: bool, M: int, N: int, K: int,
-               stream=None) -> torch.Tensor:
+               precision: int = 0, stream=None) -> torch.Tensor:
     """Split-precision tcgen05 GEMM: D[b] = op(A[b]) op(B[b]) (see include/isoloco.h)."""
     batch = A.shape[0]
     D = torch.empty((batch, M, N), dtype=torch.float32, device=A.device)
-    rc = lib().isoloco_debug_gemm(int(a_mn_major), int(b_mn_major), batch, M, N, K, A.data_ptr(), B.data_ptr(),
-                                  D.data_ptr(), _stream(stream))
+    rc = lib().isoloco_debug_gemm(int(a_mn_major), int(b_mn_major), int(precision), batch, M, N, K, A.data_ptr(),
+                                  B.data_ptr(), D.data_ptr(), _stream(stream))
     _check(rc, "isoloco_debug_gemm", hard_only=False)
     return D

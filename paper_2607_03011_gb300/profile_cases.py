@@ -3,9 +3,10 @@
     python -m paper_2607_03011_gb300.profile_cases step --workload square12 --steps 2
     python -m paper_2607_03011_gb300.profile_cases gemm --batch 48 --m 1024 --n 1024 --k 1024
 
-`step` runs IsoLoCo outer steps through the C ABI on a named workload; `square12`
-is twelve 1024 x 1024 matrices of the 180M recipe with K = 8 replicas (0.4 GB of
-replicas: larger than L2, small enough for a full ncu capture).  `gemm` runs the
+`step` runs IsoLoCo outer steps through the C ABI on a named workload; `square48`
+is the 48 square 1024 x 1024 matrices of the 180M recipe with K = 8 replicas
+(1.6 GB of replicas: larger than L2, small enough for a full ncu capture), and
+`square12` a quarter of it.  `gemm` runs the
 split-precision GEMM entry point on random inputs.
 """
 from __future__ import annotations
@@ -18,6 +19,8 @@ from . import isoloco
 from . import workloads as W
 
 EXTRA = {
+    "square48": lambda: W.custom_spec([(f"w{i}", 1024, 1024) for i in range(48)], K=8, rank=32,
+                                      shared_std=2e-5, noise_std=2e-5, momentum_std=2e-5, name="square48"),
     "square12": lambda: W.custom_spec([(f"w{i}", 1024, 1024) for i in range(12)], K=8, rank=32,
                                       shared_std=2e-5, noise_std=2e-5, momentum_std=2e-5, name="square12"),
     "tall4": lambda: W.custom_spec([("e", 32000, 1024), ("d0", 2816, 1024), ("d1", 2816, 1024), ("g", 1024, 2816)],

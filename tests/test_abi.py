@@ -60,4 +60,5 @@ def test_validation_without_gpu(lib):
     assert not h.value
     assert lib.isoloco_outer_step(None, None, None, None, None, None, None) == isoloco.ERR_INVALID
     assert lib.diloco_outer_step(None, None, None, None, None, None) == isoloco.ERR_INVALID
-    assert lib.isoloco_debug_gemm(0, 0, 0, 1, 1, 1, None, None, None, None) == isoloco.ERR_INVALID
+    assert lib.isoloco_debug_gemm(0, 0, 0, 0, 1, 1, 1, None, None, None, None) == isoloco.ERR_INVALID
+    assert lib.isoloco_debug_gemm(0, 0, 9, 1, 1, 1, 1, None, None, None, None) == isoloco.ERR_INVALID

@@ -50,6 +50,28 @@ def test_debug_gemm_layouts(iso, a_mn, b_mn, batch, M, N, K):
         assert (one_pass - R).norm() / R.norm() > 10 * err
 
 
+# precision 1: fp16, A split / B single; 2: A single / B split; 3: both split.
+# Expected relative error: the single operand's fp16 rounding (2^-12 relative per
+# entry, ~1.4e-4 in Frobenius norm on random data) for 1 and 2; ~1e-6 for 3.
+@pytest.mark.parametrize("precision,tol", [(1, 4e-4), (2, 4e-4), (3, 3e-6)])
+@pytest.mark.parametrize("a_mn,b_mn", [(0, 0), (1, 1), (0, 1)])
+@pytest.mark.parametrize("batch,M,N,K", [(2, 128, 256, 64), (2, 65, 130, 70), (1, 1024, 1024, 2816)])
+def test_debug_gemm_fp16_passes(iso, precision, tol, a_mn, b_mn, batch, M, N, K):
+    g = torch.Generator(device="cuda").manual_seed(M + N + K + precision)
+    A = torch.randn((batch, K, M) if a_mn else (batch, M, K), device="cuda", generator=g)
+    B = torch.randn((batch, K, N) if b_mn else (batch, N, K), device="cuda", generator=g)
+    D = iso.debug_gemm(A, B, a_mn, b_mn, M, N, K, precision=precision)
+    R = _ref(A, B, a_mn, b_mn)
+    err = float((D.double() - R).norm() / R.norm())
+    assert err < tol, err
+    if precision in (1, 2):
+        # matches the model: only the single operand is rounded to fp16
+        A1 = A if precision == 1 else A.half().float()
+        B1 = B if precision == 2 else B.half().float()
+        model = _ref(A1, B1, a_mn, b_mn)
+        assert float((D.double() - model).norm() / R.norm()) < 0.1 * err
+
+
 def test_debug_gemm_deterministic(iso):
     g = torch.Generator(device="cuda").manual_seed(5)
     A = torch.randn((2, 256, 512), device="cuda", generator=g)
