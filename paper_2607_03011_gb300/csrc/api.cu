@@ -24,7 +24,7 @@
 namespace isoloco {
 
 // kernels defined in the other translation units
-cudaError_t launch_gemm(const GemmParams& p, bool a_mn, bool b_mn, cudaStream_t stream);
+cudaError_t launch_gemm(const GemmParams& p, bool a_mn, bool b_mn, int max_ctas, cudaStream_t stream);
 __global__ void k_gram_finalize(const MatDesc*, const int2*, const MatState*, const float*, const int64_t*,
                                 const int64_t*, const int*, __nv_bfloat16*, __nv_bfloat16*, float*, int);
 __global__ void k_control(const MatDesc*, int, MatState*, const float*, int, int, float, uint32_t*);
@@ -290,7 +290,7 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         const int kblocks = (kdim + BK - 1) / BK;
         // split-K for long reductions: at most 256 k-blocks per split, and more splits
         // (down to 32 k-blocks each) only while the bucket alone would not fill the GPU
-        const int slots = kGemmCtasPerSm * p->num_sms;
+        const int slots = 2 * p->num_sms;
         int splits = std::max(1, (kblocks + 255) / 256);
         if (tiles * splits < slots) splits = std::max(splits, std::min(slots / std::max(1, tiles), kblocks / 32));
         int kper = (kblocks + splits - 1) / splits;
@@ -377,7 +377,7 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         (rc = dalloc(p, &p->xlo[1], plane)) ||
         (rc = dalloc(p, &p->ghi, gplane)) || (rc = dalloc(p, &p->glo, gplane)) || (rc = dalloc(p, &p->phi, gplane)) ||
         (rc = dalloc(p, &p->plo, gplane)) || (rc = dalloc(p, &p->gpart, gpart)) || (rc = dalloc(p, &p->d1d, d1)) ||
-        (rc = dalloc(p, &p->fin_part, 3 * fin)) || (rc = dalloc(p, &p->ftiles, (int64_t)ftiles.size())) ||
+        (rc = dalloc(p, &p->fin_part, 12 * fin)) || (rc = dalloc(p, &p->ftiles, (int64_t)ftiles.size())) ||
         (rc = dalloc(p, &p->tpart, tr)) || (rc = dalloc(p, &p->tchunks, tr)) ||
         (rc = dalloc(p, &p->state, p->nmat)) || (rc = dalloc(p, &p->mats_d, p->nmat)) ||
         (rc = dalloc(p, &p->gpart_off_d, p->nmat)) || (rc = dalloc(p, &p->gpart_sstride_d, p->nmat)) ||
@@ -505,7 +505,8 @@ static int flush_set(isoloco_plan* pl, int phase, LaunchSet& s, bool a_mn, bool 
             cta += g.batch * group_tiles(g) * g.splits;
             p.g[p.num_groups++] = g;
         }
-        CUDA_TRY(launch_gemm(p, a_mn, b_mn, st));
+        p.total_tiles = cta;
+        CUDA_TRY(launch_gemm(p, a_mn, b_mn, pl->num_sms, st));
     }
     return ISOLOCO_OK;
 }
@@ -962,7 +963,11 @@ int isoloco_debug_gemm(int a_mn, int b_mn, int precision, int batch, int M, int 
     g.f32_split_stride = 0;
     g.ld_f32 = N;
     gp.num_groups = 1;
-    cudaError_t e = launch_gemm(gp, a_mn != 0, b_mn != 0, st);
+    gp.total_tiles = batch * g.tiles_m * g.tiles_n;
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    cudaError_t e = launch_gemm(gp, a_mn != 0, b_mn != 0, sms, st);
     uint32_t herr = 0;
     if (e == cudaSuccess) e = cudaMemcpyAsync(&herr, err, 4, cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);

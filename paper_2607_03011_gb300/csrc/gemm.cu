@@ -99,84 +99,247 @@ __device__ __forceinline__ void sym_tile(int t, int tiles_m, int tiles_n, int& t
 
 }  // namespace
 
+// Everything a role needs to know about one output tile; every role decodes the same
+// sequence of tile indices, so the three warps agree without communicating.
+struct TileInfo {
+    int gi, b, tile, split, m0, n0, mat, kb_begin, kb_end;
+    bool run_mma, a_split, b_split;
+    float ca, cb, cc, xs;
+};
+
+// Returns false when the tile belongs to a matrix that does no work this launch.
+__device__ __forceinline__ bool decode_tile(const GemmParams& p, int t, TileInfo& ti) {
+    int gi = 0;
+    while (gi + 1 < p.num_groups && t >= p.g[gi + 1].cta_begin) ++gi;
+    const GemmGroup& g = p.g[gi];
+    int local = t - g.cta_begin;
+    ti.gi = gi;
+    ti.split = local % g.splits;
+    local /= g.splits;
+    const int ntiles = g.sym ? g.tiles_sym : g.tiles_m * g.tiles_n;
+    ti.tile = local % ntiles;
+    ti.b = local / ntiles;
+    if (ti.b >= g.batch) return false;
+    int tm, tn;
+    if (g.sym) {
+        sym_tile(ti.tile, g.tiles_m, g.tiles_n, tm, tn);
+    } else {
+        tm = ti.tile / g.tiles_n;
+        tn = ti.tile % g.tiles_n;
+    }
+    ti.m0 = tm * BM;
+    ti.n0 = tn * BN;
+    ti.mat = g.mat_base + ti.b;
+    ti.run_mma = true;
+    ti.a_split = p.a_split != 0;
+    ti.b_split = p.b_split != 0;
+    ti.ca = 0.f, ti.cb = 0.f, ti.cc = 1.f, ti.xs = 1.f;
+    if (p.gate != kGateNone) {
+        const MatState& st = p.state[ti.mat];
+        if (p.gate == kGateActive) {
+            if (st.done) return false;
+        } else {
+            if (st.mode == 0) return false;
+            if (p.epi == kEpiPoly && st.mode == 2) ti.run_mma = false;  // cubic polish: no G^2
+            if (p.split_on_polish && st.mode == 2) ti.a_split = ti.b_split = true;  // final step: 3 passes
+        }
+        ti.ca = st.a;
+        ti.cb = st.b;
+        ti.cc = st.c;
+        ti.xs = st.xscale;
+    }
+    const int total_kb = (g.K + BK - 1) / BK;
+    ti.kb_begin = ti.split * g.kblocks_per_split;
+    ti.kb_end = min(total_kb, ti.kb_begin + g.kblocks_per_split);
+    if (ti.kb_begin >= ti.kb_end) ti.run_mma = false;
+    return true;
+}
+
+// Epilogue of one tile, run by the 128 threads of warps 2..5 (thread (eg, lane) owns
+// output row m0 + 32 eg + lane).  `tacc` is the tensor-memory accumulator of the tile.
+// In symmetric mode (Gram, G^2) only entries with col >= row are produced from the
+// accumulator; each entry with col > row is also written, bitwise identical, at
+// (col, row): across a warp those mirrored stores hit 32 consecutive rows of one
+// column, so they coalesce.
+__device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInfo& ti, uint32_t tacc, bool ok,
+                                              int eg, int lane) {
+    const GemmGroup& g = p.g[ti.gi];
+    const int b = ti.b, m0 = ti.m0, n0 = ti.n0, split = ti.split;
+    const float ca = ti.ca, cb = ti.cb, cc = ti.cc, xs = ti.xs;
+    const int row = m0 + eg * 32 + lane;
+    const bool row_ok = row < g.M;
+    const bool sym = g.sym != 0;
+    const bool f32_out = (p.epi == kEpiF32) || (p.epi == kEpiGram && g.splits > 1);
+    const bool gram_fused = (p.epi == kEpiGram && g.splits == 1);
+    float s_sq = 0.f, s_tr = 0.f, s_dev = 0.f;
+    for (int c32 = 0; c32 < BN / 32; ++c32) {
+        const int col0 = n0 + c32 * 32;
+        if (col0 >= g.N) break;
+        float v[32];
+        __syncwarp();
+        if (ti.run_mma && ok) {
+            uint32_t r[32];
+            tmem_ld32(tacc + (static_cast<uint32_t>(eg * 32) << 16) + c32 * 32, r);
+            tmem_ld_wait();
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+        } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] = 0.f;
+        }
+        const int nvalid = min(32, g.N - col0);
+        const int d = row - col0;  // column index of the diagonal inside this chunk
+        // chunk entirely below the diagonal: produced by a mirror elsewhere
+        if (!row_ok || (sym && d > nvalid - 1)) continue;
+        const bool upper_all = !sym || d < 0;  // every column of the chunk has col > row
+        const int64_t goff = b * g.bf_batch_stride + static_cast<int64_t>(row) * g.ld_bf + col0;
+        if (p.epi == kEpiPoly) {
+            const uint16_t* gh = reinterpret_cast<const uint16_t*>(g.g_hi) + goff;
+            const uint16_t* gl = reinterpret_cast<const uint16_t*>(g.g_lo) + goff;
+            const bool gf16 = p.in_f16 != 0;
+            if (nvalid == 32) {
+                const uint4* h4 = reinterpret_cast<const uint4*>(gh);
+                const uint4* l4 = reinterpret_cast<const uint4*>(gl);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const uint4 hh = h4[q], ll = l4[q];
+                    const uint32_t hw[4] = {hh.x, hh.y, hh.z, hh.w};
+                    const uint32_t lw[4] = {ll.x, ll.y, ll.z, ll.w};
+#pragma unroll
+                    for (int w = 0; w < 4; ++w) {
+                        const float g0 = dec16(hw[w] & 0xFFFFu, gf16) + dec16(lw[w] & 0xFFFFu, gf16);
+                        const float g1 = dec16(hw[w] >> 16, gf16) + dec16(lw[w] >> 16, gf16);
+                        v[8 * q + 2 * w] = cc * v[8 * q + 2 * w] + cb * g0;
+                        v[8 * q + 2 * w + 1] = cc * v[8 * q + 2 * w + 1] + cb * g1;
+                    }
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                    if (j < nvalid) v[j] = cc * v[j] + cb * (dec16(gh[j], gf16) + dec16(gl[j], gf16));
+            }
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                if (j == d) v[j] += ca;
+        } else if (p.epi == kEpiXSplit) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] *= xs;
+        }
+        if (gram_fused) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                if (j < nvalid && (!sym || j >= d)) {
+                    const float x = v[j];
+                    const float e = (j == d) ? x - 1.f : x;
+                    const float w = (sym && j > d) ? 2.f : 1.f;  // mirrored entry counts twice
+                    s_sq = fmaf(w * x, x, s_sq);
+                    s_dev = fmaf(w * e, e, s_dev);
+                    if (j == d) s_tr += x;
+                }
+            }
+        }
+        if (f32_out) {
+            float* base = g.out_f32 + split * g.f32_split_stride + b * g.f32_batch_stride;
+            float* out = base + static_cast<int64_t>(row) * g.ld_f32 + col0;
+            if (upper_all && nvalid == 32 && (g.ld_f32 & 3) == 0) {
+                float4* o4 = reinterpret_cast<float4*>(out);
+#pragma unroll
+                for (int q = 0; q < 8; ++q) o4[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            } else {
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                    if (j < nvalid && (!sym || j >= d)) out[j] = v[j];
+            }
+            if (sym) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                    if (j < nvalid && j > d) base[static_cast<int64_t>(col0 + j) * g.ld_f32 + row] = v[j];
+            }
+        } else {
+            uint16_t* oh = reinterpret_cast<uint16_t*>(g.out_hi);
+            uint16_t* ol = reinterpret_cast<uint16_t*>(g.out_lo);
+            const bool of16 = p.out_f16 != 0;
+            if (upper_all) {
+                store_split_row(oh + goff, ol + goff, v, nvalid, of16);
+            } else {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+                    if (j < nvalid && j >= d) {
+                        uint16_t h, l;
+                        split16(v[j], of16, h, l);
+                        oh[goff + j] = h;
+                        ol[goff + j] = l;
+                    }
+                }
+            }
+            if (sym) {
+                const int64_t mbase = b * g.bf_batch_stride + row;
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+                    if (j < nvalid && j > d) {
+                        uint16_t h, l;
+                        split16(v[j], of16, h, l);
+                        const int64_t o = mbase + static_cast<int64_t>(col0 + j) * g.ld_bf;
+                        oh[o] = h;
+                        ol[o] = l;
+                    }
+                }
+            }
+        }
+    }
+    if (gram_fused) {
+        // fixed-order warp reduction; each epilogue warp owns one of the tile's 4 slots
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            s_sq += __shfl_xor_sync(0xffffffffu, s_sq, o);
+            s_tr += __shfl_xor_sync(0xffffffffu, s_tr, o);
+            s_dev += __shfl_xor_sync(0xffffffffu, s_dev, o);
+        }
+        if (lane == 0) {
+            const int ntiles = sym ? g.tiles_sym : g.tiles_m * g.tiles_n;
+            float* slot = g.part + ((g.part_base + static_cast<int64_t>(b) * ntiles + ti.tile) * 4 + eg) * 3;
+            slot[0] = s_sq;
+            slot[1] = s_tr;
+            slot[2] = s_dev;
+        }
+    }
+}
+
+// Persistent kernel: CTA c processes tiles c, c + gridDim.x, ... of the launch.  The TMA
+// ring runs continuously across tile boundaries, and the accumulator is double
+// buffered in tensor memory (2 x 256 columns): the epilogue of one tile overlaps the
+// MMAs of the next.
 template <bool A_MN, bool B_MN>
-__global__ void __launch_bounds__(kGemmThreads, kGemmCtasPerSm) k_gemm_split(const __grid_constant__ GemmParams p) {
+__global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_constant__ GemmParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = align1024(smem_raw);
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
     uint64_t* empty = full + kStages;
-    uint64_t* accbar = empty + kStages;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accbar + 1);
+    uint64_t* tfull = empty + kStages;   // [2] accumulator buffer ready for the epilogue
+    uint64_t* tempty = tfull + 2;        // [2] accumulator buffer released by the epilogue
+    uint64_t* drain = tempty + 2;        // teardown: every issued MMA has completed
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-    float* red = reinterpret_cast<float*>(tmem_slot + 4);  // [4 warps][3] epilogue partial sums
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
+    const int T = p.total_tiles;
 
-    // ---- locate (group, matrix, tile, split) of this CTA
-    int gi = 0;
-    while (gi + 1 < p.num_groups && static_cast<int>(blockIdx.x) >= p.g[gi + 1].cta_begin) ++gi;
-    const GemmGroup& g = p.g[gi];
-    int local = static_cast<int>(blockIdx.x) - g.cta_begin;
-    const int split = local % g.splits;
-    local /= g.splits;
-    const int ntiles = g.sym ? g.tiles_sym : g.tiles_m * g.tiles_n;
-    const int tile = local % ntiles;
-    const int b = local / ntiles;
-    if (b >= g.batch) return;
-    int tm, tn;
-    if (g.sym) {
-        sym_tile(tile, g.tiles_m, g.tiles_n, tm, tn);
-    } else {
-        tm = tile / g.tiles_n;
-        tn = tile % g.tiles_n;
-    }
-    const int m0 = tm * BM;
-    const int n0 = tn * BN;
-    const int mat = g.mat_base + b;
-
-    bool run_mma = true;
-    bool a_split = p.a_split != 0, b_split = p.b_split != 0;
-    float ca = 0.f, cb = 0.f, cc = 1.f, xs = 1.f;
-    if (p.gate != kGateNone) {
-        const MatState& st = p.state[mat];
-        if (p.gate == kGateActive) {
-            if (st.done) return;
-        } else {
-            if (st.mode == 0) return;
-            if (p.epi == kEpiPoly && st.mode == 2) run_mma = false;  // cubic polish: no G^2
-            if (p.split_on_polish && st.mode == 2) a_split = b_split = true;  // final step: 3 passes
-        }
-        ca = st.a;
-        cb = st.b;
-        cc = st.c;
-        xs = st.xscale;
-    }
-
-    const uint32_t stage_bytes = kTileABytes * (a_split ? 2u : 1u) + kTileBBytes * (b_split ? 2u : 1u);
-    const int total_kb = (g.K + BK - 1) / BK;
-    const int kb_begin = split * g.kblocks_per_split;
-    const int kb_end = min(total_kb, kb_begin + g.kblocks_per_split);
-    if (kb_begin >= kb_end) run_mma = false;
-
-    // ---- setup: barriers, tensor memory
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
         }
-        mbar_init(accbar, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&tfull[i], 1);
+            mbar_init(&tempty[i], 4);  // one arrival per epilogue warp
+        }
+        mbar_init(drain, 1);
         *abort_flag = 0;
         fence_mbar_init();
     }
-    if (warp == 0 && lane == 0 && run_mma) {
-        tma_prefetch_desc(g.a_hi);
-        tma_prefetch_desc(g.a_lo);
-        tma_prefetch_desc(g.b_hi);
-        tma_prefetch_desc(g.b_lo);
-    }
     if (warp == 1) {
-        tmem_alloc(tmem_slot, kTmemCols);
+        tmem_alloc(tmem_slot, 2 * kTmemCols);
         tmem_relinquish();
     }
     tc_fence_before();
@@ -186,48 +349,64 @@ __global__ void __launch_bounds__(kGemmThreads, kGemmCtasPerSm) k_gemm_split(con
 
     if (warp == 0) {
         // ================= TMA producer
-        if (lane == 0 && run_mma) {
+        if (lane == 0) {
             int stage = 0;
             uint32_t phase = 0;
             uint32_t issued_mask = 0, issued_parity = 0;
-            for (int kb = kb_begin; kb < kb_end; ++kb) {
-                if (*abort_flag) break;
-                if (!mbar_wait(&empty[stage], phase ^ 1u)) {
-                    *abort_flag = 1;
-                    atomicOr(p.err, kErrTimeout);
-                    break;
+            int prefetched = -1;
+            for (int t = blockIdx.x; t < T && !*abort_flag; t += gridDim.x) {
+                TileInfo ti;
+                if (!decode_tile(p, t, ti) || !ti.run_mma) continue;
+                const GemmGroup& g = p.g[ti.gi];
+                if (prefetched != ti.gi) {
+                    tma_prefetch_desc(g.a_hi);
+                    tma_prefetch_desc(g.b_hi);
+                    if (ti.a_split) tma_prefetch_desc(g.a_lo);
+                    if (ti.b_split) tma_prefetch_desc(g.b_lo);
+                    prefetched = ti.gi;
                 }
-                uint8_t* sa_hi = smem + stage * kStageBytes;
-                uint8_t* sa_lo = sa_hi + kTileABytes;
-                uint8_t* sb_hi = sa_lo + kTileABytes;
-                uint8_t* sb_lo = sb_hi + kTileBBytes;
-                mbar_arrive_expect_tx(&full[stage], stage_bytes);
-                const int k0 = kb * BK;
-                if (A_MN) {
-#pragma unroll
-                    for (int c = 0; c < BM / 64; ++c) {
-                        tma_load_3d(sa_hi + c * (BK * 128), g.a_hi, &full[stage], m0 + 64 * c, k0, b);
-                        if (a_split) tma_load_3d(sa_lo + c * (BK * 128), g.a_lo, &full[stage], m0 + 64 * c, k0, b);
+                const uint32_t stage_bytes =
+                    kTileABytes * (ti.a_split ? 2u : 1u) + kTileBBytes * (ti.b_split ? 2u : 1u);
+                for (int kb = ti.kb_begin; kb < ti.kb_end; ++kb) {
+                    if (!mbar_wait(&empty[stage], phase ^ 1u)) {
+                        *abort_flag = 1;
+                        atomicOr(p.err, kErrTimeout);
+                        break;
                     }
-                } else {
-                    tma_load_3d(sa_hi, g.a_hi, &full[stage], k0, m0, b);
-                    if (a_split) tma_load_3d(sa_lo, g.a_lo, &full[stage], k0, m0, b);
-                }
-                if (B_MN) {
+                    uint8_t* sa_hi = smem + stage * kStageBytes;
+                    uint8_t* sa_lo = sa_hi + kTileABytes;
+                    uint8_t* sb_hi = sa_lo + kTileABytes;
+                    uint8_t* sb_lo = sb_hi + kTileBBytes;
+                    mbar_arrive_expect_tx(&full[stage], stage_bytes);
+                    const int k0 = kb * BK;
+                    if (A_MN) {
 #pragma unroll
-                    for (int c = 0; c < BN / 64; ++c) {
-                        tma_load_3d(sb_hi + c * (BK * 128), g.b_hi, &full[stage], n0 + 64 * c, k0, b);
-                        if (b_split) tma_load_3d(sb_lo + c * (BK * 128), g.b_lo, &full[stage], n0 + 64 * c, k0, b);
+                        for (int c = 0; c < BM / 64; ++c) {
+                            tma_load_3d(sa_hi + c * (BK * 128), g.a_hi, &full[stage], ti.m0 + 64 * c, k0, ti.b);
+                            if (ti.a_split)
+                                tma_load_3d(sa_lo + c * (BK * 128), g.a_lo, &full[stage], ti.m0 + 64 * c, k0, ti.b);
+                        }
+                    } else {
+                        tma_load_3d(sa_hi, g.a_hi, &full[stage], k0, ti.m0, ti.b);
+                        if (ti.a_split) tma_load_3d(sa_lo, g.a_lo, &full[stage], k0, ti.m0, ti.b);
                     }
-                } else {
-                    tma_load_3d(sb_hi, g.b_hi, &full[stage], k0, n0, b);
-                    if (b_split) tma_load_3d(sb_lo, g.b_lo, &full[stage], k0, n0, b);
-                }
-                issued_mask |= 1u << stage;
-                issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
-                if (++stage == kStages) {
-                    stage = 0;
-                    phase ^= 1u;
+                    if (B_MN) {
+#pragma unroll
+                        for (int c = 0; c < BN / 64; ++c) {
+                            tma_load_3d(sb_hi + c * (BK * 128), g.b_hi, &full[stage], ti.n0 + 64 * c, k0, ti.b);
+                            if (ti.b_split)
+                                tma_load_3d(sb_lo + c * (BK * 128), g.b_lo, &full[stage], ti.n0 + 64 * c, k0, ti.b);
+                        }
+                    } else {
+                        tma_load_3d(sb_hi, g.b_hi, &full[stage], k0, ti.n0, ti.b);
+                        if (ti.b_split) tma_load_3d(sb_lo, g.b_lo, &full[stage], k0, ti.n0, ti.b);
+                    }
+                    issued_mask |= 1u << stage;
+                    issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
+                    if (++stage == kStages) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
                 }
             }
             if (*abort_flag) {
@@ -239,206 +418,87 @@ __global__ void __launch_bounds__(kGemmThreads, kGemmCtasPerSm) k_gemm_split(con
     } else if (warp == 1) {
         // ================= MMA issuer (one thread)
         if (lane == 0) {
-            if (run_mma) {
-                const uint32_t idesc = make_idesc_16bit(BM, BN, A_MN, B_MN, p.in_f16 != 0);
-                int stage = 0;
-                uint32_t phase = 0;
-                for (int kb = kb_begin; kb < kb_end; ++kb) {
-                    if (*abort_flag) break;
-                    if (!mbar_wait(&full[stage], phase)) {
-                        *abort_flag = 1;
-                        atomicOr(p.err, kErrTimeout);
-                        break;
-                    }
-                    tc_fence_after();
-                    const uint32_t sa_hi = smem_u32(smem + stage * kStageBytes);
-                    const uint32_t sa_lo = sa_hi + kTileABytes;
-                    const uint32_t sb_hi = sa_lo + kTileABytes;
-                    const uint32_t sb_lo = sb_hi + kTileBBytes;
+            const uint32_t idesc = make_idesc_16bit(BM, BN, A_MN, B_MN, p.in_f16 != 0);
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t n = 0;  // active tiles processed
+            for (int t = blockIdx.x; t < T && !*abort_flag; t += gridDim.x) {
+                TileInfo ti;
+                if (!decode_tile(p, t, ti)) continue;
+                const uint32_t buf = n & 1u, use = n >> 1;
+                ++n;
+                if (!mbar_wait(&tempty[buf], (use & 1u) ^ 1u)) {
+                    *abort_flag = 1;
+                    atomicOr(p.err, kErrTimeout);
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t tacc = tmem_base + buf * kTmemCols;
+                if (ti.run_mma) {
+                    for (int kb = ti.kb_begin; kb < ti.kb_end; ++kb) {
+                        if (!mbar_wait(&full[stage], phase)) {
+                            *abort_flag = 1;
+                            atomicOr(p.err, kErrTimeout);
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t sa_hi = smem_u32(smem + stage * kStageBytes);
+                        const uint32_t sa_lo = sa_hi + kTileABytes;
+                        const uint32_t sb_hi = sa_lo + kTileABytes;
+                        const uint32_t sb_lo = sb_hi + kTileBBytes;
 #pragma unroll
-                    for (int ks = 0; ks < BK / 16; ++ks) {
-                        const uint64_t dah = operand_desc<A_MN>(sa_hi, ks);
-                        const uint64_t dal = operand_desc<A_MN>(sa_lo, ks);
-                        const uint64_t dbh = operand_desc<B_MN>(sb_hi, ks);
-                        const uint64_t dbl = operand_desc<B_MN>(sb_lo, ks);
-                        const uint32_t acc = (kb > kb_begin || ks > 0) ? 1u : 0u;
-                        umma_16bit(tmem_base, dah, dbh, idesc, acc);
-                        if (b_split) umma_16bit(tmem_base, dah, dbl, idesc, 1u);
-                        if (a_split) umma_16bit(tmem_base, dal, dbh, idesc, 1u);
-                    }
-                    umma_commit(&empty[stage]);
-                    if (++stage == kStages) {
-                        stage = 0;
-                        phase ^= 1u;
+                        for (int ks = 0; ks < BK / 16; ++ks) {
+                            const uint64_t dah = operand_desc<A_MN>(sa_hi, ks);
+                            const uint64_t dal = operand_desc<A_MN>(sa_lo, ks);
+                            const uint64_t dbh = operand_desc<B_MN>(sb_hi, ks);
+                            const uint64_t dbl = operand_desc<B_MN>(sb_lo, ks);
+                            const uint32_t acc = (kb > ti.kb_begin || ks > 0) ? 1u : 0u;
+                            umma_16bit(tacc, dah, dbh, idesc, acc);
+                            if (ti.b_split) umma_16bit(tacc, dah, dbl, idesc, 1u);
+                            if (ti.a_split) umma_16bit(tacc, dal, dbh, idesc, 1u);
+                        }
+                        umma_commit(&empty[stage]);
+                        if (++stage == kStages) {
+                            stage = 0;
+                            phase ^= 1u;
+                        }
                     }
                 }
+                umma_commit(&tfull[buf]);  // completes once every MMA of this tile has finished
             }
-            umma_commit(accbar);  // completes once every MMA above has finished
+            umma_commit(drain);
+            (void)mbar_wait(drain, 0);
         }
     } else {
         // ================= epilogue (warps 2..5)
-        // Thread (eg, lane) owns output row `row` of the tile and walks its 256 columns
-        // in chunks of 32 (one tcgen05.ld each).  In symmetric mode (Gram, G^2) only
-        // entries with col >= row are produced from the accumulator; each entry with
-        // col > row is also written, bitwise identical, at (col, row).  Across a warp the
-        // mirrored stores hit 32 consecutive rows of one column: coalesced.
         const int eg = warp & 3;  // tensor-memory lane quarter this warp may access
-        const bool ok = __all_sync(0xffffffffu, mbar_wait(accbar, 0));
-        if (!ok && lane == 0) atomicOr(p.err, kErrTimeout);
-        __syncwarp();
-        tc_fence_after();
-        const int row = m0 + eg * 32 + lane;
-        const bool row_ok = row < g.M;
-        const bool sym = g.sym != 0;
-        const bool f32_out = (p.epi == kEpiF32) || (p.epi == kEpiGram && g.splits > 1);
-        const bool gram_fused = (p.epi == kEpiGram && g.splits == 1);
-        float s_sq = 0.f, s_tr = 0.f, s_dev = 0.f;
-        for (int c32 = 0; c32 < BN / 32; ++c32) {
-            const int col0 = n0 + c32 * 32;
-            if (col0 >= g.N) break;
-            float v[32];
+        uint32_t n = 0;
+        for (int t = blockIdx.x; t < T; t += gridDim.x) {
+            TileInfo ti;
+            if (!decode_tile(p, t, ti)) continue;
+            const uint32_t buf = n & 1u, use = n >> 1;
+            ++n;
+            const bool ok = __all_sync(0xffffffffu, mbar_wait(&tfull[buf], use & 1u));
+            if (!ok) {
+                if (lane == 0) atomicOr(p.err, kErrTimeout);
+                break;
+            }
             __syncwarp();
-            if (run_mma && ok) {
-                uint32_t r[32];
-                tmem_ld32(tmem_base + (static_cast<uint32_t>(eg * 32) << 16) + c32 * 32, r);
-                tmem_ld_wait();
-#pragma unroll
-                for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-            } else {
-#pragma unroll
-                for (int j = 0; j < 32; ++j) v[j] = 0.f;
-            }
-            const int nvalid = min(32, g.N - col0);
-            const int d = row - col0;  // column index of the diagonal inside this chunk
-            // chunk entirely below the diagonal: produced by a mirror elsewhere
-            if (!row_ok || (sym && d > nvalid - 1)) continue;
-            const bool upper_all = !sym || d < 0;  // every column of the chunk has col > row
-            const int64_t goff = b * g.bf_batch_stride + static_cast<int64_t>(row) * g.ld_bf + col0;
-            if (p.epi == kEpiPoly) {
-                const __nv_bfloat16* gh = g.g_hi + goff;
-                const __nv_bfloat16* gl = g.g_lo + goff;
-                const bool gf16 = p.in_f16 != 0;
-                if (nvalid == 32) {
-                    const uint4* h4 = reinterpret_cast<const uint4*>(gh);
-                    const uint4* l4 = reinterpret_cast<const uint4*>(gl);
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const uint4 hh = h4[q], ll = l4[q];
-                        const uint32_t hw[4] = {hh.x, hh.y, hh.z, hh.w};
-                        const uint32_t lw[4] = {ll.x, ll.y, ll.z, ll.w};
-#pragma unroll
-                        for (int w = 0; w < 4; ++w) {
-                            const float g0 = dec16(hw[w] & 0xFFFFu, gf16) + dec16(lw[w] & 0xFFFFu, gf16);
-                            const float g1 = dec16(hw[w] >> 16, gf16) + dec16(lw[w] >> 16, gf16);
-                            v[8 * q + 2 * w] = cc * v[8 * q + 2 * w] + cb * g0;
-                            v[8 * q + 2 * w + 1] = cc * v[8 * q + 2 * w + 1] + cb * g1;
-                        }
-                    }
-                } else {
-                    const uint16_t* gh16 = reinterpret_cast<const uint16_t*>(gh);
-                    const uint16_t* gl16 = reinterpret_cast<const uint16_t*>(gl);
-#pragma unroll
-                    for (int j = 0; j < 32; ++j)
-                        if (j < nvalid) v[j] = cc * v[j] + cb * (dec16(gh16[j], gf16) + dec16(gl16[j], gf16));
-                }
-#pragma unroll
-                for (int j = 0; j < 32; ++j)
-                    if (j == d) v[j] += ca;
-            } else if (p.epi == kEpiXSplit) {
-#pragma unroll
-                for (int j = 0; j < 32; ++j) v[j] *= xs;
-            }
-            if (gram_fused) {
-#pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    if (j < nvalid && (!sym || j >= d)) {
-                        const float x = v[j];
-                        const float e = (j == d) ? x - 1.f : x;
-                        const float w = (sym && j > d) ? 2.f : 1.f;  // mirrored entry counts twice
-                        s_sq = fmaf(w * x, x, s_sq);
-                        s_dev = fmaf(w * e, e, s_dev);
-                        if (j == d) s_tr += x;
-                    }
-                }
-            }
-            if (f32_out) {
-                float* base = g.out_f32 + split * g.f32_split_stride + b * g.f32_batch_stride;
-                float* out = base + static_cast<int64_t>(row) * g.ld_f32 + col0;
-                if (upper_all && nvalid == 32 && (g.ld_f32 & 3) == 0) {
-                    float4* o4 = reinterpret_cast<float4*>(out);
-#pragma unroll
-                    for (int q = 0; q < 8; ++q)
-                        o4[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-                } else {
-#pragma unroll
-                    for (int j = 0; j < 32; ++j)
-                        if (j < nvalid && (!sym || j >= d)) out[j] = v[j];
-                }
-                if (sym) {
-#pragma unroll
-                    for (int j = 0; j < 32; ++j)
-                        if (j < nvalid && j > d) base[static_cast<int64_t>(col0 + j) * g.ld_f32 + row] = v[j];
-                }
-            } else {
-                uint16_t* oh = reinterpret_cast<uint16_t*>(g.out_hi);
-                uint16_t* ol = reinterpret_cast<uint16_t*>(g.out_lo);
-                const bool of16 = p.out_f16 != 0;
-                if (upper_all) {
-                    store_split_row(oh + goff, ol + goff, v, nvalid, of16);
-                } else {
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        if (j < nvalid && j >= d) {
-                            uint16_t h, l;
-                            split16(v[j], of16, h, l);
-                            oh[goff + j] = h;
-                            ol[goff + j] = l;
-                        }
-                    }
-                }
-                if (sym) {
-                    const int64_t mbase = b * g.bf_batch_stride + row;
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        if (j < nvalid && j > d) {
-                            uint16_t h, l;
-                            split16(v[j], of16, h, l);
-                            const int64_t o = mbase + static_cast<int64_t>(col0 + j) * g.ld_bf;
-                            oh[o] = h;
-                            ol[o] = l;
-                        }
-                    }
-                }
-            }
-        }
-        if (gram_fused) {
-            // fixed-order reduction of the tile's sums over the 128 epilogue threads
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                s_sq += __shfl_xor_sync(0xffffffffu, s_sq, o);
-                s_tr += __shfl_xor_sync(0xffffffffu, s_tr, o);
-                s_dev += __shfl_xor_sync(0xffffffffu, s_dev, o);
-            }
-            if (lane == 0) {
-                red[eg * 3 + 0] = s_sq;
-                red[eg * 3 + 1] = s_tr;
-                red[eg * 3 + 2] = s_dev;
-            }
-            asm volatile("bar.sync 1, 128;" ::: "memory");
-            if (warp == 2 && lane < 3) {
-                const float t = red[lane] + red[3 + lane] + red[6 + lane] + red[9 + lane];
-                g.part[(g.part_base + static_cast<int64_t>(b) * ntiles + tile) * 3 + lane] = t;
-            }
+            tc_fence_after();
+            tile_epilogue(p, ti, tmem_base + buf * kTmemCols, ok, eg, lane);
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[buf]);
         }
     }
 
-    // ---- teardown: no tcgen05 op may be in flight when the accumulator is freed
+    // ---- teardown: the MMA thread has waited for all its MMAs (drain barrier)
     tc_fence_before();
     __syncthreads();
     if (warp == 1) {
         __syncwarp();
         tc_fence_after();
-        tmem_dealloc(tmem_base, kTmemCols);
+        tmem_dealloc(tmem_base, 2 * kTmemCols);
     }
 }
 
@@ -447,8 +507,7 @@ template <bool A_MN, bool B_MN>
 static cudaError_t launch_gemm_t(const GemmParams& p, int grid, cudaStream_t stream) {
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(k_gemm_split<A_MN, B_MN>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaError_t e = cudaFuncSetAttribute(k_gemm_split<A_MN, B_MN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              kGemmSmemBytes);
         if (e != cudaSuccess) return e;
         attr_set = true;
@@ -457,13 +516,11 @@ static cudaError_t launch_gemm_t(const GemmParams& p, int grid, cudaStream_t str
     return cudaGetLastError();
 }
 
-cudaError_t launch_gemm(const GemmParams& p, bool a_mn, bool b_mn, cudaStream_t stream) {
-    int grid = 0;
-    for (int i = 0; i < p.num_groups; ++i) {
-        const GemmGroup& g = p.g[i];
-        grid = g.cta_begin + g.batch * (g.sym ? g.tiles_sym : g.tiles_m * g.tiles_n) * g.splits;
-    }
-    if (grid <= 0) return cudaSuccess;
+// Launches one persistent GEMM over the groups of `p` (p.total_tiles tiles) on at most
+// `max_ctas` CTAs (one per SM).
+cudaError_t launch_gemm(const GemmParams& p, bool a_mn, bool b_mn, int max_ctas, cudaStream_t stream) {
+    if (p.total_tiles <= 0) return cudaSuccess;
+    const int grid = p.total_tiles < max_ctas ? p.total_tiles : max_ctas;
     if (!a_mn && !b_mn) return launch_gemm_t<false, false>(p, grid, stream);
     if (a_mn && b_mn) return launch_gemm_t<true, true>(p, grid, stream);
     if (!a_mn && b_mn) return launch_gemm_t<false, true>(p, grid, stream);

@@ -87,7 +87,11 @@ __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict
     if (threadIdx.x < 3) {
         float s = 0.f;
         for (int i = 0; i < (int)(blockDim.x >> 5); ++i) s += red[threadIdx.x][i];
-        fin_part[(md.gpart_slot + ft.y) * 3 + threadIdx.x] = s;
+        float* slot = fin_part + (md.gpart_slot + ft.y) * 12;  // 4 slots of 3 per tile
+        slot[threadIdx.x] = s;
+        slot[3 + threadIdx.x] = 0.f;
+        slot[6 + threadIdx.x] = 0.f;
+        slot[9 + threadIdx.x] = 0.f;
     }
 }
 
@@ -105,8 +109,8 @@ __global__ void k_control(const MatDesc* __restrict__ mats, int nmat, MatState* 
     }
     const MatDesc md = mats[mi];
     double sq = 0.0, tr = 0.0, dev = 0.0;
-    for (int i = lane; i < md.n_gtiles; i += 32) {
-        const float* pp = fin_part + (md.gpart_slot + i) * 3;
+    for (int i = lane; i < 4 * md.n_gtiles; i += 32) {  // 4 partial slots per Gram tile
+        const float* pp = fin_part + (md.gpart_slot * 4 + i) * 3;
         sq += pp[0];
         tr += pp[1];
         dev += pp[2];

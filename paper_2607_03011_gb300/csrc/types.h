@@ -13,13 +13,12 @@ namespace isoloco {
 constexpr int BM = 128;
 constexpr int BN = 256;
 constexpr int BK = 32;
-constexpr int kStages = 2;          // per CTA; two CTAs share an SM (measured best on GB300)
-constexpr int kGemmCtasPerSm = 2;
+constexpr int kStages = 4;  // shared-memory ring depth of the persistent GEMM (one CTA per SM)
 constexpr int kTileABytes = BM * BK * 2;                       // one bf16 plane of A
 constexpr int kTileBBytes = BN * BK * 2;                       // one bf16 plane of B
 constexpr int kStageBytes = 2 * kTileABytes + 2 * kTileBBytes;  // hi + lo of A and B
 constexpr int kGemmThreads = 192;  // warp 0 TMA, warp 1 MMA, warps 2..5 epilogue
-constexpr int kTmemCols = 256;
+constexpr int kTmemCols = 256;     // one accumulator; the kernel double-buffers (512 columns)
 constexpr int kMaxGroups = 8;
 constexpr int kFinRows = 32;  // rows of one k_gram_finalize tile (x BN columns)
 constexpr int kGemmSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
@@ -55,7 +54,7 @@ struct GemmGroup {
     int tiles_m, tiles_n, splits, kblocks_per_split;
     int sym;        // square symmetric output: compute only tiles touching col >= row
     int tiles_sym;  // number of such tiles per matrix
-    int cta_begin;  // first blockIdx.x of the group
+    int cta_begin;  // first tile index of the group in the launch's tile list
     int mat_base;   // index of the group's first matrix in the state array
     // fp32 output (kEpiF32): out_f32 + split*split_stride + b*batch_stride + row*ld + col
     float* out_f32;
@@ -92,6 +91,7 @@ struct MatState {
 struct GemmParams {
     GemmGroup g[kMaxGroups];
     int num_groups;
+    int total_tiles;      // tiles of all groups; g[i].cta_begin is group i's first tile
     int epi;
     int gate;
     int in_f16;           // operand planes are fp16 (else bf16); also the G planes of kEpiPoly
