@@ -377,7 +377,7 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         (rc = dalloc(p, &p->xlo[1], plane)) ||
         (rc = dalloc(p, &p->ghi, gplane)) || (rc = dalloc(p, &p->glo, gplane)) || (rc = dalloc(p, &p->phi, gplane)) ||
         (rc = dalloc(p, &p->plo, gplane)) || (rc = dalloc(p, &p->gpart, gpart)) || (rc = dalloc(p, &p->d1d, d1)) ||
-        (rc = dalloc(p, &p->fin_part, 12 * fin)) || (rc = dalloc(p, &p->ftiles, (int64_t)ftiles.size())) ||
+        (rc = dalloc(p, &p->fin_part, 3 * kEpiWarps * fin)) || (rc = dalloc(p, &p->ftiles, (int64_t)ftiles.size())) ||
         (rc = dalloc(p, &p->tpart, tr)) || (rc = dalloc(p, &p->tchunks, tr)) ||
         (rc = dalloc(p, &p->state, p->nmat)) || (rc = dalloc(p, &p->mats_d, p->nmat)) ||
         (rc = dalloc(p, &p->gpart_off_d, p->nmat)) || (rc = dalloc(p, &p->gpart_sstride_d, p->nmat)) ||
@@ -587,10 +587,14 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
         if ((rc = flush_set(p, ISOLOCO_PHASE_POLY, poly, false, false, st))) return rc;
         // ---- X_{t+1} = xscale * X_t P (tall) or P X_t (wide)
         // X_{t+1} is always written as fp16 planes; X is the split operand (A when tall,
-        // B when wide), P the single one except in the polish step
-        LaunchSet utall, uwide;
-        init_set(utall, kEpiXSplit, kGateStep, p, first ? Precision{0, 1, 1, 1, 0} : Precision{1, 1, 1, 0, 1});
-        init_set(uwide, kEpiXSplit, kGateStep, p, first ? Precision{0, 1, 1, 1, 0} : Precision{1, 1, 0, 1, 1});
+        // B when wide), P the single one, except in the polish step (own launch, 3 passes)
+        LaunchSet utall, uwide, ptall, pwide;
+        init_set(utall, kEpiXSplit, first ? kGateStep : kGateQuintic, p,
+                 first ? Precision{0, 1, 1, 1, 0} : Precision{1, 1, 1, 0, 0});
+        init_set(uwide, kEpiXSplit, first ? kGateStep : kGateQuintic, p,
+                 first ? Precision{0, 1, 1, 1, 0} : Precision{1, 1, 0, 1, 0});
+        init_set(ptall, kEpiXSplit, kGatePolish, p, Precision{1, 1, 1, 1, 0});
+        init_set(pwide, kEpiXSplit, kGatePolish, p, Precision{1, 1, 1, 1, 0});
         for (size_t b = 0; b < p->buckets.size(); ++b) {
             const Bucket& bk = p->buckets[b];
             const CUtensorMap* m = maps + b * kMapsPerBucket;
@@ -612,9 +616,12 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             g.bf_batch_stride = (int64_t)bk.rows * bk.ld;
             g.ld_bf = bk.ld;
             (bk.tall ? utall : uwide).add(g);
+            if (!first) (bk.tall ? ptall : pwide).add(g);
         }
         if ((rc = flush_set(p, ISOLOCO_PHASE_UPDATE, utall, false, false, st)) ||
-            (rc = flush_set(p, ISOLOCO_PHASE_UPDATE, uwide, false, true, st)))
+            (rc = flush_set(p, ISOLOCO_PHASE_UPDATE, uwide, false, true, st)) ||
+            (rc = flush_set(p, ISOLOCO_PHASE_UPDATE, ptall, false, false, st)) ||
+            (rc = flush_set(p, ISOLOCO_PHASE_UPDATE, pwide, false, true, st)))
             return rc;
     }
     { PhaseTimer tm(p, ISOLOCO_PHASE_TRACE, st, 2);

@@ -11,9 +11,9 @@
 // fp16 passes elsewhere (the operand that is not split only perturbs the iterate's
 // spectrum, which later steps correct).
 //
-// Roles (192 threads): warp 0 issues TMA loads into a kStages-deep ring of shared
+// Roles (320 threads): warp 0 issues TMA loads into a ring of shared
 // memory stages; warp 1 owns the tensor-memory accumulator and issues tcgen05.mma
-// from one thread; warps 2..5 drain the accumulator (tcgen05.ld) and run the
+// from one thread; warps 2..9 drain the accumulator (tcgen05.ld) and run the
 // epilogue.  Stage hand-off uses mbarriers: `full` (TMA bytes landed), `empty`
 // (the MMAs reading a stage finished, via tcgen05.commit), `acc` (all MMAs done).
 //
@@ -140,6 +140,8 @@ __device__ __forceinline__ bool decode_tile(const GemmParams& p, int t, TileInfo
             if (st.done) return false;
         } else {
             if (st.mode == 0) return false;
+            if (p.gate == kGateQuintic && st.mode != 1) return false;
+            if (p.gate == kGatePolish && st.mode != 2) return false;
             if (p.epi == kEpiPoly && st.mode == 2) ti.run_mma = false;  // cubic polish: no G^2
             if (p.split_on_polish && st.mode == 2) ti.a_split = ti.b_split = true;  // final step: 3 passes
         }
@@ -155,14 +157,14 @@ __device__ __forceinline__ bool decode_tile(const GemmParams& p, int t, TileInfo
     return true;
 }
 
-// Epilogue of one tile, run by the 128 threads of warps 2..5 (thread (eg, lane) owns
+// Epilogue of one tile's column half, run by four warps (thread (eg, lane) owns
 // output row m0 + 32 eg + lane).  `tacc` is the tensor-memory accumulator of the tile.
 // In symmetric mode (Gram, G^2) only entries with col >= row are produced from the
 // accumulator; each entry with col > row is also written, bitwise identical, at
 // (col, row): across a warp those mirrored stores hit 32 consecutive rows of one
 // column, so they coalesce.
 __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInfo& ti, uint32_t tacc, bool ok,
-                                              int eg, int lane) {
+                                              int eg, int half, int lane) {
     const GemmGroup& g = p.g[ti.gi];
     const int b = ti.b, m0 = ti.m0, n0 = ti.n0, split = ti.split;
     const float ca = ti.ca, cb = ti.cb, cc = ti.cc, xs = ti.xs;
@@ -172,7 +174,7 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
     const bool f32_out = (p.epi == kEpiF32) || (p.epi == kEpiGram && g.splits > 1);
     const bool gram_fused = (p.epi == kEpiGram && g.splits == 1);
     float s_sq = 0.f, s_tr = 0.f, s_dev = 0.f;
-    for (int c32 = 0; c32 < BN / 32; ++c32) {
+    for (int c32 = half * (BN / 64); c32 < (half + 1) * (BN / 64); ++c32) {
         const int col0 = n0 + c32 * 32;
         if (col0 >= g.N) break;
         float v[32];
@@ -288,7 +290,7 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
         }
     }
     if (gram_fused) {
-        // fixed-order warp reduction; each epilogue warp owns one of the tile's 4 slots
+        // fixed-order warp reduction; each epilogue warp owns one of the tile's kEpiWarps slots
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
             s_sq += __shfl_xor_sync(0xffffffffu, s_sq, o);
@@ -297,7 +299,8 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
         }
         if (lane == 0) {
             const int ntiles = sym ? g.tiles_sym : g.tiles_m * g.tiles_n;
-            float* slot = g.part + ((g.part_base + static_cast<int64_t>(b) * ntiles + ti.tile) * 4 + eg) * 3;
+            float* slot = g.part + ((g.part_base + static_cast<int64_t>(b) * ntiles + ti.tile) * kEpiWarps +
+                                    half * 4 + eg) * 3;
             slot[0] = s_sq;
             slot[1] = s_tr;
             slot[2] = s_dev;
@@ -313,9 +316,9 @@ template <bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_constant__ GemmParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = align1024(smem_raw);
-    uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
-    uint64_t* empty = full + kStages;
-    uint64_t* tfull = empty + kStages;   // [2] accumulator buffer ready for the epilogue
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + kRingBytes);
+    uint64_t* empty = full + kMaxStages;
+    uint64_t* tfull = empty + kMaxStages;  // [2] accumulator buffer ready for the epilogue
     uint64_t* tempty = tfull + 2;        // [2] accumulator buffer released by the epilogue
     uint64_t* drain = tempty + 2;        // teardown: every issued MMA has completed
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
@@ -324,15 +327,19 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const int T = p.total_tiles;
+    // ring geometry of this launch: room for the planes its tiles can load
+    const uint32_t stage_stride = kTileABytes * (p.a_split || p.split_on_polish ? 2u : 1u) +
+                                  kTileBBytes * (p.b_split || p.split_on_polish ? 2u : 1u);
+    const int nstages = min(kMaxStages, static_cast<int>(kRingBytes / stage_stride));
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kStages; ++s) {
+        for (int s = 0; s < nstages; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&tfull[i], 1);
-            mbar_init(&tempty[i], 4);  // one arrival per epilogue warp
+            mbar_init(&tempty[i], kEpiWarps);  // one arrival per epilogue warp
         }
         mbar_init(drain, 1);
         *abort_flag = 0;
@@ -373,9 +380,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                         atomicOr(p.err, kErrTimeout);
                         break;
                     }
-                    uint8_t* sa_hi = smem + stage * kStageBytes;
+                    uint8_t* sa_hi = smem + stage * stage_stride;
                     uint8_t* sa_lo = sa_hi + kTileABytes;
-                    uint8_t* sb_hi = sa_lo + kTileABytes;
+                    uint8_t* sb_hi = sa_hi + kTileABytes * (ti.a_split ? 2u : 1u);
                     uint8_t* sb_lo = sb_hi + kTileBBytes;
                     mbar_arrive_expect_tx(&full[stage], stage_bytes);
                     const int k0 = kb * BK;
@@ -403,7 +410,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                     }
                     issued_mask |= 1u << stage;
                     issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
-                    if (++stage == kStages) {
+                    if (++stage == nstages) {
                         stage = 0;
                         phase ^= 1u;
                     }
@@ -411,7 +418,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
             }
             if (*abort_flag) {
                 // Let the copies already in flight land before the CTA exits.
-                for (int s = 0; s < kStages; ++s)
+                for (int s = 0; s < nstages; ++s)
                     if (issued_mask & (1u << s)) (void)mbar_wait(&full[s], (issued_parity >> s) & 1u);
             }
         }
@@ -442,9 +449,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                             break;
                         }
                         tc_fence_after();
-                        const uint32_t sa_hi = smem_u32(smem + stage * kStageBytes);
+                        const uint32_t sa_hi = smem_u32(smem + stage * stage_stride);
                         const uint32_t sa_lo = sa_hi + kTileABytes;
-                        const uint32_t sb_hi = sa_lo + kTileABytes;
+                        const uint32_t sb_hi = sa_hi + kTileABytes * (ti.a_split ? 2u : 1u);
                         const uint32_t sb_lo = sb_hi + kTileBBytes;
 #pragma unroll
                         for (int ks = 0; ks < BK / 16; ++ks) {
@@ -458,7 +465,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                             if (ti.a_split) umma_16bit(tacc, dal, dbh, idesc, 1u);
                         }
                         umma_commit(&empty[stage]);
-                        if (++stage == kStages) {
+                        if (++stage == nstages) {
                             stage = 0;
                             phase ^= 1u;
                         }
@@ -470,8 +477,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
             (void)mbar_wait(drain, 0);
         }
     } else {
-        // ================= epilogue (warps 2..5)
+        // ================= epilogue (warps 2..9): warp w reads TMEM lanes 32 (w % 4) ..,
+        // warps 2..5 take columns 0..127 of the tile and warps 6..9 columns 128..255
         const int eg = warp & 3;  // tensor-memory lane quarter this warp may access
+        const int half = (warp - 2) >> 2;
         uint32_t n = 0;
         for (int t = blockIdx.x; t < T; t += gridDim.x) {
             TileInfo ti;
@@ -485,7 +494,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
             }
             __syncwarp();
             tc_fence_after();
-            tile_epilogue(p, ti, tmem_base + buf * kTmemCols, ok, eg, lane);
+            tile_epilogue(p, ti, tmem_base + buf * kTmemCols, ok, eg, half, lane);
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&tempty[buf]);

@@ -87,11 +87,9 @@ __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict
     if (threadIdx.x < 3) {
         float s = 0.f;
         for (int i = 0; i < (int)(blockDim.x >> 5); ++i) s += red[threadIdx.x][i];
-        float* slot = fin_part + (md.gpart_slot + ft.y) * 12;  // 4 slots of 3 per tile
+        float* slot = fin_part + (md.gpart_slot + ft.y) * kEpiWarps * 3;  // kEpiWarps slots of 3 per tile
         slot[threadIdx.x] = s;
-        slot[3 + threadIdx.x] = 0.f;
-        slot[6 + threadIdx.x] = 0.f;
-        slot[9 + threadIdx.x] = 0.f;
+        for (int w = 1; w < kEpiWarps; ++w) slot[3 * w + threadIdx.x] = 0.f;
     }
 }
 
@@ -109,8 +107,8 @@ __global__ void k_control(const MatDesc* __restrict__ mats, int nmat, MatState* 
     }
     const MatDesc md = mats[mi];
     double sq = 0.0, tr = 0.0, dev = 0.0;
-    for (int i = lane; i < 4 * md.n_gtiles; i += 32) {  // 4 partial slots per Gram tile
-        const float* pp = fin_part + (md.gpart_slot * 4 + i) * 3;
+    for (int i = lane; i < kEpiWarps * md.n_gtiles; i += 32) {  // kEpiWarps partial slots per Gram tile
+        const float* pp = fin_part + (md.gpart_slot * kEpiWarps + i) * 3;
         sq += pp[0];
         tr += pp[1];
         dev += pp[2];

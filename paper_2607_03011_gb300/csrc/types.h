@@ -13,15 +13,19 @@ namespace isoloco {
 constexpr int BM = 128;
 constexpr int BN = 256;
 constexpr int BK = 32;
-constexpr int kStages = 4;  // shared-memory ring depth of the persistent GEMM (one CTA per SM)
+// Shared-memory ring of the persistent GEMM (one CTA per SM): as many stages of the
+// launch's plane set as fit in kRingBytes (4 of 48 KB for three passes, 6 of 32 KB for two).
+constexpr int kMaxStages = 8;
+constexpr int kRingBytes = 4 * (2 * BM * BK * 2 + 2 * BN * BK * 2);
 constexpr int kTileABytes = BM * BK * 2;                       // one bf16 plane of A
 constexpr int kTileBBytes = BN * BK * 2;                       // one bf16 plane of B
-constexpr int kStageBytes = 2 * kTileABytes + 2 * kTileBBytes;  // hi + lo of A and B
-constexpr int kGemmThreads = 192;  // warp 0 TMA, warp 1 MMA, warps 2..5 epilogue
+
+constexpr int kEpiWarps = 8;       // two warps per tensor-memory lane quarter
+constexpr int kGemmThreads = 64 + 32 * kEpiWarps;  // warp 0 TMA, warp 1 MMA, warps 2.. epilogue
 constexpr int kTmemCols = 256;     // one accumulator; the kernel double-buffers (512 columns)
 constexpr int kMaxGroups = 8;
 constexpr int kFinRows = 32;  // rows of one k_gram_finalize tile (x BN columns)
-constexpr int kGemmSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+constexpr int kGemmSmemBytes = kRingBytes + 1024 /*align*/ + 256 /*barriers*/;
 
 // Epilogue of the split-precision GEMM.
 enum EpiMode : int {
@@ -37,6 +41,8 @@ enum GateMode : int {
     kGateNone = 0,    // all (debug GEMM)
     kGateActive = 1,  // matrices not yet done (Gram)
     kGateStep = 2,    // matrices whose mode this iteration is quintic or polish
+    kGateQuintic = 3, // matrices taking a quintic step
+    kGatePolish = 4,  // matrices taking the final polish step
 };
 
 // First tile column of tile row tm that touches the upper triangle of a square output.
