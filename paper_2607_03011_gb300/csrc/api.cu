@@ -46,11 +46,14 @@ constexpr int kDefaultMaxIter = 28;
 constexpr float kDefaultTol = 4e-3f;
 
 // Roles of the tensor maps of one bucket.
-enum MapRole { kRoleKA = 0, kRoleKB = 1, kRoleMN = 2 };
-constexpr int kMapsPerBucket = 26;  // 3 sources x 3 roles x 2 planes + G (2x2) + P (2x2)
+enum MapRole { kRoleKA = 0, kRoleKB = 1, kRoleMN = 2, kRoleST = 3 };
+// 3 sources x 3 roles x 2 planes + G (2x2) + P (2x2) + store maps (X0, X1, G, P) x 2 planes
+constexpr int kMapsPerBucket = 34;
 inline int src_map(int src, int role, int plane) { return (src * 3 + role) * 2 + plane; }
 inline int g_map(int role, int plane) { return 18 + role * 2 + plane; }
 inline int p_map(int role, int plane) { return 22 + role * 2 + plane; }
+// store maps (32 x 32 boxes): which 0 = X0, 1 = X1, 2 = G, 3 = P
+inline int st_map(int which, int plane) { return 26 + which * 2 + plane; }
 
 struct Bucket {
     int rows, cols, ld, n, ld_n, count;
@@ -153,6 +156,8 @@ static bool make_map(CUtensorMap* m, const void* base, int cols, int rows, int c
     CUtensorMapSwizzle sw;
     if (role == kRoleMN) {
         box[0] = 64; box[1] = BK; sw = CU_TENSOR_MAP_SWIZZLE_128B;
+    } else if (role == kRoleST) {
+        box[0] = 32; box[1] = 32; sw = CU_TENSOR_MAP_SWIZZLE_64B;
     } else {
         box[0] = BK; box[1] = (role == kRoleKA) ? BM : BN;
         sw = (BK * 2 == 128) ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
@@ -430,6 +435,17 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
                                   bk.count, bk.ld_n, role))
                         return fail(ISOLOCO_ERR_CUDA, "cuTensorMapEncodeTiled failed (Gram planes)");
                 }
+            for (int pl = 0; pl < 2; ++pl) {
+                if (!make_map(&m[st_map(0, pl)], (pl == 0 ? p->xhi[0] : p->xlo[0]) + bk.plane_off, bk.cols, bk.rows,
+                              bk.count, bk.ld, kRoleST) ||
+                    !make_map(&m[st_map(1, pl)], (pl == 0 ? p->xhi[1] : p->xlo[1]) + bk.plane_off, bk.cols, bk.rows,
+                              bk.count, bk.ld, kRoleST) ||
+                    !make_map(&m[st_map(2, pl)], (pl == 0 ? p->ghi : p->glo) + bk.gplane_off, bk.n, bk.n, bk.count,
+                              bk.ld_n, kRoleST) ||
+                    !make_map(&m[st_map(3, pl)], (pl == 0 ? p->phi : p->plo) + bk.gplane_off, bk.n, bk.n, bk.count,
+                              bk.ld_n, kRoleST))
+                    return fail(ISOLOCO_ERR_CUDA, "cuTensorMapEncodeTiled failed (store maps)");
+            }
         }
         CUDA_TRY(cudaMemcpy(p->tmaps_d, maps.data(), sizeof(CUtensorMap) * maps.size(), cudaMemcpyHostToDevice));
     }
@@ -541,6 +557,8 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             g.ld_f32 = bk.ld_n;
             g.out_hi = p->ghi + bk.gplane_off;
             g.out_lo = p->glo + bk.gplane_off;
+            g.st_hi = m + st_map(2, 0);
+            g.st_lo = m + st_map(2, 1);
             g.bf_batch_stride = (int64_t)bk.n * bk.ld_n;
             g.ld_bf = bk.ld_n;
             g.part = p->fin_part;
@@ -577,6 +595,8 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             set_group_common(g, bk.n, bk.n, bk.n, bk.count, 1, bk.mat_base);
             g.out_hi = p->phi + bk.gplane_off;
             g.out_lo = p->plo + bk.gplane_off;
+            g.st_hi = m + st_map(3, 0);
+            g.st_lo = m + st_map(3, 1);
             g.bf_batch_stride = (int64_t)bk.n * bk.ld_n;
             g.ld_bf = bk.ld_n;
             g.g_hi = p->ghi + bk.gplane_off;
@@ -587,14 +607,10 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
         if ((rc = flush_set(p, ISOLOCO_PHASE_POLY, poly, false, false, st))) return rc;
         // ---- X_{t+1} = xscale * X_t P (tall) or P X_t (wide)
         // X_{t+1} is always written as fp16 planes; X is the split operand (A when tall,
-        // B when wide), P the single one, except in the polish step (own launch, 3 passes)
-        LaunchSet utall, uwide, ptall, pwide;
-        init_set(utall, kEpiXSplit, first ? kGateStep : kGateQuintic, p,
-                 first ? Precision{0, 1, 1, 1, 0} : Precision{1, 1, 1, 0, 0});
-        init_set(uwide, kEpiXSplit, first ? kGateStep : kGateQuintic, p,
-                 first ? Precision{0, 1, 1, 1, 0} : Precision{1, 1, 0, 1, 0});
-        init_set(ptall, kEpiXSplit, kGatePolish, p, Precision{1, 1, 1, 1, 0});
-        init_set(pwide, kEpiXSplit, kGatePolish, p, Precision{1, 1, 1, 1, 0});
+        // B when wide), P the single one except in the polish step (3 passes)
+        LaunchSet utall, uwide;
+        init_set(utall, kEpiXSplit, kGateStep, p, first ? Precision{0, 1, 1, 1, 0} : Precision{1, 1, 1, 0, 1});
+        init_set(uwide, kEpiXSplit, kGateStep, p, first ? Precision{0, 1, 1, 1, 0} : Precision{1, 1, 0, 1, 1});
         for (size_t b = 0; b < p->buckets.size(); ++b) {
             const Bucket& bk = p->buckets[b];
             const CUtensorMap* m = maps + b * kMapsPerBucket;
@@ -613,15 +629,14 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             set_group_common(g, bk.rows, bk.cols, bk.n, bk.count, 1, bk.mat_base);
             g.out_hi = p->xhi[dst] + bk.plane_off;
             g.out_lo = p->xlo[dst] + bk.plane_off;
+            g.st_hi = m + st_map(dst, 0);
+            g.st_lo = m + st_map(dst, 1);
             g.bf_batch_stride = (int64_t)bk.rows * bk.ld;
             g.ld_bf = bk.ld;
             (bk.tall ? utall : uwide).add(g);
-            if (!first) (bk.tall ? ptall : pwide).add(g);
         }
         if ((rc = flush_set(p, ISOLOCO_PHASE_UPDATE, utall, false, false, st)) ||
-            (rc = flush_set(p, ISOLOCO_PHASE_UPDATE, uwide, false, true, st)) ||
-            (rc = flush_set(p, ISOLOCO_PHASE_UPDATE, ptall, false, false, st)) ||
-            (rc = flush_set(p, ISOLOCO_PHASE_UPDATE, pwide, false, true, st)))
+            (rc = flush_set(p, ISOLOCO_PHASE_UPDATE, uwide, false, true, st)))
             return rc;
     }
     { PhaseTimer tm(p, ISOLOCO_PHASE_TRACE, st, 2);

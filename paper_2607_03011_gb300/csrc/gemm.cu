@@ -48,39 +48,6 @@ __device__ __forceinline__ uint64_t operand_desc(uint32_t plane_addr, int ks) {
     }
 }
 
-// Stores 32 values of one row as hi/lo planes (bf16 or fp16 bits).
-__device__ __forceinline__ void store_split_row(uint16_t* hi_row, uint16_t* lo_row, const float* v,
-                                                int ncols_valid, bool f16) {
-    if (ncols_valid >= 32) {
-        uint32_t h[16], l[16];
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            uint16_t h0, l0, h1, l1;
-            split16(v[2 * j], f16, h0, l0);
-            split16(v[2 * j + 1], f16, h1, l1);
-            h[j] = static_cast<uint32_t>(h0) | (static_cast<uint32_t>(h1) << 16);
-            l[j] = static_cast<uint32_t>(l0) | (static_cast<uint32_t>(l1) << 16);
-        }
-        uint4* hp = reinterpret_cast<uint4*>(hi_row);
-        uint4* lp = reinterpret_cast<uint4*>(lo_row);
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            hp[q] = make_uint4(h[4 * q], h[4 * q + 1], h[4 * q + 2], h[4 * q + 3]);
-            lp[q] = make_uint4(l[4 * q], l[4 * q + 1], l[4 * q + 2], l[4 * q + 3]);
-        }
-    } else {
-#pragma unroll
-        for (int j = 0; j < 32; ++j) {
-            if (j < ncols_valid) {
-                uint16_t h0, l0;
-                split16(v[j], f16, h0, l0);
-                hi_row[j] = h0;
-                lo_row[j] = l0;
-            }
-        }
-    }
-}
-
 // Symmetric outputs: the t-th of the tiles that touch the upper triangle (col >= row),
 // in row-major order of tiles.
 __device__ __forceinline__ void sym_tile(int t, int tiles_m, int tiles_n, int& tm, int& tn) {
@@ -157,26 +124,41 @@ __device__ __forceinline__ bool decode_tile(const GemmParams& p, int t, TileInfo
     return true;
 }
 
+// Byte offset of element (r, c) in a 32 x 32 block of 16-bit values stored with 64-byte
+// rows and the 64-byte swizzle (16-byte chunk index XOR (r / 2) mod 4), the layout a TMA
+// store with CU_TENSOR_MAP_SWIZZLE_64B reads.
+__device__ __forceinline__ uint32_t stg_off(int r, int c) {
+    return static_cast<uint32_t>(r * 64 + ((((c >> 3) ^ (r >> 1)) & 3) << 4) + (c & 7) * 2);
+}
+
 // Epilogue of one tile's column half, run by four warps (thread (eg, lane) owns
 // output row m0 + 32 eg + lane).  `tacc` is the tensor-memory accumulator of the tile.
-// In symmetric mode (Gram, G^2) only entries with col >= row are produced from the
-// accumulator; each entry with col > row is also written, bitwise identical, at
-// (col, row): across a warp those mirrored stores hit 32 consecutive rows of one
-// column, so they coalesce.
+// 16-bit outputs leave through the warp's shared-memory staging blocks `stg` and TMA
+// stores, one 32 x 32 block at a time.  In symmetric mode (Gram, G^2) blocks below the
+// diagonal are skipped, a block above it is also stored transposed at (col, row), and the
+// diagonal block is made symmetric in shared memory (its upper half mirrored) before its
+// single store, so every entry is written once and the matrix is bitwise symmetric.
 __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInfo& ti, uint32_t tacc, bool ok,
-                                              int eg, int half, int lane) {
+                                              int eg, int half, int lane, uint8_t* stg) {
     const GemmGroup& g = p.g[ti.gi];
     const int b = ti.b, m0 = ti.m0, n0 = ti.n0, split = ti.split;
     const float ca = ti.ca, cb = ti.cb, cc = ti.cc, xs = ti.xs;
-    const int row = m0 + eg * 32 + lane;
+    const int row_base = m0 + eg * 32;
+    const int row = row_base + lane;
     const bool row_ok = row < g.M;
     const bool sym = g.sym != 0;
     const bool f32_out = (p.epi == kEpiF32) || (p.epi == kEpiGram && g.splits > 1);
     const bool gram_fused = (p.epi == kEpiGram && g.splits == 1);
+    const bool of16 = p.out_f16 != 0;
+    const int nplanes = (g.st_lo != nullptr) ? 2 : 1;
+    uint8_t* sd = stg;                      // direct block
+    uint8_t* sm = stg + kStageBlockBytes;   // transposed (mirror) block
     float s_sq = 0.f, s_tr = 0.f, s_dev = 0.f;
     for (int c32 = half * (BN / 64); c32 < (half + 1) * (BN / 64); ++c32) {
         const int col0 = n0 + c32 * 32;
         if (col0 >= g.N) break;
+        if (sym && col0 < row_base) continue;  // block below the diagonal (warp-uniform)
+        const bool diag = sym && col0 == row_base;
         float v[32];
         __syncwarp();
         if (ti.run_mma && ok) {
@@ -190,12 +172,9 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
             for (int j = 0; j < 32; ++j) v[j] = 0.f;
         }
         const int nvalid = min(32, g.N - col0);
-        const int d = row - col0;  // column index of the diagonal inside this chunk
-        // chunk entirely below the diagonal: produced by a mirror elsewhere
-        if (!row_ok || (sym && d > nvalid - 1)) continue;
-        const bool upper_all = !sym || d < 0;  // every column of the chunk has col > row
-        const int64_t goff = b * g.bf_batch_stride + static_cast<int64_t>(row) * g.ld_bf + col0;
-        if (p.epi == kEpiPoly) {
+        const int d = row - col0;  // column index of this lane's diagonal entry in the block
+        if (p.epi == kEpiPoly && row_ok) {
+            const int64_t goff = b * g.bf_batch_stride + static_cast<int64_t>(row) * g.ld_bf + col0;
             const uint16_t* gh = reinterpret_cast<const uint16_t*>(g.g_hi) + goff;
             const uint16_t* gl = reinterpret_cast<const uint16_t*>(g.g_lo) + goff;
             const bool gf16 = p.in_f16 != 0;
@@ -227,7 +206,7 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
 #pragma unroll
             for (int j = 0; j < 32; ++j) v[j] *= xs;
         }
-        if (gram_fused) {
+        if (gram_fused && row_ok) {
 #pragma unroll
             for (int j = 0; j < 32; ++j) {
                 if (j < nvalid && (!sym || j >= d)) {
@@ -241,9 +220,10 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
             }
         }
         if (f32_out) {
+            if (!row_ok) continue;
             float* base = g.out_f32 + split * g.f32_split_stride + b * g.f32_batch_stride;
             float* out = base + static_cast<int64_t>(row) * g.ld_f32 + col0;
-            if (upper_all && nvalid == 32 && (g.ld_f32 & 3) == 0) {
+            if (!diag && nvalid == 32 && (g.ld_f32 & 3) == 0) {
                 float4* o4 = reinterpret_cast<float4*>(out);
 #pragma unroll
                 for (int q = 0; q < 8; ++q) o4[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
@@ -257,35 +237,49 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
                 for (int j = 0; j < 32; ++j)
                     if (j < nvalid && j > d) base[static_cast<int64_t>(col0 + j) * g.ld_f32 + row] = v[j];
             }
-        } else {
-            uint16_t* oh = reinterpret_cast<uint16_t*>(g.out_hi);
-            uint16_t* ol = reinterpret_cast<uint16_t*>(g.out_lo);
-            const bool of16 = p.out_f16 != 0;
-            if (upper_all) {
-                store_split_row(oh + goff, ol + goff, v, nvalid, of16);
-            } else {
+            continue;
+        }
+        // ---- 16-bit hi (and lo) planes through shared memory and TMA stores
+        uint32_t hw[16], lw[16];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+            uint16_t h0, l0, h1, l1;
+            split16(v[2 * j], of16, h0, l0);
+            split16(v[2 * j + 1], of16, h1, l1);
+            hw[j] = static_cast<uint32_t>(h0) | (static_cast<uint32_t>(h1) << 16);
+            lw[j] = static_cast<uint32_t>(l0) | (static_cast<uint32_t>(l1) << 16);
+        }
+        for (int plane = 0; plane < nplanes; ++plane) {
+            const uint32_t* w = plane ? lw : hw;
+            if (lane == 0) bulk_wait_read0();  // the staging blocks are free again
+            __syncwarp();
+            if (diag) {
 #pragma unroll
                 for (int j = 0; j < 32; ++j) {
-                    if (j < nvalid && j >= d) {
-                        uint16_t h, l;
-                        split16(v[j], of16, h, l);
-                        oh[goff + j] = h;
-                        ol[goff + j] = l;
+                    const uint16_t x = static_cast<uint16_t>((j & 1) ? (w[j >> 1] >> 16) : (w[j >> 1] & 0xFFFFu));
+                    if (j >= lane) *reinterpret_cast<uint16_t*>(sd + stg_off(lane, j)) = x;
+                    if (j > lane) *reinterpret_cast<uint16_t*>(sd + stg_off(j, lane)) = x;
+                }
+            } else {
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    *reinterpret_cast<uint4*>(sd + lane * 64 + ((((q ^ (lane >> 1)) & 3)) << 4)) =
+                        make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+                if (sym) {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const uint16_t x = static_cast<uint16_t>((j & 1) ? (w[j >> 1] >> 16) : (w[j >> 1] & 0xFFFFu));
+                        *reinterpret_cast<uint16_t*>(sm + stg_off(j, lane)) = x;
                     }
                 }
             }
-            if (sym) {
-                const int64_t mbase = b * g.bf_batch_stride + row;
-#pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    if (j < nvalid && j > d) {
-                        uint16_t h, l;
-                        split16(v[j], of16, h, l);
-                        const int64_t o = mbase + static_cast<int64_t>(col0 + j) * g.ld_bf;
-                        oh[o] = h;
-                        ol[o] = l;
-                    }
-                }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                const CUtensorMap* map = plane ? g.st_lo : g.st_hi;
+                tma_store_3d(map, sd, col0, row_base, b);
+                if (sym && !diag) tma_store_3d(map, sm, row_base, col0, b);
+                bulk_commit();
             }
         }
     }
@@ -316,7 +310,8 @@ template <bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_constant__ GemmParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = align1024(smem_raw);
-    uint64_t* full = reinterpret_cast<uint64_t*>(smem + kRingBytes);
+    uint8_t* staging = smem + kRingBytes;  // kEpiWarps x (direct, mirror) blocks
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + kRingBytes + kEpiStagingBytes);
     uint64_t* empty = full + kMaxStages;
     uint64_t* tfull = empty + kMaxStages;  // [2] accumulator buffer ready for the epilogue
     uint64_t* tempty = tfull + 2;        // [2] accumulator buffer released by the epilogue
@@ -494,11 +489,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
             }
             __syncwarp();
             tc_fence_after();
-            tile_epilogue(p, ti, tmem_base + buf * kTmemCols, ok, eg, half, lane);
+            tile_epilogue(p, ti, tmem_base + buf * kTmemCols, ok, eg, half, lane,
+                          staging + (warp - 2) * 2 * kStageBlockBytes);
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&tempty[buf]);
         }
+        if (lane == 0) bulk_wait0();  // this warp's TMA stores have completed
+        __syncwarp();
     }
 
     // ---- teardown: the MMA thread has waited for all its MMAs (drain barrier)

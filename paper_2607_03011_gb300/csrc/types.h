@@ -25,7 +25,11 @@ constexpr int kGemmThreads = 64 + 32 * kEpiWarps;  // warp 0 TMA, warp 1 MMA, wa
 constexpr int kTmemCols = 256;     // one accumulator; the kernel double-buffers (512 columns)
 constexpr int kMaxGroups = 8;
 constexpr int kFinRows = 32;  // rows of one k_gram_finalize tile (x BN columns)
-constexpr int kGemmSmemBytes = kRingBytes + 1024 /*align*/ + 256 /*barriers*/;
+// Epilogue staging: per epilogue warp a 32 x 32 16-bit block and its transpose (2 KB each,
+// 64-byte swizzled rows), written to global memory by TMA stores.
+constexpr int kStageBlockBytes = 32 * 32 * 2;
+constexpr int kEpiStagingBytes = kEpiWarps * 2 * kStageBlockBytes;
+constexpr int kGemmSmemBytes = kRingBytes + kEpiStagingBytes + 1024 /*align*/ + 256 /*barriers*/;
 
 // Epilogue of the split-precision GEMM.
 enum EpiMode : int {
@@ -66,9 +70,12 @@ struct GemmGroup {
     float* out_f32;
     int64_t f32_split_stride, f32_batch_stride;
     int ld_f32;
-    // bf16 hi/lo output (kEpiPoly, kEpiXSplit)
+    // 16-bit hi/lo output planes (kEpiGram, kEpiPoly, kEpiXSplit) and their TMA store maps
+    // (32 x 32 boxes, 64-byte swizzle); out_lo/st_lo may be null when no lo plane is kept
     __nv_bfloat16* out_hi;
     __nv_bfloat16* out_lo;
+    const CUtensorMap* st_hi;
+    const CUtensorMap* st_lo;
     int64_t bf_batch_stride;
     int ld_bf;
     // kEpiPoly: the Gram matrix G as bf16 hi/lo planes (same indexing as the output)

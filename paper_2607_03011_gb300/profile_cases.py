@@ -44,12 +44,12 @@ def run_step(workload: str, steps: int) -> None:
         raise SystemExit(1)
 
 
-def run_gemm(batch, m, n, k, a_mn, b_mn, reps) -> None:
+def run_gemm(batch, m, n, k, a_mn, b_mn, reps, precision=0) -> None:
     g = torch.Generator(device="cuda").manual_seed(0)
     A = torch.randn((batch, k, m) if a_mn else (batch, m, k), device="cuda", generator=g)
     B = torch.randn((batch, k, n) if b_mn else (batch, n, k), device="cuda", generator=g)
     for _ in range(reps):
-        isoloco.debug_gemm(A, B, a_mn, b_mn, m, n, k)
+        isoloco.debug_gemm(A, B, a_mn, b_mn, m, n, k, precision=precision)
     torch.cuda.synchronize()
     print("gemm ok")
 
@@ -68,11 +68,12 @@ def main():
     gm.add_argument("--a-mn", type=int, default=0)
     gm.add_argument("--b-mn", type=int, default=0)
     gm.add_argument("--reps", type=int, default=2)
+    gm.add_argument("--precision", type=int, default=0)
     a = ap.parse_args()
     if a.cmd == "step":
         run_step(a.workload, a.steps)
     else:
-        run_gemm(a.batch, a.m, a.n, a.k, a.a_mn, a.b_mn, a.reps)
+        run_gemm(a.batch, a.m, a.n, a.k, a.a_mn, a.b_mn, a.reps, a.precision)
 
 
 if __name__ == "__main__":
