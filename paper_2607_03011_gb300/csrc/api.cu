@@ -26,7 +26,8 @@ namespace isoloco {
 // kernels defined in the other translation units
 cudaError_t launch_gemm(const GemmParams& p, bool a_mn, bool b_mn, int max_ctas, cudaStream_t stream);
 __global__ void k_gram_finalize(const MatDesc*, const int2*, const MatState*, const float*, const int64_t*,
-                                const int64_t*, const int*, __nv_bfloat16*, __nv_bfloat16*, float*, int);
+                                const int64_t*, const int*, __nv_bfloat16*, __nv_bfloat16*, float*, int,
+                                __nv_bfloat16*);
 __global__ void k_control(const MatDesc*, int, MatState*, const float*, int, int, float, uint32_t*);
 __global__ void k_trace_partial(const MatDesc*, const int4*, const MatState*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, const __nv_bfloat16*,
@@ -48,12 +49,15 @@ constexpr float kDefaultTol = 4e-3f;
 // Roles of the tensor maps of one bucket.
 enum MapRole { kRoleKA = 0, kRoleKB = 1, kRoleMN = 2, kRoleST = 3 };
 // 3 sources x 3 roles x 2 planes + G (2x2) + P (2x2) + store maps (X0, X1, G, P) x 2 planes
-constexpr int kMapsPerBucket = 34;
+// + Y (operand KB, store)
+constexpr int kMapsPerBucket = 36;
 inline int src_map(int src, int role, int plane) { return (src * 3 + role) * 2 + plane; }
 inline int g_map(int role, int plane) { return 18 + role * 2 + plane; }
 inline int p_map(int role, int plane) { return 22 + role * 2 + plane; }
 // store maps (32 x 32 boxes): which 0 = X0, 1 = X1, 2 = G, 3 = P
 inline int st_map(int which, int plane) { return 26 + which * 2 + plane; }
+inline int y_map() { return 34; }     // Y as the B operand (K-major, 256 rows)
+inline int y_st_map() { return 35; }  // Y store map
 
 struct Bucket {
     int rows, cols, ld, n, ld_n, count;
@@ -84,6 +88,7 @@ struct isoloco_plan {
     int64_t ws_bytes = 0;
     __nv_bfloat16 *dhi = nullptr, *dlo = nullptr, *xhi[2] = {nullptr, nullptr}, *xlo[2] = {nullptr, nullptr};
     __nv_bfloat16 *ghi = nullptr, *glo = nullptr, *phi = nullptr, *plo = nullptr;
+    __nv_bfloat16* ypl = nullptr;  // Y = b I + c G of the next quintic step (hi plane only)
     float* gpart = nullptr;
     float* d1d = nullptr;
     float* fin_part = nullptr;
@@ -381,7 +386,7 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         (rc = dalloc(p, &p->xlo[0], plane)) || (rc = dalloc(p, &p->xhi[1], plane)) ||
         (rc = dalloc(p, &p->xlo[1], plane)) ||
         (rc = dalloc(p, &p->ghi, gplane)) || (rc = dalloc(p, &p->glo, gplane)) || (rc = dalloc(p, &p->phi, gplane)) ||
-        (rc = dalloc(p, &p->plo, gplane)) || (rc = dalloc(p, &p->gpart, gpart)) || (rc = dalloc(p, &p->d1d, d1)) ||
+        (rc = dalloc(p, &p->plo, gplane)) || (rc = dalloc(p, &p->ypl, gplane)) || (rc = dalloc(p, &p->gpart, gpart)) || (rc = dalloc(p, &p->d1d, d1)) ||
         (rc = dalloc(p, &p->fin_part, 3 * kEpiWarps * fin)) || (rc = dalloc(p, &p->ftiles, (int64_t)ftiles.size())) ||
         (rc = dalloc(p, &p->tpart, tr)) || (rc = dalloc(p, &p->tchunks, tr)) ||
         (rc = dalloc(p, &p->state, p->nmat)) || (rc = dalloc(p, &p->mats_d, p->nmat)) ||
@@ -397,7 +402,7 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
     for (void* a : {(void*)p->dhi, (void*)p->dlo, (void*)p->xhi[0], (void*)p->xlo[0], (void*)p->xhi[1],
                     (void*)p->xlo[1]})
         CUDA_TRY(cudaMemset(a, 0, std::max<int64_t>(1, plane) * 2));
-    for (void* a : {(void*)p->ghi, (void*)p->glo, (void*)p->phi, (void*)p->plo})
+    for (void* a : {(void*)p->ghi, (void*)p->glo, (void*)p->phi, (void*)p->plo, (void*)p->ypl})
         CUDA_TRY(cudaMemset(a, 0, std::max<int64_t>(1, gplane) * 2));
     CUDA_TRY(cudaMemset(p->err_d, 0, 4));
     if (p->nmat) {
@@ -446,6 +451,9 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
                               bk.ld_n, kRoleST))
                     return fail(ISOLOCO_ERR_CUDA, "cuTensorMapEncodeTiled failed (store maps)");
             }
+            if (!make_map(&m[y_map()], p->ypl + bk.gplane_off, bk.n, bk.n, bk.count, bk.ld_n, kRoleKB) ||
+                !make_map(&m[y_st_map()], p->ypl + bk.gplane_off, bk.n, bk.n, bk.count, bk.ld_n, kRoleST))
+                return fail(ISOLOCO_ERR_CUDA, "cuTensorMapEncodeTiled failed (Y maps)");
         }
         CUDA_TRY(cudaMemcpy(p->tmaps_d, maps.data(), sizeof(CUtensorMap) * maps.size(), cudaMemcpyHostToDevice));
     }
@@ -489,6 +497,9 @@ struct LaunchSet {
 struct Precision {
     int in_f16, out_f16, a_split, b_split, split_on_polish;
 };
+
+// Iterations after the first write Y = b I + c G in the Gram epilogue and form
+// P = a I + G Y (Horner) in the G^2 launch: no G reads in that epilogue.
 
 static void init_set(LaunchSet& s, int epi, int gate, isoloco_plan* pl, Precision pr) {
     memset(&s.p, 0, sizeof(s.p));
@@ -540,6 +551,7 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
         LaunchSet tall, wide;
         init_set(tall, kEpiGram, kGateActive, p, gram_pr);
         init_set(wide, kEpiGram, kGateActive, p, gram_pr);
+        tall.p.gram_y = wide.p.gram_y = first ? 0 : 1;
         for (size_t b = 0; b < p->buckets.size(); ++b) {
             const Bucket& bk = p->buckets[b];
             const CUtensorMap* m = maps + b * kMapsPerBucket;
@@ -559,6 +571,7 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             g.out_lo = p->glo + bk.gplane_off;
             g.st_hi = m + st_map(2, 0);
             g.st_lo = m + st_map(2, 1);
+            g.st_y = m + y_st_map();
             g.bf_batch_stride = (int64_t)bk.n * bk.ld_n;
             g.ld_bf = bk.ld_n;
             g.part = p->fin_part;
@@ -574,7 +587,7 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             PhaseTimer tm(p, ISOLOCO_PHASE_FINALIZE, st);
             k_gram_finalize<<<p->nftiles, 256, 0, st>>>(p->mats_d, p->ftiles, p->state, p->gpart, p->gpart_off_d,
                                                         p->gpart_sstride_d, p->nsplit_d, p->ghi, p->glo,
-                                                        p->fin_part, first ? 0 : 1);
+                                                        p->fin_part, first ? 0 : 1, first ? nullptr : p->ypl);
             CUDA_TRY(cudaGetLastError());
         }
         { PhaseTimer tm(p, ISOLOCO_PHASE_CONTROL, st);
@@ -584,13 +597,14 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
         // ---- P = a I + b G + c G^2
         LaunchSet poly;
         init_set(poly, kEpiPoly, kGateStep, p, first ? Precision{0, 0, 1, 1, 0} : Precision{1, 1, 1, 0, 0});
+        poly.p.poly_horner = first ? 0 : 1;
         for (size_t b = 0; b < p->buckets.size(); ++b) {
             const Bucket& bk = p->buckets[b];
             const CUtensorMap* m = maps + b * kMapsPerBucket;
             GemmGroup g{};
             g.a_hi = m + g_map(kRoleKA, 0);
             g.a_lo = m + g_map(kRoleKA, 1);
-            g.b_hi = m + g_map(kRoleKB, 0);
+            g.b_hi = first ? m + g_map(kRoleKB, 0) : m + y_map();  // G G (t = 0) or G Y
             g.b_lo = m + g_map(kRoleKB, 1);
             set_group_common(g, bk.n, bk.n, bk.n, bk.count, 1, bk.mat_base);
             g.out_hi = p->phi + bk.gplane_off;

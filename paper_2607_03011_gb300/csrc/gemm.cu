@@ -24,6 +24,7 @@
 #include <cstdio>
 
 #include "common.cuh"
+#include "ns_schedule.h"
 #include "types.h"
 
 namespace isoloco {
@@ -71,7 +72,9 @@ __device__ __forceinline__ void sym_tile(int t, int tiles_m, int tiles_n, int& t
 struct TileInfo {
     int gi, b, tile, split, m0, n0, mat, kb_begin, kb_end;
     bool run_mma, a_split, b_split;
+    bool horner;     // kEpiPoly: P = acc + a I (the MMA computed G Y); else P = a I + b G + c acc
     float ca, cb, cc, xs;
+    float yb, yc;    // kEpiGram with p.gram_y: Y = yb I + yc G for the next quintic step
 };
 
 // Returns false when the tile belongs to a matrix that does no work this launch.
@@ -100,16 +103,23 @@ __device__ __forceinline__ bool decode_tile(const GemmParams& p, int t, TileInfo
     ti.run_mma = true;
     ti.a_split = p.a_split != 0;
     ti.b_split = p.b_split != 0;
-    ti.ca = 0.f, ti.cb = 0.f, ti.cc = 1.f, ti.xs = 1.f;
+    ti.ca = 0.f, ti.cb = 0.f, ti.cc = 1.f, ti.xs = 1.f, ti.yb = 0.f, ti.yc = 0.f;
+    ti.horner = false;
     if (p.gate != kGateNone) {
         const MatState& st = p.state[ti.mat];
         if (p.gate == kGateActive) {
             if (st.done) return false;
+            if (p.gram_y) {  // coefficients of the quintic step this Gram may lead to
+                const int k = st.step % kSchedSteps;
+                ti.yb = kSched[k][1];
+                ti.yc = kSched[k][2];
+            }
         } else {
             if (st.mode == 0) return false;
             if (p.gate == kGateQuintic && st.mode != 1) return false;
             if (p.gate == kGatePolish && st.mode != 2) return false;
             if (p.epi == kEpiPoly && st.mode == 2) ti.run_mma = false;  // cubic polish: no G^2
+            ti.horner = (p.epi == kEpiPoly && p.poly_horner && st.mode == 1);
             if (p.split_on_polish && st.mode == 2) ti.a_split = ti.b_split = true;  // final step: 3 passes
         }
         ti.ca = st.a;
@@ -131,6 +141,44 @@ __device__ __forceinline__ uint32_t stg_off(int r, int c) {
     return static_cast<uint32_t>(r * 64 + ((((c >> 3) ^ (r >> 1)) & 3) << 4) + (c & 7) * 2);
 }
 
+// One warp writes a 32 x 32 block of 16-bit values (lane = row, w = the lane's 32 values
+// packed in pairs) to its staging block(s) and stores it with TMA at (col0, row_base, b):
+// the diagonal block is symmetrised in shared memory; an off-diagonal block of a symmetric
+// output is also stored transposed at (row_base, col0, b).
+__device__ __forceinline__ void stage_store_block(const uint32_t (&w)[16], const CUtensorMap* map, uint8_t* sd,
+                                                  uint8_t* sm, bool diag, bool sym, int lane, int col0,
+                                                  int row_base, int b) {
+    if (lane == 0) bulk_wait_read0();  // the staging blocks are free again
+    __syncwarp();
+    if (diag) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+            const uint16_t x = static_cast<uint16_t>((j & 1) ? (w[j >> 1] >> 16) : (w[j >> 1] & 0xFFFFu));
+            if (j >= lane) *reinterpret_cast<uint16_t*>(sd + stg_off(lane, j)) = x;
+            if (j > lane) *reinterpret_cast<uint16_t*>(sd + stg_off(j, lane)) = x;
+        }
+    } else {
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+            *reinterpret_cast<uint4*>(sd + lane * 64 + ((((q ^ (lane >> 1)) & 3)) << 4)) =
+                make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+        if (sym) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                const uint16_t x = static_cast<uint16_t>((j & 1) ? (w[j >> 1] >> 16) : (w[j >> 1] & 0xFFFFu));
+                *reinterpret_cast<uint16_t*>(sm + stg_off(j, lane)) = x;
+            }
+        }
+    }
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+        tma_store_3d(map, sd, col0, row_base, b);
+        if (sym && !diag) tma_store_3d(map, sm, row_base, col0, b);
+        bulk_commit();
+    }
+}
+
 // Epilogue of one tile's column half, run by four warps (thread (eg, lane) owns
 // output row m0 + 32 eg + lane).  `tacc` is the tensor-memory accumulator of the tile.
 // 16-bit outputs leave through the warp's shared-memory staging blocks `stg` and TMA
@@ -150,7 +198,10 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
     const bool f32_out = (p.epi == kEpiF32) || (p.epi == kEpiGram && g.splits > 1);
     const bool gram_fused = (p.epi == kEpiGram && g.splits == 1);
     const bool of16 = p.out_f16 != 0;
-    const int nplanes = (g.st_lo != nullptr) ? 2 : 1;
+    // planes written: hi, lo (if kept; not for a Horner-form P, whose lo plane nobody reads),
+    // and for the Gram with p.gram_y the plane Y = yb I + yc G (hi only)
+    const bool write_y = (p.epi == kEpiGram && p.gram_y);
+    const int nplanes = (ti.horner || g.st_lo == nullptr) ? 1 : 2;
     uint8_t* sd = stg;                      // direct block
     uint8_t* sm = stg + kStageBlockBytes;   // transposed (mirror) block
     float s_sq = 0.f, s_tr = 0.f, s_dev = 0.f;
@@ -173,7 +224,11 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
         }
         const int nvalid = min(32, g.N - col0);
         const int d = row - col0;  // column index of this lane's diagonal entry in the block
-        if (p.epi == kEpiPoly && row_ok) {
+        if (ti.horner) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                if (j == d) v[j] += ca;
+        } else if (p.epi == kEpiPoly && row_ok) {
             const int64_t goff = b * g.bf_batch_stride + static_cast<int64_t>(row) * g.ld_bf + col0;
             const uint16_t* gh = reinterpret_cast<const uint16_t*>(g.g_hi) + goff;
             const uint16_t* gl = reinterpret_cast<const uint16_t*>(g.g_lo) + goff;
@@ -239,7 +294,7 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
             }
             continue;
         }
-        // ---- 16-bit hi (and lo) planes through shared memory and TMA stores
+        // ---- 16-bit planes through shared memory and TMA stores
         uint32_t hw[16], lw[16];
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
@@ -249,38 +304,18 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
             hw[j] = static_cast<uint32_t>(h0) | (static_cast<uint32_t>(h1) << 16);
             lw[j] = static_cast<uint32_t>(l0) | (static_cast<uint32_t>(l1) << 16);
         }
-        for (int plane = 0; plane < nplanes; ++plane) {
-            const uint32_t* w = plane ? lw : hw;
-            if (lane == 0) bulk_wait_read0();  // the staging blocks are free again
-            __syncwarp();
-            if (diag) {
+        stage_store_block(hw, g.st_hi, sd, sm, diag, sym, lane, col0, row_base, b);
+        if (nplanes > 1) stage_store_block(lw, g.st_lo, sd, sm, diag, sym, lane, col0, row_base, b);
+        if (write_y) {
+            // Y = yb I + yc G, hi plane only (it is the single operand of G Y)
 #pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    const uint16_t x = static_cast<uint16_t>((j & 1) ? (w[j >> 1] >> 16) : (w[j >> 1] & 0xFFFFu));
-                    if (j >= lane) *reinterpret_cast<uint16_t*>(sd + stg_off(lane, j)) = x;
-                    if (j > lane) *reinterpret_cast<uint16_t*>(sd + stg_off(j, lane)) = x;
-                }
-            } else {
-#pragma unroll
-                for (int q = 0; q < 4; ++q)
-                    *reinterpret_cast<uint4*>(sd + lane * 64 + ((((q ^ (lane >> 1)) & 3)) << 4)) =
-                        make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
-                if (sym) {
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        const uint16_t x = static_cast<uint16_t>((j & 1) ? (w[j >> 1] >> 16) : (w[j >> 1] & 0xFFFFu));
-                        *reinterpret_cast<uint16_t*>(sm + stg_off(j, lane)) = x;
-                    }
-                }
+            for (int j = 0; j < 16; ++j) {
+                uint16_t y0, y1, unused;
+                split16(ti.yc * v[2 * j] + (2 * j == d ? ti.yb : 0.f), of16, y0, unused);
+                split16(ti.yc * v[2 * j + 1] + (2 * j + 1 == d ? ti.yb : 0.f), of16, y1, unused);
+                lw[j] = static_cast<uint32_t>(y0) | (static_cast<uint32_t>(y1) << 16);
             }
-            fence_proxy_async_smem();
-            __syncwarp();
-            if (lane == 0) {
-                const CUtensorMap* map = plane ? g.st_lo : g.st_hi;
-                tma_store_3d(map, sd, col0, row_base, b);
-                if (sym && !diag) tma_store_3d(map, sm, row_base, col0, b);
-                bulk_commit();
-            }
+            stage_store_block(lw, g.st_y, sd, sm, diag, sym, lane, col0, row_base, b);
         }
     }
     if (gram_fused) {

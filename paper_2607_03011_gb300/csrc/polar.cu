@@ -45,10 +45,14 @@ __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict
                                                        const int* __restrict__ nsplit,
                                                        __nv_bfloat16* __restrict__ ghi,
                                                        __nv_bfloat16* __restrict__ glo,
-                                                       float* __restrict__ fin_part, int out_f16) {
+                                                       float* __restrict__ fin_part, int out_f16,
+                                                       __nv_bfloat16* __restrict__ ypl) {
     const int2 ft = ftiles[blockIdx.x];
     const int mi = ft.x;
     if (state[mi].done) return;
+    // ypl != null: also write Y = yb I + yc G (hi plane) for the quintic step that may follow
+    const int ks = state[mi].step % kSchedSteps;
+    const float yb = kSched[ks][1], yc = kSched[ks][2];
     const MatDesc md = mats[mi];
     const int n = md.n, ld = md.ld_n;
     const int tiles_c = (n + BN - 1) / BN;
@@ -68,6 +72,11 @@ __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict
         split16(v, out_f16 != 0, h, l);
         reinterpret_cast<uint16_t*>(ghi)[md.gslot + idx] = h;
         reinterpret_cast<uint16_t*>(glo)[md.gslot + idx] = l;
+        if (ypl) {
+            uint16_t yh, yl;
+            split16(yc * v + (r == c ? yb : 0.f), out_f16 != 0, yh, yl);
+            reinterpret_cast<uint16_t*>(ypl)[md.gslot + idx] = yh;
+        }
         sq += v * v;
         const float dlt = (r == c) ? 1.f : 0.f;
         tr += (r == c) ? v : 0.f;

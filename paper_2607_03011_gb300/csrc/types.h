@@ -76,6 +76,7 @@ struct GemmGroup {
     __nv_bfloat16* out_lo;
     const CUtensorMap* st_hi;
     const CUtensorMap* st_lo;
+    const CUtensorMap* st_y;  // kEpiGram with gram_y: store map of the Y plane
     int64_t bf_batch_stride;
     int ld_bf;
     // kEpiPoly: the Gram matrix G as bf16 hi/lo planes (same indexing as the output)
@@ -111,6 +112,8 @@ struct GemmParams {
     int out_f16;          // hi/lo output planes are fp16 (else bf16)
     int a_split, b_split; // operand carries a lo plane (adds one tensor pass each)
     int split_on_polish;  // matrices in the polish step use both lo planes
+    int gram_y;           // kEpiGram: also write Y = b I + c G for the next quintic step
+    int poly_horner;      // kEpiPoly: B is Y, so P = G Y + a I (quintic steps)
     MatState* state;
     uint32_t* err;
 };
