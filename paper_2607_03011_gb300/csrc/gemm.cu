@@ -145,15 +145,10 @@ __device__ __forceinline__ uint32_t stg_off(int r, int c) {
 // packed in pairs) to its staging block(s) and stores it with TMA at (col0, row_base, b):
 // the diagonal block is symmetrised in shared memory; an off-diagonal block of a symmetric
 // output is also stored transposed at (row_base, col0, b).
-// Two staging sets alternate (`set` flips per call): before writing a set, the store group
-// committed two calls ago (the previous user of this set) must have finished reading it.
-__device__ __forceinline__ void stage_store_block(const uint32_t (&w)[16], const CUtensorMap* map, uint8_t* stg,
-                                                  uint32_t& set, bool diag, bool sym, int lane, int col0,
+__device__ __forceinline__ void stage_store_block(const uint32_t (&w)[16], const CUtensorMap* map, uint8_t* sd,
+                                                  uint8_t* sm, bool diag, bool sym, int lane, int col0,
                                                   int row_base, int b) {
-    uint8_t* sd = stg + set * 2 * kStageBlockBytes;
-    uint8_t* sm = sd + kStageBlockBytes;
-    set ^= 1u;
-    if (lane == 0) bulk_wait_read1();
+    if (lane == 0) bulk_wait_read0();  // the staging blocks are free again
     __syncwarp();
     if (diag) {
 #pragma unroll
@@ -192,7 +187,7 @@ __device__ __forceinline__ void stage_store_block(const uint32_t (&w)[16], const
 // diagonal block is made symmetric in shared memory (its upper half mirrored) before its
 // single store, so every entry is written once and the matrix is bitwise symmetric.
 __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInfo& ti, uint32_t tacc, bool ok,
-                                              int eg, int half, int lane, uint8_t* stg, uint32_t& set) {
+                                              int eg, int half, int lane, uint8_t* stg) {
     const GemmGroup& g = p.g[ti.gi];
     const int b = ti.b, m0 = ti.m0, n0 = ti.n0, split = ti.split;
     const float ca = ti.ca, cb = ti.cb, cc = ti.cc, xs = ti.xs;
@@ -207,6 +202,8 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
     // and for the Gram with p.gram_y the plane Y = yb I + yc G (hi only)
     const bool write_y = (p.epi == kEpiGram && p.gram_y);
     const int nplanes = (ti.horner || g.st_lo == nullptr) ? 1 : 2;
+    uint8_t* sd = stg;                      // direct block
+    uint8_t* sm = stg + kStageBlockBytes;   // transposed (mirror) block
     float s_sq = 0.f, s_tr = 0.f, s_dev = 0.f;
     for (int c32 = half * (BN / 64); c32 < (half + 1) * (BN / 64); ++c32) {
         const int col0 = n0 + c32 * 32;
@@ -307,8 +304,8 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
             hw[j] = static_cast<uint32_t>(h0) | (static_cast<uint32_t>(h1) << 16);
             lw[j] = static_cast<uint32_t>(l0) | (static_cast<uint32_t>(l1) << 16);
         }
-        stage_store_block(hw, g.st_hi, stg, set, diag, sym, lane, col0, row_base, b);
-        if (nplanes > 1) stage_store_block(lw, g.st_lo, stg, set, diag, sym, lane, col0, row_base, b);
+        stage_store_block(hw, g.st_hi, sd, sm, diag, sym, lane, col0, row_base, b);
+        if (nplanes > 1) stage_store_block(lw, g.st_lo, sd, sm, diag, sym, lane, col0, row_base, b);
         if (write_y) {
             // Y = yb I + yc G, hi plane only (it is the single operand of G Y)
 #pragma unroll
@@ -318,7 +315,7 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
                 split16(ti.yc * v[2 * j + 1] + (2 * j + 1 == d ? ti.yb : 0.f), of16, y1, unused);
                 lw[j] = static_cast<uint32_t>(y0) | (static_cast<uint32_t>(y1) << 16);
             }
-            stage_store_block(lw, g.st_y, stg, set, diag, sym, lane, col0, row_base, b);
+            stage_store_block(lw, g.st_y, sd, sm, diag, sym, lane, col0, row_base, b);
         }
     }
     if (gram_fused) {
@@ -514,7 +511,6 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
         // warps 2..5 take columns 0..127 of the tile and warps 6..9 columns 128..255
         const int eg = warp & 3;  // tensor-memory lane quarter this warp may access
         const int half = (warp - 2) >> 2;
-        uint32_t set = 0;  // staging set of the next block
         uint32_t n = 0;
         for (int t = blockIdx.x; t < T; t += gridDim.x) {
             TileInfo ti;
@@ -529,7 +525,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
             __syncwarp();
             tc_fence_after();
             tile_epilogue(p, ti, tmem_base + buf * kTmemCols, ok, eg, half, lane,
-                          staging + (warp - 2) * 4 * kStageBlockBytes, set);
+                          staging + (warp - 2) * 2 * kStageBlockBytes);
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&tempty[buf]);

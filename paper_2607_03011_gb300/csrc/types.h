@@ -14,9 +14,9 @@ constexpr int BM = 128;
 constexpr int BN = 256;
 constexpr int BK = 32;
 // Shared-memory ring of the persistent GEMM (one CTA per SM): as many stages of the
-// launch's plane set as fit in kRingBytes (3 of 48 KB for three passes, 5 of 32 KB for two).
+// launch's plane set as fit in kRingBytes (4 of 48 KB for three passes, 6 of 32 KB for two).
 constexpr int kMaxStages = 8;
-constexpr int kRingBytes = 160 * 1024;
+constexpr int kRingBytes = 4 * (2 * BM * BK * 2 + 2 * BN * BK * 2);
 constexpr int kTileABytes = BM * BK * 2;                       // one bf16 plane of A
 constexpr int kTileBBytes = BN * BK * 2;                       // one bf16 plane of B
 
@@ -25,10 +25,10 @@ constexpr int kGemmThreads = 64 + 32 * kEpiWarps;  // warp 0 TMA, warp 1 MMA, wa
 constexpr int kTmemCols = 256;     // one accumulator; the kernel double-buffers (512 columns)
 constexpr int kMaxGroups = 8;
 constexpr int kFinRows = 32;  // rows of one k_gram_finalize tile (x BN columns)
-// Epilogue staging: per epilogue warp two sets (double buffer) of a 32 x 32 16-bit block
-// and its transpose (2 KB each, 64-byte swizzled rows), written out by TMA stores.
+// Epilogue staging: per epilogue warp a 32 x 32 16-bit block and its transpose (2 KB each,
+// 64-byte swizzled rows), written to global memory by TMA stores.
 constexpr int kStageBlockBytes = 32 * 32 * 2;
-constexpr int kEpiStagingBytes = kEpiWarps * 4 * kStageBlockBytes;
+constexpr int kEpiStagingBytes = kEpiWarps * 2 * kStageBlockBytes;
 constexpr int kGemmSmemBytes = kRingBytes + kEpiStagingBytes + 1024 /*align*/ + 256 /*barriers*/;
 
 // Epilogue of the split-precision GEMM.
