@@ -67,35 +67,11 @@ __device__ __forceinline__ void sym_tile(int t, int tiles_m, int tiles_n, int& t
 
 }  // namespace
 
-struct TileInfo;
-
-// TMA loads of one A plane (BM rows x BK) or one B plane (BN rows x BK) of a k-block.
-template <bool MN, class TI>
-__device__ __forceinline__ void load_a_plane(uint8_t* dst, const CUtensorMap* map, uint64_t* bar, const TI& ti, int k0) {
-    if (MN) {
-#pragma unroll
-        for (int c = 0; c < BM / 64; ++c) tma_load_3d(dst + c * (BK * 128), map, bar, ti.m0 + 64 * c, k0, ti.b);
-    } else {
-        tma_load_3d(dst, map, bar, k0, ti.m0, ti.b);
-    }
-}
-
-template <bool MN, class TI>
-__device__ __forceinline__ void load_b_plane(uint8_t* dst, const CUtensorMap* map, uint64_t* bar, const TI& ti, int k0) {
-    if (MN) {
-#pragma unroll
-        for (int c = 0; c < BN / 64; ++c) tma_load_3d(dst + c * (BK * 128), map, bar, ti.n0 + 64 * c, k0, ti.b);
-    } else {
-        tma_load_3d(dst, map, bar, k0, ti.n0, ti.b);
-    }
-}
-
 // Everything a role needs to know about one output tile; every role decodes the same
 // sequence of tile indices, so the three warps agree without communicating.
 struct TileInfo {
     int gi, b, tile, split, m0, n0, mat, kb_begin, kb_end;
-    bool run_mma, a_split, b_split;  // planes of the first sub-stage of every k-block
-    bool extra;      // a second sub-stage per k-block carries the remaining third pass
+    bool run_mma, a_split, b_split;
     bool horner;     // kEpiPoly: P = acc + a I (the MMA computed G Y); else P = a I + b G + c acc
     float ca, cb, cc, xs;
     float yb, yc;    // kEpiGram with p.gram_y: Y = yb I + yc G for the next quintic step
@@ -129,7 +105,6 @@ __device__ __forceinline__ bool decode_tile(const GemmParams& p, int t, TileInfo
     ti.b_split = p.b_split != 0;
     ti.ca = 0.f, ti.cb = 0.f, ti.cc = 1.f, ti.xs = 1.f, ti.yb = 0.f, ti.yc = 0.f;
     ti.horner = false;
-    ti.extra = false;
     if (p.gate != kGateNone) {
         const MatState& st = p.state[ti.mat];
         if (p.gate == kGateActive) {
@@ -145,9 +120,7 @@ __device__ __forceinline__ bool decode_tile(const GemmParams& p, int t, TileInfo
             if (p.gate == kGatePolish && st.mode != 2) return false;
             if (p.epi == kEpiPoly && st.mode == 2) ti.run_mma = false;  // cubic polish: no G^2
             ti.horner = (p.epi == kEpiPoly && p.poly_horner && st.mode == 1);
-            // final polish step: three passes; the launch's ring only holds its two-pass plane
-            // set, so the third pass comes in its own sub-stage
-            if (p.split_on_polish && st.mode == 2 && !(ti.a_split && ti.b_split)) ti.extra = true;
+            if (p.split_on_polish && st.mode == 2) ti.a_split = ti.b_split = true;  // final step: 3 passes
         }
         ti.ca = st.a;
         ti.cb = st.b;
@@ -385,7 +358,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
     const int lane = threadIdx.x & 31;
     const int T = p.total_tiles;
     // ring geometry of this launch: room for the planes its tiles can load
-    const uint32_t stage_stride = kTileABytes * (p.a_split ? 2u : 1u) + kTileBBytes * (p.b_split ? 2u : 1u);
+    const uint32_t stage_stride = kTileABytes * (p.a_split || p.split_on_polish ? 2u : 1u) +
+                                  kTileBBytes * (p.b_split || p.split_on_polish ? 2u : 1u);
     const int nstages = min(kMaxStages, static_cast<int>(kRingBytes / stage_stride));
 
     if (threadIdx.x == 0) {
@@ -424,43 +398,51 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                 if (prefetched != ti.gi) {
                     tma_prefetch_desc(g.a_hi);
                     tma_prefetch_desc(g.b_hi);
-                    if (ti.a_split || ti.extra) tma_prefetch_desc(g.a_lo);
-                    if (ti.b_split || ti.extra) tma_prefetch_desc(g.b_lo);
+                    if (ti.a_split) tma_prefetch_desc(g.a_lo);
+                    if (ti.b_split) tma_prefetch_desc(g.b_lo);
                     prefetched = ti.gi;
                 }
-                const int nsub = ti.extra ? 2 : 1;
-                bool stop = false;
-                for (int kb = ti.kb_begin; kb < ti.kb_end && !stop; ++kb) {
+                const uint32_t stage_bytes =
+                    kTileABytes * (ti.a_split ? 2u : 1u) + kTileBBytes * (ti.b_split ? 2u : 1u);
+                for (int kb = ti.kb_begin; kb < ti.kb_end; ++kb) {
+                    if (!mbar_wait(&empty[stage], phase ^ 1u)) {
+                        *abort_flag = 1;
+                        atomicOr(p.err, kErrTimeout);
+                        break;
+                    }
+                    uint8_t* sa_hi = smem + stage * stage_stride;
+                    uint8_t* sa_lo = sa_hi + kTileABytes;
+                    uint8_t* sb_hi = sa_hi + kTileABytes * (ti.a_split ? 2u : 1u);
+                    uint8_t* sb_lo = sb_hi + kTileBBytes;
+                    mbar_arrive_expect_tx(&full[stage], stage_bytes);
                     const int k0 = kb * BK;
-                    for (int sub = 0; sub < nsub; ++sub) {
-                        if (!mbar_wait(&empty[stage], phase ^ 1u)) {
-                            *abort_flag = 1;
-                            atomicOr(p.err, kErrTimeout);
-                            stop = true;
-                            break;
+                    if (A_MN) {
+#pragma unroll
+                        for (int c = 0; c < BM / 64; ++c) {
+                            tma_load_3d(sa_hi + c * (BK * 128), g.a_hi, &full[stage], ti.m0 + 64 * c, k0, ti.b);
+                            if (ti.a_split)
+                                tma_load_3d(sa_lo + c * (BK * 128), g.a_lo, &full[stage], ti.m0 + 64 * c, k0, ti.b);
                         }
-                        uint8_t* base = smem + stage * stage_stride;
-                        if (sub == 0) {
-                            // A_hi [A_lo] B_hi [B_lo]
-                            uint8_t* sb = base + kTileABytes * (ti.a_split ? 2u : 1u);
-                            mbar_arrive_expect_tx(&full[stage], kTileABytes * (ti.a_split ? 2u : 1u) +
-                                                                    kTileBBytes * (ti.b_split ? 2u : 1u));
-                            load_a_plane<A_MN>(base, g.a_hi, &full[stage], ti, k0);
-                            if (ti.a_split) load_a_plane<A_MN>(base + kTileABytes, g.a_lo, &full[stage], ti, k0);
-                            load_b_plane<B_MN>(sb, g.b_hi, &full[stage], ti, k0);
-                            if (ti.b_split) load_b_plane<B_MN>(sb + kTileBBytes, g.b_lo, &full[stage], ti, k0);
-                        } else {
-                            // the remaining pass: A_hi B_lo when A was split, else A_lo B_hi
-                            mbar_arrive_expect_tx(&full[stage], kTileABytes + kTileBBytes);
-                            load_a_plane<A_MN>(base, ti.a_split ? g.a_hi : g.a_lo, &full[stage], ti, k0);
-                            load_b_plane<B_MN>(base + kTileABytes, ti.a_split ? g.b_lo : g.b_hi, &full[stage], ti, k0);
+                    } else {
+                        tma_load_3d(sa_hi, g.a_hi, &full[stage], k0, ti.m0, ti.b);
+                        if (ti.a_split) tma_load_3d(sa_lo, g.a_lo, &full[stage], k0, ti.m0, ti.b);
+                    }
+                    if (B_MN) {
+#pragma unroll
+                        for (int c = 0; c < BN / 64; ++c) {
+                            tma_load_3d(sb_hi + c * (BK * 128), g.b_hi, &full[stage], ti.n0 + 64 * c, k0, ti.b);
+                            if (ti.b_split)
+                                tma_load_3d(sb_lo + c * (BK * 128), g.b_lo, &full[stage], ti.n0 + 64 * c, k0, ti.b);
                         }
-                        issued_mask |= 1u << stage;
-                        issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
-                        if (++stage == nstages) {
-                            stage = 0;
-                            phase ^= 1u;
-                        }
+                    } else {
+                        tma_load_3d(sb_hi, g.b_hi, &full[stage], k0, ti.n0, ti.b);
+                        if (ti.b_split) tma_load_3d(sb_lo, g.b_lo, &full[stage], k0, ti.n0, ti.b);
+                    }
+                    issued_mask |= 1u << stage;
+                    issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
+                    if (++stage == nstages) {
+                        stage = 0;
+                        phase ^= 1u;
                     }
                 }
             }
@@ -490,44 +472,32 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                 tc_fence_after();
                 const uint32_t tacc = tmem_base + buf * kTmemCols;
                 if (ti.run_mma) {
-                    const int nsub = ti.extra ? 2 : 1;
-                    bool stop = false;
-                    for (int kb = ti.kb_begin; kb < ti.kb_end && !stop; ++kb) {
-                        for (int sub = 0; sub < nsub; ++sub) {
-                            if (!mbar_wait(&full[stage], phase)) {
-                                *abort_flag = 1;
-                                atomicOr(p.err, kErrTimeout);
-                                stop = true;
-                                break;
-                            }
-                            tc_fence_after();
-                            const uint32_t base = smem_u32(smem + stage * stage_stride);
-                            if (sub == 0) {
-                                const uint32_t sa_lo = base + kTileABytes;
-                                const uint32_t sb_hi = base + kTileABytes * (ti.a_split ? 2u : 1u);
-                                const uint32_t sb_lo = sb_hi + kTileBBytes;
+                    for (int kb = ti.kb_begin; kb < ti.kb_end; ++kb) {
+                        if (!mbar_wait(&full[stage], phase)) {
+                            *abort_flag = 1;
+                            atomicOr(p.err, kErrTimeout);
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t sa_hi = smem_u32(smem + stage * stage_stride);
+                        const uint32_t sa_lo = sa_hi + kTileABytes;
+                        const uint32_t sb_hi = sa_hi + kTileABytes * (ti.a_split ? 2u : 1u);
+                        const uint32_t sb_lo = sb_hi + kTileBBytes;
 #pragma unroll
-                                for (int ks = 0; ks < BK / 16; ++ks) {
-                                    const uint64_t dah = operand_desc<A_MN>(base, ks);
-                                    const uint64_t dal = operand_desc<A_MN>(sa_lo, ks);
-                                    const uint64_t dbh = operand_desc<B_MN>(sb_hi, ks);
-                                    const uint64_t dbl = operand_desc<B_MN>(sb_lo, ks);
-                                    const uint32_t acc = (kb > ti.kb_begin || ks > 0) ? 1u : 0u;
-                                    umma_16bit(tacc, dah, dbh, idesc, acc);
-                                    if (ti.b_split) umma_16bit(tacc, dah, dbl, idesc, 1u);
-                                    if (ti.a_split) umma_16bit(tacc, dal, dbh, idesc, 1u);
-                                }
-                            } else {
-#pragma unroll
-                                for (int ks = 0; ks < BK / 16; ++ks)
-                                    umma_16bit(tacc, operand_desc<A_MN>(base, ks),
-                                               operand_desc<B_MN>(base + kTileABytes, ks), idesc, 1u);
-                            }
-                            umma_commit(&empty[stage]);
-                            if (++stage == nstages) {
-                                stage = 0;
-                                phase ^= 1u;
-                            }
+                        for (int ks = 0; ks < BK / 16; ++ks) {
+                            const uint64_t dah = operand_desc<A_MN>(sa_hi, ks);
+                            const uint64_t dal = operand_desc<A_MN>(sa_lo, ks);
+                            const uint64_t dbh = operand_desc<B_MN>(sb_hi, ks);
+                            const uint64_t dbl = operand_desc<B_MN>(sb_lo, ks);
+                            const uint32_t acc = (kb > ti.kb_begin || ks > 0) ? 1u : 0u;
+                            umma_16bit(tacc, dah, dbh, idesc, acc);
+                            if (ti.b_split) umma_16bit(tacc, dah, dbl, idesc, 1u);
+                            if (ti.a_split) umma_16bit(tacc, dal, dbh, idesc, 1u);
+                        }
+                        umma_commit(&empty[stage]);
+                        if (++stage == nstages) {
+                            stage = 0;
+                            phase ^= 1u;
                         }
                     }
                 }
