@@ -456,6 +456,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
         // ================= MMA issuer (one thread)
         if (lane == 0) {
             const uint32_t idesc = make_idesc_16bit(BM, BN, A_MN, B_MN, p.in_f16 != 0);
+            const uint64_t desc_a0 = operand_desc<A_MN>(smem_u32(smem), 0);
+            const uint64_t desc_b0 = operand_desc<B_MN>(smem_u32(smem), 0);
+            // start-address step of one 16-deep K slice: 2048 bytes MN-major, 32 bytes K-major
+            constexpr uint64_t kDescStepA = A_MN ? (2048 >> 4) : (32 >> 4);
+            constexpr uint64_t kDescStepB = B_MN ? (2048 >> 4) : (32 >> 4);
             int stage = 0;
             uint32_t phase = 0;
             uint32_t n = 0;  // active tiles processed
@@ -472,6 +477,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                 tc_fence_after();
                 const uint32_t tacc = tmem_base + buf * kTmemCols;
                 if (ti.run_mma) {
+                    // descriptors of this tile's planes in stage 0; a stage or a 16-deep K
+                    // slice only moves the start address (14-bit field in 16-byte units; every
+                    // shared address is below 256 KB, so the sum never carries out of it)
+                    const uint64_t a_hi0 = desc_a0;
+                    const uint64_t a_lo0 = desc_a0 + (kTileABytes >> 4);
+                    const uint64_t b_hi0 = desc_b0 + ((kTileABytes * (ti.a_split ? 2u : 1u)) >> 4);
+                    const uint64_t b_lo0 = b_hi0 + (kTileBBytes >> 4);
+                    const bool bs = ti.b_split, as = ti.a_split;
+                    uint32_t acc = 0u;
                     for (int kb = ti.kb_begin; kb < ti.kb_end; ++kb) {
                         if (!mbar_wait(&full[stage], phase)) {
                             *abort_flag = 1;
@@ -479,20 +493,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                             break;
                         }
                         tc_fence_after();
-                        const uint32_t sa_hi = smem_u32(smem + stage * stage_stride);
-                        const uint32_t sa_lo = sa_hi + kTileABytes;
-                        const uint32_t sb_hi = sa_hi + kTileABytes * (ti.a_split ? 2u : 1u);
-                        const uint32_t sb_lo = sb_hi + kTileBBytes;
+                        const uint64_t so = static_cast<uint64_t>(stage) * (stage_stride >> 4);
 #pragma unroll
                         for (int ks = 0; ks < BK / 16; ++ks) {
-                            const uint64_t dah = operand_desc<A_MN>(sa_hi, ks);
-                            const uint64_t dal = operand_desc<A_MN>(sa_lo, ks);
-                            const uint64_t dbh = operand_desc<B_MN>(sb_hi, ks);
-                            const uint64_t dbl = operand_desc<B_MN>(sb_lo, ks);
-                            const uint32_t acc = (kb > ti.kb_begin || ks > 0) ? 1u : 0u;
-                            umma_16bit(tacc, dah, dbh, idesc, acc);
-                            if (ti.b_split) umma_16bit(tacc, dah, dbl, idesc, 1u);
-                            if (ti.a_split) umma_16bit(tacc, dal, dbh, idesc, 1u);
+                            const uint64_t da = so + ks * kDescStepA, db = so + ks * kDescStepB;
+                            umma_16bit(tacc, a_hi0 + da, b_hi0 + db, idesc, acc);
+                            acc = 1u;
+                            if (bs) umma_16bit(tacc, a_hi0 + da, b_lo0 + db, idesc, 1u);
+                            if (as) umma_16bit(tacc, a_lo0 + da, b_hi0 + db, idesc, 1u);
                         }
                         umma_commit(&empty[stage]);
                         if (++stage == nstages) {
