@@ -28,12 +28,14 @@ cudaError_t launch_gemm(const GemmParams& p, bool a_mn, bool b_mn, int max_ctas,
 __global__ void k_gram_finalize(const MatDesc*, const int2*, const MatState*, const float*, const int64_t*,
                                 const int64_t*, const int*, __nv_bfloat16*, __nv_bfloat16*, float*, int,
                                 __nv_bfloat16*);
-__global__ void k_control(const MatDesc*, int, MatState*, const float*, int, int, float, uint32_t*);
+__global__ void k_control(const MatDesc*, int, MatState*, const float*, int, int, float, uint32_t*, const int*,
+                          const int*, int, int*, int*, int*, int*);
 __global__ void k_trace_partial(const MatDesc*, const int4*, const MatState*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, double*);
 __global__ void k_trace_final(const MatDesc*, int, MatState*, const double*);
-__global__ void k_reset_state(MatState*, int, uint32_t*);
+__global__ void k_reset_state(MatState*, int, uint32_t*, const MatDesc*, const int*, const int*, int, int*, int*,
+                              int*, int);
 __global__ void k_reduce(const Chunk*, const MatDesc*, ReplicaPtrs, int, int, const float*, float,
                          __nv_bfloat16*, __nv_bfloat16*, float*, uint32_t*);
 __global__ void k_apply(const Chunk*, const MatDesc*, const MatState*, UpdateSrc, int, float, float, float,
@@ -44,6 +46,7 @@ __global__ void k_split_planes(const float*, int64_t, int, int, int, __nv_bfloat
 constexpr int kChunkElems = 16384;
 constexpr int kTraceChunkElems = 16384;
 constexpr int kDefaultMaxIter = 28;
+constexpr int kLaunchCounters = 4096;  // dynamic-scheduler counters, one per GEMM launch of a step
 constexpr float kDefaultTol = 4e-3f;
 
 // Roles of the tensor maps of one bucket.
@@ -97,6 +100,15 @@ struct isoloco_plan {
     int4* tchunks = nullptr;
     MatState* state = nullptr;
     MatDesc* mats_d = nullptr;
+    // work lists (per shape bucket) rebuilt by k_control, and the GEMM tile counters
+    int* bucket_first_d = nullptr;
+    int* bucket_count_d = nullptr;
+    int* list_gram = nullptr;
+    int* cnt_gram = nullptr;
+    int* list_step = nullptr;
+    int* cnt_step = nullptr;
+    int* counters = nullptr;
+    int launch_seq = 0;
     int64_t* gpart_off_d = nullptr;
     int64_t* gpart_sstride_d = nullptr;
     int* nsplit_d = nullptr;
@@ -392,7 +404,13 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         (rc = dalloc(p, &p->state, p->nmat)) || (rc = dalloc(p, &p->mats_d, p->nmat)) ||
         (rc = dalloc(p, &p->gpart_off_d, p->nmat)) || (rc = dalloc(p, &p->gpart_sstride_d, p->nmat)) ||
         (rc = dalloc(p, &p->nsplit_d, p->nmat)) || (rc = dalloc(p, &p->chunks_d, p->nchunks)) ||
-        (rc = dalloc(p, &p->err_d, 1)) ||
+        (rc = dalloc(p, &p->err_d, 1)) || (rc = dalloc(p, &p->list_gram, p->nmat)) ||
+        (rc = dalloc(p, &p->list_step, p->nmat)) ||
+        (rc = dalloc(p, &p->bucket_first_d, (int64_t)p->buckets.size())) ||
+        (rc = dalloc(p, &p->bucket_count_d, (int64_t)p->buckets.size())) ||
+        (rc = dalloc(p, &p->cnt_gram, (int64_t)p->buckets.size())) ||
+        (rc = dalloc(p, &p->cnt_step, (int64_t)p->buckets.size())) ||
+        (rc = dalloc(p, &p->counters, kLaunchCounters)) ||
         (rc = dalloc(p, &p->tmaps_d, (int64_t)kMapsPerBucket * std::max<size_t>(1, p->buckets.size()))))
         return rc;
     CUDA_TRY(cudaHostAlloc(reinterpret_cast<void**>(&p->err_h), sizeof(uint32_t), cudaHostAllocDefault));
@@ -416,6 +434,15 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
     }
     if (p->nchunks)
         CUDA_TRY(cudaMemcpy(p->chunks_d, chunks.data(), sizeof(Chunk) * p->nchunks, cudaMemcpyHostToDevice));
+    if (!p->buckets.empty()) {
+        std::vector<int> bf, bc;
+        for (const Bucket& bk : p->buckets) {
+            bf.push_back(bk.mat_base);
+            bc.push_back(bk.count);
+        }
+        CUDA_TRY(cudaMemcpy(p->bucket_first_d, bf.data(), sizeof(int) * bf.size(), cudaMemcpyHostToDevice));
+        CUDA_TRY(cudaMemcpy(p->bucket_count_d, bc.data(), sizeof(int) * bc.size(), cudaMemcpyHostToDevice));
+    }
 
     // --- tensor maps
     if (!p->buckets.empty()) {
@@ -511,6 +538,8 @@ static void init_set(LaunchSet& s, int epi, int gate, isoloco_plan* pl, Precisio
     s.p.split_on_polish = pr.split_on_polish;
     s.p.epi = epi;
     s.p.gate = gate;
+    s.p.list = (gate == kGateActive) ? pl->list_gram : pl->list_step;
+    s.p.cnt = (gate == kGateActive) ? pl->cnt_gram : pl->cnt_step;
     s.p.state = pl->state;
     s.p.err = pl->err_d;
 }
@@ -533,6 +562,7 @@ static int flush_set(isoloco_plan* pl, int phase, LaunchSet& s, bool a_mn, bool 
             p.g[p.num_groups++] = g;
         }
         p.total_tiles = cta;
+        p.counter = pl->counters + (pl->launch_seq++ % kLaunchCounters);
         CUDA_TRY(launch_gemm(p, a_mn, b_mn, pl->num_sms, st));
     }
     return ISOLOCO_OK;
@@ -563,6 +593,7 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             g.b_hi = m + src_map(src, role_b, 0);
             g.b_lo = m + src_map(src, role_b, 1);
             set_group_common(g, bk.n, bk.n, bk.tall ? bk.rows : bk.cols, bk.count, bk.splits, bk.mat_base);
+            g.bucket = (int)b;
             g.out_f32 = p->gpart + bk.gpart_off;
             g.f32_batch_stride = (int64_t)bk.n * bk.ld_n;
             g.f32_split_stride = (int64_t)bk.count * bk.n * bk.ld_n;
@@ -591,8 +622,9 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             CUDA_TRY(cudaGetLastError());
         }
         { PhaseTimer tm(p, ISOLOCO_PHASE_CONTROL, st);
-        k_control<<<(p->nmat + 7) / 8, 256, 0, st>>>(p->mats_d, p->nmat, p->state, p->fin_part, t, max_iter, tol,
-                                                     p->err_d); }
+        k_control<<<1, 1024, 0, st>>>(p->mats_d, p->nmat, p->state, p->fin_part, t, max_iter, tol, p->err_d,
+                                      p->bucket_first_d, p->bucket_count_d, (int)p->buckets.size(), p->list_gram,
+                                      p->cnt_gram, p->list_step, p->cnt_step); }
         CUDA_TRY(cudaGetLastError());
         // ---- P = a I + b G + c G^2
         LaunchSet poly;
@@ -607,6 +639,7 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             g.b_hi = first ? m + g_map(kRoleKB, 0) : m + y_map();  // G G (t = 0) or G Y
             g.b_lo = m + g_map(kRoleKB, 1);
             set_group_common(g, bk.n, bk.n, bk.n, bk.count, 1, bk.mat_base);
+            g.bucket = (int)b;
             g.out_hi = p->phi + bk.gplane_off;
             g.out_lo = p->plo + bk.gplane_off;
             g.st_hi = m + st_map(3, 0);
@@ -641,6 +674,7 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
                 g.b_lo = m + src_map(src, kRoleMN, 1);
             }
             set_group_common(g, bk.rows, bk.cols, bk.n, bk.count, 1, bk.mat_base);
+            g.bucket = (int)b;
             g.out_hi = p->xhi[dst] + bk.plane_off;
             g.out_lo = p->xlo[dst] + bk.plane_off;
             g.st_hi = m + st_map(dst, 0);
@@ -701,7 +735,10 @@ static int run_isoc_step(isoloco_plan* p, int merge, float* theta, float* mom, c
     const float* th_src = merge ? base : theta;
     const float scale = merge ? -1.f : (o.reduce_mean ? 1.f / (float)p->K : 1.f);
     { PhaseTimer tm(p, ISOLOCO_PHASE_OTHER, st);
-    k_reset_state<<<(std::max(1, p->nmat) + 255) / 256, 256, 0, st>>>(p->state, p->nmat, p->err_d); }
+    k_reset_state<<<(std::max(1, p->nmat) + 255) / 256, 256, 0, st>>>(
+        p->state, p->nmat, p->err_d, p->mats_d, p->bucket_first_d, p->bucket_count_d, (int)p->buckets.size(),
+        p->list_gram, p->cnt_gram, p->counters, kLaunchCounters); }
+    p->launch_seq = 0;
     CUDA_TRY(cudaGetLastError());
     if (p->nchunks) {
         PhaseTimer tm(p, ISOLOCO_PHASE_REDUCE, st);
@@ -964,13 +1001,13 @@ int isoloco_debug_gemm(int a_mn, int b_mn, int precision, int batch, int M, int 
         cudaFree(ah); cudaFree(al); cudaFree(bh); cudaFree(bl); cudaFree(maps_d); cudaFree(dummy_state); cudaFree(err);
     };
     if (cudaMalloc(&ah, asz * 2) || cudaMalloc(&al, asz * 2) || cudaMalloc(&bh, bsz * 2) || cudaMalloc(&bl, bsz * 2) ||
-        cudaMalloc(&maps_d, 4 * sizeof(CUtensorMap)) || cudaMalloc(&err, 4)) {
+        cudaMalloc(&maps_d, 4 * sizeof(CUtensorMap)) || cudaMalloc(&err, 8)) {
         cleanup();
         return fail(ISOLOCO_ERR_OOM, "debug_gemm scratch allocation failed");
     }
     cudaMemsetAsync(ah, 0, asz * 2, st); cudaMemsetAsync(al, 0, asz * 2, st);
     cudaMemsetAsync(bh, 0, bsz * 2, st); cudaMemsetAsync(bl, 0, bsz * 2, st);
-    cudaMemsetAsync(err, 0, 4, st);
+    cudaMemsetAsync(err, 0, 8, st);  // err word and the tile counter
     const int f16 = precision > 0 ? 1 : 0;
     k_split_planes<<<1024, 256, 0, st>>>(A, (int64_t)batch * a_rows * a_cols, a_rows, a_cols, lda, ah, al, f16);
     k_split_planes<<<1024, 256, 0, st>>>(B, (int64_t)batch * b_rows * b_cols, b_rows, b_cols, ldb, bh, bl, f16);
@@ -1000,6 +1037,7 @@ int isoloco_debug_gemm(int a_mn, int b_mn, int precision, int batch, int M, int 
     g.ld_f32 = N;
     gp.num_groups = 1;
     gp.total_tiles = batch * g.tiles_m * g.tiles_n;
+    gp.counter = reinterpret_cast<int*>(err) + 1;
     int dev = 0, sms = 148;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);

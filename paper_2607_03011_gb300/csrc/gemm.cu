@@ -77,18 +77,29 @@ struct TileInfo {
     float yb, yc;    // kEpiGram with p.gram_y: Y = yb I + yc G for the next quintic step
 };
 
-// Returns false when the tile belongs to a matrix that does no work this launch.
-__device__ __forceinline__ bool decode_tile(const GemmParams& p, int t, TileInfo& ti) {
+// Active-tile prefix of the launch: group i owns active tiles [pre[i], pre[i + 1]).
+__device__ __forceinline__ void active_prefix(const GemmParams& p, int* pre) {
+    pre[0] = 0;
+    for (int i = 0; i < p.num_groups; ++i) {
+        const GemmGroup& g = p.g[i];
+        const int mats = p.list ? p.cnt[g.bucket] : g.batch;
+        pre[i + 1] = pre[i] + mats * (g.sym ? g.tiles_sym : g.tiles_m * g.tiles_n) * g.splits;
+    }
+}
+
+// Decodes active tile t.  Returns false when the matrix does no work in this launch.
+__device__ __forceinline__ bool decode_tile(const GemmParams& p, const int* pre, int t, TileInfo& ti) {
     int gi = 0;
-    while (gi + 1 < p.num_groups && t >= p.g[gi + 1].cta_begin) ++gi;
+    while (gi + 1 < p.num_groups && t >= pre[gi + 1]) ++gi;
     const GemmGroup& g = p.g[gi];
-    int local = t - g.cta_begin;
+    int local = t - pre[gi];
     ti.gi = gi;
     ti.split = local % g.splits;
     local /= g.splits;
     const int ntiles = g.sym ? g.tiles_sym : g.tiles_m * g.tiles_n;
     ti.tile = local % ntiles;
-    ti.b = local / ntiles;
+    const int j = local / ntiles;
+    ti.b = p.list ? p.list[g.mat_base + j] : j;
     if (ti.b >= g.batch) return false;
     int tm, tn;
     if (g.sym) {
@@ -351,12 +362,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
     uint64_t* tfull = empty + kMaxStages;  // [2] accumulator buffer ready for the epilogue
     uint64_t* tempty = tfull + 2;        // [2] accumulator buffer released by the epilogue
     uint64_t* drain = tempty + 2;        // teardown: every issued MMA has completed
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+    uint64_t* tq_full = drain + 1;       // [kTileQueue] tile index written by the producer
+    uint64_t* tq_empty = tq_full + kTileQueue;  // [kTileQueue] read by the MMA and epilogue warps
+    int* tq_tile = reinterpret_cast<int*>(tq_empty + kTileQueue);
+    int* pre = tq_tile + kTileQueue;     // [kMaxGroups + 1] active-tile prefix
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pre + kMaxGroups + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int T = p.total_tiles;
     // ring geometry of this launch: room for the planes its tiles can load
     const uint32_t stage_stride = kTileABytes * (p.a_split || p.split_on_polish ? 2u : 1u) +
                                   kTileBBytes * (p.b_split || p.split_on_polish ? 2u : 1u);
@@ -372,6 +386,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
             mbar_init(&tempty[i], kEpiWarps);  // one arrival per epilogue warp
         }
         mbar_init(drain, 1);
+        for (int q = 0; q < kTileQueue; ++q) {
+            mbar_init(&tq_full[q], 1);
+            mbar_init(&tq_empty[q], 1 + kEpiWarps);  // the MMA thread and one lane per epilogue warp
+        }
+        active_prefix(p, pre);
         *abort_flag = 0;
         fence_mbar_init();
     }
@@ -391,9 +410,28 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
             uint32_t phase = 0;
             uint32_t issued_mask = 0, issued_parity = 0;
             int prefetched = -1;
-            for (int t = blockIdx.x; t < T && !*abort_flag; t += gridDim.x) {
+            const int T = pre[p.num_groups];
+            int q = 0;
+            uint32_t qphase = 0;
+            int t = blockIdx.x;
+            for (;;) {
+                // publish the next tile (or -1: no more) to the MMA and epilogue warps
+                const int tile = (t < T && !*abort_flag) ? t : -1;
+                if (!mbar_wait(&tq_empty[q], qphase ^ 1u)) {
+                    *abort_flag = 1;
+                    atomicOr(p.err, kErrTimeout);
+                    break;
+                }
+                tq_tile[q] = tile;
+                mbar_arrive(&tq_full[q]);
+                if (++q == kTileQueue) {
+                    q = 0;
+                    qphase ^= 1u;
+                }
+                if (tile < 0) break;
+                t = atomicAdd(p.counter, 1) + static_cast<int>(gridDim.x);  // claimed early
                 TileInfo ti;
-                if (!decode_tile(p, t, ti) || !ti.run_mma) continue;
+                if (!decode_tile(p, pre, tile, ti) || !ti.run_mma) continue;
                 const GemmGroup& g = p.g[ti.gi];
                 if (prefetched != ti.gi) {
                     tma_prefetch_desc(g.a_hi);
@@ -464,9 +502,23 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
             int stage = 0;
             uint32_t phase = 0;
             uint32_t n = 0;  // active tiles processed
-            for (int t = blockIdx.x; t < T && !*abort_flag; t += gridDim.x) {
+            int q = 0;
+            uint32_t qphase = 0;
+            for (;;) {
+                if (!mbar_wait(&tq_full[q], qphase)) {
+                    *abort_flag = 1;
+                    atomicOr(p.err, kErrTimeout);
+                    break;
+                }
+                const int tile = tq_tile[q];
+                mbar_arrive(&tq_empty[q]);
+                if (++q == kTileQueue) {
+                    q = 0;
+                    qphase ^= 1u;
+                }
+                if (tile < 0 || *abort_flag) break;
                 TileInfo ti;
-                if (!decode_tile(p, t, ti)) continue;
+                if (!decode_tile(p, pre, tile, ti)) continue;
                 const uint32_t buf = n & 1u, use = n >> 1;
                 ++n;
                 if (!mbar_wait(&tempty[buf], (use & 1u) ^ 1u)) {
@@ -520,9 +572,31 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
         const int eg = warp & 3;  // tensor-memory lane quarter this warp may access
         const int half = (warp - 2) >> 2;
         uint32_t n = 0;
-        for (int t = blockIdx.x; t < T; t += gridDim.x) {
+        int q = 0;
+        uint32_t qphase = 0;
+        for (;;) {
+            int tile = -1;
+            int got = 1;
+            if (lane == 0) {
+                got = mbar_wait(&tq_full[q], qphase) ? 1 : 0;
+                if (got) {
+                    tile = tq_tile[q];
+                    mbar_arrive(&tq_empty[q]);
+                }
+            }
+            tile = __shfl_sync(0xffffffffu, tile, 0);
+            got = __shfl_sync(0xffffffffu, got, 0);
+            if (++q == kTileQueue) {
+                q = 0;
+                qphase ^= 1u;
+            }
+            if (!got) {
+                if (lane == 0) atomicOr(p.err, kErrTimeout);
+                break;
+            }
+            if (tile < 0) break;
             TileInfo ti;
-            if (!decode_tile(p, t, ti)) continue;
+            if (!decode_tile(p, pre, tile, ti)) continue;
             const uint32_t buf = n & 1u, use = n >> 1;
             ++n;
             const bool ok = __all_sync(0xffffffffu, mbar_wait(&tfull[buf], use & 1u));

@@ -102,13 +102,10 @@ __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict
     }
 }
 
-// One warp per matrix.  t: iteration index (0 = first Gram of Delta itself).
-__global__ void k_control(const MatDesc* __restrict__ mats, int nmat, MatState* __restrict__ state,
-                          const float* __restrict__ fin_part, int t, int max_iter, float tol,
-                          uint32_t* __restrict__ err) {
-    const int mi = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    const int lane = threadIdx.x & 31;
-    if (mi >= nmat) return;
+// Decision for matrix mi, taken by one warp.  t: iteration index (0 = first Gram of Delta).
+__device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatState* __restrict__ state,
+                               const float* __restrict__ fin_part, int t, int max_iter, float tol,
+                               uint32_t* __restrict__ err, int lane) {
     MatState& st = state[mi];
     if (st.done) {
         if (lane == 0) st.mode = 0;
@@ -179,6 +176,50 @@ __global__ void k_control(const MatDesc* __restrict__ mats, int nmat, MatState* 
         st.c = static_cast<float>(kSched[k][2] * gscale * gscale);
         st.step += 1;
         st.iters += 1;
+    }
+}
+
+
+// One block of 1024 threads.  Warp w takes the decisions of matrices w, w + 32, ...; then
+// warp b compacts, for shape bucket b, the matrices that still need a Gram (not done) and
+// those that take a step this iteration (mode != 0), in matrix order.  GEMM launches only
+// enumerate the listed matrices.
+__global__ void __launch_bounds__(1024) k_control(const MatDesc* __restrict__ mats, int nmat,
+                                                  MatState* __restrict__ state,
+                                                  const float* __restrict__ fin_part, int t, int max_iter,
+                                                  float tol, uint32_t* __restrict__ err,
+                                                  const int* __restrict__ bucket_first,
+                                                  const int* __restrict__ bucket_count, int nbuckets,
+                                                  int* __restrict__ list_gram, int* __restrict__ cnt_gram,
+                                                  int* __restrict__ list_step, int* __restrict__ cnt_step) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int mi = warp; mi < nmat; mi += 32) {
+        control_matrix(mats, mi, state, fin_part, t, max_iter, tol, err, lane);
+        __syncwarp();
+    }
+    __syncthreads();
+    for (int bk = warp; bk < nbuckets; bk += 32) {
+        const int first = bucket_first[bk], count = bucket_count[bk];
+        int ng = 0, ns = 0;
+        for (int j0 = 0; j0 < count; j0 += 32) {
+            const int j = j0 + lane;
+            bool g_on = false, s_on = false;
+            if (j < count) {
+                const MatState& st = state[first + j];
+                g_on = (st.done == 0);
+                s_on = (st.mode != 0);
+            }
+            const unsigned bg = __ballot_sync(0xffffffffu, g_on), bs = __ballot_sync(0xffffffffu, s_on);
+            const unsigned below = (1u << lane) - 1u;
+            if (g_on) list_gram[first + ng + __popc(bg & below)] = j;
+            if (s_on) list_step[first + ns + __popc(bs & below)] = j;
+            ng += __popc(bg);
+            ns += __popc(bs);
+        }
+        if (lane == 0) {
+            cnt_gram[bk] = ng;
+            cnt_step[bk] = ns;
+        }
     }
 }
 
@@ -267,10 +308,17 @@ __global__ void k_trace_final(const MatDesc* __restrict__ mats, int nmat, MatSta
     }
 }
 
-// Resets the per-matrix state before a step.
-__global__ void k_reset_state(MatState* state, int nmat, uint32_t* err) {
+// Resets the per-matrix state before a step: every matrix is active for the first Gram,
+// and the GEMM launches' tile counters restart at zero.
+__global__ void k_reset_state(MatState* state, int nmat, uint32_t* err, const MatDesc* __restrict__ mats,
+                              const int* __restrict__ bucket_first, const int* __restrict__ bucket_count,
+                              int nbuckets, int* __restrict__ list_gram, int* __restrict__ cnt_gram,
+                              int* __restrict__ counters, int ncounters) {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i == 0) *err = 0u;
+    for (int c = i; c < ncounters; c += gridDim.x * blockDim.x) counters[c] = 0;
+    if (i < nbuckets) cnt_gram[i] = bucket_count[i];
+    if (i < nmat) list_gram[i] = i - bucket_first[mats[i].bucket];
     if (i >= nmat) return;
     MatState s;
     s.a = s.b = s.c = 0.f;

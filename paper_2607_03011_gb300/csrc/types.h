@@ -29,7 +29,8 @@ constexpr int kFinRows = 32;  // rows of one k_gram_finalize tile (x BN columns)
 // 64-byte swizzled rows), written to global memory by TMA stores.
 constexpr int kStageBlockBytes = 32 * 32 * 2;
 constexpr int kEpiStagingBytes = kEpiWarps * 2 * kStageBlockBytes;
-constexpr int kGemmSmemBytes = kRingBytes + kEpiStagingBytes + 1024 /*align*/ + 256 /*barriers*/;
+constexpr int kTileQueue = 8;  // tiles handed from the producer warp to the MMA and epilogue warps
+constexpr int kGemmSmemBytes = kRingBytes + kEpiStagingBytes + 1024 /*align*/ + 512 /*barriers, queues*/;
 
 // Epilogue of the split-precision GEMM.
 enum EpiMode : int {
@@ -64,8 +65,9 @@ struct GemmGroup {
     int tiles_m, tiles_n, splits, kblocks_per_split;
     int sym;        // square symmetric output: compute only tiles touching col >= row
     int tiles_sym;  // number of such tiles per matrix
-    int cta_begin;  // first tile index of the group in the launch's tile list
+    int cta_begin;  // (host bookkeeping) first tile of the group when every matrix is active
     int mat_base;   // index of the group's first matrix in the state array
+    int bucket;     // shape bucket: index into the work-list counts
     // fp32 output (kEpiF32): out_f32 + split*split_stride + b*batch_stride + row*ld + col
     float* out_f32;
     int64_t f32_split_stride, f32_batch_stride;
@@ -105,7 +107,12 @@ struct MatState {
 struct GemmParams {
     GemmGroup g[kMaxGroups];
     int num_groups;
-    int total_tiles;      // tiles of all groups; g[i].cta_begin is group i's first tile
+    int total_tiles;      // tiles of all groups when every matrix is active (grid sizing)
+    // Work list of this launch (null: every matrix of every group): for group i, the
+    // matrices list[g.mat_base + j], j < cnt[g.bucket] (indices within the group).
+    const int* list;
+    const int* cnt;
+    int* counter;         // dynamic tile scheduler of this launch (zeroed before the step)
     int epi;
     int gate;
     int in_f16;           // operand planes are fp16 (else bf16); also the G planes of kEpiPoly
