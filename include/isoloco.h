@@ -157,6 +157,38 @@ int isoloco_plan_num_matrices(isoloco_plan_t plan);
 int isoloco_debug_gemm(int a_mn_major, int b_mn_major, int precision, int batch, int M, int N,
                        int K, const float* A, const float* B, float* D, void* stream);
 
+/* The same GEMM as isoloco_debug_gemm (same arguments, same kernels, bitwise the
+ * same D), for callers that must not allocate device memory.  The paper has no
+ * counterpart: this is a library service, not part of the method.
+ *
+ * Who needs it: a caller whose process has handed the device's free memory to
+ * another allocator (a training framework's caching pool that reserved the HBM
+ * up front), so that a cudaMalloc here would fail or force that pool to give
+ * memory back; and a caller in the middle of an overlapped step, where the
+ * implicit device-wide synchronization of cudaMalloc / cudaFree would stall the
+ * work queued on its other streams.  This entry point calls neither, nor any
+ * other allocating routine: its scratch (the hi/lo operand planes, the four
+ * tensor maps, an error word and a tile counter) lives in one static device
+ * array of the library, 16 MiB per device, whose address is looked up once per
+ * device.
+ *
+ * Limit: 1024 + 2 * R(2 * batch * a_rows * round8(a_cols))
+ *             + 2 * R(2 * batch * b_rows * round8(b_cols)) <= 16 MiB,
+ * with (a_rows, a_cols) = (K, M) if a_mn_major else (M, K), likewise B with N,
+ * and R() rounding up to 256 bytes.  E.g. batch 1, M = N = K = 1024 fits;
+ * M = N = K = 2048 does not.  Larger operands return ISOLOCO_ERR_INVALID with a
+ * message giving the bytes needed, before anything is launched.
+ *
+ * Every call on a device shares that one array.  The call zeroes the error word
+ * and the tile counter on `stream` before its kernels and synchronizes `stream`
+ * before returning, so calls made one after another are safe.  Calls whose GPU
+ * work can overlap (from several host threads, or on streams that are not
+ * ordered with one another) race on the shared scratch and give wrong results;
+ * such callers must serialize them. */
+int isoloco_debug_gemm_noalloc(int a_mn_major, int b_mn_major, int precision, int batch, int M,
+                               int N, int K, const float* A, const float* B, float* D,
+                               void* stream);
+
 /* Phases of the launch sequence, for isoloco_profile_read. */
 enum {
     ISOLOCO_PHASE_REDUCE = 0,   /* pseudo-gradient reduction (HBM stream) */

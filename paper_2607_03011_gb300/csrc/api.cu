@@ -14,6 +14,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <map>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -1048,6 +1049,117 @@ int isoloco_debug_gemm(int a_mn, int b_mn, int precision, int batch, int M, int 
     cleanup();
     if (e != cudaSuccess) return fail(ISOLOCO_ERR_CUDA, std::string("debug_gemm: ") + cudaGetErrorString(e));
     if (herr & kErrTimeout) return fail(ISOLOCO_ERR_TIMEOUT, "debug_gemm: device wait timed out");
+    return ISOLOCO_OK;
+}
+
+}  // extern "C"
+
+// ================================================================== GEMM without allocation
+// Scratch of isoloco_debug_gemm_noalloc: one array per device, shared by every call.
+//   [0, 4)     error word      \  zeroed by every call before its launches
+//   [4, 8)     tile counter    /
+//   [256, 768) the four tensor maps (A hi, A lo, B hi, B lo), written by every call
+//   [1024, ..) A hi, A lo, B hi, B lo planes, each starting on a 256-byte boundary and
+//              fully written by the split kernel before the GEMM reads them
+namespace {
+constexpr int64_t kNoAllocScratchBytes = int64_t(16) << 20;  // 16 MiB
+constexpr int64_t kNoAllocMapsOffset = 256;
+constexpr int64_t kNoAllocPlanesOffset = 1024;
+constexpr int kNoAllocMaxDevices = 64;
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+std::mutex g_noalloc_mutex;
+unsigned char* g_noalloc_ptr[kNoAllocMaxDevices] = {};
+
+// Address of the scratch array in the current device's context, looked up once per device.
+int noalloc_scratch(unsigned char** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return fail(ISOLOCO_ERR_CUDA, std::string("cudaGetDevice: ") + cudaGetErrorString(e));
+    if (dev < 0 || dev >= kNoAllocMaxDevices) return fail(ISOLOCO_ERR_INVALID, "device ordinal beyond 63");
+    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+    if (!g_noalloc_ptr[dev]) {
+        void* ptr = nullptr;
+        e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
+        if (e != cudaSuccess || !ptr)
+            return fail(ISOLOCO_ERR_CUDA, std::string("cudaGetSymbolAddress(scratch): ") + cudaGetErrorString(e));
+        g_noalloc_ptr[dev] = static_cast<unsigned char*>(ptr);
+    }
+    *out = g_noalloc_ptr[dev];
+    return ISOLOCO_OK;
+}
+}  // namespace
+
+extern "C" {
+
+int isoloco_debug_gemm_noalloc(int a_mn, int b_mn, int precision, int batch, int M, int N, int K, const float* A,
+                               const float* B, float* D, void* stream) {
+    if (precision < 0 || precision > 3) return fail(ISOLOCO_ERR_INVALID, "bad debug_gemm_noalloc precision");
+    if (batch <= 0 || M <= 0 || N <= 0 || K <= 0 || !A || !B || !D)
+        return fail(ISOLOCO_ERR_INVALID, "bad debug_gemm_noalloc arguments");
+    const int a_rows = a_mn ? K : M, a_cols = a_mn ? M : K;
+    const int b_rows = b_mn ? K : N, b_cols = b_mn ? N : K;
+    const int lda = (int)round_up(a_cols, 8), ldb = (int)round_up(b_cols, 8);
+    const int64_t asz = (int64_t)batch * a_rows * lda, bsz = (int64_t)batch * b_rows * ldb;
+    const int64_t a_bytes = round_up(asz * 2, 256), b_bytes = round_up(bsz * 2, 256);
+    const int64_t need = kNoAllocPlanesOffset + 2 * a_bytes + 2 * b_bytes;
+    if (need > kNoAllocScratchBytes) {
+        char msg[200];
+        snprintf(msg, sizeof(msg),
+                 "debug_gemm_noalloc: these operands need %lld bytes of scratch; the static scratch holds %lld",
+                 (long long)need, (long long)kNoAllocScratchBytes);
+        return fail(ISOLOCO_ERR_INVALID, msg);
+    }
+    unsigned char* base = nullptr;
+    int rc = noalloc_scratch(&base);
+    if (rc != ISOLOCO_OK) return rc;
+    uint32_t* err = reinterpret_cast<uint32_t*>(base);
+    CUtensorMap* maps_d = reinterpret_cast<CUtensorMap*>(base + kNoAllocMapsOffset);
+    __nv_bfloat16* ah = reinterpret_cast<__nv_bfloat16*>(base + kNoAllocPlanesOffset);
+    __nv_bfloat16* al = reinterpret_cast<__nv_bfloat16*>(base + kNoAllocPlanesOffset + a_bytes);
+    __nv_bfloat16* bh = reinterpret_cast<__nv_bfloat16*>(base + kNoAllocPlanesOffset + 2 * a_bytes);
+    __nv_bfloat16* bl = reinterpret_cast<__nv_bfloat16*>(base + kNoAllocPlanesOffset + 2 * a_bytes + b_bytes);
+
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    CUtensorMap maps[4];
+    const int ra = a_mn ? kRoleMN : kRoleKA, rb = b_mn ? kRoleMN : kRoleKB;
+    if (!make_map(&maps[0], ah, a_cols, a_rows, batch, lda, ra) || !make_map(&maps[1], al, a_cols, a_rows, batch, lda, ra) ||
+        !make_map(&maps[2], bh, b_cols, b_rows, batch, ldb, rb) || !make_map(&maps[3], bl, b_cols, b_rows, batch, ldb, rb))
+        return fail(ISOLOCO_ERR_CUDA, "cuTensorMapEncodeTiled failed");
+    CUDA_TRY(cudaMemsetAsync(err, 0, 8, st));  // error word and tile counter
+    CUDA_TRY(cudaMemcpyAsync(maps_d, maps, sizeof(maps), cudaMemcpyHostToDevice, st));
+    const int f16 = precision > 0 ? 1 : 0;
+    k_split_planes<<<1024, 256, 0, st>>>(A, (int64_t)batch * a_rows * a_cols, a_rows, a_cols, lda, ah, al, f16);
+    k_split_planes<<<1024, 256, 0, st>>>(B, (int64_t)batch * b_rows * b_cols, b_rows, b_cols, ldb, bh, bl, f16);
+    CUDA_TRY(cudaGetLastError());
+    GemmParams gp;
+    memset(&gp, 0, sizeof(gp));
+    gp.epi = kEpiF32;
+    gp.gate = kGateNone;
+    gp.in_f16 = f16;
+    gp.a_split = (precision == 0 || precision == 1 || precision == 3) ? 1 : 0;
+    gp.b_split = (precision == 0 || precision == 2 || precision == 3) ? 1 : 0;
+    gp.err = err;
+    GemmGroup& g = gp.g[0];
+    g.a_hi = maps_d; g.a_lo = maps_d + 1; g.b_hi = maps_d + 2; g.b_lo = maps_d + 3;
+    set_group_common(g, M, N, K, batch, 1, 0);
+    g.cta_begin = 0;
+    g.out_f32 = D;
+    g.f32_batch_stride = (int64_t)M * N;
+    g.f32_split_stride = 0;
+    g.ld_f32 = N;
+    gp.num_groups = 1;
+    gp.total_tiles = batch * g.tiles_m * g.tiles_n;
+    gp.counter = reinterpret_cast<int*>(err) + 1;
+    int dev = 0, sms = 148;
+    CUDA_TRY(cudaGetDevice(&dev));
+    CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    CUDA_TRY(launch_gemm(gp, a_mn != 0, b_mn != 0, sms, st));
+    uint32_t herr = 0;
+    CUDA_TRY(cudaMemcpyAsync(&herr, err, 4, cudaMemcpyDeviceToHost, st));
+    CUDA_TRY(cudaStreamSynchronize(st));
+    if (herr & kErrTimeout) return fail(ISOLOCO_ERR_TIMEOUT, "debug_gemm_noalloc: device wait timed out");
     return ISOLOCO_OK;
 }
 

@@ -81,6 +81,7 @@ def lib():
             L.isoloco_plan_launches.restype = ctypes.c_int64
             L.isoloco_debug_gemm.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                              ctypes.c_int, ctypes.c_int, _vp, _vp, _vp, _vp]
+            L.isoloco_debug_gemm_noalloc.argtypes = L.isoloco_debug_gemm.argtypes
             _lib = L
     return _lib
 
@@ -246,3 +247,14 @@ def debug_gemm(A: torch.Tensor, B: torch.Tensor, a_mn_major: bool, b_mn_major: b
                                   B.data_ptr(), D.data_ptr(), _stream(stream))
     _check(rc, "isoloco_debug_gemm", hard_only=False)
     return D
+
+
+def debug_gemm_noalloc(A: torch.Tensor, B: torch.Tensor, D: torch.Tensor, a_mn_major: bool, b_mn_major: bool,
+                       M: int, N: int, K: int, precision: int = 0, stream=None) -> int:
+    """The same GEMM as debug_gemm into the caller's D, with the library's static scratch
+    (no device allocation; see isoloco_debug_gemm_noalloc in include/isoloco.h)."""
+    if D.dtype != torch.float32 or D.numel() < A.shape[0] * M * N:
+        raise ValueError("D must be fp32 with room for batch x M x N")
+    rc = lib().isoloco_debug_gemm_noalloc(int(a_mn_major), int(b_mn_major), int(precision), A.shape[0], M, N, K,
+                                          A.data_ptr(), B.data_ptr(), D.data_ptr(), _stream(stream))
+    return _check(rc, "isoloco_debug_gemm_noalloc", hard_only=False)
