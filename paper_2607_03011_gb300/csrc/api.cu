@@ -177,7 +177,7 @@ static bool make_map(CUtensorMap* m, const void* base, int cols, int rows, int c
     } else if (role == kRoleST) {
         box[0] = 32; box[1] = 32; sw = CU_TENSOR_MAP_SWIZZLE_64B;
     } else {
-        box[0] = BK; box[1] = (role == kRoleKA) ? BM : BN;
+        box[0] = BK; box[1] = (role == kRoleKA) ? BM : kBRows;
         sw = (BK * 2 == 128) ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
     }
     box[2] = 1;
@@ -192,7 +192,7 @@ static inline int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * 
 
 // Output tiles of an n x n symmetric product that touch the upper triangle.
 static int sym_tiles(int n) {
-    const int tm_n = (n + BM - 1) / BM, tn_n = (n + BN - 1) / BN;
+    const int tm_n = (n + kTileM - 1) / kTileM, tn_n = (n + BN - 1) / BN;
     int c = 0;
     for (int tm = 0; tm < tm_n; ++tm) c += tn_n - sym_first_tile_n(tm);
     return c;
@@ -313,7 +313,8 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         const int kblocks = (kdim + BK - 1) / BK;
         // split-K for long reductions: at most 256 k-blocks per split, and more splits
         // (down to 32 k-blocks each) only while the bucket alone would not fill the GPU
-        const int slots = 2 * p->num_sms;
+        // (two output tiles per SM, or per pair of SMs with pair MMAs)
+        const int slots = 2 * p->num_sms / (kPairMma ? 2 : 1);
         int splits = std::max(1, (kblocks + 255) / 256);
         if (tiles * splits < slots) splits = std::max(splits, std::min(slots / std::max(1, tiles), kblocks / 32));
         int kper = (kblocks + splits - 1) / splits;
@@ -400,7 +401,7 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         (rc = dalloc(p, &p->xlo[1], plane)) ||
         (rc = dalloc(p, &p->ghi, gplane)) || (rc = dalloc(p, &p->glo, gplane)) || (rc = dalloc(p, &p->phi, gplane)) ||
         (rc = dalloc(p, &p->plo, gplane)) || (rc = dalloc(p, &p->ypl, gplane)) || (rc = dalloc(p, &p->gpart, gpart)) || (rc = dalloc(p, &p->d1d, d1)) ||
-        (rc = dalloc(p, &p->fin_part, 3 * kEpiWarps * fin)) || (rc = dalloc(p, &p->ftiles, (int64_t)ftiles.size())) ||
+        (rc = dalloc(p, &p->fin_part, 3 * kPartSlots * fin)) || (rc = dalloc(p, &p->ftiles, (int64_t)ftiles.size())) ||
         (rc = dalloc(p, &p->tpart, tr)) || (rc = dalloc(p, &p->tchunks, tr)) ||
         (rc = dalloc(p, &p->state, p->nmat)) || (rc = dalloc(p, &p->mats_d, p->nmat)) ||
         (rc = dalloc(p, &p->gpart_off_d, p->nmat)) || (rc = dalloc(p, &p->gpart_sstride_d, p->nmat)) ||
@@ -495,7 +496,7 @@ static void set_group_common(GemmGroup& g, int M, int N, int K, int batch, int s
     g.N = N;
     g.K = K;
     g.batch = batch;
-    g.tiles_m = (M + BM - 1) / BM;
+    g.tiles_m = (M + kTileM - 1) / kTileM;
     g.tiles_n = (N + BN - 1) / BN;
     const int kblocks = (K + BK - 1) / BK;
     g.kblocks_per_split = (kblocks + splits - 1) / splits;

@@ -87,8 +87,10 @@ __device__ __forceinline__ void active_prefix(const GemmParams& p, int* pre) {
     }
 }
 
-// Decodes active tile t.  Returns false when the matrix does no work in this launch.
-__device__ __forceinline__ bool decode_tile(const GemmParams& p, const int* pre, int t, TileInfo& ti) {
+// Decodes active tile t for the CTA of rank `crank` in its pair (0 without pairs).
+// Returns false when the matrix does no work in this launch.
+__device__ __forceinline__ bool decode_tile(const GemmParams& p, const int* pre, int t, uint32_t crank,
+                                            TileInfo& ti) {
     int gi = 0;
     while (gi + 1 < p.num_groups && t >= pre[gi + 1]) ++gi;
     const GemmGroup& g = p.g[gi];
@@ -108,7 +110,7 @@ __device__ __forceinline__ bool decode_tile(const GemmParams& p, const int* pre,
         tm = ti.tile / g.tiles_n;
         tn = ti.tile % g.tiles_n;
     }
-    ti.m0 = tm * BM;
+    ti.m0 = tm * kTileM + static_cast<int>(crank) * BM;  // this CTA's rows of the tile
     ti.n0 = tn * BN;
     ti.mat = g.mat_base + ti.b;
     ti.run_mma = true;
@@ -198,7 +200,7 @@ __device__ __forceinline__ void stage_store_block(const uint32_t (&w)[16], const
 // diagonal block is made symmetric in shared memory (its upper half mirrored) before its
 // single store, so every entry is written once and the matrix is bitwise symmetric.
 __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInfo& ti, uint32_t tacc, bool ok,
-                                              int eg, int half, int lane, uint8_t* stg) {
+                                              int eg, int half, int lane, uint32_t crank, uint8_t* stg) {
     const GemmGroup& g = p.g[ti.gi];
     const int b = ti.b, m0 = ti.m0, n0 = ti.n0, split = ti.split;
     const float ca = ti.ca, cb = ti.cb, cc = ti.cc, xs = ti.xs;
@@ -339,8 +341,8 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
         }
         if (lane == 0) {
             const int ntiles = sym ? g.tiles_sym : g.tiles_m * g.tiles_n;
-            float* slot = g.part + ((g.part_base + static_cast<int64_t>(b) * ntiles + ti.tile) * kEpiWarps +
-                                    half * 4 + eg) * 3;
+            float* slot = g.part + ((g.part_base + static_cast<int64_t>(b) * ntiles + ti.tile) * kPartSlots +
+                                    static_cast<int>(crank) * kEpiWarps + half * 4 + eg) * 3;
             slot[0] = s_sq;
             slot[1] = s_tr;
             slot[2] = s_dev;
@@ -348,10 +350,16 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
     }
 }
 
-// Persistent kernel: CTA c processes tiles c, c + gridDim.x, ... of the launch.  The TMA
-// ring runs continuously across tile boundaries, and the accumulator is double
-// buffered in tensor memory (2 x 256 columns): the epilogue of one tile overlaps the
-// MMAs of the next.
+// Persistent kernel.  Without pairs, CTA c starts with tile c and claims further tiles
+// from the launch's counter.  With kPairMma the grid is made of clusters of two CTAs
+// (ranks 0 and 1, on neighbouring SMs); cluster c processes tiles c, c + clusters, ...
+// and both CTAs walk that sequence together: each loads its rows of A and its half of B,
+// the TMA bytes of both complete on rank 0's `full` barrier, rank 0 alone issues the
+// cta_group::2 MMAs, whose commits arrive on the `empty` / `tfull` barriers of both CTAs,
+// and each CTA's epilogue drains its own half of the accumulator and reports to rank 0's
+// `tempty`.  The TMA ring runs continuously across tile boundaries, and the accumulator
+// is double buffered in tensor memory (2 x 256 columns): the epilogue of one tile
+// overlaps the MMAs of the next.
 template <bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_constant__ GemmParams p) {
     extern __shared__ uint8_t smem_raw[];
@@ -371,6 +379,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
+    const uint32_t crank = kPairMma ? cluster_ctarank() : 0u;  // rank in the CTA pair
+    const bool leader = crank == 0;                              // issues the MMAs
     // ring geometry of this launch: room for the planes its tiles can load
     const uint32_t stage_stride = kTileABytes * (p.a_split || p.split_on_polish ? 2u : 1u) +
                                   kTileBBytes * (p.b_split || p.split_on_polish ? 2u : 1u);
@@ -383,7 +393,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&tfull[i], 1);
-            mbar_init(&tempty[i], kEpiWarps);  // one arrival per epilogue warp
+            mbar_init(&tempty[i], kEpiWarps * (kPairMma ? 2 : 1));  // one arrival per epilogue warp of the pair
         }
         mbar_init(drain, 1);
         for (int q = 0; q < kTileQueue; ++q) {
@@ -395,11 +405,17 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
         fence_mbar_init();
     }
     if (warp == 1) {
-        tmem_alloc(tmem_slot, 2 * kTmemCols);
-        tmem_relinquish();
+        if (kPairMma) {
+            tmem_alloc_pair(tmem_slot, 2 * kTmemCols);
+            tmem_relinquish_pair();
+        } else {
+            tmem_alloc(tmem_slot, 2 * kTmemCols);
+            tmem_relinquish();
+        }
     }
     tc_fence_before();
     __syncthreads();
+    if (kPairMma) cluster_sync();  // both CTAs' barriers exist before either signals the other's
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
 
@@ -413,7 +429,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
             const int T = pre[p.num_groups];
             int q = 0;
             uint32_t qphase = 0;
-            int t = blockIdx.x;
+            // first tile; without pairs later ones come from the launch's counter, with pairs
+            // cluster c takes tiles c, c + clusters, ... (both CTAs of the pair agree)
+            const int tile_stride = kPairMma ? static_cast<int>(gridDim.x >> 1) : 0;
+            int t = kPairMma ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
             for (;;) {
                 // publish the next tile (or -1: no more) to the MMA and epilogue warps
                 const int tile = (t < T && !*abort_flag) ? t : -1;
@@ -429,9 +448,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                     qphase ^= 1u;
                 }
                 if (tile < 0) break;
-                t = atomicAdd(p.counter, 1) + static_cast<int>(gridDim.x);  // claimed early
+                if (kPairMma)
+                    t += tile_stride;
+                else
+                    t = atomicAdd(p.counter, 1) + static_cast<int>(gridDim.x);  // claimed early
                 TileInfo ti;
-                if (!decode_tile(p, pre, tile, ti) || !ti.run_mma) continue;
+                if (!decode_tile(p, pre, tile, crank, ti) || !ti.run_mma) continue;
                 const GemmGroup& g = p.g[ti.gi];
                 if (prefetched != ti.gi) {
                     tma_prefetch_desc(g.a_hi);
@@ -442,6 +464,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                 }
                 const uint32_t stage_bytes =
                     kTileABytes * (ti.a_split ? 2u : 1u) + kTileBBytes * (ti.b_split ? 2u : 1u);
+                const int nb0 = ti.n0 + static_cast<int>(crank) * kBRows;  // this CTA's rows of B
                 for (int kb = ti.kb_begin; kb < ti.kb_end; ++kb) {
                     if (!mbar_wait(&empty[stage], phase ^ 1u)) {
                         *abort_flag = 1;
@@ -452,29 +475,35 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                     uint8_t* sa_lo = sa_hi + kTileABytes;
                     uint8_t* sb_hi = sa_hi + kTileABytes * (ti.a_split ? 2u : 1u);
                     uint8_t* sb_lo = sb_hi + kTileBBytes;
-                    mbar_arrive_expect_tx(&full[stage], stage_bytes);
+                    // rank 0's barrier expects the bytes of both CTAs of the pair
+                    if (leader) mbar_arrive_expect_tx(&full[stage], stage_bytes * (kPairMma ? 2u : 1u));
+                    const uint32_t fbar = kPairMma ? mapa_shared(smem_u32(&full[stage]), 0) : 0u;
+                    auto load = [&](uint8_t* dst, const CUtensorMap* map, int c0, int c1) {
+                        if (kPairMma)
+                            tma_load_3d_pair(dst, map, fbar, c0, c1, ti.b);
+                        else
+                            tma_load_3d(dst, map, &full[stage], c0, c1, ti.b);
+                    };
                     const int k0 = kb * BK;
                     if (A_MN) {
 #pragma unroll
                         for (int c = 0; c < BM / 64; ++c) {
-                            tma_load_3d(sa_hi + c * (BK * 128), g.a_hi, &full[stage], ti.m0 + 64 * c, k0, ti.b);
-                            if (ti.a_split)
-                                tma_load_3d(sa_lo + c * (BK * 128), g.a_lo, &full[stage], ti.m0 + 64 * c, k0, ti.b);
+                            load(sa_hi + c * (BK * 128), g.a_hi, ti.m0 + 64 * c, k0);
+                            if (ti.a_split) load(sa_lo + c * (BK * 128), g.a_lo, ti.m0 + 64 * c, k0);
                         }
                     } else {
-                        tma_load_3d(sa_hi, g.a_hi, &full[stage], k0, ti.m0, ti.b);
-                        if (ti.a_split) tma_load_3d(sa_lo, g.a_lo, &full[stage], k0, ti.m0, ti.b);
+                        load(sa_hi, g.a_hi, k0, ti.m0);
+                        if (ti.a_split) load(sa_lo, g.a_lo, k0, ti.m0);
                     }
                     if (B_MN) {
 #pragma unroll
-                        for (int c = 0; c < BN / 64; ++c) {
-                            tma_load_3d(sb_hi + c * (BK * 128), g.b_hi, &full[stage], ti.n0 + 64 * c, k0, ti.b);
-                            if (ti.b_split)
-                                tma_load_3d(sb_lo + c * (BK * 128), g.b_lo, &full[stage], ti.n0 + 64 * c, k0, ti.b);
+                        for (int c = 0; c < kBRows / 64; ++c) {
+                            load(sb_hi + c * (BK * 128), g.b_hi, nb0 + 64 * c, k0);
+                            if (ti.b_split) load(sb_lo + c * (BK * 128), g.b_lo, nb0 + 64 * c, k0);
                         }
                     } else {
-                        tma_load_3d(sb_hi, g.b_hi, &full[stage], k0, ti.n0, ti.b);
-                        if (ti.b_split) tma_load_3d(sb_lo, g.b_lo, &full[stage], k0, ti.n0, ti.b);
+                        load(sb_hi, g.b_hi, k0, nb0);
+                        if (ti.b_split) load(sb_lo, g.b_lo, k0, nb0);
                     }
                     issued_mask |= 1u << stage;
                     issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
@@ -485,15 +514,41 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                 }
             }
             if (*abort_flag) {
-                // Let the copies already in flight land before the CTA exits.
-                for (int s = 0; s < nstages; ++s)
-                    if (issued_mask & (1u << s)) (void)mbar_wait(&full[s], (issued_parity >> s) & 1u);
+                // Let the copies already in flight land before the CTA exits (rank 0's
+                // barriers also count rank 1's copies; rank 1 cannot observe its own, so it
+                // leaves them a generous margin).
+                if (leader) {
+                    for (int s = 0; s < nstages; ++s)
+                        if (issued_mask & (1u << s)) (void)mbar_wait(&full[s], (issued_parity >> s) & 1u);
+                } else {
+                    const uint64_t t0 = globaltimer_ns();
+                    while (globaltimer_ns() - t0 < 100000ull) {
+                    }
+                }
             }
         }
     } else if (warp == 1) {
-        // ================= MMA issuer (one thread)
-        if (lane == 0) {
-            const uint32_t idesc = make_idesc_16bit(BM, BN, A_MN, B_MN, p.in_f16 != 0);
+        // ================= MMA issuer (one thread; with pairs only in rank 0)
+        if (lane == 0 && kPairMma && !leader) {
+            // rank 1 issues no MMAs; it only keeps its tile queue moving
+            int q = 0;
+            uint32_t qphase = 0;
+            for (;;) {
+                if (!mbar_wait(&tq_full[q], qphase)) {
+                    *abort_flag = 1;
+                    atomicOr(p.err, kErrTimeout);
+                    break;
+                }
+                const int tile = tq_tile[q];
+                mbar_arrive(&tq_empty[q]);
+                if (++q == kTileQueue) {
+                    q = 0;
+                    qphase ^= 1u;
+                }
+                if (tile < 0) break;
+            }
+        } else if (lane == 0) {
+            const uint32_t idesc = make_idesc_16bit(kTileM, BN, A_MN, B_MN, p.in_f16 != 0);
             const uint64_t desc_a0 = operand_desc<A_MN>(smem_u32(smem), 0);
             const uint64_t desc_b0 = operand_desc<B_MN>(smem_u32(smem), 0);
             // start-address step of one 16-deep K slice: 2048 bytes MN-major, 32 bytes K-major
@@ -518,7 +573,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                 }
                 if (tile < 0 || *abort_flag) break;
                 TileInfo ti;
-                if (!decode_tile(p, pre, tile, ti)) continue;
+                if (!decode_tile(p, pre, tile, crank, ti)) continue;
                 const uint32_t buf = n & 1u, use = n >> 1;
                 ++n;
                 if (!mbar_wait(&tempty[buf], (use & 1u) ^ 1u)) {
@@ -549,21 +604,38 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
 #pragma unroll
                         for (int ks = 0; ks < BK / 16; ++ks) {
                             const uint64_t da = so + ks * kDescStepA, db = so + ks * kDescStepB;
-                            umma_16bit(tacc, a_hi0 + da, b_hi0 + db, idesc, acc);
+                            if (kPairMma) {
+                                umma_16bit_pair(tacc, a_hi0 + da, b_hi0 + db, idesc, acc);
+                                if (bs) umma_16bit_pair(tacc, a_hi0 + da, b_lo0 + db, idesc, 1u);
+                                if (as) umma_16bit_pair(tacc, a_lo0 + da, b_hi0 + db, idesc, 1u);
+                            } else {
+                                umma_16bit(tacc, a_hi0 + da, b_hi0 + db, idesc, acc);
+                                if (bs) umma_16bit(tacc, a_hi0 + da, b_lo0 + db, idesc, 1u);
+                                if (as) umma_16bit(tacc, a_lo0 + da, b_hi0 + db, idesc, 1u);
+                            }
                             acc = 1u;
-                            if (bs) umma_16bit(tacc, a_hi0 + da, b_lo0 + db, idesc, 1u);
-                            if (as) umma_16bit(tacc, a_lo0 + da, b_hi0 + db, idesc, 1u);
                         }
-                        umma_commit(&empty[stage]);
+                        // the stage is free in both CTAs once these MMAs have read it
+                        if (kPairMma)
+                            umma_commit_pair_mc(&empty[stage], 0x3);
+                        else
+                            umma_commit(&empty[stage]);
                         if (++stage == nstages) {
                             stage = 0;
                             phase ^= 1u;
                         }
                     }
                 }
-                umma_commit(&tfull[buf]);  // completes once every MMA of this tile has finished
+                // completes once every MMA of this tile has finished (in both CTAs' barriers)
+                if (kPairMma)
+                    umma_commit_pair_mc(&tfull[buf], 0x3);
+                else
+                    umma_commit(&tfull[buf]);
             }
-            umma_commit(drain);
+            if (kPairMma)
+                umma_commit_pair(drain);
+            else
+                umma_commit(drain);
             (void)mbar_wait(drain, 0);
         }
     } else {
@@ -596,7 +668,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
             }
             if (tile < 0) break;
             TileInfo ti;
-            if (!decode_tile(p, pre, tile, ti)) continue;
+            if (!decode_tile(p, pre, tile, crank, ti)) continue;
             const uint32_t buf = n & 1u, use = n >> 1;
             ++n;
             const bool ok = __all_sync(0xffffffffu, mbar_wait(&tfull[buf], use & 1u));
@@ -606,49 +678,96 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
             }
             __syncwarp();
             tc_fence_after();
-            tile_epilogue(p, ti, tmem_base + buf * kTmemCols, ok, eg, half, lane,
+            tile_epilogue(p, ti, tmem_base + buf * kTmemCols, ok, eg, half, lane, crank,
                           staging + (warp - 2) * 2 * kStageBlockBytes);
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&tempty[buf]);
+            if (lane == 0) {
+                if (leader)
+                    mbar_arrive(&tempty[buf]);
+                else
+                    mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[buf]), 0));  // rank 0 issues the MMAs
+            }
         }
         if (lane == 0) bulk_wait0();  // this warp's TMA stores have completed
         __syncwarp();
     }
 
-    // ---- teardown: the MMA thread has waited for all its MMAs (drain barrier)
+    // ---- teardown: the MMA thread has waited for all its MMAs (drain barrier); with
+    // pairs neither CTA leaves (or frees tensor memory) while rank 0's MMAs could still
+    // read rank 1's shared memory or write its tensor memory
     tc_fence_before();
     __syncthreads();
+    if (kPairMma) cluster_sync();
     if (warp == 1) {
         __syncwarp();
         tc_fence_after();
-        tmem_dealloc(tmem_base, 2 * kTmemCols);
+        if (kPairMma)
+            tmem_dealloc_pair(tmem_base, 2 * kTmemCols);
+        else
+            tmem_dealloc(tmem_base, 2 * kTmemCols);
     }
 }
 
 // ------------------------------------------------------------------ host launcher
 template <bool A_MN, bool B_MN>
-static cudaError_t launch_gemm_t(const GemmParams& p, int grid, cudaStream_t stream) {
+static cudaError_t launch_gemm_t(const GemmParams& p, int max_ctas, cudaStream_t stream) {
+    static int max_clusters = 0;  // clusters of two that can be resident at once
     static bool attr_set = false;
     if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(k_gemm_split<A_MN, B_MN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              kGemmSmemBytes);
         if (e != cudaSuccess) return e;
+        if (kPairMma) {
+            cudaLaunchConfig_t cfg = {};
+            cudaLaunchAttribute at[1];
+            at[0].id = cudaLaunchAttributeClusterDimension;
+            at[0].val.clusterDim.x = 2;
+            at[0].val.clusterDim.y = 1;
+            at[0].val.clusterDim.z = 1;
+            cfg.gridDim = dim3(static_cast<unsigned>(max_ctas & ~1));
+            cfg.blockDim = dim3(kGemmThreads);
+            cfg.dynamicSmemBytes = kGemmSmemBytes;
+            cfg.attrs = at;
+            cfg.numAttrs = 1;
+            int n = 0;
+            e = cudaOccupancyMaxActiveClusters(&n, k_gemm_split<A_MN, B_MN>, &cfg);
+            if (e != cudaSuccess) return e;
+            max_clusters = n > 0 ? n : 1;
+        }
         attr_set = true;
     }
-    k_gemm_split<A_MN, B_MN><<<grid, kGemmThreads, kGemmSmemBytes, stream>>>(p);
-    return cudaGetLastError();
+    if (!kPairMma) {
+        const int grid = p.total_tiles < max_ctas ? p.total_tiles : max_ctas;
+        k_gemm_split<A_MN, B_MN><<<grid, kGemmThreads, kGemmSmemBytes, stream>>>(p);
+        return cudaGetLastError();
+    }
+    int clusters = p.total_tiles;
+    clusters = clusters < max_clusters ? clusters : max_clusters;
+    clusters = clusters < max_ctas / 2 ? clusters : (max_ctas / 2 > 0 ? max_ctas / 2 : 1);
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 2;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3(static_cast<unsigned>(2 * clusters));
+    cfg.blockDim = dim3(kGemmThreads);
+    cfg.dynamicSmemBytes = kGemmSmemBytes;
+    cfg.stream = stream;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k_gemm_split<A_MN, B_MN>, p);
 }
 
-// Launches one persistent GEMM over the groups of `p` (p.total_tiles tiles) on at most
-// `max_ctas` CTAs (one per SM).
+// Launches one persistent GEMM over the groups of `p` (p.total_tiles output tiles) on at
+// most `max_ctas` CTAs (one per SM; with kPairMma, clusters of two CTAs per tile).
 cudaError_t launch_gemm(const GemmParams& p, bool a_mn, bool b_mn, int max_ctas, cudaStream_t stream) {
     if (p.total_tiles <= 0) return cudaSuccess;
-    const int grid = p.total_tiles < max_ctas ? p.total_tiles : max_ctas;
-    if (!a_mn && !b_mn) return launch_gemm_t<false, false>(p, grid, stream);
-    if (a_mn && b_mn) return launch_gemm_t<true, true>(p, grid, stream);
-    if (!a_mn && b_mn) return launch_gemm_t<false, true>(p, grid, stream);
-    return launch_gemm_t<true, false>(p, grid, stream);
+    if (!a_mn && !b_mn) return launch_gemm_t<false, false>(p, max_ctas, stream);
+    if (a_mn && b_mn) return launch_gemm_t<true, true>(p, max_ctas, stream);
+    if (!a_mn && b_mn) return launch_gemm_t<false, true>(p, max_ctas, stream);
+    return launch_gemm_t<true, false>(p, max_ctas, stream);
 }
 
 }  // namespace isoloco

@@ -96,9 +96,9 @@ __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict
     if (threadIdx.x < 3) {
         float s = 0.f;
         for (int i = 0; i < (int)(blockDim.x >> 5); ++i) s += red[threadIdx.x][i];
-        float* slot = fin_part + (md.gpart_slot + ft.y) * kEpiWarps * 3;  // kEpiWarps slots of 3 per tile
+        float* slot = fin_part + (md.gpart_slot + ft.y) * kPartSlots * 3;  // kPartSlots slots of 3 per tile
         slot[threadIdx.x] = s;
-        for (int w = 1; w < kEpiWarps; ++w) slot[3 * w + threadIdx.x] = 0.f;
+        for (int w = 1; w < kPartSlots; ++w) slot[3 * w + threadIdx.x] = 0.f;
     }
 }
 
@@ -116,8 +116,8 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
     // non-negative terms (relative error ~1e-6, far below the tolerance this sum is
     // tested against), and fp32 keeps one SM off GB300's narrow fp64 pipe.
     float sqf = 0.f, trf = 0.f, devf = 0.f;
-    for (int i = lane; i < kEpiWarps * md.n_gtiles; i += 32) {  // kEpiWarps partial slots per Gram tile
-        const float* pp = fin_part + (md.gpart_slot * kEpiWarps + i) * 3;
+    for (int i = lane; i < kPartSlots * md.n_gtiles; i += 32) {  // kPartSlots partial slots per Gram tile
+        const float* pp = fin_part + (md.gpart_slot * kPartSlots + i) * 3;
         sqf += pp[0];
         trf += pp[1];
         devf += pp[2];

@@ -8,19 +8,27 @@
 namespace isoloco {
 
 // ------------------------------------------------------------------ GEMM tiles
-// One CTA computes a BM x BN fp32 tile in tensor memory from bf16 hi/lo operand
-// planes staged BK deep per pipeline stage.
+// One CTA holds a BM x BN fp32 tile in tensor memory, computed from 16-bit hi/lo
+// operand planes staged BK deep per pipeline stage.  With kPairMma a pair of CTAs on
+// neighbouring SMs (a cluster of two) computes one kTileM x BN = 256 x 256 output tile
+// with tcgen05 cta_group::2: each CTA stages its own BM rows of A and half of B's BN
+// rows, so one SM's shared memory supplies 8 KB instead of 12 KB per 16-deep MMA step
+// (the single-SM M128 x N256 tile is bound by shared-memory bandwidth, not the tensor pipe).
+constexpr bool kPairMma = true;
 constexpr int BM = 128;
 constexpr int BN = 256;
 constexpr int BK = 32;
+constexpr int kTileM = kPairMma ? 2 * BM : BM;  // rows of one output tile
+constexpr int kBRows = kPairMma ? BN / 2 : BN;  // rows of B (N extent) staged by one CTA
 // Shared-memory ring of the persistent GEMM (one CTA per SM): as many stages of the
-// launch's plane set as fit in kRingBytes (4 of 48 KB for three passes, 6 of 32 KB for two).
-constexpr int kMaxStages = 8;
-constexpr int kRingBytes = 4 * (2 * BM * BK * 2 + 2 * BN * BK * 2);
+// launch's plane set as fit in kRingBytes, at most kMaxStages.
+constexpr int kMaxStages = 12;
+constexpr int kRingBytes = 192 * 1024;
 constexpr int kTileABytes = BM * BK * 2;                       // one bf16 plane of A
-constexpr int kTileBBytes = BN * BK * 2;                       // one bf16 plane of B
+constexpr int kTileBBytes = kBRows * BK * 2;                   // one bf16 plane of this CTA's B
 
 constexpr int kEpiWarps = 8;       // two warps per tensor-memory lane quarter
+constexpr int kPartSlots = kEpiWarps * (kPairMma ? 2 : 1);  // Gram partial sums per output tile
 constexpr int kGemmThreads = 64 + 32 * kEpiWarps;  // warp 0 TMA, warp 1 MMA, warps 2.. epilogue
 constexpr int kTmemCols = 256;     // one accumulator; the kernel double-buffers (512 columns)
 constexpr int kMaxGroups = 8;
@@ -52,7 +60,7 @@ enum GateMode : int {
 
 // First tile column of tile row tm that touches the upper triangle of a square output.
 __host__ __device__ constexpr int sym_first_tile_n(int tm) {
-    return (tm * BM - BN + 1) <= 0 ? 0 : (tm * BM - BN + 1 + BN - 1) / BN;
+    return (tm * kTileM - BN + 1) <= 0 ? 0 : (tm * kTileM - BN + 1 + BN - 1) / BN;
 }
 
 struct GemmGroup {
