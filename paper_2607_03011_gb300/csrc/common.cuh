@@ -109,6 +109,15 @@ __device__ __forceinline__ void bulk_wait_read0() {
     asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
 
+// Same, allowing the most recent 1 (or 3) bulk groups to still be reading.
+__device__ __forceinline__ void bulk_wait_read1() {
+    asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
+
+__device__ __forceinline__ void bulk_wait_read3() {
+    asm volatile("cp.async.bulk.wait_group.read 3;" ::: "memory");
+}
+
 // Waits until the bulk stores of this thread have completed.
 __device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
@@ -306,6 +315,34 @@ __device__ __forceinline__ void split16(float x, bool f16, uint16_t& hi, uint16_
         hi = __bfloat16_as_ushort(h);
         lo = __bfloat16_as_ushort(__float2bfloat16_rn(x - __bfloat162float(h)));
     }
+}
+
+// Two values at once (packed conversions; the same roundings as split16): hi / lo words
+// with a's bits in the low half.
+__device__ __forceinline__ void split16x2(float a, float b, bool f16, uint32_t& hi, uint32_t& lo) {
+    if (f16) {
+        const __half2 h = __floats2half2_rn(a, b);
+        const float2 hf = __half22float2(h);
+        const __half2 l = __floats2half2_rn(a - hf.x, b - hf.y);
+        hi = *reinterpret_cast<const uint32_t*>(&h);
+        lo = *reinterpret_cast<const uint32_t*>(&l);
+    } else {
+        const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+        const float2 hf = __bfloat1622float2(h);
+        const __nv_bfloat162 l = __floats2bfloat162_rn(a - hf.x, b - hf.y);
+        hi = *reinterpret_cast<const uint32_t*>(&h);
+        lo = *reinterpret_cast<const uint32_t*>(&l);
+    }
+}
+
+// Round-to-nearest 16-bit pair (a in the low half).
+__device__ __forceinline__ uint32_t round16x2(float a, float b, bool f16) {
+    if (f16) {
+        const __half2 h = __floats2half2_rn(a, b);
+        return *reinterpret_cast<const uint32_t*>(&h);
+    }
+    const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<const uint32_t*>(&h);
 }
 
 __device__ __forceinline__ float dec16(uint32_t bits, bool f16) {

@@ -155,13 +155,26 @@ __device__ __forceinline__ uint32_t stg_off(int r, int c) {
 }
 
 // One warp writes a 32 x 32 block of 16-bit values (lane = row, w = the lane's 32 values
-// packed in pairs) to its staging block(s) and stores it with TMA at (col0, row_base, b):
-// the diagonal block is symmetrised in shared memory; an off-diagonal block of a symmetric
-// output is also stored transposed at (row_base, col0, b).
-__device__ __forceinline__ void stage_store_block(const uint32_t (&w)[16], const CUtensorMap* map, uint8_t* sd,
-                                                  uint8_t* sm, bool diag, bool sym, int lane, int col0,
+// packed in pairs) to staging and stores it with TMA at (col0, row_base, b): the diagonal
+// block is symmetrised in shared memory; an off-diagonal block of a symmetric output is
+// also stored transposed at (row_base, col0, b).  `stg` holds the warp's kStageBlocks
+// blocks and `seq` counts its stores (one bulk group each): a symmetric store takes the
+// pair (seq & 1) once the store before the previous one has read it, any other store the
+// block (seq & 3) once the store four back has.
+__device__ __forceinline__ void stage_store_block(const uint32_t (&w)[16], const CUtensorMap* map, uint8_t* stg,
+                                                  uint32_t& seq, bool diag, bool sym, int lane, int col0,
                                                   int row_base, int b) {
-    if (lane == 0) bulk_wait_read0();  // the staging blocks are free again
+    static_assert(kStageBlocks == 4, "block rotation below assumes four staging blocks per warp");
+    uint8_t* sd;
+    if (sym) {
+        sd = stg + (seq & 1u) * 2u * kStageBlockBytes;
+        if (lane == 0) bulk_wait_read1();
+    } else {
+        sd = stg + (seq & 3u) * kStageBlockBytes;
+        if (lane == 0) bulk_wait_read3();
+    }
+    uint8_t* sm = sd + kStageBlockBytes;  // transposed block (symmetric outputs only)
+    ++seq;
     __syncwarp();
     if (diag) {
 #pragma unroll
@@ -176,10 +189,15 @@ __device__ __forceinline__ void stage_store_block(const uint32_t (&w)[16], const
             *reinterpret_cast<uint4*>(sd + lane * 64 + ((((q ^ (lane >> 1)) & 3)) << 4)) =
                 make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
         if (sym) {
+            // transposed block T(r, c) = value of lane c at column r: for rows 2i and 2i + 1,
+            // even lanes c form (own, partner) column 2i and odd lanes (partner, own) column
+            // 2i + 1 from the packed pair w[i] and the partner lane's, one 32-bit store each
+            const uint32_t sel = (lane & 1) ? 0x3276u : 0x5410u;
+            const int r_odd = lane & 1, c_even = lane & ~1;
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
-                const uint16_t x = static_cast<uint16_t>((j & 1) ? (w[j >> 1] >> 16) : (w[j >> 1] & 0xFFFFu));
-                *reinterpret_cast<uint16_t*>(sm + stg_off(j, lane)) = x;
+            for (int i = 0; i < 16; ++i) {
+                const uint32_t other = __shfl_xor_sync(0xffffffffu, w[i], 1);
+                *reinterpret_cast<uint32_t*>(sm + stg_off(2 * i + r_odd, c_even)) = __byte_perm(w[i], other, sel);
             }
         }
     }
@@ -200,7 +218,8 @@ __device__ __forceinline__ void stage_store_block(const uint32_t (&w)[16], const
 // diagonal block is made symmetric in shared memory (its upper half mirrored) before its
 // single store, so every entry is written once and the matrix is bitwise symmetric.
 __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInfo& ti, uint32_t tacc, bool ok,
-                                              int eg, int half, int lane, uint32_t crank, uint8_t* stg) {
+                                              int eg, int half, int lane, uint32_t crank, uint8_t* stg,
+                                              uint32_t& sseq) {
     const GemmGroup& g = p.g[ti.gi];
     const int b = ti.b, m0 = ti.m0, n0 = ti.n0, split = ti.split;
     const float ca = ti.ca, cb = ti.cb, cc = ti.cc, xs = ti.xs;
@@ -215,8 +234,6 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
     // and for the Gram with p.gram_y the plane Y = yb I + yc G (hi only)
     const bool write_y = (p.epi == kEpiGram && p.gram_y);
     const int nplanes = (ti.horner || g.st_lo == nullptr) ? 1 : 2;
-    uint8_t* sd = stg;                      // direct block
-    uint8_t* sm = stg + kStageBlockBytes;   // transposed (mirror) block
     float s_sq = 0.f, s_tr = 0.f, s_dev = 0.f;
     for (int c32 = half * (BN / 64); c32 < (half + 1) * (BN / 64); ++c32) {
         const int col0 = n0 + c32 * 32;
@@ -274,7 +291,14 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
 #pragma unroll
             for (int j = 0; j < 32; ++j) v[j] *= xs;
         }
-        if (gram_fused && row_ok) {
+        if (gram_fused && row_ok && sym && !diag && nvalid == 32) {
+            // block strictly above the diagonal: every entry counts twice and (G - I) = G
+            float ss = 0.f;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) ss = fmaf(v[j], v[j], ss);
+            s_sq = fmaf(2.f, ss, s_sq);
+            s_dev = fmaf(2.f, ss, s_dev);
+        } else if (gram_fused && row_ok) {
 #pragma unroll
             for (int j = 0; j < 32; ++j) {
                 if (j < nvalid && (!sym || j >= d)) {
@@ -310,25 +334,21 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
         // ---- 16-bit planes through shared memory and TMA stores
         uint32_t hw[16], lw[16];
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            uint16_t h0, l0, h1, l1;
-            split16(v[2 * j], of16, h0, l0);
-            split16(v[2 * j + 1], of16, h1, l1);
-            hw[j] = static_cast<uint32_t>(h0) | (static_cast<uint32_t>(h1) << 16);
-            lw[j] = static_cast<uint32_t>(l0) | (static_cast<uint32_t>(l1) << 16);
-        }
-        stage_store_block(hw, g.st_hi, sd, sm, diag, sym, lane, col0, row_base, b);
-        if (nplanes > 1) stage_store_block(lw, g.st_lo, sd, sm, diag, sym, lane, col0, row_base, b);
+        for (int j = 0; j < 16; ++j) split16x2(v[2 * j], v[2 * j + 1], of16, hw[j], lw[j]);
+        stage_store_block(hw, g.st_hi, stg, sseq, diag, sym, lane, col0, row_base, b);
+        if (nplanes > 1) stage_store_block(lw, g.st_lo, stg, sseq, diag, sym, lane, col0, row_base, b);
         if (write_y) {
             // Y = yb I + yc G, hi plane only (it is the single operand of G Y)
+            if (diag) {
 #pragma unroll
-            for (int j = 0; j < 16; ++j) {
-                uint16_t y0, y1, unused;
-                split16(ti.yc * v[2 * j] + (2 * j == d ? ti.yb : 0.f), of16, y0, unused);
-                split16(ti.yc * v[2 * j + 1] + (2 * j + 1 == d ? ti.yb : 0.f), of16, y1, unused);
-                lw[j] = static_cast<uint32_t>(y0) | (static_cast<uint32_t>(y1) << 16);
+                for (int j = 0; j < 16; ++j)
+                    lw[j] = round16x2(ti.yc * v[2 * j] + (2 * j == d ? ti.yb : 0.f),
+                                      ti.yc * v[2 * j + 1] + (2 * j + 1 == d ? ti.yb : 0.f), of16);
+            } else {
+#pragma unroll
+                for (int j = 0; j < 16; ++j) lw[j] = round16x2(ti.yc * v[2 * j], ti.yc * v[2 * j + 1], of16);
             }
-            stage_store_block(lw, g.st_y, sd, sm, diag, sym, lane, col0, row_base, b);
+            stage_store_block(lw, g.st_y, stg, sseq, diag, sym, lane, col0, row_base, b);
         }
     }
     if (gram_fused) {
@@ -644,6 +664,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
         const int eg = warp & 3;  // tensor-memory lane quarter this warp may access
         const int half = (warp - 2) >> 2;
         uint32_t n = 0;
+        uint32_t sseq = 0;  // this warp's staged stores so far (staging block rotation)
         int q = 0;
         uint32_t qphase = 0;
         for (;;) {
@@ -679,7 +700,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
             __syncwarp();
             tc_fence_after();
             tile_epilogue(p, ti, tmem_base + buf * kTmemCols, ok, eg, half, lane, crank,
-                          staging + (warp - 2) * 2 * kStageBlockBytes);
+                          staging + (warp - 2) * kStageBlocks * kStageBlockBytes, sseq);
             tc_fence_before();
             __syncwarp();
             if (lane == 0) {

@@ -23,7 +23,7 @@ constexpr int kBRows = kPairMma ? BN / 2 : BN;  // rows of B (N extent) staged b
 // Shared-memory ring of the persistent GEMM (one CTA per SM): as many stages of the
 // launch's plane set as fit in kRingBytes, at most kMaxStages.
 constexpr int kMaxStages = 12;
-constexpr int kRingBytes = 192 * 1024;
+constexpr int kRingBytes = 160 * 1024;
 constexpr int kTileABytes = BM * BK * 2;                       // one bf16 plane of A
 constexpr int kTileBBytes = kBRows * BK * 2;                   // one bf16 plane of this CTA's B
 
@@ -33,10 +33,13 @@ constexpr int kGemmThreads = 64 + 32 * kEpiWarps;  // warp 0 TMA, warp 1 MMA, wa
 constexpr int kTmemCols = 256;     // one accumulator; the kernel double-buffers (512 columns)
 constexpr int kMaxGroups = 8;
 constexpr int kFinRows = 32;  // rows of one k_gram_finalize tile (x BN columns)
-// Epilogue staging: per epilogue warp a 32 x 32 16-bit block and its transpose (2 KB each,
-// 64-byte swizzled rows), written to global memory by TMA stores.
+// Epilogue staging: per epilogue warp kStageBlocks blocks of 32 x 32 16-bit values (2 KB,
+// 64-byte swizzled rows), written to global memory by TMA stores.  A symmetric output
+// uses them as two (direct, transposed) pairs, anything else as four single blocks, so
+// that a warp fills one while the TMA stores of the others still read shared memory.
 constexpr int kStageBlockBytes = 32 * 32 * 2;
-constexpr int kEpiStagingBytes = kEpiWarps * 2 * kStageBlockBytes;
+constexpr int kStageBlocks = 4;
+constexpr int kEpiStagingBytes = kEpiWarps * kStageBlocks * kStageBlockBytes;
 constexpr int kTileQueue = 8;  // tiles handed from the producer warp to the MMA and epilogue warps
 constexpr int kGemmSmemBytes = kRingBytes + kEpiStagingBytes + 1024 /*align*/ + 512 /*barriers, queues*/;
 
