@@ -169,8 +169,13 @@ int isoloco_debug_gemm(int a_mn_major, int b_mn_major, int precision, int batch,
  * work queued on its other streams.  This entry point calls neither, nor any
  * other allocating routine: its scratch (the hi/lo operand planes, the four
  * tensor maps, an error word and a tile counter) lives in one static device
- * array of the library, 16 MiB per device, whose address is looked up once per
- * device.
+ * array of the library, 16 MiB per device, held by every GPU that loads the
+ * library until the process exits.
+ *
+ * Set-up: the first call on a device (with that device current) looks up the
+ * array's device address with cudaGetSymbolAddress and keeps it for later
+ * calls; a failure there returns ISOLOCO_ERR_CUDA.  Make that first call on each
+ * device before any stream capture begins.
  *
  * Limit: 1024 + 2 * R(2 * batch * a_rows * round8(a_cols))
  *             + 2 * R(2 * batch * b_rows * round8(b_cols)) <= 16 MiB,

@@ -1073,7 +1073,10 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratch
 std::mutex g_noalloc_mutex;
 unsigned char* g_noalloc_ptr[kNoAllocMaxDevices] = {};
 
-// Address of the scratch array in the current device's context, looked up once per device.
+// Address of the scratch array in the current device's context.  In host code the name
+// g_noalloc_scratch stands for a host-side shadow, not a device address, so kernels are
+// given this looked-up pointer instead.  The first call on a device (that device
+// current) does the lookup; later calls reuse it.
 int noalloc_scratch(unsigned char** out) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
