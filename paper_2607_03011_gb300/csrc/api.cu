@@ -30,7 +30,7 @@ __global__ void k_gram_finalize(const MatDesc*, const int2*, const MatState*, co
                                 const int64_t*, const int*, __nv_bfloat16*, __nv_bfloat16*, float*, int,
                                 __nv_bfloat16*);
 __global__ void k_control(const MatDesc*, int, MatState*, const float*, int, int, float, uint32_t*, const int*,
-                          const int*, int, int*, int*, int*, int*);
+                          const int*, int, int*, int*, int*, int*, cudaGraphConditionalHandle, int, long long*);
 __global__ void k_trace_partial(const MatDesc*, const int4*, const MatState*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, double*);
@@ -118,6 +118,15 @@ struct isoloco_plan {
     uint32_t* err_h = nullptr;  // pinned
     CUtensorMap* tmaps_d = nullptr;
     cudaEvent_t done_ev = nullptr;
+    // iterations 1, 2, ... of the polar loop as one CUDA graph: a while-conditional node
+    // whose body (two iterations) runs until k_control reports no matrix left to iterate
+    cudaStream_t cap_st = nullptr;  // private stream the body is captured on
+    cudaGraph_t graph = nullptr;
+    cudaGraphExec_t gexec = nullptr;
+    int g_max_iter = -1;
+    float g_tol = 0.f;
+    int64_t body_launches = 0;      // kernels in one run of the body
+    long long* loopc = nullptr;     // device: [0] body runs in this call, [1] body runs ever
     // phase timing (isoloco_profile_enable) and launch counting
     bool prof = false;
     std::vector<std::pair<cudaEvent_t, cudaEvent_t>> pend[ISOLOCO_NUM_PHASES];
@@ -225,6 +234,9 @@ static void free_plan(isoloco_plan* p) {
     for (cudaEvent_t e : p->ev_pool) cudaEventDestroy(e);
     if (p->err_h) cudaFreeHost(p->err_h);
     if (p->done_ev) cudaEventDestroy(p->done_ev);
+    if (p->gexec) cudaGraphExecDestroy(p->gexec);
+    if (p->graph) cudaGraphDestroy(p->graph);
+    if (p->cap_st) cudaStreamDestroy(p->cap_st);
     delete p;
 }
 
@@ -412,12 +424,14 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         (rc = dalloc(p, &p->bucket_count_d, (int64_t)p->buckets.size())) ||
         (rc = dalloc(p, &p->cnt_gram, (int64_t)p->buckets.size())) ||
         (rc = dalloc(p, &p->cnt_step, (int64_t)p->buckets.size())) ||
-        (rc = dalloc(p, &p->counters, kLaunchCounters)) ||
+        (rc = dalloc(p, &p->counters, kLaunchCounters)) || (rc = dalloc(p, &p->loopc, 2)) ||
         (rc = dalloc(p, &p->tmaps_d, (int64_t)kMapsPerBucket * std::max<size_t>(1, p->buckets.size()))))
         return rc;
     CUDA_TRY(cudaHostAlloc(reinterpret_cast<void**>(&p->err_h), sizeof(uint32_t), cudaHostAllocDefault));
     *p->err_h = 0;
     CUDA_TRY(cudaEventCreateWithFlags(&p->done_ev, cudaEventDisableTiming));
+    CUDA_TRY(cudaStreamCreateWithFlags(&p->cap_st, cudaStreamNonBlocking));
+    CUDA_TRY(cudaMemset(p->loopc, 0, 2 * sizeof(long long)));
     // zero the planes once so that padding columns hold zeros
     for (void* a : {(void*)p->dhi, (void*)p->dlo, (void*)p->xhi[0], (void*)p->xlo[0], (void*)p->xhi[1],
                     (void*)p->xlo[1]})
@@ -570,11 +584,13 @@ static int flush_set(isoloco_plan* pl, int phase, LaunchSet& s, bool a_mn, bool 
     return ISOLOCO_OK;
 }
 
-// The polar iteration for every matrix, from Delta (planes dhi/dlo) to Q and sigma_bar.
-static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) {
-    if (p->nmat == 0) return ISOLOCO_OK;
+// Iteration t of the polar loop for every matrix still active: Gram, convergence test
+// and choice of the step (k_control), polynomial, update.  With set_cond, k_control also
+// sets the graph condition `cond` (graph body only).
+static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cudaStream_t st,
+                           cudaGraphConditionalHandle cond, int set_cond) {
     const CUtensorMap* maps = p->tmaps_d;
-    for (int t = 0; t <= max_iter; ++t) {
+    {
         const int src = (t == 0) ? 0 : 1 + (t & 1);  // Delta, X0 or X1 as the current iterate
         const int dst = (t + 1) & 1;
         // ---- Gram G = X^T X (tall, MN-major operands) or X X^T (wide, K-major)
@@ -626,7 +642,7 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
         { PhaseTimer tm(p, ISOLOCO_PHASE_CONTROL, st);
         k_control<<<1, 1024, 0, st>>>(p->mats_d, p->nmat, p->state, p->fin_part, t, max_iter, tol, p->err_d,
                                       p->bucket_first_d, p->bucket_count_d, (int)p->buckets.size(), p->list_gram,
-                                      p->cnt_gram, p->list_step, p->cnt_step); }
+                                      p->cnt_gram, p->list_step, p->cnt_step, cond, set_cond, p->loopc); }
         CUDA_TRY(cudaGetLastError());
         // ---- P = a I + b G + c G^2
         LaunchSet poly;
@@ -688,6 +704,98 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
         if ((rc = flush_set(p, ISOLOCO_PHASE_UPDATE, utall, false, false, st)) ||
             (rc = flush_set(p, ISOLOCO_PHASE_UPDATE, uwide, false, true, st)))
             return rc;
+    }
+    return ISOLOCO_OK;
+}
+
+// Captures iterations 1 and 2 (the buffer parity of every later odd / even pair) as the
+// body of a while-conditional graph node; the body's second k_control keeps the loop
+// going while some matrix is not done.  Built once per plan and (max_iter, tol).
+static int build_polar_graph(isoloco_plan* p, int max_iter, float tol) {
+    if (p->gexec) cudaGraphExecDestroy(p->gexec);
+    if (p->graph) cudaGraphDestroy(p->graph);
+    p->gexec = nullptr;
+    p->graph = nullptr;
+    p->g_max_iter = -1;
+    cudaGraph_t g = nullptr;
+    CUDA_TRY(cudaGraphCreate(&g, 0));
+    cudaGraphConditionalHandle h;
+    cudaError_t e = cudaGraphConditionalHandleCreate(&h, g, 1, cudaGraphCondAssignDefault);
+    cudaGraphNodeParams np = {cudaGraphNodeTypeConditional};
+    np.conditional.handle = h;
+    np.conditional.type = cudaGraphCondTypeWhile;
+    np.conditional.size = 1;
+    cudaGraphNode_t node = nullptr;
+    if (e == cudaSuccess) e = cudaGraphAddNode(&node, g, nullptr, nullptr, 0, &np);
+    if (e != cudaSuccess) {
+        cudaGraphDestroy(g);
+        return fail(ISOLOCO_ERR_CUDA, std::string("polar graph: ") + cudaGetErrorString(e));
+    }
+    cudaGraph_t body = np.conditional.phGraph_out[0];
+    // the captured launches are counted per run of the body, not at capture time
+    const int64_t launches0 = p->launches;
+    int64_t prof_n0[ISOLOCO_NUM_PHASES];
+    memcpy(prof_n0, p->prof_n, sizeof(prof_n0));
+    e = cudaStreamBeginCaptureToGraph(p->cap_st, body, nullptr, nullptr, 0, cudaStreamCaptureModeThreadLocal);
+    int rc = ISOLOCO_OK;
+    if (e == cudaSuccess) {
+        rc = polar_iteration(p, 1, max_iter, tol, p->cap_st, h, 0);
+        if (rc == ISOLOCO_OK) rc = polar_iteration(p, 2, max_iter, tol, p->cap_st, h, 1);
+        cudaGraph_t captured = nullptr;
+        const cudaError_t e2 = cudaStreamEndCapture(p->cap_st, &captured);
+        if (e2 != cudaSuccess && rc == ISOLOCO_OK) rc = fail(ISOLOCO_ERR_CUDA, std::string("polar graph capture: ") + cudaGetErrorString(e2));
+    } else {
+        rc = fail(ISOLOCO_ERR_CUDA, std::string("polar graph capture: ") + cudaGetErrorString(e));
+    }
+    p->body_launches = p->launches - launches0;
+    p->launches = launches0;
+    memcpy(p->prof_n, prof_n0, sizeof(prof_n0));
+    if (rc == ISOLOCO_OK) {
+        e = cudaGraphInstantiate(&p->gexec, g, 0);
+        if (e != cudaSuccess) rc = fail(ISOLOCO_ERR_CUDA, std::string("polar graph instantiate: ") + cudaGetErrorString(e));
+    }
+    if (rc != ISOLOCO_OK) {
+        (void)cudaGetLastError();
+        cudaGraphDestroy(g);
+        p->gexec = nullptr;
+        return rc;
+    }
+    p->graph = g;
+    p->g_max_iter = max_iter;
+    p->g_tol = tol;
+    return ISOLOCO_OK;
+}
+
+// The polar iteration for every matrix, from Delta (planes dhi/dlo) to Q and sigma_bar.
+// Iteration 0 is launched directly; the rest run as one graph launch that stops as soon
+// as every matrix is done.  With phase profiling on (events cannot sit inside the graph
+// body), or when `st` is itself being captured, iterations 1 .. max_iter are launched one
+// by one instead (empty launches once every matrix is done).
+static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) {
+    if (p->nmat == 0) return ISOLOCO_OK;
+    int rc = polar_iteration(p, 0, max_iter, tol, st, 0, 0);
+    if (rc) return rc;
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    CUDA_TRY(cudaStreamIsCapturing(st, &cs));
+    const bool use_graph = kPairMma && !p->prof && cs == cudaStreamCaptureStatusNone;
+    if (use_graph) {
+        if (!p->gexec || p->g_max_iter != max_iter || p->g_tol != tol)
+            if ((rc = build_polar_graph(p, max_iter, tol))) return rc;
+        CUDA_TRY(cudaGraphLaunch(p->gexec, st));
+    } else {
+        std::vector<int> cnt(p->buckets.size());
+        for (int t = 1; t <= max_iter; ++t) {
+            if ((rc = polar_iteration(p, t, max_iter, tol, st, 0, 0))) return rc;
+            if (p->prof && cs == cudaStreamCaptureStatusNone && !cnt.empty()) {
+                // profiling: stop, as the graph does, once no matrix is left (the wait for
+                // the count lies between the phases' events)
+                CUDA_TRY(cudaMemcpyAsync(cnt.data(), p->cnt_gram, sizeof(int) * cnt.size(), cudaMemcpyDeviceToHost, st));
+                CUDA_TRY(cudaStreamSynchronize(st));
+                int active = 0;
+                for (int c : cnt) active += c;
+                if (active == 0) break;
+            }
+        }
     }
     { PhaseTimer tm(p, ISOLOCO_PHASE_TRACE, st, 2);
     k_trace_partial<<<p->ntchunks, 256, 0, st>>>(p->mats_d, p->tchunks, p->state, p->dhi, p->dlo, p->xhi[0],
@@ -962,7 +1070,14 @@ int isoloco_profile_read(isoloco_plan_t p, void* stream, double* ms, int64_t* la
     return ISOLOCO_OK;
 }
 
-int64_t isoloco_plan_launches(isoloco_plan_t p) { return p ? p->launches : 0; }
+int64_t isoloco_plan_launches(isoloco_plan_t p) {
+    if (!p) return 0;
+    // kernels launched directly, plus those of every run of the polar graph's body
+    long long runs[2] = {0, 0};
+    if (p->body_launches > 0 && cudaMemcpy(runs, p->loopc, sizeof(runs), cudaMemcpyDeviceToHost) != cudaSuccess)
+        runs[1] = 0;
+    return p->launches + p->body_launches * static_cast<int64_t>(runs[1]);
+}
 
 int isoloco_read_diag(isoloco_plan_t p, void* stream, float* sigma_bar, int32_t* iters, int32_t* status,
                       float* resid) {

@@ -61,26 +61,75 @@ __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict
     const int64_t sstride = gpart_split_stride[mi];
     const int splits = nsplit[mi];
 
+    // each thread owns 4-column groups (float4) of the tile; 8 independent loads per split
+    // are in flight per thread.  Columns beyond n (row padding) are neither read as data
+    // nor written.
+    static_assert((kFinRows * BN / 4) % (8 * 256) == 0, "tile = 8 column groups per thread");
+    constexpr int kGroups = kFinRows * BN / 4 / 256;  // column groups per thread (blockDim 256)
     float sq = 0.f, tr = 0.f, dev = 0.f;
-    for (int e = threadIdx.x; e < kFinRows * BN; e += blockDim.x) {
+    float4 acc[kGroups];
+    int64_t idx[kGroups];
+    bool any[kGroups];
+#pragma unroll
+    for (int i = 0; i < kGroups; ++i) {
+        const int e = (threadIdx.x + i * 256) * 4;
         const int r = r0 + e / BN, c = c0 + e % BN;
-        if (r >= n || c >= n) continue;
-        const int64_t idx = static_cast<int64_t>(r) * ld + c;
-        float v = 0.f;
-        for (int s = 0; s < splits; ++s) v += gpart[poff + s * sstride + idx];
-        uint16_t h, l;
-        split16(v, out_f16 != 0, h, l);
-        reinterpret_cast<uint16_t*>(ghi)[md.gslot + idx] = h;
-        reinterpret_cast<uint16_t*>(glo)[md.gslot + idx] = l;
-        if (ypl) {
-            uint16_t yh, yl;
-            split16(yc * v + (r == c ? yb : 0.f), out_f16 != 0, yh, yl);
-            reinterpret_cast<uint16_t*>(ypl)[md.gslot + idx] = yh;
+        any[i] = r < n && c < n;
+        idx[i] = static_cast<int64_t>(r) * ld + c;
+        acc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    for (int sp = 0; sp < splits; ++sp) {
+        const float* base = gpart + poff + sp * sstride;
+        float4 t[kGroups];
+#pragma unroll
+        for (int i = 0; i < kGroups; ++i)
+            t[i] = any[i] ? __ldg(reinterpret_cast<const float4*>(base + idx[i])) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int i = 0; i < kGroups; ++i) {
+            acc[i].x += t[i].x;
+            acc[i].y += t[i].y;
+            acc[i].z += t[i].z;
+            acc[i].w += t[i].w;
         }
-        sq += v * v;
-        const float dlt = (r == c) ? 1.f : 0.f;
-        tr += (r == c) ? v : 0.f;
-        dev += (v - dlt) * (v - dlt);
+    }
+    const bool of16 = out_f16 != 0;
+#pragma unroll
+    for (int i = 0; i < kGroups; ++i) {
+        if (!any[i]) continue;
+        const int e = (threadIdx.x + i * 256) * 4;
+        const int r = r0 + e / BN, c = c0 + e % BN;
+        const float v[4] = {acc[i].x, acc[i].y, acc[i].z, acc[i].w};
+        uint32_t hw[2], lw[2], yw[2];
+        split16x2(v[0], v[1], of16, hw[0], lw[0]);
+        split16x2(v[2], v[3], of16, hw[1], lw[1]);
+        if (ypl) {
+            yw[0] = round16x2(yc * v[0] + (r == c ? yb : 0.f), yc * v[1] + (r == c + 1 ? yb : 0.f), of16);
+            yw[1] = round16x2(yc * v[2] + (r == c + 2 ? yb : 0.f), yc * v[3] + (r == c + 3 ? yb : 0.f), of16);
+        }
+        const int64_t o = md.gslot + idx[i];
+        if (c + 3 < n) {
+            *reinterpret_cast<uint2*>(reinterpret_cast<uint16_t*>(ghi) + o) = make_uint2(hw[0], hw[1]);
+            *reinterpret_cast<uint2*>(reinterpret_cast<uint16_t*>(glo) + o) = make_uint2(lw[0], lw[1]);
+            if (ypl) *reinterpret_cast<uint2*>(reinterpret_cast<uint16_t*>(ypl) + o) = make_uint2(yw[0], yw[1]);
+        } else {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                if (c + q >= n) break;
+                const int sh = (q & 1) * 16;
+                reinterpret_cast<uint16_t*>(ghi)[o + q] = static_cast<uint16_t>(hw[q >> 1] >> sh);
+                reinterpret_cast<uint16_t*>(glo)[o + q] = static_cast<uint16_t>(lw[q >> 1] >> sh);
+                if (ypl) reinterpret_cast<uint16_t*>(ypl)[o + q] = static_cast<uint16_t>(yw[q >> 1] >> sh);
+            }
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            if (c + q >= n) break;
+            const float x = v[q];
+            const bool dg = (r == c + q);
+            sq += x * x;
+            tr += dg ? x : 0.f;
+            dev += dg ? (x - 1.f) * (x - 1.f) : x * x;
+        }
     }
     __shared__ float red[3][8];
     sq = warp_sum_f(sq);
@@ -187,7 +236,10 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
 // One block of 1024 threads.  Warp w takes the decisions of matrices w, w + 32, ...; then
 // warp b compacts, for shape bucket b, the matrices that still need a Gram (not done) and
 // those that take a step this iteration (mode != 0), in matrix order.  GEMM launches only
-// enumerate the listed matrices.
+// enumerate the listed matrices.  As the last kernel of the polar graph's loop body
+// (set_cond), it also sets the loop's condition: run the body again while some matrix is
+// not done, at most until the iteration count passes max_iter (loopc[0] counts body runs
+// in this call, reset at t = 0; loopc[1] counts them over the plan's life).
 __global__ void __launch_bounds__(1024) k_control(const MatDesc* __restrict__ mats, int nmat,
                                                   MatState* __restrict__ state,
                                                   const float* __restrict__ fin_part, int t, int max_iter,
@@ -195,8 +247,11 @@ __global__ void __launch_bounds__(1024) k_control(const MatDesc* __restrict__ ma
                                                   const int* __restrict__ bucket_first,
                                                   const int* __restrict__ bucket_count, int nbuckets,
                                                   int* __restrict__ list_gram, int* __restrict__ cnt_gram,
-                                                  int* __restrict__ list_step, int* __restrict__ cnt_step) {
+                                                  int* __restrict__ list_step, int* __restrict__ cnt_step,
+                                                  cudaGraphConditionalHandle cond, int set_cond,
+                                                  long long* __restrict__ loopc) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (t == 0 && threadIdx.x == 0) loopc[0] = 0;
     for (int mi = warp; mi < nmat; mi += 32) {
         control_matrix(mats, mi, state, fin_part, t, max_iter, tol, err, lane);
         __syncwarp();
@@ -223,6 +278,17 @@ __global__ void __launch_bounds__(1024) k_control(const MatDesc* __restrict__ ma
         if (lane == 0) {
             cnt_gram[bk] = ng;
             cnt_step[bk] = ns;
+        }
+    }
+    if (set_cond) {
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            int active = 0;
+            for (int bk = 0; bk < nbuckets; ++bk) active += cnt_gram[bk];
+            const long long runs = ++loopc[0];
+            ++loopc[1];
+            const bool more = active > 0 && 2 * runs < static_cast<long long>(max_iter) + 2;
+            cudaGraphSetConditional(cond, more ? 1u : 0u);
         }
     }
 }

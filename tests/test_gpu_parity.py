@@ -158,6 +158,28 @@ def test_deterministic(iso):
     assert torch.equal(r1[1], r2[1]) and torch.equal(r1[2], r2[2]) and torch.equal(r1[3], r2[3])
 
 
+def test_graph_loop_matches_per_launch_loop(iso):
+    """The polar loop runs as one CUDA graph whose while-node stops once every matrix is
+    done; under phase profiling it runs launch by launch instead.  Both give the same bits,
+    the graph running at most one extra (empty) iteration, and a new max_iter rebuilds it."""
+    spec = W.custom_spec(RAGGED, K=3, rank=2, momentum_std=1e-4)
+    wl = W.make_workload(spec, seed=11, device="cuda")
+    plan = iso.Plan(wl.table, wl.N, wl.K)
+    for max_iter in (0, 20):
+        l0 = plan.launches
+        g = run_gpu(iso, wl, 1.0, 0.7, 0.9, plan=plan, max_iter=max_iter)
+        lg = plan.launches - l0
+        plan.profile(True)
+        l0 = plan.launches
+        h = run_gpu(iso, wl, 1.0, 0.7, 0.9, plan=plan, max_iter=max_iter)
+        lh = plan.launches - l0
+        plan.profile(False)
+        assert g[0] == h[0] == 0
+        assert torch.equal(g[1], h[1]) and torch.equal(g[2], h[2]) and torch.equal(g[3], h[3])
+        assert g[4]["iters"] == h[4]["iters"] and g[4]["sigma_bar"] == h[4]["sigma_bar"]
+        assert lh <= lg <= lh + lh // 2, (lg, lh)
+
+
 def test_diloco_outer_step(iso):
     spec = W.custom_spec(RAGGED, K=3, rank=2, momentum_std=1e-4)
     wl = W.make_workload(spec, seed=6, device="cuda")
