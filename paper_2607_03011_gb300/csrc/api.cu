@@ -334,9 +334,11 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         bk.splits = splits;
         const int64_t mat_elems = (int64_t)bk.rows * bk.ld;
         const int64_t g_elems = (int64_t)bk.n * bk.ld_n;
-        // Gram partial-sum slots per matrix: one per computed Gram tile (upper-triangle
-        // tiles) when the Gram's epilogue produces them, one per finalize tile otherwise
-        const int gtiles = splits > 1 ? ((bk.n + kFinRows - 1) / kFinRows) * ((bk.n + BN - 1) / BN) : sym_tiles(bk.n);
+        // Gram partial sums per matrix, in groups of kPartSlots slots: one group per computed
+        // Gram tile (upper-triangle tiles) when the Gram's epilogue produces them; with
+        // split-K one slot per finalize tile, packed, the rest of the last group zero
+        const int nft = splits > 1 ? ((bk.n + kFinRows - 1) / kFinRows) * ((bk.n + BN - 1) / BN) : 0;
+        const int gtiles = splits > 1 ? (nft + kPartSlots - 1) / kPartSlots : sym_tiles(bk.n);
         for (int j = 0; j < bk.count; ++j) {
             const int pi = members[b][j];
             MatDesc md{};
@@ -351,12 +353,14 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
             md.gslot = gplane + j * g_elems;
             md.gpart_slot = fin;
             md.n_gtiles = gtiles;
+            // near-square (|rows - cols| < min / 16): the deep polar schedule
+            md.deep = (std::abs(bk.rows - bk.cols) * 16 < bk.n) ? 1 : 0;
             md.trace_part = tr;
             const int rows_per = std::max(1, kTraceChunkElems / bk.cols);
             md.n_tchunks = (bk.rows + rows_per - 1) / rows_per;
             const int mi = (int)p->mats_h.size();
             if (splits > 1)
-                for (int t = 0; t < md.n_gtiles; ++t) ftiles.push_back(make_int2(mi, t));
+                for (int t = 0; t < nft; ++t) ftiles.push_back(make_int2(mi, t));
             for (int c = 0; c < md.n_tchunks; ++c) {
                 const int r0 = c * rows_per;
                 tchunks.push_back(make_int4(mi, r0, std::min(rows_per, bk.rows - r0), c));
@@ -439,6 +443,9 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
     for (void* a : {(void*)p->ghi, (void*)p->glo, (void*)p->phi, (void*)p->plo, (void*)p->ypl})
         CUDA_TRY(cudaMemset(a, 0, std::max<int64_t>(1, gplane) * 2));
     CUDA_TRY(cudaMemset(p->err_d, 0, 4));
+    // Gram partial sums: slots that no kernel writes (the tail of a split-K matrix's last
+    // group) must read as zero
+    if (fin > 0) CUDA_TRY(cudaMemset(p->fin_part, 0, sizeof(float) * 3 * kPartSlots * fin));
     if (p->nmat) {
         CUDA_TRY(cudaMemcpy(p->mats_d, p->mats_h.data(), sizeof(MatDesc) * p->nmat, cudaMemcpyHostToDevice));
         CUDA_TRY(cudaMemcpy(p->gpart_off_d, gpoff.data(), sizeof(int64_t) * p->nmat, cudaMemcpyHostToDevice));

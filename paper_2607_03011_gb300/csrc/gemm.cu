@@ -123,9 +123,8 @@ __device__ __forceinline__ bool decode_tile(const GemmParams& p, const int* pre,
         if (p.gate == kGateActive) {
             if (st.done) return false;
             if (p.gram_y) {  // coefficients of the quintic step this Gram may lead to
-                const int k = st.step % kSchedSteps;
-                ti.yb = kSched[k][1];
-                ti.yc = kSched[k][2];
+                ti.yb = st.yb;
+                ti.yc = st.yc;
             }
         } else {
             if (st.mode == 0) return false;

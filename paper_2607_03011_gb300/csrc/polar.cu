@@ -51,8 +51,7 @@ __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict
     const int mi = ft.x;
     if (state[mi].done) return;
     // ypl != null: also write Y = yb I + yc G (hi plane) for the quintic step that may follow
-    const int ks = state[mi].step % kSchedSteps;
-    const float yb = kSched[ks][1], yc = kSched[ks][2];
+    const float yb = state[mi].yb, yc = state[mi].yc;
     const MatDesc md = mats[mi];
     const int n = md.n, ld = md.ld_n;
     const int tiles_c = (n + BN - 1) / BN;
@@ -145,10 +144,20 @@ __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict
     if (threadIdx.x < 3) {
         float s = 0.f;
         for (int i = 0; i < (int)(blockDim.x >> 5); ++i) s += red[threadIdx.x][i];
-        float* slot = fin_part + (md.gpart_slot + ft.y) * kPartSlots * 3;  // kPartSlots slots of 3 per tile
-        slot[threadIdx.x] = s;
-        for (int w = 1; w < kPartSlots; ++w) slot[3 * w + threadIdx.x] = 0.f;
+        // one slot of 3 per finalize tile, packed after the matrix's first slot
+        fin_part[(static_cast<int64_t>(md.gpart_slot) * kPartSlots + ft.y) * 3 + threadIdx.x] = s;
     }
+}
+
+// Coefficients (a, b, c) of quintic step `step` of a matrix.  Near-square matrices (deep)
+// start with one round of the deep schedule, which reaches singular values down to 1e-6
+// of the normalisation; whatever was below that has grown by the product of its linear
+// coefficients (~4e6) and sits above the standard schedule's 1e-3 floor, so later rounds
+// (and every round of the other matrices) use the standard schedule.
+__device__ __forceinline__ const float* sched_row(bool deep, int step) {
+    if (deep && step < kSchedDeepSteps) return kSchedDeep[step];
+    const int k = (deep ? step - kSchedDeepSteps : step) % kSchedSteps;
+    return kSched[k];
 }
 
 // Decision for matrix mi, taken by one warp.  t: iteration index (0 = first Gram of Delta).
@@ -164,13 +173,24 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
     // fp32 lane sums and a fixed shuffle tree: each lane adds at most a few dozen
     // non-negative terms (relative error ~1e-6, far below the tolerance this sum is
     // tested against), and fp32 keeps one SM off GB300's narrow fp64 pipe.
-    float sqf = 0.f, trf = 0.f, devf = 0.f;
-    for (int i = lane; i < kPartSlots * md.n_gtiles; i += 32) {  // kPartSlots partial slots per Gram tile
-        const float* pp = fin_part + (md.gpart_slot * kPartSlots + i) * 3;
-        sqf += pp[0];
-        trf += pp[1];
-        devf += pp[2];
+    // four independent accumulators per lane keep four slots' loads in flight
+    const int nslots = kPartSlots * md.n_gtiles;
+    const float* pp = fin_part + static_cast<int64_t>(md.gpart_slot) * kPartSlots * 3;
+    float a_sq[4] = {0.f, 0.f, 0.f, 0.f}, a_tr[4] = {0.f, 0.f, 0.f, 0.f}, a_dev[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int i0 = lane; i0 < nslots; i0 += 128) {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int i = i0 + 32 * u;
+            if (i < nslots) {
+                a_sq[u] += pp[3 * i];
+                a_tr[u] += pp[3 * i + 1];
+                a_dev[u] += pp[3 * i + 2];
+            }
+        }
     }
+    float sqf = (a_sq[0] + a_sq[1]) + (a_sq[2] + a_sq[3]);
+    float trf = (a_tr[0] + a_tr[1]) + (a_tr[2] + a_tr[3]);
+    float devf = (a_dev[0] + a_dev[1]) + (a_dev[2] + a_dev[3]);
     sqf = warp_sum_f(sqf);
     trf = warp_sum_f(trf);
     devf = warp_sum_f(devf);
@@ -222,13 +242,17 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
         st.status = kErrNotConverged;
         atomicOr(err, kErrNotConverged);
     } else {
-        const int k = st.step % kSchedSteps;
+        const float* q = sched_row(md.deep != 0, st.step);
         st.mode = 1;
-        st.a = kSched[k][0];
-        st.b = static_cast<float>(kSched[k][1] * gscale);
-        st.c = static_cast<float>(kSched[k][2] * gscale * gscale);
+        st.a = q[0];
+        st.b = static_cast<float>(q[1] * gscale);
+        st.c = static_cast<float>(q[2] * gscale * gscale);
         st.step += 1;
         st.iters += 1;
+        // the next Gram writes Y = b I + c G of the step after this one (X normalised by then)
+        const float* qn = sched_row(md.deep != 0, st.step);
+        st.yb = qn[1];
+        st.yc = qn[2];
     }
 }
 
@@ -400,6 +424,7 @@ __global__ void k_reset_state(MatState* state, int nmat, uint32_t* err, const Ma
     s.iters = 0;
     s.done = 0;
     s.final_buf = 2;
+    s.yb = s.yc = 0.f;
     s.status = 0;
     s.trace = 0.0;
     state[i] = s;

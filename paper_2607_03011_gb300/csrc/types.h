@@ -111,6 +111,7 @@ struct MatState {
     int iters;        // GEMM iterations used
     int done;         // 1 once finished
     int final_buf;    // ping-pong buffer holding Q (0/1), or 2 when Q = 0
+    float yb, yc;     // Y = yb I + yc G for the quintic step the next Gram leads to
     int status;       // 0, or kErrNotConverged
     double trace;     // tr(Q^T Delta)
 };
@@ -147,7 +148,8 @@ struct MatDesc {
     int64_t gslot;         // element offset of the matrix in the n x n planes
     int64_t gpart_slot;    // first partial (3 floats each) of the finalize pass
     int64_t trace_part;    // first partial of the trace pass
-    int n_gtiles;          // finalize tiles of this matrix
+    int n_gtiles;          // groups of kPartSlots Gram partial sums of this matrix
+    int deep;              // 1: near-square, polar steps from the deep schedule
     int n_tchunks;         // trace chunks of this matrix
 };
 
