@@ -6,8 +6,10 @@
 `step` runs IsoLoCo outer steps through the C ABI on a named workload; `square48`
 is the 48 square 1024 x 1024 matrices of the 180M recipe with K = 8 replicas
 (1.6 GB of replicas: larger than L2, small enough for a full ncu capture), and
-`square12` a quarter of it.  `gemm` runs the
-split-precision GEMM entry point on random inputs.
+`square12` a quarter of it; with --per-launch the polar iterations are launched one
+by one (phase profiling on) instead of as the library's CUDA graph, so that every
+kernel is a plain launch.  `gemm` runs the split-precision GEMM entry point on random
+inputs.
 """
 from __future__ import annotations
 
@@ -28,10 +30,12 @@ EXTRA = {
 }
 
 
-def run_step(workload: str, steps: int) -> None:
+def run_step(workload: str, steps: int, per_launch: bool = False) -> None:
     spec = EXTRA[workload]() if workload in EXTRA else W.SPECS[workload]
     wl = W.make_workload(spec, seed=0, device="cuda")
     plan = isoloco.Plan(wl.table, wl.N, wl.K, wl.replicas.dtype)
+    if per_launch:
+        plan.profile(True)
     opts = isoloco.make_opts(spec.alpha, spec.outer_lr, spec.momentum)
     th0, b0 = wl.theta.clone(), wl.momentum.clone()
     for _ in range(steps):
@@ -60,6 +64,7 @@ def main():
     s = sub.add_parser("step")
     s.add_argument("--workload", default="square12")
     s.add_argument("--steps", type=int, default=2)
+    s.add_argument("--per-launch", action="store_true")
     gm = sub.add_parser("gemm")
     gm.add_argument("--batch", type=int, default=48)
     gm.add_argument("--m", type=int, default=1024)
@@ -71,7 +76,7 @@ def main():
     gm.add_argument("--precision", type=int, default=0)
     a = ap.parse_args()
     if a.cmd == "step":
-        run_step(a.workload, a.steps)
+        run_step(a.workload, a.steps, a.per_launch)
     else:
         run_gemm(a.batch, a.m, a.n, a.k, a.a_mn, a.b_mn, a.reps, a.precision)
 
