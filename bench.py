@@ -162,7 +162,8 @@ def stream_bytes(table, K, replica_bytes):
 
 
 # --------------------------------------------------------------------------- CPU oracle arm
-CPU_SAMPLE = ["layers.0.attn_norm", "layers.0.wq", "layers.0.ffn_norm", "layers.0.w_gate", "layers.0.w_down"]
+CPU_SAMPLE = ["layers.0.attn_norm", "layers.0.wq", "layers.0.wk", "layers.0.ffn_norm", "layers.0.w_gate", "layers.0.w_up",
+              "layers.0.w_down"]
 REF_SAMPLE = ["layers.0.attn_norm", "layers.0.wq", "layers.0.ffn_norm"]
 
 
