@@ -219,15 +219,16 @@ def test_host_buffer_entry_point(iso):
     assert torch.equal(th_h, th.cpu()) and torch.equal(b_h, b.cpu())
 
 
-def test_llama_180m_k8_sampled(iso):
-    """The benchmarked configuration (180M shapes, K = 8), full size on the GPU,
-    checked on one matrix of each shape bucket plus every 1-D tensor."""
-    wl = W.make_workload("llama_180m_k8", seed=0, device="cuda")
+def sampled_parity(iso, workload, pick_names):
+    """A configuration at full size on the GPU (the launch configuration bench.py times),
+    checked against the oracle on the sampled matrices plus every 1-D tensor (each matrix's
+    Iso-C and each element's Nesterov step are independent of the others)."""
+    wl = W.make_workload(workload, seed=0, device="cuda")
     sp = wl.spec
     rc, th, b, upd, diag, plan = run_gpu(iso, wl, sp.alpha, sp.outer_lr, sp.momentum)
     assert rc == 0
     names = [s[0] for s in sp.shapes]
-    pick = [names.index(n) for n in ("layers.0.wq", "layers.5.w_gate", "layers.11.w_down", "head")]
+    pick = [names.index(n) for n in pick_names]
     pick += [i for i, s in enumerate(sp.shapes) if s[2] == 0]
     # the oracle gets only the sampled tensors, re-packed densely (host copies of the inputs)
     sub_table, parts, off = [], [], 0
@@ -247,4 +248,22 @@ def test_llama_180m_k8_sampled(iso):
     worst = check_step(sub_table, th[idx].double().cpu().numpy(), b[idx].double().cpu().numpy(),
                        upd[idx].double().cpu().numpy(), sig, ref)
     assert all(s == 0 for s in diag["status"])
-    print("worst errors", worst, "iterations", sorted(set(diag["iters"])))
+    print(workload, "worst errors", worst, "iterations", sorted(set(diag["iters"])))
+    del wl, th, b, upd, plan
+    torch.cuda.empty_cache()
+
+
+def test_llama_180m_k8_sampled(iso):
+    """The benchmarked configuration (180M shapes, K = 8): one matrix of each shape bucket."""
+    sampled_parity(iso, "llama_180m_k8", ("layers.0.wq", "layers.5.w_gate", "layers.11.w_down", "head"))
+
+
+@pytest.mark.parametrize("workload,pick", [
+    ("llama_180m_k16", ("layers.3.wk", "layers.7.w_up", "layers.0.w_down")),
+    ("llama_1b_k8", ("layers.0.wq", "layers.11.w_gate", "layers.23.w_down")),
+    ("llama_3b_k4", ("layers.0.wv",)),   # bf16 replicas; 3072-wide matrices keep the oracle sample small
+])
+def test_larger_configs_sampled(iso, workload, pick):
+    """The other configurations at full size (up to 3.4e9 parameters with 4 bf16 replicas),
+    sampled matrices plus every 1-D tensor."""
+    sampled_parity(iso, workload, pick)
