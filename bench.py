@@ -91,16 +91,22 @@ class ClockSampler:
 
 
 # --------------------------------------------------------------------------- accounting
-def gemm_flops(table, diag):
+def gemm_flops(table, diag, fast=False):
     """Algorithmic (single-pass) FLOPs of the polar GEMMs of one step, per phase, from
     the per-matrix iteration counts: a full Gram 2*r*n^2 per iteration (symmetry not
     discounted), G^2 = 2*n^3 per quintic step, an update 2*r*n^2 per iteration
-    (r = long side, n = short side of the matrix)."""
+    (r = long side, n = short side of the matrix).  The fast variant runs `it` quintic
+    steps and no polish."""
     out = {"gram": 0.0, "poly": 0.0, "update": 0.0}
     mats = [(r, c) for (_, r, c) in table if c > 0]
     for (r, c), it, st in zip(mats, diag["iters"], diag["status"]):
         big, small = max(r, c), min(r, c)
         gram1, sq1 = 2.0 * big * small * small, 2.0 * small ** 3
+        if fast:
+            out["gram"] += it * gram1
+            out["poly"] += it * sq1
+            out["update"] += it * gram1
+            continue
         if it == 0:
             out["gram"] += gram1  # one Gram, then found zero
             continue
@@ -111,7 +117,7 @@ def gemm_flops(table, diag):
     return out
 
 
-BM, BN, BK = 128, 256, 32
+BM, BN, BK = 256, 256, 32   # output tile of one CTA pair (tcgen05 cta_group::2)
 
 
 def _sym_tiles(n):
@@ -123,7 +129,7 @@ def _sym_tiles(n):
     return c
 
 
-def gemm_exec_flops(table, diag):
+def gemm_exec_flops(table, diag, fast=False):
     """Tensor-core FLOPs the GEMM launches execute per phase: 2*BM*BN*K_padded per
     computed tile and per 16-bit pass (3 passes at iteration 0 and in the final polish
     update, 2 elsewhere), symmetric Grams/G^2 on their upper-triangle tiles only."""
@@ -135,6 +141,11 @@ def gemm_exec_flops(table, diag):
         gram1 = _sym_tiles(n) * BM * BN * 2.0 * kpad_big
         poly1 = _sym_tiles(n) * BM * BN * 2.0 * kpad_n
         upd1 = (-(-r // BM)) * (-(-c // BN)) * BM * BN * 2.0 * kpad_n
+        if fast:   # `it` quintic steps, every one with three passes; no polish
+            out["gram"] += 3 * gram1 * it
+            out["poly"] += 3 * poly1 * it
+            out["update"] += 3 * upd1 * it
+            continue
         if it == 0:
             out["gram"] += 3 * gram1
             continue
@@ -222,6 +233,8 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--fast-steps", type=int, default=0,
+                    help="time the fast variant of Sec. 4.3 (k fixed polar steps, rms sigma_bar); 0 = exact")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     if args.impl == "reference":
@@ -248,7 +261,7 @@ def main():
     spec = W.SPECS[args.workload]
     wl = W.make_workload(spec, seed=rank, device="cuda")
     plan = isoloco.Plan(wl.table, wl.N, wl.K, wl.replicas.dtype)
-    opts = isoloco.make_opts(spec.alpha, spec.outer_lr, spec.momentum)
+    opts = isoloco.make_opts(spec.alpha, spec.outer_lr, spec.momentum, fast_steps=args.fast_steps)
     theta0, mom0 = wl.theta.clone(), wl.momentum.clone()
     th, b = wl.theta, wl.momentum
     stream = torch.cuda.current_stream()
@@ -332,8 +345,8 @@ def main():
         return 0
 
     peaks, peak_src = load_peaks()
-    fl = gemm_flops(wl.table, diag)
-    fx = gemm_exec_flops(wl.table, diag)
+    fl = gemm_flops(wl.table, diag, fast=args.fast_steps > 0)
+    fx = gemm_exec_flops(wl.table, diag, fast=args.fast_steps > 0)
     flops = sum(fl.values()) * args.steps
     xflops = sum(fx.values()) * args.steps
     gemm_ms = prof["gram"][0] + prof["poly"][0] + prof["update"][0]
@@ -399,7 +412,9 @@ def main():
                                                                       wl.replicas.element_size() / 1e9),
                    "timing": "sum of per-step CUDA-event intervals on the launch stream; theta/B "
                              "restored between steps outside the intervals",
-                   "parallelism": f"replicas x{world}"},
+                   "parallelism": f"replicas x{world}",
+                   "iso_c": ("exact polar, sigma_bar = tr(Q^T Delta)/r" if not args.fast_steps else
+                             f"fast variant: {args.fast_steps} fixed polar steps, sigma_bar = ||Delta||_F/sqrt(r)")},
         "status": isoloco.STATUS_NAMES.get(status, status),
         "polar_iters": {"min": min(iters), "max": max(iters), "mean": sum(iters) / len(iters)},
         "phases_ms_per_step": phases_ms, "phases_algorithmic_tflops": phases_tflops,

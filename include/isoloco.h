@@ -76,6 +76,12 @@ typedef struct {
     int max_iter;     /* cap on quintic polar steps per matrix; <= 0 selects 28. */
     float tol;        /* convergence test ||X^T X - I||_F / sqrt(n) < tol; <= 0 selects 4e-3. */
     int sync;         /* 1: synchronize `stream` and return the step's device status. */
+    int fast_steps;   /* 0: exact Iso-C (polar factor to convergence, sigma_bar = tr(Q^T Delta) / r).
+                       * k in 1..64: the fast variant of Sec. 4.3 -- exactly k quintic steps of
+                       * the standard schedule from X_0 = Delta / ||Delta^T Delta||_F^(1/2) (steps
+                       * after its seventh repeat the seventh), no convergence test and no
+                       * polish, and sigma_bar = ||Delta||_F / sqrt(r) (the RMS of the singular
+                       * values); the paper runs 5. */
 } isoloco_opts_t;
 
 /* Fills *opts with alpha = 1, outer_lr = 0.7, momentum = 0.9 (the paper's DiLoCo

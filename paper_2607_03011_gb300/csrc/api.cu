@@ -30,7 +30,8 @@ __global__ void k_gram_finalize(const MatDesc*, const int2*, const MatState*, co
                                 const int64_t*, const int*, __nv_bfloat16*, __nv_bfloat16*, float*, int,
                                 __nv_bfloat16*);
 __global__ void k_control(const MatDesc*, int, MatState*, const float*, int, int, float, uint32_t*, const int*,
-                          const int*, int, int*, int*, int*, int*, cudaGraphConditionalHandle, int, long long*);
+                          const int*, int, int*, int*, int*, int*, cudaGraphConditionalHandle, int, long long*,
+                          int);
 __global__ void k_trace_partial(const MatDesc*, const int4*, const MatState*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, double*);
@@ -125,6 +126,8 @@ struct isoloco_plan {
     cudaGraphExec_t gexec = nullptr;
     int g_max_iter = -1;
     float g_tol = 0.f;
+    int g_fast = -1;
+    int fast_steps = 0;             // this call's fast-variant step count (0: exact Iso-C)
     int64_t body_launches = 0;      // kernels in one run of the body
     long long* loopc = nullptr;     // device: [0] body runs in this call, [1] body runs ever
     // phase timing (isoloco_profile_enable) and launch counting
@@ -602,11 +605,18 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
         const int dst = (t + 1) & 1;
         // ---- Gram G = X^T X (tall, MN-major operands) or X X^T (wide, K-major)
         const bool first = (t == 0);
-        const Precision gram_pr = first ? Precision{0, 0, 1, 1, 0} : Precision{1, 1, 1, 0, 0};
+        // The fast variant stops after a fixed number of steps, so nothing corrects a step's
+        // rounding afterwards: every step splits both operands (fp16 three passes) and the
+        // polynomial is formed from G's hi/lo planes (no single-plane Y).  The converging
+        // path keeps one operand single from iteration 1 on (its rounding only perturbs the
+        // spectrum, which later steps correct).
+        const bool full = p->fast_steps > 0;
+        const Precision gram_pr = first ? Precision{0, 0, 1, 1, 0}
+                                        : (full ? Precision{1, 1, 1, 1, 0} : Precision{1, 1, 1, 0, 0});
         LaunchSet tall, wide;
         init_set(tall, kEpiGram, kGateActive, p, gram_pr);
         init_set(wide, kEpiGram, kGateActive, p, gram_pr);
-        tall.p.gram_y = wide.p.gram_y = first ? 0 : 1;
+        tall.p.gram_y = wide.p.gram_y = (first || full) ? 0 : 1;
         for (size_t b = 0; b < p->buckets.size(); ++b) {
             const Bucket& bk = p->buckets[b];
             const CUtensorMap* m = maps + b * kMapsPerBucket;
@@ -643,25 +653,27 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
             PhaseTimer tm(p, ISOLOCO_PHASE_FINALIZE, st);
             k_gram_finalize<<<p->nftiles, 256, 0, st>>>(p->mats_d, p->ftiles, p->state, p->gpart, p->gpart_off_d,
                                                         p->gpart_sstride_d, p->nsplit_d, p->ghi, p->glo,
-                                                        p->fin_part, first ? 0 : 1, first ? nullptr : p->ypl);
+                                                        p->fin_part, first ? 0 : 1, (first || full) ? nullptr : p->ypl);
             CUDA_TRY(cudaGetLastError());
         }
         { PhaseTimer tm(p, ISOLOCO_PHASE_CONTROL, st);
         k_control<<<1, 1024, 0, st>>>(p->mats_d, p->nmat, p->state, p->fin_part, t, max_iter, tol, p->err_d,
                                       p->bucket_first_d, p->bucket_count_d, (int)p->buckets.size(), p->list_gram,
-                                      p->cnt_gram, p->list_step, p->cnt_step, cond, set_cond, p->loopc); }
+                                      p->cnt_gram, p->list_step, p->cnt_step, cond, set_cond, p->loopc,
+                                      p->fast_steps); }
         CUDA_TRY(cudaGetLastError());
         // ---- P = a I + b G + c G^2
         LaunchSet poly;
-        init_set(poly, kEpiPoly, kGateStep, p, first ? Precision{0, 0, 1, 1, 0} : Precision{1, 1, 1, 0, 0});
-        poly.p.poly_horner = first ? 0 : 1;
+        init_set(poly, kEpiPoly, kGateStep, p,
+                 first ? Precision{0, 0, 1, 1, 0} : (full ? Precision{1, 1, 1, 1, 0} : Precision{1, 1, 1, 0, 0}));
+        poly.p.poly_horner = (first || full) ? 0 : 1;
         for (size_t b = 0; b < p->buckets.size(); ++b) {
             const Bucket& bk = p->buckets[b];
             const CUtensorMap* m = maps + b * kMapsPerBucket;
             GemmGroup g{};
             g.a_hi = m + g_map(kRoleKA, 0);
             g.a_lo = m + g_map(kRoleKA, 1);
-            g.b_hi = first ? m + g_map(kRoleKB, 0) : m + y_map();  // G G (t = 0) or G Y
+            g.b_hi = (first || full) ? m + g_map(kRoleKB, 0) : m + y_map();  // G G or G Y (Horner)
             g.b_lo = m + g_map(kRoleKB, 1);
             set_group_common(g, bk.n, bk.n, bk.n, bk.count, 1, bk.mat_base);
             g.bucket = (int)b;
@@ -681,8 +693,10 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
         // X_{t+1} is always written as fp16 planes; X is the split operand (A when tall,
         // B when wide), P the single one except in the polish step (3 passes)
         LaunchSet utall, uwide;
-        init_set(utall, kEpiXSplit, kGateStep, p, first ? Precision{0, 1, 1, 1, 0} : Precision{1, 1, 1, 0, 1});
-        init_set(uwide, kEpiXSplit, kGateStep, p, first ? Precision{0, 1, 1, 1, 0} : Precision{1, 1, 0, 1, 1});
+        init_set(utall, kEpiXSplit, kGateStep, p,
+                 first ? Precision{0, 1, 1, 1, 0} : (full ? Precision{1, 1, 1, 1, 0} : Precision{1, 1, 1, 0, 1}));
+        init_set(uwide, kEpiXSplit, kGateStep, p,
+                 first ? Precision{0, 1, 1, 1, 0} : (full ? Precision{1, 1, 1, 1, 0} : Precision{1, 1, 0, 1, 1}));
         for (size_t b = 0; b < p->buckets.size(); ++b) {
             const Bucket& bk = p->buckets[b];
             const CUtensorMap* m = maps + b * kMapsPerBucket;
@@ -770,6 +784,7 @@ static int build_polar_graph(isoloco_plan* p, int max_iter, float tol) {
     p->graph = g;
     p->g_max_iter = max_iter;
     p->g_tol = tol;
+    p->g_fast = p->fast_steps;
     return ISOLOCO_OK;
 }
 
@@ -786,7 +801,7 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
     CUDA_TRY(cudaStreamIsCapturing(st, &cs));
     const bool use_graph = kPairMma && !p->prof && cs == cudaStreamCaptureStatusNone;
     if (use_graph) {
-        if (!p->gexec || p->g_max_iter != max_iter || p->g_tol != tol)
+        if (!p->gexec || p->g_max_iter != max_iter || p->g_tol != tol || p->g_fast != p->fast_steps)
             if ((rc = build_polar_graph(p, max_iter, tol))) return rc;
         CUDA_TRY(cudaGraphLaunch(p->gexec, st));
     } else {
@@ -804,6 +819,7 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             }
         }
     }
+    if (p->fast_steps) return ISOLOCO_OK;  // the fast variant's sigma_bar comes from ||Delta||_F
     { PhaseTimer tm(p, ISOLOCO_PHASE_TRACE, st, 2);
     k_trace_partial<<<p->ntchunks, 256, 0, st>>>(p->mats_d, p->tchunks, p->state, p->dhi, p->dlo, p->xhi[0],
                                                  p->xlo[0], p->xhi[1], p->xlo[1], p->tpart);
@@ -826,6 +842,7 @@ static int check_opts(const isoloco_opts_t* o, isoloco_opts_t* out) {
     if (out->max_iter <= 0) out->max_iter = kDefaultMaxIter;
     if (out->max_iter > 200) return fail(ISOLOCO_ERR_INVALID, "max_iter must be <= 200");
     if (!(out->tol > 0.f)) out->tol = kDefaultTol;
+    if (out->fast_steps < 0 || out->fast_steps > 64) return fail(ISOLOCO_ERR_INVALID, "fast_steps must be in 0..64");
     return ISOLOCO_OK;
 }
 
@@ -863,7 +880,8 @@ static int run_isoc_step(isoloco_plan* p, int merge, float* theta, float* mom, c
                                              p->dlo, p->d1d, p->err_d);
         CUDA_TRY(cudaGetLastError());
     }
-    if ((rc = run_polar(p, o.max_iter, o.tol, st))) return rc;
+    p->fast_steps = merge ? 0 : o.fast_steps;
+    if ((rc = run_polar(p, p->fast_steps ? std::max(o.max_iter, o.fast_steps) : o.max_iter, o.tol, st))) return rc;
     UpdateSrc us;
     us.qh[0] = p->xhi[0];
     us.qh[1] = p->xhi[1];
@@ -897,6 +915,7 @@ int isoloco_opts_default(isoloco_opts_t* o) {
     o->max_iter = kDefaultMaxIter;
     o->tol = kDefaultTol;
     o->sync = 0;
+    o->fast_steps = 0;
     return ISOLOCO_OK;
 }
 

@@ -163,7 +163,7 @@ __device__ __forceinline__ const float* sched_row(bool deep, int step) {
 // Decision for matrix mi, taken by one warp.  t: iteration index (0 = first Gram of Delta).
 __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatState* __restrict__ state,
                                const float* __restrict__ fin_part, int t, int max_iter, float tol,
-                               uint32_t* __restrict__ err, int lane) {
+                               uint32_t* __restrict__ err, int lane, int fast_steps) {
     MatState& st = state[mi];
     if (st.done) {
         if (lane == 0) st.mode = 0;
@@ -212,6 +212,9 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
         }
         gscale = 1.0 / s2;
         xscale = 1.0 / sqrt(s2);
+        // fast variant (Sec. 4.3): sigma_bar = RMS of the singular values = ||Delta||_F / sqrt(r),
+        // with ||Delta||_F^2 = tr(Delta^T Delta), the trace of this Gram
+        if (fast_steps) st.sigma_bar = static_cast<float>(sqrt(fmax(0.0, tr) / n));
         // ||G/s2 - I||_F^2 = ||G||^2/s2^2 - 2 tr(G)/s2 + n, with ||G||^2/s2^2 = 1
         d = sqrt(fmax(0.0, 1.0 - 2.0 * tr * gscale + n) / n);
     } else {
@@ -226,7 +229,22 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
         st.final_buf = 2;
         return;
     }
-    if (d < tol) {
+    if (fast_steps) {
+        // fast variant: a fixed number of standard quintic steps, no test, no polish (steps
+        // after the schedule's last repeat it); the last one leaves Q in the buffer its
+        // update writes
+        const float* q = kSched[st.step < kSchedSteps ? st.step : kSchedSteps - 1];
+        st.mode = 1;
+        st.a = q[0];
+        st.b = static_cast<float>(q[1] * gscale);
+        st.c = static_cast<float>(q[2] * gscale * gscale);
+        st.step += 1;
+        st.iters += 1;
+        if (st.iters >= fast_steps) {
+            st.done = 1;
+            st.final_buf = (t + 1) & 1;
+        }
+    } else if (d < tol) {
         // Cubic polish p(x) = 1.5 x - 0.5 x^3 on singular values already near 1.
         st.mode = 2;
         st.a = 1.5f;
@@ -273,11 +291,11 @@ __global__ void __launch_bounds__(1024) k_control(const MatDesc* __restrict__ ma
                                                   int* __restrict__ list_gram, int* __restrict__ cnt_gram,
                                                   int* __restrict__ list_step, int* __restrict__ cnt_step,
                                                   cudaGraphConditionalHandle cond, int set_cond,
-                                                  long long* __restrict__ loopc) {
+                                                  long long* __restrict__ loopc, int fast_steps) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (t == 0 && threadIdx.x == 0) loopc[0] = 0;
     for (int mi = warp; mi < nmat; mi += 32) {
-        control_matrix(mats, mi, state, fin_part, t, max_iter, tol, err, lane);
+        control_matrix(mats, mi, state, fin_part, t, max_iter, tol, err, lane, fast_steps);
         __syncwarp();
     }
     __syncthreads();

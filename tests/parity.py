@@ -14,6 +14,19 @@ def oracle_step(table, theta, mom, reps, alpha, eta, mu, only=None, reduce_mean=
                                      reduce_mean=reduce_mean)
 
 
+def oracle_fast_step(table, theta, mom, reps, alpha, eta, mu, steps, only=None):
+    """The fast variant (Sec. 4.3) in fp64: the oracle's reduction, then its own fixed-step
+    schedule (oracle/fast_ns.py) on every 2-D tensor and Nesterov."""
+    from oracle import fast_ns
+    th = theta.detach().cpu().numpy().astype(np.float32)
+    b = mom.detach().cpu().numpy().astype(np.float32)
+    delta = oracle.pseudo_gradient(th, W.replicas_as_numpy(reps), mode=0)
+    ref = fast_ns.isoloco_outer_step_fast(table, th, b, delta, alpha, eta, mu, fast_ns.fast_schedule(steps),
+                                          only=only)
+    ref["theta_in"] = th.astype(np.float64)
+    return ref
+
+
 def rel_fro(a, b):
     a = np.asarray(a, np.float64); b = np.asarray(b, np.float64)
     nb = np.linalg.norm(b)

@@ -11,7 +11,7 @@ import torch
 
 import oracle
 from paper_2607_03011_gb300 import workloads as W
-from parity import check_step, elementwise_rel, oracle_step, rel_fro
+from parity import check_step, elementwise_rel, oracle_fast_step, oracle_step, rel_fro
 
 pytestmark = pytest.mark.gpu
 
@@ -24,13 +24,14 @@ def iso():
 
 
 def run_gpu(iso, wl, alpha, eta, mu, reps=None, theta=None, mom=None, max_iter=0, reduce_mean=True,
-            plan=None):
+            plan=None, fast_steps=0):
     plan = plan or iso.Plan(wl.table, wl.N, wl.K, wl.replicas.dtype)
     th = (wl.theta if theta is None else theta).clone()
     b = (wl.momentum if mom is None else mom).clone()
     upd = torch.empty_like(th)
     rc = plan.outer_step(th, b, wl.replicas if reps is None else reps,
-                         iso.make_opts(alpha, eta, mu, reduce_mean=reduce_mean, max_iter=max_iter, sync=True),
+                         iso.make_opts(alpha, eta, mu, reduce_mean=reduce_mean, max_iter=max_iter, sync=True,
+                                       fast_steps=fast_steps),
                          update_out=upd)
     diag = plan.read_diag()
     return rc, th, b, upd, diag, plan
@@ -180,6 +181,39 @@ def test_graph_loop_matches_per_launch_loop(iso):
         assert lh <= lg <= lh + lh // 2, (lg, lh)
 
 
+# ---- the fast variant of Sec. 4.3: a fixed number of quintic steps, sigma_bar = ||Delta||_F / sqrt(r)
+
+@pytest.mark.parametrize("steps", [5, 3, 8])
+def test_fast_variant_ragged(iso, steps):
+    """Odd and even step counts (Q in either ping-pong buffer), ragged tiles, 1-D tensors."""
+    spec = W.custom_spec(RAGGED, K=3, rank=2, momentum_std=1e-4)
+    wl = W.make_workload(spec, seed=11, device="cuda")
+    rc, th, b, upd, diag, _ = run_gpu(iso, wl, 1.0, 0.7, 0.9, fast_steps=steps)
+    assert rc == 0
+    assert diag["iters"] == [steps] * len(diag["iters"]) and not any(diag["status"])
+    ref = oracle_fast_step(wl.table, wl.theta, wl.momentum, wl.replicas, 1.0, 0.7, 0.9, steps)
+    check_step(wl.table, th.double().cpu().numpy(), b.double().cpu().numpy(), upd.double().cpu().numpy(),
+               diag["sigma_bar"], ref)
+
+
+def test_fast_variant_tiny(iso):
+    wl = W.make_workload("tiny", seed=0, device="cuda")
+    sp = wl.spec
+    rc, th, b, upd, diag, _ = run_gpu(iso, wl, sp.alpha, sp.outer_lr, sp.momentum, fast_steps=5)
+    assert rc == 0
+    ref = oracle_fast_step(wl.table, wl.theta, wl.momentum, wl.replicas, sp.alpha, sp.outer_lr, sp.momentum, 5)
+    check_step(wl.table, th.double().cpu().numpy(), b.double().cpu().numpy(), upd.double().cpu().numpy(),
+               diag["sigma_bar"], ref)
+    # the fast update is not the exact one: the rms proxy exceeds the mean singular value
+    exact = run_gpu(iso, wl, sp.alpha, sp.outer_lr, sp.momentum)[4]
+    assert all(f > e for f, e in zip(diag["sigma_bar"], exact["sigma_bar"]))
+
+
+def test_fast_variant_180m_sampled(iso):
+    """The benchmarked configuration at full size with the paper's 5 fixed steps."""
+    sampled_parity(iso, "llama_180m_k8", ("layers.0.wq", "layers.5.w_gate", "layers.11.w_down"), fast_steps=5)
+
+
 def test_diloco_outer_step(iso):
     spec = W.custom_spec(RAGGED, K=3, rank=2, momentum_std=1e-4)
     wl = W.make_workload(spec, seed=6, device="cuda")
@@ -219,13 +253,13 @@ def test_host_buffer_entry_point(iso):
     assert torch.equal(th_h, th.cpu()) and torch.equal(b_h, b.cpu())
 
 
-def sampled_parity(iso, workload, pick_names):
+def sampled_parity(iso, workload, pick_names, fast_steps=0):
     """A configuration at full size on the GPU (the launch configuration bench.py times),
     checked against the oracle on the sampled matrices plus every 1-D tensor (each matrix's
     Iso-C and each element's Nesterov step are independent of the others)."""
     wl = W.make_workload(workload, seed=0, device="cuda")
     sp = wl.spec
-    rc, th, b, upd, diag, plan = run_gpu(iso, wl, sp.alpha, sp.outer_lr, sp.momentum)
+    rc, th, b, upd, diag, plan = run_gpu(iso, wl, sp.alpha, sp.outer_lr, sp.momentum, fast_steps=fast_steps)
     assert rc == 0
     names = [s[0] for s in sp.shapes]
     pick = [names.index(n) for n in pick_names]
@@ -239,9 +273,13 @@ def sampled_parity(iso, workload, pick_names):
         parts.append((o, n))
         off += n
     idx = torch.cat([torch.arange(o, o + n, device="cuda") for o, n in parts])
-    ref = oracle.isoloco_outer_step(sub_table, wl.theta[idx].cpu().numpy(), wl.momentum[idx].cpu().numpy(),
-                                    W.replicas_as_numpy(wl.replicas[:, idx]), alpha=sp.alpha,
-                                    eta=sp.outer_lr, mu=sp.momentum)
+    if fast_steps:
+        ref = oracle_fast_step(sub_table, wl.theta[idx], wl.momentum[idx], wl.replicas[:, idx], sp.alpha,
+                               sp.outer_lr, sp.momentum, fast_steps)
+    else:
+        ref = oracle.isoloco_outer_step(sub_table, wl.theta[idx].cpu().numpy(), wl.momentum[idx].cpu().numpy(),
+                                        W.replicas_as_numpy(wl.replicas[:, idx]), alpha=sp.alpha,
+                                        eta=sp.outer_lr, mu=sp.momentum)
     ref["theta_in"] = wl.theta[idx].double().cpu().numpy()
     mat_index = {p: j for j, p in enumerate([i for i, s in enumerate(sp.shapes) if s[2] > 0])}
     sig = [diag["sigma_bar"][mat_index[i]] for i in pick if sp.shapes[i][2] > 0]
