@@ -82,6 +82,16 @@ typedef struct {
                        * after its seventh repeat the seventh), no convergence test and no
                        * polish, and sigma_bar = ||Delta||_F / sqrt(r) (the RMS of the singular
                        * values); the paper runs 5. */
+    /* The ablations of Sec. 4.5 and App. B (all 0 by default = Alg. 2): */
+    int orth_target;   /* 0: Iso-C of Delta.  1: of the momentum update instead: B <- mu B + Delta,
+                        * P <- Delta + mu B (or P <- B with standard momentum), then
+                        * theta <- theta - eta * Iso(P) for 2-D tensors and theta - eta * P for
+                        * 1-D ones (sigma_bar = tr(Q^T P) / r). */
+    int momentum_kind; /* 0: Nesterov (Alg. 2).  1: standard momentum, B <- mu B + U and
+                        * theta <- theta - eta B. */
+    int scale_kind;    /* 0: the Iso-C scale sigma_bar.  1: Muon's spectral scale, U = alpha *
+                        * sqrt(rows / cols) * Q for a rows x cols tensor (App. B; sigma_bar is
+                        * then not computed). */
 } isoloco_opts_t;
 
 /* Fills *opts with alpha = 1, outer_lr = 0.7, momentum = 0.9 (the paper's DiLoCo

@@ -40,8 +40,10 @@ __global__ void k_reset_state(MatState*, int, uint32_t*, const MatDesc*, const i
                               int*, int);
 __global__ void k_reduce(const Chunk*, const MatDesc*, ReplicaPtrs, int, int, const float*, float,
                          __nv_bfloat16*, __nv_bfloat16*, float*, uint32_t*);
+__global__ void k_reduce_p(const Chunk*, const MatDesc*, ReplicaPtrs, int, int, const float*, float,
+                           __nv_bfloat16*, __nv_bfloat16*, float*, uint32_t*, int, float, const float*, float*);
 __global__ void k_apply(const Chunk*, const MatDesc*, const MatState*, UpdateSrc, int, float, float, float,
-                        float*, float*, const float*, float*, float*, const uint32_t*);
+                        float*, float*, const float*, float*, float*, const uint32_t*, int, int, int, const float*);
 __global__ void k_diloco(ReplicaPtrs, int, int, float*, float*, int64_t, float, float, float, uint32_t*);
 __global__ void k_split_planes(const float*, int64_t, int, int, int, __nv_bfloat16*, __nv_bfloat16*, int);
 
@@ -128,6 +130,8 @@ struct isoloco_plan {
     float g_tol = 0.f;
     int g_fast = -1;
     int fast_steps = 0;             // this call's fast-variant step count (0: exact Iso-C)
+    bool skip_trace = false;        // this call needs no tr(Q^T Delta) (fast variant, spectral scale)
+    float* bnew = nullptr;          // B' of the orthogonalise-P ablation (allocated on first use)
     int64_t body_launches = 0;      // kernels in one run of the body
     long long* loopc = nullptr;     // device: [0] body runs in this call, [1] body runs ever
     // phase timing (isoloco_profile_enable) and launch counting
@@ -819,7 +823,7 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             }
         }
     }
-    if (p->fast_steps) return ISOLOCO_OK;  // the fast variant's sigma_bar comes from ||Delta||_F
+    if (p->skip_trace) return ISOLOCO_OK;  // sigma_bar from ||Delta||_F (fast) or not used (spectral)
     { PhaseTimer tm(p, ISOLOCO_PHASE_TRACE, st, 2);
     k_trace_partial<<<p->ntchunks, 256, 0, st>>>(p->mats_d, p->tchunks, p->state, p->dhi, p->dlo, p->xhi[0],
                                                  p->xlo[0], p->xhi[1], p->xlo[1], p->tpart);
@@ -843,6 +847,9 @@ static int check_opts(const isoloco_opts_t* o, isoloco_opts_t* out) {
     if (out->max_iter > 200) return fail(ISOLOCO_ERR_INVALID, "max_iter must be <= 200");
     if (!(out->tol > 0.f)) out->tol = kDefaultTol;
     if (out->fast_steps < 0 || out->fast_steps > 64) return fail(ISOLOCO_ERR_INVALID, "fast_steps must be in 0..64");
+    if (out->orth_target < 0 || out->orth_target > 1 || out->momentum_kind < 0 || out->momentum_kind > 1 ||
+        out->scale_kind < 0 || out->scale_kind > 1)
+        return fail(ISOLOCO_ERR_INVALID, "orth_target, momentum_kind and scale_kind must be 0 or 1");
     return ISOLOCO_OK;
 }
 
@@ -868,6 +875,13 @@ static int run_isoc_step(isoloco_plan* p, int merge, float* theta, float* mom, c
     CUDA_TRY(cudaSetDevice(p->device));
     const float* th_src = merge ? base : theta;
     const float scale = merge ? -1.f : (o.reduce_mean ? 1.f / (float)p->K : 1.f);
+    // orthogonalise-P ablation: the reduce pass takes the momentum step on the raw Delta and
+    // keeps B' aside, so that a non-finite Delta still leaves B untouched
+    const int pmode = (!merge && o.orth_target) ? (o.momentum_kind ? 2 : 1) : 0;
+    if (pmode && !p->bnew) {
+        const int rc2 = dalloc(p, &p->bnew, p->N);
+        if (rc2) return rc2;
+    }
     { PhaseTimer tm(p, ISOLOCO_PHASE_OTHER, st);
     k_reset_state<<<(std::max(1, p->nmat) + 255) / 256, 256, 0, st>>>(
         p->state, p->nmat, p->err_d, p->mats_d, p->bucket_first_d, p->bucket_count_d, (int)p->buckets.size(),
@@ -876,11 +890,16 @@ static int run_isoc_step(isoloco_plan* p, int merge, float* theta, float* mom, c
     CUDA_TRY(cudaGetLastError());
     if (p->nchunks) {
         PhaseTimer tm(p, ISOLOCO_PHASE_REDUCE, st);
-        k_reduce<<<p->nchunks, 256, 0, st>>>(p->chunks_d, p->mats_d, rp, p->K, p->dtype, th_src, scale, p->dhi,
-                                             p->dlo, p->d1d, p->err_d);
+        if (pmode)
+            k_reduce_p<<<p->nchunks, 256, 0, st>>>(p->chunks_d, p->mats_d, rp, p->K, p->dtype, th_src, scale,
+                                                   p->dhi, p->dlo, p->d1d, p->err_d, pmode, o.momentum, mom, p->bnew);
+        else
+            k_reduce<<<p->nchunks, 256, 0, st>>>(p->chunks_d, p->mats_d, rp, p->K, p->dtype, th_src, scale, p->dhi,
+                                                 p->dlo, p->d1d, p->err_d);
         CUDA_TRY(cudaGetLastError());
     }
     p->fast_steps = merge ? 0 : o.fast_steps;
+    p->skip_trace = !merge && (o.fast_steps > 0 || o.scale_kind == 1);
     if ((rc = run_polar(p, p->fast_steps ? std::max(o.max_iter, o.fast_steps) : o.max_iter, o.tol, st))) return rc;
     UpdateSrc us;
     us.qh[0] = p->xhi[0];
@@ -892,10 +911,11 @@ static int run_isoc_step(isoloco_plan* p, int merge, float* theta, float* mom, c
         PhaseTimer tm(p, ISOLOCO_PHASE_APPLY, st);
         if (merge)
             k_apply<<<p->nchunks, 256, 0, st>>>(p->chunks_d, p->mats_d, p->state, us, 1, alpha_merge, 0.f, 0.f,
-                                                nullptr, nullptr, base, out, nullptr, p->err_d);
+                                                nullptr, nullptr, base, out, nullptr, p->err_d, 0, 0, 0, nullptr);
         else
             k_apply<<<p->nchunks, 256, 0, st>>>(p->chunks_d, p->mats_d, p->state, us, 0, o.alpha, o.outer_lr,
-                                                o.momentum, theta, mom, nullptr, nullptr, upd_out, p->err_d);
+                                                o.momentum, theta, mom, nullptr, nullptr, upd_out, p->err_d,
+                                                o.momentum_kind, pmode, o.scale_kind, p->bnew);
         CUDA_TRY(cudaGetLastError());
     }
     return finish_call(p, st, o.sync);
@@ -916,6 +936,9 @@ int isoloco_opts_default(isoloco_opts_t* o) {
     o->tol = kDefaultTol;
     o->sync = 0;
     o->fast_steps = 0;
+    o->orth_target = 0;
+    o->momentum_kind = 0;
+    o->scale_kind = 0;
     return ISOLOCO_OK;
 }
 

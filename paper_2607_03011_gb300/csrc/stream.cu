@@ -35,15 +35,28 @@ __device__ __forceinline__ void raise_nonfinite(bool bad, uint32_t* err) {
     if (__any_sync(0xffffffffu, bad) && (threadIdx.x & 31) == 0) atomicOr(err, kErrNonFinite);
 }
 
-// grid: one CTA per chunk.
-__global__ void __launch_bounds__(kStreamThreads) k_reduce(const Chunk* __restrict__ chunks,
-                                                           const MatDesc* __restrict__ mats,
-                                                           ReplicaPtrs reps, int K, int dtype,
-                                                           const float* __restrict__ theta, float scale,
-                                                           __nv_bfloat16* __restrict__ dhi,
-                                                           __nv_bfloat16* __restrict__ dlo,
-                                                           float* __restrict__ d1d,
-                                                           uint32_t* __restrict__ err) {
+// The value the polar iteration (2-D) or the apply pass (1-D) receives for one element of
+// Delta: Delta itself, or with pmode (orthogonalise the update P instead of Delta) the
+// momentum step taken first on the raw Delta, B' = mu B + Delta (written to bnew), and
+// P = Delta + mu B' (pmode 1, Nesterov) or P = B' (pmode 2, standard momentum).
+__device__ __forceinline__ float reduce_out(float d, int pmode, float mu, const float* __restrict__ mom,
+                                            float* __restrict__ bnew, int64_t i) {
+    if (!pmode) return d;
+    const float nb = fmaf(mu, __ldg(mom + i), d);
+    bnew[i] = nb;
+    return pmode == 1 ? fmaf(mu, nb, d) : nb;
+}
+
+// One CTA per chunk.  PM: the orthogonalise-P ablation (its own kernel, so that the
+// default reduction keeps its registers).
+template <bool PM>
+__device__ __forceinline__ void reduce_chunk(const Chunk* __restrict__ chunks, const MatDesc* __restrict__ mats,
+                                             const ReplicaPtrs& reps, int K, int dtype,
+                                             const float* __restrict__ theta, float scale,
+                                             __nv_bfloat16* __restrict__ dhi, __nv_bfloat16* __restrict__ dlo,
+                                             float* __restrict__ d1d, uint32_t* __restrict__ err, int pmode_arg,
+                                             float mu, const float* __restrict__ mom, float* __restrict__ bnew) {
+    const int pmode = PM ? pmode_arg : 0;
     const Chunk ch = chunks[blockIdx.x];
     bool bad = false;
     const int64_t f0 = ch.flat_begin;
@@ -52,7 +65,7 @@ __global__ void __launch_bounds__(kStreamThreads) k_reduce(const Chunk* __restri
             const float th = __ldg(theta + f0 + e);
             float s = 0.f;
             for (int k = 0; k < K; ++k) s += th - ld_rep1(reps.p[k], dtype, f0 + e);
-            const float d = s * scale;
+            const float d = reduce_out(s * scale, pmode, mu, mom, bnew, f0 + e);
             bad |= !isfinite(d);
             d1d[ch.dst + e] = d;
         }
@@ -75,7 +88,11 @@ __global__ void __launch_bounds__(kStreamThreads) k_reduce(const Chunk* __restri
                     s.z += th.z - r.z;
                     s.w += th.w - r.w;
                 }
-                const float d[4] = {s.x * scale, s.y * scale, s.z * scale, s.w * scale};
+                float d[4] = {s.x * scale, s.y * scale, s.z * scale, s.w * scale};
+                if (PM) {
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) d[j] = reduce_out(d[j], pmode, mu, mom, bnew, i + j);
+                }
                 __nv_bfloat16 h[4], l[4];
 #pragma unroll
                 for (int j = 0; j < 4; ++j) {
@@ -91,7 +108,7 @@ __global__ void __launch_bounds__(kStreamThreads) k_reduce(const Chunk* __restri
                 const float th = __ldg(theta + i);
                 float s = 0.f;
                 for (int k = 0; k < K; ++k) s += th - ld_rep1(reps.p[k], dtype, i);
-                const float d = s * scale;
+                const float d = reduce_out(s * scale, pmode, mu, mom, bnew, i);
                 bad |= !isfinite(d);
                 const int pe = ch.elem_begin + e;
                 const int64_t o = md.slot + static_cast<int64_t>(pe / md.cols) * md.ld + pe % md.cols;
@@ -105,8 +122,37 @@ __global__ void __launch_bounds__(kStreamThreads) k_reduce(const Chunk* __restri
     raise_nonfinite(bad, err);
 }
 
+__global__ void __launch_bounds__(kStreamThreads) k_reduce(const Chunk* __restrict__ chunks,
+                                                           const MatDesc* __restrict__ mats,
+                                                           ReplicaPtrs reps, int K, int dtype,
+                                                           const float* __restrict__ theta, float scale,
+                                                           __nv_bfloat16* __restrict__ dhi,
+                                                           __nv_bfloat16* __restrict__ dlo,
+                                                           float* __restrict__ d1d,
+                                                           uint32_t* __restrict__ err) {
+    reduce_chunk<false>(chunks, mats, reps, K, dtype, theta, scale, dhi, dlo, d1d, err, 0, 0.f, nullptr, nullptr);
+}
 
-// grid: one CTA per chunk.  mode 0: Nesterov (theta, B in place); mode 1: merge output.
+// pmode 1 (Nesterov) or 2 (standard momentum); mom is read, B' goes to bnew.
+__global__ void __launch_bounds__(kStreamThreads) k_reduce_p(const Chunk* __restrict__ chunks,
+                                                             const MatDesc* __restrict__ mats,
+                                                             ReplicaPtrs reps, int K, int dtype,
+                                                             const float* __restrict__ theta, float scale,
+                                                             __nv_bfloat16* __restrict__ dhi,
+                                                             __nv_bfloat16* __restrict__ dlo,
+                                                             float* __restrict__ d1d,
+                                                             uint32_t* __restrict__ err, int pmode, float mu,
+                                                             const float* __restrict__ mom,
+                                                             float* __restrict__ bnew) {
+    reduce_chunk<true>(chunks, mats, reps, K, dtype, theta, scale, dhi, dlo, d1d, err, pmode, mu, mom, bnew);
+}
+
+
+// grid: one CTA per chunk.  mode 0: outer update of theta and B in place; mode 1: merge
+// output.  Mode 0 variants (the ablations of Sec. 4.5 and App. B): mom_kind 0 Nesterov
+// (Alg. 2), 1 standard momentum (B <- mu B + U, theta <- theta - eta B); pmode != 0: U is
+// already the orthogonalised update P (theta <- theta - eta U, B <- bnew from the reduce
+// pass); spectral: 2-D tensors scale Q by sqrt(rows / cols) instead of sigma_bar.
 __global__ void __launch_bounds__(kStreamThreads) k_apply(const Chunk* __restrict__ chunks,
                                                           const MatDesc* __restrict__ mats,
                                                           const MatState* __restrict__ state,
@@ -117,7 +163,9 @@ __global__ void __launch_bounds__(kStreamThreads) k_apply(const Chunk* __restric
                                                           const float* __restrict__ base,
                                                           float* __restrict__ out,
                                                           float* __restrict__ upd_out,
-                                                          const uint32_t* __restrict__ err) {
+                                                          const uint32_t* __restrict__ err, int mom_kind,
+                                                          int pmode, int spectral,
+                                                          const float* __restrict__ bnew) {
     if (*err & kErrNonFinite) return;  // leave theta and B untouched
     const Chunk ch = chunks[blockIdx.x];
     const int64_t f0 = ch.flat_begin;
@@ -136,7 +184,7 @@ __global__ void __launch_bounds__(kStreamThreads) k_apply(const Chunk* __restric
             qh = src.qh[st.final_buf] + md.slot;
             ql = src.ql[st.final_buf] + md.slot;
         }
-        ucoef = alpha * st.sigma_bar;
+        ucoef = alpha * (spectral ? sqrtf(static_cast<float>(md.rows) / static_cast<float>(md.cols)) : st.sigma_bar);
         contiguous = (md.ld == md.cols);
     } else if (mode == 1) {
         ucoef = alpha;  // Eq. 1: base + lambda * sum tau for non-matrix tensors
@@ -170,12 +218,25 @@ __global__ void __launch_bounds__(kStreamThreads) k_apply(const Chunk* __restric
             }
             if (mode == 0) {
                 const float4 th = *reinterpret_cast<const float4*>(theta + i);
-                const float4 bb = *reinterpret_cast<const float4*>(mom + i);
                 float4 nb, nt;
-                nb.x = fmaf(mu, bb.x, u[0]); nt.x = th.x - eta * fmaf(mu, nb.x, u[0]);
-                nb.y = fmaf(mu, bb.y, u[1]); nt.y = th.y - eta * fmaf(mu, nb.y, u[1]);
-                nb.z = fmaf(mu, bb.z, u[2]); nt.z = th.z - eta * fmaf(mu, nb.z, u[2]);
-                nb.w = fmaf(mu, bb.w, u[3]); nt.w = th.w - eta * fmaf(mu, nb.w, u[3]);
+                if (pmode) {
+                    nb = *reinterpret_cast<const float4*>(bnew + i);
+                    nt = make_float4(th.x - eta * u[0], th.y - eta * u[1], th.z - eta * u[2], th.w - eta * u[3]);
+                } else {
+                    const float4 bb = *reinterpret_cast<const float4*>(mom + i);
+                    nb.x = fmaf(mu, bb.x, u[0]);
+                    nb.y = fmaf(mu, bb.y, u[1]);
+                    nb.z = fmaf(mu, bb.z, u[2]);
+                    nb.w = fmaf(mu, bb.w, u[3]);
+                    if (mom_kind == 1) {
+                        nt = make_float4(th.x - eta * nb.x, th.y - eta * nb.y, th.z - eta * nb.z, th.w - eta * nb.w);
+                    } else {
+                        nt.x = th.x - eta * fmaf(mu, nb.x, u[0]);
+                        nt.y = th.y - eta * fmaf(mu, nb.y, u[1]);
+                        nt.z = th.z - eta * fmaf(mu, nb.z, u[2]);
+                        nt.w = th.w - eta * fmaf(mu, nb.w, u[3]);
+                    }
+                }
                 *reinterpret_cast<float4*>(mom + i) = nb;
                 *reinterpret_cast<float4*>(theta + i) = nt;
             } else {
@@ -189,9 +250,14 @@ __global__ void __launch_bounds__(kStreamThreads) k_apply(const Chunk* __restric
             const int64_t i = f0 + e;
             const float u = uval(e);
             if (mode == 0) {
-                const float nb = fmaf(mu, mom[i], u);
-                theta[i] = theta[i] - eta * fmaf(mu, nb, u);
-                mom[i] = nb;
+                if (pmode) {
+                    theta[i] = theta[i] - eta * u;
+                    mom[i] = bnew[i];
+                } else {
+                    const float nb = fmaf(mu, mom[i], u);
+                    theta[i] = theta[i] - eta * (mom_kind == 1 ? nb : fmaf(mu, nb, u));
+                    mom[i] = nb;
+                }
             } else {
                 out[i] = base[i] + u;
             }

@@ -45,7 +45,8 @@ class Param(ctypes.Structure):
 class Opts(ctypes.Structure):
     _fields_ = [("alpha", ctypes.c_float), ("outer_lr", ctypes.c_float), ("momentum", ctypes.c_float),
                 ("reduce_mean", ctypes.c_int), ("max_iter", ctypes.c_int), ("tol", ctypes.c_float),
-                ("sync", ctypes.c_int), ("fast_steps", ctypes.c_int)]
+                ("sync", ctypes.c_int), ("fast_steps", ctypes.c_int), ("orth_target", ctypes.c_int),
+                ("momentum_kind", ctypes.c_int), ("scale_kind", ctypes.c_int)]
 
 
 _lib = None
@@ -107,13 +108,15 @@ def _stream(stream=None) -> int:
 
 
 def make_opts(alpha=1.0, outer_lr=0.7, momentum=0.9, reduce_mean=True, max_iter=0, tol=0.0,
-              sync=False, fast_steps=0) -> Opts:
-    """Options of an outer step; fast_steps > 0 selects the fixed-step variant of Sec. 4.3."""
+              sync=False, fast_steps=0, orth_target=0, momentum_kind=0, scale_kind=0) -> Opts:
+    """Options of an outer step; fast_steps > 0 selects the fixed-step variant of Sec. 4.3,
+    the last three the ablations of Sec. 4.5 / App. B (see include/isoloco.h)."""
     o = Opts()
     lib().isoloco_opts_default(ctypes.byref(o))
     o.alpha, o.outer_lr, o.momentum = float(alpha), float(outer_lr), float(momentum)
     o.reduce_mean, o.max_iter, o.tol, o.sync = int(bool(reduce_mean)), int(max_iter), float(tol), int(bool(sync))
     o.fast_steps = int(fast_steps)
+    o.orth_target, o.momentum_kind, o.scale_kind = int(orth_target), int(momentum_kind), int(scale_kind)
     return o
 
 

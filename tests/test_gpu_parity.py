@@ -24,14 +24,14 @@ def iso():
 
 
 def run_gpu(iso, wl, alpha, eta, mu, reps=None, theta=None, mom=None, max_iter=0, reduce_mean=True,
-            plan=None, fast_steps=0):
+            plan=None, fast_steps=0, **ablation):
     plan = plan or iso.Plan(wl.table, wl.N, wl.K, wl.replicas.dtype)
     th = (wl.theta if theta is None else theta).clone()
     b = (wl.momentum if mom is None else mom).clone()
     upd = torch.empty_like(th)
     rc = plan.outer_step(th, b, wl.replicas if reps is None else reps,
                          iso.make_opts(alpha, eta, mu, reduce_mean=reduce_mean, max_iter=max_iter, sync=True,
-                                       fast_steps=fast_steps),
+                                       fast_steps=fast_steps, **ablation),
                          update_out=upd)
     diag = plan.read_diag()
     return rc, th, b, upd, diag, plan
@@ -212,6 +212,53 @@ def test_fast_variant_tiny(iso):
 def test_fast_variant_180m_sampled(iso):
     """The benchmarked configuration at full size with the paper's 5 fixed steps."""
     sampled_parity(iso, "llama_180m_k8", ("layers.0.wq", "layers.5.w_gate", "layers.11.w_down"), fast_steps=5)
+
+
+# ---- the ablations of Sec. 4.5 and App. B
+
+ABLATIONS = [
+    {"orth_target": 1},                                  # Iso-C of the Nesterov update P
+    {"orth_target": 1, "momentum_kind": 1},              # ... with standard momentum (P = B')
+    {"momentum_kind": 1},                                # standard momentum on Iso-C(Delta)
+    {"scale_kind": 1},                                   # Muon's spectral scale sqrt(rows / cols)
+    {"scale_kind": 1, "fast_steps": 5},                  # fixed steps + spectral scale (Muon-like)
+    {"orth_target": 1, "fast_steps": 5},
+]
+
+
+@pytest.mark.parametrize("flags", ABLATIONS, ids=lambda f: "-".join(f"{k}{v}" for k, v in f.items()))
+def test_ablation_variants(iso, flags):
+    from oracle import variants
+    spec = W.custom_spec(RAGGED, K=3, rank=2, momentum_std=1e-4)
+    wl = W.make_workload(spec, seed=11, device="cuda")
+    rc, th, b, upd, diag, _ = run_gpu(iso, wl, 1.3, 0.7, 0.9, **flags)
+    assert rc == 0
+    ref = variants.isoloco_outer_step_variant(
+        wl.table, wl.theta.cpu().numpy(), wl.momentum.cpu().numpy(), W.replicas_as_numpy(wl.replicas),
+        alpha=1.3, eta=0.7, mu=0.9, **flags)
+    ref["theta_in"] = wl.theta.double().cpu().numpy()
+    sigma = diag["sigma_bar"]
+    if flags.get("scale_kind"):
+        # the spectral scale needs no sigma_bar, so the library does not compute it
+        sigma = [s for s, (_, r, c) in zip(ref["sigma_bar"], wl.table) if c > 0]
+        ref["sigma_bar"] = np.asarray(ref["sigma_bar"])
+    check_step(wl.table, th.double().cpu().numpy(), b.double().cpu().numpy(), upd.double().cpu().numpy(),
+               sigma, ref)
+
+
+def test_excluded_matrix_is_listed_as_1d(iso):
+    """Sec. 4.5's exclusion of embedding/head from Iso-C: the caller lists the tensor as 1-D."""
+    spec = W.custom_spec([("embed", 96, 64), ("w", 64, 48), ("head", 64, 96), ("norm", 64, 0)], K=2, rank=2)
+    wl = W.make_workload(spec, seed=3, device="cuda")
+    table = [(o, r * c, 0) if i in (0, 2) else (o, r, c) for i, (o, r, c) in enumerate(wl.table)]
+    plan = iso.Plan(table, wl.N, wl.K)
+    assert plan.num_matrices == 1
+    rc, th, b, upd, diag, _ = run_gpu(iso, wl, 1.0, 0.7, 0.9, plan=plan)
+    assert rc == 0
+    ref = oracle_step(table, wl.theta, wl.momentum, wl.replicas, 1.0, 0.7, 0.9)
+    ref["theta_in"] = wl.theta.double().cpu().numpy()
+    check_step(table, th.double().cpu().numpy(), b.double().cpu().numpy(), upd.double().cpu().numpy(),
+               diag["sigma_bar"], ref)
 
 
 def test_diloco_outer_step(iso):
