@@ -117,7 +117,7 @@ def gemm_flops(table, diag, fast=False):
     return out
 
 
-BM, BN, BK = 256, 256, 32   # output tile of one CTA pair (tcgen05 cta_group::2)
+BM, BN, BK = 256, 256, 64   # output tile of one CTA pair (tcgen05 cta_group::2), stage depth
 
 
 def _sym_tiles(n):

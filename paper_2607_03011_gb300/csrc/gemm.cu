@@ -163,14 +163,24 @@ __device__ __forceinline__ uint32_t stg_off(int r, int c) {
 __device__ __forceinline__ void stage_store_block(const uint32_t (&w)[16], const CUtensorMap* map, uint8_t* stg,
                                                   uint32_t& seq, bool diag, bool sym, int lane, int col0,
                                                   int row_base, int b) {
-    static_assert(kStageBlocks == 4, "block rotation below assumes four staging blocks per warp");
+    static_assert(kStageBlocks == 4 || kStageBlocks == 2, "block rotation below handles two or four blocks");
     uint8_t* sd;
-    if (sym) {
-        sd = stg + (seq & 1u) * 2u * kStageBlockBytes;
-        if (lane == 0) bulk_wait_read1();
+    if (kStageBlocks == 4) {
+        if (sym) {
+            sd = stg + (seq & 1u) * 2u * kStageBlockBytes;
+            if (lane == 0) bulk_wait_read1();
+        } else {
+            sd = stg + (seq & 3u) * kStageBlockBytes;
+            if (lane == 0) bulk_wait_read3();
+        }
     } else {
-        sd = stg + (seq & 3u) * kStageBlockBytes;
-        if (lane == 0) bulk_wait_read3();
+        if (sym) {
+            sd = stg;
+            if (lane == 0) bulk_wait_read0();
+        } else {
+            sd = stg + (seq & 1u) * kStageBlockBytes;
+            if (lane == 0) bulk_wait_read1();
+        }
     }
     uint8_t* sm = sd + kStageBlockBytes;  // transposed block (symmetric outputs only)
     ++seq;

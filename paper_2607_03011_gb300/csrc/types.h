@@ -12,18 +12,20 @@ namespace isoloco {
 // operand planes staged BK deep per pipeline stage.  With kPairMma a pair of CTAs on
 // neighbouring SMs (a cluster of two) computes one kTileM x BN = 256 x 256 output tile
 // with tcgen05 cta_group::2: each CTA stages its own BM rows of A and half of B's BN
-// rows, so one SM's shared memory supplies 8 KB instead of 12 KB per 16-deep MMA step
-// (the single-SM M128 x N256 tile is bound by shared-memory bandwidth, not the tensor pipe).
+// rows, so an SM loads and stages 8 KB instead of 12 KB per 16-deep MMA step.
+// BK = 64: one TMA instruction moves twice the bytes of a 32-deep stage; with 32-deep
+// stages the single producer thread's issue rate held back the MN-major operands (a Gram
+// stage needs six 64 x 32 boxes).
 constexpr bool kPairMma = true;
 constexpr int BM = 128;
 constexpr int BN = 256;
-constexpr int BK = 32;
+constexpr int BK = 64;
 constexpr int kTileM = kPairMma ? 2 * BM : BM;  // rows of one output tile
 constexpr int kBRows = kPairMma ? BN / 2 : BN;  // rows of B (N extent) staged by one CTA
 // Shared-memory ring of the persistent GEMM (one CTA per SM): as many stages of the
 // launch's plane set as fit in kRingBytes, at most kMaxStages.
 constexpr int kMaxStages = 12;
-constexpr int kRingBytes = 160 * 1024;
+constexpr int kRingBytes = 192 * 1024;
 constexpr int kTileABytes = BM * BK * 2;                       // one bf16 plane of A
 constexpr int kTileBBytes = kBRows * BK * 2;                   // one bf16 plane of this CTA's B
 
@@ -34,11 +36,13 @@ constexpr int kTmemCols = 256;     // one accumulator; the kernel double-buffers
 constexpr int kMaxGroups = 8;
 constexpr int kFinRows = 32;  // rows of one k_gram_finalize tile (x BN columns)
 // Epilogue staging: per epilogue warp kStageBlocks blocks of 32 x 32 16-bit values (2 KB,
-// 64-byte swizzled rows), written to global memory by TMA stores.  A symmetric output
-// uses them as two (direct, transposed) pairs, anything else as four single blocks, so
-// that a warp fills one while the TMA stores of the others still read shared memory.
+// 64-byte swizzled rows), written to global memory by TMA stores.  With four, a symmetric
+// output uses them as two (direct, transposed) pairs and anything else as four single
+// blocks, so that a warp fills one while the TMA stores of the others still read shared
+// memory; with two (the setting: the epilogue keeps up with the main loop, and the ring
+// gets the 32 KB), one pair, or two alternating single blocks.
 constexpr int kStageBlockBytes = 32 * 32 * 2;
-constexpr int kStageBlocks = 4;
+constexpr int kStageBlocks = 2;
 constexpr int kEpiStagingBytes = kEpiWarps * kStageBlocks * kStageBlockBytes;
 constexpr int kTileQueue = 8;  // tiles handed from the producer warp to the MMA and epilogue warps
 constexpr int kGemmSmemBytes = kRingBytes + kEpiStagingBytes + 1024 /*align*/ + 512 /*barriers, queues*/;
