@@ -151,13 +151,18 @@ __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict
 
 // Coefficients (a, b, c) of quintic step `step` of a matrix.  Near-square matrices (deep)
 // start with one round of the deep schedule, which reaches singular values down to 1e-6
-// of the normalisation; whatever was below that has grown by the product of its linear
-// coefficients (~4e6) and sits above the standard schedule's 1e-3 floor, so later rounds
-// (and every round of the other matrices) use the standard schedule.
+// of the normalisation.  Whatever was below that has grown by the product of its linear
+// coefficients (~4e6): from 1e-8 up it is above 0.038, inside the design interval of the
+// standard schedule's third step, so the next round starts there (5 steps instead of 7);
+// any later round, and every round of the other matrices, is the full standard schedule.
+// (Singular values under 1e-8 of s are below what the split arithmetic resolves.)
+constexpr int kDeepRestart = 2;  // first standard step after the deep round
 __device__ __forceinline__ const float* sched_row(bool deep, int step) {
-    if (deep && step < kSchedDeepSteps) return kSchedDeep[step];
-    const int k = (deep ? step - kSchedDeepSteps : step) % kSchedSteps;
-    return kSched[k];
+    if (!deep) return kSched[step % kSchedSteps];
+    if (step < kSchedDeepSteps) return kSchedDeep[step];
+    const int kk = step - kSchedDeepSteps;
+    if (kk < kSchedSteps - kDeepRestart) return kSched[kDeepRestart + kk];
+    return kSched[(kk - (kSchedSteps - kDeepRestart)) % kSchedSteps];
 }
 
 // Decision for matrix mi, taken by one warp.  t: iteration index (0 = first Gram of Delta).
