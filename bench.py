@@ -222,6 +222,180 @@ def run_reference(args):
     return 0
 
 
+# --------------------------------------------------------------------------- DiLoCo arm
+AGG_CODE = {"mean": 0, "ties": 1, "dare": 2}
+AGG_KERNELS = {"mean": "k_diloco", "ties": "k_ties_hist (4 radix-select passes) + k_ties_merge",
+               "dare": "k_dare"}
+
+
+def diloco_bytes(agg, N, K, eb):
+    """Algorithmic HBM bytes of one DiLoCo step per phase: the streaming pass reads theta,
+    B and the K replicas and writes theta and B; TIES's trim reads theta and the replicas
+    once per radix pass (4 passes)."""
+    out = {"diloco": (16 + K * eb) * N}
+    if agg == "ties":
+        out["trim"] = 4 * (4 + K * eb) * N
+    return out
+
+
+def oracle_merging_sample(workload: str, names, agg: str, sparsity: float, seed: int = 0):
+    """The oracle's DiLoCo step with a merging rule on a sample of the workload's tensors
+    (TIES trims within the sample).  Returns (params, seconds, description)."""
+    import oracle
+    from oracle import merging
+    from paper_2607_03011_gb300 import workloads as W
+    base = W.SPECS[workload]
+    shapes = [s for s in base.shapes if s[0] in names]
+    spec = W.custom_spec(shapes, K=base.K, rank=base.rank, shared_std=base.shared_std,
+                         noise_std=base.noise_std, momentum_std=base.momentum_std,
+                         replica_dtype=base.replica_dtype, name=base.name + "_sample")
+    wl = W.make_workload(spec, seed=seed, device="cpu")
+    reps = W.replicas_as_numpy(wl.replicas)
+    th, b = wl.theta.numpy(), wl.momentum.numpy()
+    t0 = time.perf_counter()
+    if agg == "mean":
+        oracle.diloco_outer_step(th, b, reps, eta=base.outer_lr, mu=base.momentum)
+    else:
+        merging.merged_outer_step(th, b, reps, agg, sparsity=sparsity, seed=1, eta=base.outer_lr,
+                                  mu=base.momentum)
+    dt = time.perf_counter() - t0
+    return wl.N, dt, "+".join(f"{n}:{r}x{c}" if c else f"{n}:{r}" for (n, r, c) in shapes)
+
+
+def run_diloco(args, torch, isoloco, wl, plan, world, rank, local, dist, barrier):
+    """Times diloco_outer_step (Alg. 1) with the chosen merging rule on the workload."""
+    spec = wl.spec
+    agg = args.aggregator
+    opts = isoloco.make_opts(outer_lr=spec.outer_lr, momentum=spec.momentum, aggregator=AGG_CODE[agg],
+                             sparsity=args.sparsity if agg != "mean" else 0.0, seed=1)
+    theta0, mom0 = wl.theta.clone(), wl.momentum.clone()
+    th, b = wl.theta, wl.momentum
+    stream = torch.cuda.current_stream()
+
+    def restore():
+        th.copy_(theta0)
+        b.copy_(mom0)
+
+    for _ in range(args.warmup):
+        restore()
+        plan.diloco_outer_step(th, b, wl.replicas, opts)
+    if plan.last_status() != 0:
+        raise RuntimeError(f"warm-up step status {isoloco.STATUS_NAMES.get(plan.last_status())}")
+    launches0 = plan.launches
+    clocks = ClockSampler(local)
+    torch.cuda.synchronize()
+    barrier()
+    clocks.start()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    for i in range(args.steps):
+        restore()
+        ev[i][0].record(stream)
+        plan.diloco_outer_step(th, b, wl.replicas, opts)
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop()
+    status = plan.last_status()
+    step_ms = [a.elapsed_time(z) for a, z in ev]
+    total_ms = sum(step_ms)
+    launches = plan.launches - launches0
+    plan.profile(True)
+    for i in range(args.steps):
+        restore()
+        plan.diloco_outer_step(th, b, wl.replicas, opts)
+    torch.cuda.synchronize()
+    prof = plan.profile_read()
+    plan.profile(False)
+    if dist is not None:
+        t = torch.tensor([total_ms], device="cuda", dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+    value = world * wl.N * args.steps / (total_ms / 1000.0)
+
+    # end to end: pinned host buffers copied in and out on the stream around the call
+    e2e = None
+    if not args.no_e2e and rank == 0:
+        th_h, b_h = theta0.cpu().pin_memory(), mom0.cpu().pin_memory()
+        reps_h = wl.replicas.cpu().pin_memory()
+        th_d, b_d = torch.empty_like(th), torch.empty_like(b)
+        reps_d = torch.empty_like(wl.replicas)
+        e_ms = []
+        for _ in range(1 + args.e2e_steps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            th_d.copy_(th_h, non_blocking=True)
+            b_d.copy_(b_h, non_blocking=True)
+            reps_d.copy_(reps_h, non_blocking=True)
+            plan.diloco_outer_step(th_d, b_d, reps_d, opts)
+            th_h.copy_(th_d, non_blocking=True)
+            b_h.copy_(b_d, non_blocking=True)
+            e1.record(stream)
+            e1.synchronize()
+            e_ms.append(e0.elapsed_time(e1))
+            th_h.copy_(theta0.cpu())
+            b_h.copy_(mom0.cpu())
+        e_ms = e_ms[1:]
+        eb = wl.replicas.element_size()
+        e2e = {"value": wl.N / (statistics.median(e_ms) / 1000.0), "unit": UNIT,
+               "h2d_bytes_per_step": int(wl.N * (8 + wl.K * eb)), "d2h_bytes_per_step": int(wl.N * 8),
+               "ms_per_step": statistics.median(e_ms),
+               "api": "diloco_outer_step on device copies of pinned host buffers (copies on the same stream)"}
+        del reps_h, reps_d
+
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return 0
+    peaks, peak_src = load_peaks()
+    hbm = peaks["hbm_gbs"]
+    eb = wl.replicas.element_size()
+    nb = diloco_bytes(agg, wl.N, wl.K, eb)
+    phases = {}
+    for ph, nbytes in nb.items():
+        ms, n = prof[ph]
+        gb = nbytes * args.steps / (ms / 1000.0) / 1e9 if ms > 0 else 0.0
+        phases[ph] = {"achieved": gb, "frac": gb / hbm, "bytes_per_step": nbytes, "ms_per_step": ms / args.steps,
+                      "launches_per_step": n / args.steps}
+    dom = max(phases, key=lambda k: phases[k]["ms_per_step"])
+    roofline = {"bound": "hbm", "kernel": {"diloco": "k_diloco" if agg == "mean" else
+                                           ("k_ties_merge" if agg == "ties" else "k_dare"),
+                                           "trim": "k_ties_hist x4 + k_ties_select x4 + k_ties_init"}[dom],
+                "achieved": phases[dom]["achieved"], "peak": hbm, "unit": "GB/s", "frac": phases[dom]["frac"],
+                "traffic": None, "peak_source": f"{peak_src} hbm_gbs",
+                "kernel_times": "per-phase CUDA events on the launch stream, in a profiled pass of the same "
+                                "steps right after the timed region",
+                "phases": phases}
+    cpu = None
+    if not args.no_cpu_baseline and world == 1:
+        import oracle
+        oracle.build()
+        nparams, dt, desc = oracle_merging_sample(args.workload, CPU_SAMPLE, agg, args.sparsity)
+        cpu = {"value": nparams / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+               "sample": f"oracle DiLoCo step ({agg}) on {desc} ({nparams} params, {dt:.1f} s), "
+                         "same generator recipe"}
+    line = {
+        "metric": f"DiLoCo outer-step ({agg} aggregation) params/s at {args.workload}", "value": value,
+        "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": args.workload, "params": wl.N, "K": wl.K, "aggregator": agg,
+                   "sparsity": args.sparsity if agg != "mean" else 0.0,
+                   "replica_dtype": str(wl.replicas.dtype).replace("torch.", ""),
+                   "outer_lr": spec.outer_lr, "momentum": spec.momentum,
+                   "l2": "inputs larger than L2 (K replicas = %.1f GB)" % (wl.replicas.numel() * eb / 1e9),
+                   "timing": "sum of per-step CUDA-event intervals on the launch stream; theta/B restored "
+                             "between steps outside the intervals",
+                   "parallelism": f"replicas x{world}"},
+        "status": isoloco.STATUS_NAMES.get(status, status),
+        "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
+        "clocks": clk, "step_ms": [round(x, 3) for x in step_ms],
+    }
+    print(json.dumps(line))
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
 # --------------------------------------------------------------------------- GPU arm
 def main():
     ap = argparse.ArgumentParser()
@@ -235,6 +409,10 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--fast-steps", type=int, default=0,
                     help="time the fast variant of Sec. 4.3 (k fixed polar steps, rms sigma_bar); 0 = exact")
+    ap.add_argument("--aggregator", default="iso_c", choices=["iso_c", "mean", "ties", "dare"],
+                    help="iso_c: the IsoLoCo step (Alg. 2, default); mean / ties / dare: the DiLoCo step "
+                         "(Alg. 1) with that merging rule (Sec. 3.2)")
+    ap.add_argument("--sparsity", type=float, default=0.1, help="TIES / DARE sparsity (0.1: Sec. 5.1's best)")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     if args.impl == "reference":
@@ -261,6 +439,8 @@ def main():
     spec = W.SPECS[args.workload]
     wl = W.make_workload(spec, seed=rank, device="cuda")
     plan = isoloco.Plan(wl.table, wl.N, wl.K, wl.replicas.dtype)
+    if args.aggregator != "iso_c":
+        return run_diloco(args, torch, isoloco, wl, plan, world, rank, local, dist, barrier)
     opts = isoloco.make_opts(spec.alpha, spec.outer_lr, spec.momentum, fast_steps=args.fast_steps)
     theta0, mom0 = wl.theta.clone(), wl.momentum.clone()
     th, b = wl.theta, wl.momentum

@@ -92,6 +92,23 @@ typedef struct {
     int scale_kind;    /* 0: the Iso-C scale sigma_bar.  1: Muon's spectral scale, U = alpha *
                         * sqrt(rows / cols) * Q for a rows x cols tensor (App. B; sigma_bar is
                         * then not computed). */
+    /* The merging aggregators of Sec. 3.2, used by diloco_outer_step in place of the mean
+     * of the Delta_k (the outer optimiser stays Nesterov; momentum = 0 is the paper's SGD): */
+    int aggregator;    /* 0: mean (Alg. 1).
+                        * 1: TIES -- trim: each worker keeps its n_keep = N - floor(sparsity * N)
+                        *    largest |Delta_k| over all N entries (entries equal to the
+                        *    n_keep-th largest are kept too); elect: sign of P + N, P and N the
+                        *    fp32 sums, in worker order, of an entry's kept positive and kept
+                        *    negative values; merge: U = the mean of the kept values of the
+                        *    elected sign (0 when P + N = 0).
+                        * 2: DARE -- drop each entry of each Delta_k with probability
+                        *    `sparsity`, rescale the rest by 1 / (1 - sparsity), and average
+                        *    (or sum, reduce_mean = 0). */
+    float sparsity;    /* in [0, 1) */
+    unsigned int seed; /* DARE's drops: entry i (flat index) of worker k is dropped when
+                        * u < sparsity, u = top 24 bits of SplitMix64 output number
+                        * k * n_total + i + 1 from state `seed` (Steele, Lea and Flood 2014),
+                        * times 2^-24. */
 } isoloco_opts_t;
 
 /* Fills *opts with alpha = 1, outer_lr = 0.7, momentum = 0.9 (the paper's DiLoCo
@@ -134,7 +151,10 @@ int isoloco_outer_step_host(isoloco_plan_t plan, float* theta_host, float* momen
 
 /* DiLoCo outer step, Alg. 1 with Nesterov SGD: one streaming pass over every
  * parameter (no Iso-C).  Elementwise, so a non-finite input only affects its own
- * element; the step's status reports it. */
+ * element; the step's status reports it.  opts->aggregator selects the merging rule of
+ * Sec. 3.2 that replaces the mean (TIES: 4 extra read passes over the replicas for the
+ * trim, then one pass; DARE: one pass).  The table is not used: every entry of
+ * [0, n_total) is updated.  Errors: INVALID for a bad aggregator or sparsity. */
 int diloco_outer_step(isoloco_plan_t plan, float* theta, float* momentum,
                       const void* const* replicas, const isoloco_opts_t* opts, void* stream);
 
@@ -220,9 +240,10 @@ enum {
     ISOLOCO_PHASE_UPDATE = 5,   /* X P (or P X) GEMMs */
     ISOLOCO_PHASE_TRACE = 6,    /* sigma_bar = tr(Q^T Delta) / n */
     ISOLOCO_PHASE_APPLY = 7,    /* Nesterov update / merge output (HBM stream) */
-    ISOLOCO_PHASE_DILOCO = 8,   /* fused DiLoCo pass */
+    ISOLOCO_PHASE_DILOCO = 8,   /* fused DiLoCo pass (mean, DARE, or TIES's merge pass) */
     ISOLOCO_PHASE_OTHER = 9,
-    ISOLOCO_NUM_PHASES = 10
+    ISOLOCO_PHASE_TRIM = 10,    /* TIES trim: per-worker radix select of the threshold */
+    ISOLOCO_NUM_PHASES = 11
 };
 
 /* Per-phase timing.  enable != 0 makes every later call record a CUDA event pair

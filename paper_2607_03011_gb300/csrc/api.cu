@@ -45,6 +45,14 @@ __global__ void k_reduce_p(const Chunk*, const MatDesc*, ReplicaPtrs, int, int, 
 __global__ void k_apply(const Chunk*, const MatDesc*, const MatState*, UpdateSrc, int, float, float, float,
                         float*, float*, const float*, float*, float*, const uint32_t*, int, int, int, const float*);
 __global__ void k_diloco(ReplicaPtrs, int, int, float*, float*, int64_t, float, float, float, uint32_t*);
+__global__ void k_dare(ReplicaPtrs, int, int, float*, float*, int64_t, float, float, float, unsigned int, float,
+                       float, uint32_t*);
+__global__ void k_ties_init(int, uint64_t, unsigned long long*, uint64_t*, uint64_t*);
+__global__ void k_ties_hist(ReplicaPtrs, int, int, const float*, int64_t, int, const uint64_t*,
+                            unsigned long long*);
+__global__ void k_ties_select(int, int, unsigned long long*, uint64_t*, uint64_t*);
+__global__ void k_ties_merge(ReplicaPtrs, int, int, float*, float*, int64_t, const uint64_t*, float, float,
+                             uint32_t*);
 __global__ void k_split_planes(const float*, int64_t, int, int, int, __nv_bfloat16*, __nv_bfloat16*, int);
 
 constexpr int kChunkElems = 16384;
@@ -141,6 +149,10 @@ struct isoloco_plan {
     double prof_ms[ISOLOCO_NUM_PHASES] = {0};
     int64_t prof_n[ISOLOCO_NUM_PHASES] = {0};
     int64_t launches = 0;
+    // TIES trim: per-worker radix-select histogram (K x 256), rank and chosen key prefix
+    unsigned long long* ties_hist = nullptr;
+    uint64_t* ties_rank = nullptr;
+    uint64_t* ties_prefix = nullptr;
     // staging for the host-buffer entry point (allocated on first use)
     float* st_theta = nullptr;
     float* st_mom = nullptr;
@@ -436,11 +448,15 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         (rc = dalloc(p, &p->cnt_gram, (int64_t)p->buckets.size())) ||
         (rc = dalloc(p, &p->cnt_step, (int64_t)p->buckets.size())) ||
         (rc = dalloc(p, &p->counters, kLaunchCounters)) || (rc = dalloc(p, &p->loopc, 2)) ||
+        (rc = dalloc(p, &p->ties_hist, (int64_t)p->K * 256)) || (rc = dalloc(p, &p->ties_rank, p->K)) ||
+        (rc = dalloc(p, &p->ties_prefix, p->K)) ||
         (rc = dalloc(p, &p->tmaps_d, (int64_t)kMapsPerBucket * std::max<size_t>(1, p->buckets.size()))))
         return rc;
     CUDA_TRY(cudaHostAlloc(reinterpret_cast<void**>(&p->err_h), sizeof(uint32_t), cudaHostAllocDefault));
     *p->err_h = 0;
     CUDA_TRY(cudaEventCreateWithFlags(&p->done_ev, cudaEventDisableTiming));
+    if (p->K * 256 * 4 > 48 * 1024)  // TIES histogram: K x 256 shared counters
+        CUDA_TRY(cudaFuncSetAttribute(k_ties_hist, cudaFuncAttributeMaxDynamicSharedMemorySize, p->K * 256 * 4));
     CUDA_TRY(cudaStreamCreateWithFlags(&p->cap_st, cudaStreamNonBlocking));
     CUDA_TRY(cudaMemset(p->loopc, 0, 2 * sizeof(long long)));
     // zero the planes once so that padding columns hold zeros
@@ -850,6 +866,9 @@ static int check_opts(const isoloco_opts_t* o, isoloco_opts_t* out) {
     if (out->orth_target < 0 || out->orth_target > 1 || out->momentum_kind < 0 || out->momentum_kind > 1 ||
         out->scale_kind < 0 || out->scale_kind > 1)
         return fail(ISOLOCO_ERR_INVALID, "orth_target, momentum_kind and scale_kind must be 0 or 1");
+    if (out->aggregator < 0 || out->aggregator > 2) return fail(ISOLOCO_ERR_INVALID, "aggregator must be 0, 1 or 2");
+    if (!(out->sparsity >= 0.f && out->sparsity < 1.f))
+        return fail(ISOLOCO_ERR_INVALID, "sparsity must be in [0, 1)");
     return ISOLOCO_OK;
 }
 
@@ -939,6 +958,9 @@ int isoloco_opts_default(isoloco_opts_t* o) {
     o->orth_target = 0;
     o->momentum_kind = 0;
     o->scale_kind = 0;
+    o->aggregator = 0;
+    o->sparsity = 0.f;
+    o->seed = 0u;
     return ISOLOCO_OK;
 }
 
@@ -1030,9 +1052,32 @@ int diloco_outer_step(isoloco_plan_t p, float* theta, float* momentum, const voi
     CUDA_TRY(cudaMemsetAsync(p->err_d, 0, 4, st));
     const float scale = o.reduce_mean ? 1.f / (float)p->K : 1.f;
     const int grid = p->num_sms * 8;
-    { PhaseTimer tm(p, ISOLOCO_PHASE_DILOCO, st);
-    k_diloco<<<grid, 256, 0, st>>>(rp, p->K, p->dtype, theta, momentum, p->N, scale, o.outer_lr, o.momentum,
-                                   p->err_d); }
+    if (o.aggregator == 0) {
+        PhaseTimer tm(p, ISOLOCO_PHASE_DILOCO, st);
+        k_diloco<<<grid, 256, 0, st>>>(rp, p->K, p->dtype, theta, momentum, p->N, scale, o.outer_lr, o.momentum,
+                                       p->err_d);
+    } else if (o.aggregator == 2) {
+        PhaseTimer tm(p, ISOLOCO_PHASE_DILOCO, st);
+        k_dare<<<grid, 256, 0, st>>>(rp, p->K, p->dtype, theta, momentum, p->N, scale, o.sparsity,
+                                     1.f / (1.f - o.sparsity), o.seed, o.outer_lr, o.momentum, p->err_d);
+    } else {
+        // keep the n_keep largest |Delta_k| of each worker; n_keep = N keeps all (threshold 0)
+        const uint64_t n_keep = (uint64_t)(p->N - (int64_t)std::floor((double)o.sparsity * (double)p->N));
+        const bool select = n_keep < (uint64_t)p->N;
+        {
+            PhaseTimer tm(p, ISOLOCO_PHASE_TRIM, st, select ? 9 : 1);
+            k_ties_init<<<1, 256, 0, st>>>(p->K, n_keep, p->ties_hist, p->ties_rank, p->ties_prefix);
+            const int smem = p->K * 256 * 4;
+            for (int pass = 0; select && pass < 4; ++pass) {
+                k_ties_hist<<<grid, 256, smem, st>>>(rp, p->K, p->dtype, theta, p->N, pass, p->ties_prefix,
+                                                     p->ties_hist);
+                k_ties_select<<<1, 64, 0, st>>>(p->K, pass, p->ties_hist, p->ties_rank, p->ties_prefix);
+            }
+        }
+        PhaseTimer tm(p, ISOLOCO_PHASE_DILOCO, st);
+        k_ties_merge<<<grid, 256, 0, st>>>(rp, p->K, p->dtype, theta, momentum, p->N, p->ties_prefix, o.outer_lr,
+                                           o.momentum, p->err_d);
+    }
     CUDA_TRY(cudaGetLastError());
     return finish_call(p, st, o.sync);
 }

@@ -11,6 +11,11 @@
 //  k_diloco       : Alg. 1 with Nesterov SGD fused into a single pass over all
 //                   parameters (reduction + update, no workspace).
 //                   Mode 1: Iso-C merge output base + alpha IsoC(T) / base + alpha T (Eq. 1).
+//  k_dare         : Alg. 1 with DARE aggregation (Sec. 3.2): random drop and rescale of
+//                   each Delta_k, then the mean and the outer step, one pass.
+//  k_ties_*       : Alg. 1 with TIES aggregation (Sec. 3.2): per-worker magnitude trim by
+//                   radix select over all N entries (4 histogram passes), then sign
+//                   election, disjoint mean and the outer step in one pass.
 //  k_split_planes : fp32 -> bf16 hi/lo planes (tests of the split-precision GEMM).
 #include "common.cuh"
 #include "types.h"
@@ -310,6 +315,247 @@ __global__ void __launch_bounds__(kStreamThreads) k_diloco(ReplicaPtrs reps, int
             const float nb = fmaf(mu, mom[i], d);
             theta[i] = th - eta * fmaf(mu, nb, d);
             mom[i] = nb;
+        }
+    }
+    raise_nonfinite(bad, err);
+}
+
+// ---------------------------------------------------------------- merging aggregators
+// Sec. 3.2 replaces DiLoCo's mean of the Delta_k by a model-merging rule.  These kernels
+// compute the merged direction U over all N entries and take the outer step
+// B <- mu B + U, theta <- theta - eta (U + mu B) (mu = 0: the SGD step of Sec. 5.1).
+
+// SplitMix64 (Steele, Lea and Flood, 2014): output number n (n >= 1) from state s.
+__device__ __forceinline__ uint64_t splitmix64(uint64_t s, uint64_t n) {
+    uint64_t z = s + n * 0x9E3779B97F4A7C15ull;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+// DARE's mask bit: keep entry i of worker k when the top 24 bits of SplitMix64 output
+// k * N + i + 1, times 2^-24, are >= p.
+__device__ __forceinline__ bool dare_keep(unsigned int seed, int k, int64_t N, int64_t i, float p) {
+    const uint64_t z = splitmix64(seed, static_cast<uint64_t>(k) * static_cast<uint64_t>(N) +
+                                            static_cast<uint64_t>(i) + 1ull);
+    return static_cast<float>(z >> 40) * 0x1p-24f >= p;
+}
+
+__device__ __forceinline__ void nesterov1(float& th, float& b, float u, float eta, float mu) {
+    const float nb = fmaf(mu, b, u);
+    th = th - eta * fmaf(mu, nb, u);
+    b = nb;
+}
+
+// DARE: U = scale * sum_k keep_scale * m_k * Delta_k, keep_scale = 1 / (1 - p), scale =
+// 1 / K (mean) or 1.  Grid-stride over float4 vectors of all N entries, scalar tail in CTA 0.
+__global__ void __launch_bounds__(kStreamThreads) k_dare(ReplicaPtrs reps, int K, int dtype,
+                                                         float* __restrict__ theta, float* __restrict__ mom,
+                                                         int64_t N, float scale, float p, float keep_scale,
+                                                         unsigned int seed, float eta, float mu,
+                                                         uint32_t* __restrict__ err) {
+    bool bad = false;
+    const int64_t nv = N >> 2;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t v = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; v < nv; v += stride) {
+        const int64_t i = 4 * v;
+        float4 th = *reinterpret_cast<const float4*>(theta + i);
+        float4 bb = *reinterpret_cast<const float4*>(mom + i);
+        float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+        float chk = 0.f;  // every Delta_k entry, dropped or not, for the non-finite test
+        for (int k = 0; k < K; ++k) {
+            const float4 r = ld_rep4(reps.p[k], dtype, i);
+            const float4 d = make_float4(th.x - r.x, th.y - r.y, th.z - r.z, th.w - r.w);
+            chk += (d.x + d.y) + (d.z + d.w);
+            if (dare_keep(seed, k, N, i + 0, p)) s.x += d.x * keep_scale;
+            if (dare_keep(seed, k, N, i + 1, p)) s.y += d.y * keep_scale;
+            if (dare_keep(seed, k, N, i + 2, p)) s.z += d.z * keep_scale;
+            if (dare_keep(seed, k, N, i + 3, p)) s.w += d.w * keep_scale;
+        }
+        s.x *= scale; s.y *= scale; s.z *= scale; s.w *= scale;
+        bad |= !isfinite(chk);
+        nesterov1(th.x, bb.x, s.x, eta, mu);
+        nesterov1(th.y, bb.y, s.y, eta, mu);
+        nesterov1(th.z, bb.z, s.z, eta, mu);
+        nesterov1(th.w, bb.w, s.w, eta, mu);
+        *reinterpret_cast<float4*>(mom + i) = bb;
+        *reinterpret_cast<float4*>(theta + i) = th;
+    }
+    if (blockIdx.x == 0) {
+        for (int64_t i = 4 * nv + threadIdx.x; i < N; i += blockDim.x) {
+            float th = theta[i], bb = mom[i], s = 0.f, chk = 0.f;
+            for (int k = 0; k < K; ++k) {
+                const float d = th - ld_rep1(reps.p[k], dtype, i);
+                chk += d;
+                if (dare_keep(seed, k, N, i, p)) s += d * keep_scale;
+            }
+            s *= scale;
+            bad |= !isfinite(chk);
+            nesterov1(th, bb, s, eta, mu);
+            theta[i] = th;
+            mom[i] = bb;
+        }
+    }
+    raise_nonfinite(bad, err);
+}
+
+// TIES trim: per worker k, the key (fp32 bits of |Delta_k|, ordered like the magnitudes) of
+// the rank-th largest magnitude over all N entries, by four radix passes over the 31 key
+// bits: [30:23], [22:15], [14:7], [6:0].  prefix[k] collects the chosen digits; rank[k]
+// starts at the number of entries kept, N - floor(sparsity * N).
+__host__ __device__ constexpr int ties_shift(int pass) { return pass == 0 ? 23 : pass == 1 ? 15 : pass == 2 ? 7 : 0; }
+__host__ __device__ constexpr int ties_bins(int pass) { return pass == 3 ? 128 : 256; }
+
+// Counts, per worker, the digit of this pass of every key whose higher digits equal the
+// prefix chosen so far.  Shared histogram K x 256; keys sharing a bin within a warp are
+// counted by one atomic (most magnitudes fall in a few exponent bins).
+__device__ __forceinline__ void ties_count(uint32_t* sh, int k, uint32_t key, bool valid, int hs, uint32_t phi,
+                                           int shift, uint32_t mask) {
+    const bool m = valid && (key >> hs) == phi;
+    const uint32_t bin = m ? ((key >> shift) & mask) : 0xFFFFFFFFu;
+    const unsigned peers = __match_any_sync(0xffffffffu, bin);
+    if (m && (threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&sh[k * 256 + bin], static_cast<uint32_t>(__popc(peers)));
+}
+
+__global__ void __launch_bounds__(kStreamThreads) k_ties_hist(ReplicaPtrs reps, int K, int dtype,
+                                                              const float* __restrict__ theta, int64_t N, int pass,
+                                                              const uint64_t* __restrict__ prefix,
+                                                              unsigned long long* __restrict__ hist) {
+    extern __shared__ uint32_t sh[];
+    __shared__ uint32_t phi_s[kMaxK];
+    const int shift = ties_shift(pass);
+    const int hs = pass == 0 ? 31 : ties_shift(pass - 1);
+    const uint32_t mask = static_cast<uint32_t>(ties_bins(pass) - 1);
+    for (int j = threadIdx.x; j < K * 256; j += blockDim.x) sh[j] = 0u;
+    for (int k = threadIdx.x; k < K; k += blockDim.x) phi_s[k] = static_cast<uint32_t>(prefix[k]) >> hs;
+    __syncthreads();
+    const int64_t nv = N >> 2;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    // warp-uniform trip count: every lane runs every iteration (match_any over the full warp)
+    const int64_t wbase = blockIdx.x * static_cast<int64_t>(blockDim.x) + (threadIdx.x & ~31);
+    const int lane = threadIdx.x & 31;
+    for (int64_t vb = wbase; vb < nv; vb += stride) {
+        const int64_t v = vb + lane;
+        const bool valid = v < nv;
+        const int64_t i = 4 * (valid ? v : 0);
+        const float4 th = __ldg(reinterpret_cast<const float4*>(theta + i));
+        for (int k = 0; k < K; ++k) {
+            const float4 r = ld_rep4(reps.p[k], dtype, i);
+            const uint32_t ph = phi_s[k];
+            ties_count(sh, k, __float_as_uint(fabsf(th.x - r.x)), valid, hs, ph, shift, mask);
+            ties_count(sh, k, __float_as_uint(fabsf(th.y - r.y)), valid, hs, ph, shift, mask);
+            ties_count(sh, k, __float_as_uint(fabsf(th.z - r.z)), valid, hs, ph, shift, mask);
+            ties_count(sh, k, __float_as_uint(fabsf(th.w - r.w)), valid, hs, ph, shift, mask);
+        }
+    }
+    if (blockIdx.x == 0 && threadIdx.x < 32) {
+        const int64_t i = 4 * nv + lane;
+        const bool valid = i < N;
+        const float th = valid ? __ldg(theta + i) : 0.f;
+        for (int k = 0; k < K; ++k) {
+            const float r = valid ? ld_rep1(reps.p[k], dtype, i) : 0.f;
+            ties_count(sh, k, __float_as_uint(fabsf(th - r)), valid, hs, phi_s[k], shift, mask);
+        }
+    }
+    __syncthreads();
+    for (int j = threadIdx.x; j < K * 256; j += blockDim.x)
+        if (sh[j]) atomicAdd(&hist[j], static_cast<unsigned long long>(sh[j]));
+}
+
+// rank[k] = n_keep, prefix[k] = 0, histogram cleared.  One CTA.
+__global__ void k_ties_init(int K, uint64_t n_keep, unsigned long long* __restrict__ hist,
+                            uint64_t* __restrict__ rank, uint64_t* __restrict__ prefix) {
+    for (int j = threadIdx.x; j < K * 256; j += blockDim.x) hist[j] = 0ull;
+    for (int k = threadIdx.x; k < K; k += blockDim.x) {
+        rank[k] = n_keep;
+        prefix[k] = 0ull;
+    }
+}
+
+// One thread per worker: the bin holding the rank-th largest key (counting from the top),
+// appended to the prefix; the histogram is cleared for the next pass.
+__global__ void k_ties_select(int K, int pass, unsigned long long* __restrict__ hist, uint64_t* __restrict__ rank,
+                              uint64_t* __restrict__ prefix) {
+    const int k = blockIdx.x * blockDim.x + threadIdx.x;
+    if (k >= K) return;
+    unsigned long long* h = hist + static_cast<int64_t>(k) * 256;
+    uint64_t r = rank[k];
+    int digit = 0;
+    for (int b = ties_bins(pass) - 1; b >= 0; --b) {
+        const uint64_t c = h[b];
+        if (r <= c) {
+            digit = b;
+            break;
+        }
+        r -= c;
+    }
+    rank[k] = r;
+    prefix[k] |= static_cast<uint64_t>(digit) << ties_shift(pass);
+    for (int b = 0; b < 256; ++b) h[b] = 0ull;
+}
+
+// TIES elect and disjoint merge.  Entry kept when its key >= thr[k] (ties kept).  P and N
+// are the fp32 sums, in worker order, of the kept positive and negative values; the elected
+// sign is that of P + N, and U the mean of the kept values of that sign (0 if P + N = 0).
+__device__ __forceinline__ float ties_u(float P, float Nn, int cp, int cn) {
+    const float S = __fadd_rn(P, Nn);
+    return S > 0.f ? __fdiv_rn(P, static_cast<float>(cp)) : S < 0.f ? __fdiv_rn(Nn, static_cast<float>(cn)) : 0.f;
+}
+
+__device__ __forceinline__ void ties_acc(float d, uint32_t t, float& P, float& Nn, int& cp, int& cn) {
+    if (__float_as_uint(fabsf(d)) >= t) {
+        if (d > 0.f) { P = __fadd_rn(P, d); ++cp; }
+        if (d < 0.f) { Nn = __fadd_rn(Nn, d); ++cn; }
+    }
+}
+
+__global__ void __launch_bounds__(kStreamThreads) k_ties_merge(ReplicaPtrs reps, int K, int dtype,
+                                                               float* __restrict__ theta, float* __restrict__ mom,
+                                                               int64_t N, const uint64_t* __restrict__ thr,
+                                                               float eta, float mu, uint32_t* __restrict__ err) {
+    __shared__ uint32_t thr_s[kMaxK];
+    for (int k = threadIdx.x; k < K; k += blockDim.x) thr_s[k] = static_cast<uint32_t>(thr[k]);
+    __syncthreads();
+    bool bad = false;
+    const int64_t nv = N >> 2;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t v = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; v < nv; v += stride) {
+        const int64_t i = 4 * v;
+        float4 th = *reinterpret_cast<const float4*>(theta + i);
+        float4 bb = *reinterpret_cast<const float4*>(mom + i);
+        float P[4] = {0.f, 0.f, 0.f, 0.f}, Nn[4] = {0.f, 0.f, 0.f, 0.f}, T = 0.f;
+        int cp[4] = {0, 0, 0, 0}, cn[4] = {0, 0, 0, 0};
+        for (int k = 0; k < K; ++k) {
+            const float4 r = ld_rep4(reps.p[k], dtype, i);
+            const uint32_t t = thr_s[k];
+            const float d[4] = {th.x - r.x, th.y - r.y, th.z - r.z, th.w - r.w};
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                T += d[j];
+                ties_acc(d[j], t, P[j], Nn[j], cp[j], cn[j]);
+            }
+        }
+        bad |= !isfinite(T);
+        nesterov1(th.x, bb.x, ties_u(P[0], Nn[0], cp[0], cn[0]), eta, mu);
+        nesterov1(th.y, bb.y, ties_u(P[1], Nn[1], cp[1], cn[1]), eta, mu);
+        nesterov1(th.z, bb.z, ties_u(P[2], Nn[2], cp[2], cn[2]), eta, mu);
+        nesterov1(th.w, bb.w, ties_u(P[3], Nn[3], cp[3], cn[3]), eta, mu);
+        *reinterpret_cast<float4*>(mom + i) = bb;
+        *reinterpret_cast<float4*>(theta + i) = th;
+    }
+    if (blockIdx.x == 0) {
+        for (int64_t i = 4 * nv + threadIdx.x; i < N; i += blockDim.x) {
+            float th = theta[i], bb = mom[i], P = 0.f, Nn = 0.f, T = 0.f;
+            int cp = 0, cn = 0;
+            for (int k = 0; k < K; ++k) {
+                const float d = th - ld_rep1(reps.p[k], dtype, i);
+                T += d;
+                ties_acc(d, thr_s[k], P, Nn, cp, cn);
+            }
+            bad |= !isfinite(T);
+            nesterov1(th, bb, ties_u(P, Nn, cp, cn), eta, mu);
+            theta[i] = th;
+            mom[i] = bb;
         }
     }
     raise_nonfinite(bad, err);

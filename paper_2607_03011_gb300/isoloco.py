@@ -17,7 +17,7 @@ import torch
 
 from . import _build
 
-PHASES = ["reduce", "gram", "finalize", "control", "poly", "update", "trace", "apply", "diloco", "other"]
+PHASES = ["reduce", "gram", "finalize", "control", "poly", "update", "trace", "apply", "diloco", "other", "trim"]
 
 OK = 0
 ERR_INVALID = -1
@@ -46,7 +46,8 @@ class Opts(ctypes.Structure):
     _fields_ = [("alpha", ctypes.c_float), ("outer_lr", ctypes.c_float), ("momentum", ctypes.c_float),
                 ("reduce_mean", ctypes.c_int), ("max_iter", ctypes.c_int), ("tol", ctypes.c_float),
                 ("sync", ctypes.c_int), ("fast_steps", ctypes.c_int), ("orth_target", ctypes.c_int),
-                ("momentum_kind", ctypes.c_int), ("scale_kind", ctypes.c_int)]
+                ("momentum_kind", ctypes.c_int), ("scale_kind", ctypes.c_int), ("aggregator", ctypes.c_int),
+                ("sparsity", ctypes.c_float), ("seed", ctypes.c_uint)]
 
 
 _lib = None
@@ -108,15 +109,19 @@ def _stream(stream=None) -> int:
 
 
 def make_opts(alpha=1.0, outer_lr=0.7, momentum=0.9, reduce_mean=True, max_iter=0, tol=0.0,
-              sync=False, fast_steps=0, orth_target=0, momentum_kind=0, scale_kind=0) -> Opts:
+              sync=False, fast_steps=0, orth_target=0, momentum_kind=0, scale_kind=0, aggregator=0,
+              sparsity=0.0, seed=0) -> Opts:
     """Options of an outer step; fast_steps > 0 selects the fixed-step variant of Sec. 4.3,
-    the last three the ablations of Sec. 4.5 / App. B (see include/isoloco.h)."""
+    orth_target / momentum_kind / scale_kind the ablations of Sec. 4.5 / App. B, and
+    aggregator / sparsity / seed the merging rule of diloco_outer_step (Sec. 3.2: 0 mean,
+    1 TIES, 2 DARE); see include/isoloco.h."""
     o = Opts()
     lib().isoloco_opts_default(ctypes.byref(o))
     o.alpha, o.outer_lr, o.momentum = float(alpha), float(outer_lr), float(momentum)
     o.reduce_mean, o.max_iter, o.tol, o.sync = int(bool(reduce_mean)), int(max_iter), float(tol), int(bool(sync))
     o.fast_steps = int(fast_steps)
     o.orth_target, o.momentum_kind, o.scale_kind = int(orth_target), int(momentum_kind), int(scale_kind)
+    o.aggregator, o.sparsity, o.seed = int(aggregator), float(sparsity), int(seed) & 0xFFFFFFFF
     return o
 
 
