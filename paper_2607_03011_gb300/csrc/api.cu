@@ -45,8 +45,8 @@ __global__ void k_reduce_p(const Chunk*, const MatDesc*, ReplicaPtrs, int, int, 
 __global__ void k_apply(const Chunk*, const MatDesc*, const MatState*, UpdateSrc, int, float, float, float,
                         float*, float*, const float*, float*, float*, const uint32_t*, int, int, int, const float*);
 __global__ void k_diloco(ReplicaPtrs, int, int, float*, float*, int64_t, float, float, float, uint32_t*);
-__global__ void k_dare(ReplicaPtrs, int, int, float*, float*, int64_t, float, float, float, unsigned int, float,
-                       float, uint32_t*);
+__global__ void k_dare(ReplicaPtrs, int, int, float*, float*, int64_t, float, uint32_t, float, unsigned int,
+                       uint64_t, float, float, uint32_t*);
 __global__ void k_ties_init(int, uint64_t, unsigned long long*, uint64_t*, uint64_t*);
 __global__ void k_ties_hist(ReplicaPtrs, int, int, const float*, int64_t, int, const uint64_t*,
                             unsigned long long*);
@@ -1058,8 +1058,11 @@ int diloco_outer_step(isoloco_plan_t p, float* theta, float* momentum, const voi
                                        p->err_d);
     } else if (o.aggregator == 2) {
         PhaseTimer tm(p, ISOLOCO_PHASE_DILOCO, st);
-        k_dare<<<grid, 256, 0, st>>>(rp, p->K, p->dtype, theta, momentum, p->N, scale, o.sparsity,
-                                     1.f / (1.f - o.sparsity), o.seed, o.outer_lr, o.momentum, p->err_d);
+        // keep when top24 >= ceil(p * 2^24) (exact in double); draw numbers step by N * GAMMA
+        const uint32_t pthr = (uint32_t)std::ceil((double)o.sparsity * 16777216.0);
+        const uint64_t ng = (uint64_t)p->N * 0x9E3779B97F4A7C15ull;
+        k_dare<<<grid, 256, 0, st>>>(rp, p->K, p->dtype, theta, momentum, p->N, scale, pthr,
+                                     1.f / (1.f - o.sparsity), o.seed, ng, o.outer_lr, o.momentum, p->err_d);
     } else {
         // keep the n_keep largest |Delta_k| of each worker; n_keep = N keeps all (threshold 0)
         const uint64_t n_keep = (uint64_t)(p->N - (int64_t)std::floor((double)o.sparsity * (double)p->N));

@@ -325,20 +325,17 @@ __global__ void __launch_bounds__(kStreamThreads) k_diloco(ReplicaPtrs reps, int
 // compute the merged direction U over all N entries and take the outer step
 // B <- mu B + U, theta <- theta - eta (U + mu B) (mu = 0: the SGD step of Sec. 5.1).
 
-// SplitMix64 (Steele, Lea and Flood, 2014): output number n (n >= 1) from state s.
-__device__ __forceinline__ uint64_t splitmix64(uint64_t s, uint64_t n) {
-    uint64_t z = s + n * 0x9E3779B97F4A7C15ull;
+// SplitMix64 (Steele, Lea and Flood, 2014): output number n (n >= 1) from state s is
+// mix(s + n * GAMMA), mix = xor-shift 30, * M1, xor-shift 27, * M2, xor-shift 31.  DARE uses
+// only the top 24 bits of an output: the last xor-shift leaves bits 63..33 as they are, and
+// the top half of the last product is umulhi(lo, M2lo) + lo * M2hi + hi * M2lo (mod 2^32).
+constexpr uint64_t kSmGamma = 0x9E3779B97F4A7C15ull;
+__device__ __forceinline__ uint32_t splitmix64_top24(uint64_t z /* s + n * GAMMA */) {
     z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
-    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
-    return z ^ (z >> 31);
-}
-
-// DARE's mask bit: keep entry i of worker k when the top 24 bits of SplitMix64 output
-// k * N + i + 1, times 2^-24, are >= p.
-__device__ __forceinline__ bool dare_keep(unsigned int seed, int k, int64_t N, int64_t i, float p) {
-    const uint64_t z = splitmix64(seed, static_cast<uint64_t>(k) * static_cast<uint64_t>(N) +
-                                            static_cast<uint64_t>(i) + 1ull);
-    return static_cast<float>(z >> 40) * 0x1p-24f >= p;
+    z ^= z >> 27;
+    const uint32_t lo = static_cast<uint32_t>(z), hi = static_cast<uint32_t>(z >> 32);
+    const uint32_t m_lo = 0x133111EBu, m_hi = 0x94D049BBu;
+    return (__umulhi(lo, m_lo) + lo * m_hi + hi * m_lo) >> 8;
 }
 
 __device__ __forceinline__ void nesterov1(float& th, float& b, float u, float eta, float mu) {
@@ -348,11 +345,14 @@ __device__ __forceinline__ void nesterov1(float& th, float& b, float u, float et
 }
 
 // DARE: U = scale * sum_k keep_scale * m_k * Delta_k, keep_scale = 1 / (1 - p), scale =
-// 1 / K (mean) or 1.  Grid-stride over float4 vectors of all N entries, scalar tail in CTA 0.
+// 1 / K (mean) or 1.  Entry i of worker k is kept when the top 24 bits of SplitMix64 output
+// k * N + i + 1 (state seed) are >= pthr = ceil(p * 2^24), i.e. when that value times 2^-24
+// is >= p.  ng = N * GAMMA (mod 2^64) steps the draw number from one worker to the next.
+// Grid-stride over float4 vectors of all N entries, scalar tail in CTA 0.
 __global__ void __launch_bounds__(kStreamThreads) k_dare(ReplicaPtrs reps, int K, int dtype,
                                                          float* __restrict__ theta, float* __restrict__ mom,
-                                                         int64_t N, float scale, float p, float keep_scale,
-                                                         unsigned int seed, float eta, float mu,
+                                                         int64_t N, float scale, uint32_t pthr, float keep_scale,
+                                                         unsigned int seed, uint64_t ng, float eta, float mu,
                                                          uint32_t* __restrict__ err) {
     bool bad = false;
     const int64_t nv = N >> 2;
@@ -363,14 +363,15 @@ __global__ void __launch_bounds__(kStreamThreads) k_dare(ReplicaPtrs reps, int K
         float4 bb = *reinterpret_cast<const float4*>(mom + i);
         float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
         float chk = 0.f;  // every Delta_k entry, dropped or not, for the non-finite test
-        for (int k = 0; k < K; ++k) {
+        uint64_t z = seed + static_cast<uint64_t>(i + 1) * kSmGamma;  // draw k * N + i + 1, k = 0
+        for (int k = 0; k < K; ++k, z += ng) {
             const float4 r = ld_rep4(reps.p[k], dtype, i);
             const float4 d = make_float4(th.x - r.x, th.y - r.y, th.z - r.z, th.w - r.w);
             chk += (d.x + d.y) + (d.z + d.w);
-            if (dare_keep(seed, k, N, i + 0, p)) s.x += d.x * keep_scale;
-            if (dare_keep(seed, k, N, i + 1, p)) s.y += d.y * keep_scale;
-            if (dare_keep(seed, k, N, i + 2, p)) s.z += d.z * keep_scale;
-            if (dare_keep(seed, k, N, i + 3, p)) s.w += d.w * keep_scale;
+            if (splitmix64_top24(z) >= pthr) s.x += d.x * keep_scale;
+            if (splitmix64_top24(z + kSmGamma) >= pthr) s.y += d.y * keep_scale;
+            if (splitmix64_top24(z + 2 * kSmGamma) >= pthr) s.z += d.z * keep_scale;
+            if (splitmix64_top24(z + 3 * kSmGamma) >= pthr) s.w += d.w * keep_scale;
         }
         s.x *= scale; s.y *= scale; s.z *= scale; s.w *= scale;
         bad |= !isfinite(chk);
@@ -384,10 +385,11 @@ __global__ void __launch_bounds__(kStreamThreads) k_dare(ReplicaPtrs reps, int K
     if (blockIdx.x == 0) {
         for (int64_t i = 4 * nv + threadIdx.x; i < N; i += blockDim.x) {
             float th = theta[i], bb = mom[i], s = 0.f, chk = 0.f;
-            for (int k = 0; k < K; ++k) {
+            uint64_t z = seed + static_cast<uint64_t>(i + 1) * kSmGamma;
+            for (int k = 0; k < K; ++k, z += ng) {
                 const float d = th - ld_rep1(reps.p[k], dtype, i);
                 chk += d;
-                if (dare_keep(seed, k, N, i, p)) s += d * keep_scale;
+                if (splitmix64_top24(z) >= pthr) s += d * keep_scale;
             }
             s *= scale;
             bad |= !isfinite(chk);
