@@ -413,6 +413,9 @@ def main():
                     help="iso_c: the IsoLoCo step (Alg. 2, default); mean / ties / dare: the DiLoCo step "
                          "(Alg. 1) with that merging rule (Sec. 3.2)")
     ap.add_argument("--sparsity", type=float, default=0.1, help="TIES / DARE sparsity (0.1: Sec. 5.1's best)")
+    ap.add_argument("--spectrum", default="iso_c", choices=["iso_c", "clip_high", "clip_low"],
+                    help="the IsoLoCo step's spectrum map (Sec. 4.5): every singular value to the mean (Iso-C), "
+                         "or only those above (clip_high) / below (clip_low) it")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     if args.impl == "reference":
@@ -441,7 +444,9 @@ def main():
     plan = isoloco.Plan(wl.table, wl.N, wl.K, wl.replicas.dtype)
     if args.aggregator != "iso_c":
         return run_diloco(args, torch, isoloco, wl, plan, world, rank, local, dist, barrier)
-    opts = isoloco.make_opts(spec.alpha, spec.outer_lr, spec.momentum, fast_steps=args.fast_steps)
+    spectrum_kind = {"iso_c": 0, "clip_high": 1, "clip_low": 2}[args.spectrum]
+    opts = isoloco.make_opts(spec.alpha, spec.outer_lr, spec.momentum, fast_steps=args.fast_steps,
+                             spectrum_kind=spectrum_kind)
     theta0, mom0 = wl.theta.clone(), wl.momentum.clone()
     th, b = wl.theta, wl.momentum
     stream = torch.cuda.current_stream()
@@ -594,7 +599,8 @@ def main():
                              "restored between steps outside the intervals",
                    "parallelism": f"replicas x{world}",
                    "iso_c": ("exact polar, sigma_bar = tr(Q^T Delta)/r" if not args.fast_steps else
-                             f"fast variant: {args.fast_steps} fixed polar steps, sigma_bar = ||Delta||_F/sqrt(r)")},
+                             f"fast variant: {args.fast_steps} fixed polar steps, sigma_bar = ||Delta||_F/sqrt(r)"),
+                   "spectrum": args.spectrum},
         "status": isoloco.STATUS_NAMES.get(status, status),
         "polar_iters": {"min": min(iters), "max": max(iters), "mean": sum(iters) / len(iters)},
         "phases_ms_per_step": phases_ms, "phases_algorithmic_tflops": phases_tflops,

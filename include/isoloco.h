@@ -109,6 +109,13 @@ typedef struct {
                         * u < sparsity, u = top 24 bits of SplitMix64 output number
                         * k * n_total + i + 1 from state `seed` (Steele, Lea and Flood 2014),
                         * times 2^-24. */
+    int spectrum_kind; /* isoloco_outer_step's spectrum map (Sec. 4.5): 0: Iso-C, every
+                        * singular value set to sigma_bar (Alg. 2).  1: clip_high, only the
+                        * singular values above sigma_bar set to it, U = alpha * U_D
+                        * diag(min(s_i, sigma_bar)) V_D^T.  2: clip_low, only those below,
+                        * max(s_i, sigma_bar).  1 and 2 need fast_steps = 0 and scale_kind = 0;
+                        * their first call allocates an auxiliary plan (the n x n matrices
+                        * H - sigma_bar I, H = Q^T Delta) and its buffers. */
 } isoloco_opts_t;
 
 /* Fills *opts with alpha = 1, outer_lr = 0.7, momentum = 0.9 (the paper's DiLoCo
@@ -243,7 +250,8 @@ enum {
     ISOLOCO_PHASE_DILOCO = 8,   /* fused DiLoCo pass (mean, DARE, or TIES's merge pass) */
     ISOLOCO_PHASE_OTHER = 9,
     ISOLOCO_PHASE_TRIM = 10,    /* TIES trim: per-worker radix select of the threshold */
-    ISOLOCO_NUM_PHASES = 11
+    ISOLOCO_PHASE_CLIP = 11,    /* clip_high / clip_low: H, sign(H - sigma_bar I), E P_sel */
+    ISOLOCO_NUM_PHASES = 12
 };
 
 /* Per-phase timing.  enable != 0 makes every later call record a CUDA event pair

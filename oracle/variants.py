@@ -12,6 +12,10 @@ Alg. 2's outer step, with the choices the paper's ablations vary:
   RMS ||X||_F / sqrt(r)); scale_kind 1: Muon's spectral scale sqrt(rows / cols) (App. B).
 * fast_steps k > 0: the polar factor by k fixed quintic steps (oracle/fast_ns.py) instead
   of the SVD.
+* spectrum_kind 1 (clip_high) / 2 (clip_low), Sec. 4.5: only the singular values above /
+  below their mean sigma_bar are set to it, the others kept: U = alpha * U_D diag(f(s)) V_D^T
+  with f(s) = min(s, sigma_bar) / max(s, sigma_bar), from the oracle's SVD.  Singular values
+  that the SVD finds zero (below r * eps * s_max) stay zero, as in Iso-C's partial isometry.
 * Excluding a 2-D tensor from Iso-C (Sec. 4.5) is a table choice: it is listed as a 1-D
   tensor of rows * cols elements and updated with Delta.
 
@@ -20,13 +24,15 @@ reduction and the SVD-based Iso-C are the pinned C oracle's (oracle/isoloco_orac
 
 Parity status: pinned (``tests/test_oracle_variants.py``: default flags reproduce the
 oracle's Alg. 2, mu = 0 collapses every momentum choice to Eq. 2, closed forms on
-c * orthogonal inputs, a hand-worked standard-momentum scalar).
+c * orthogonal inputs, a hand-worked standard-momentum scalar; the clip variants by a
+diagonal worked example, clip_high + clip_low = Delta + Iso-C(Delta), their spectra against
+LAPACK's, and orthogonal equivariance).
 """
 from __future__ import annotations
 
 import numpy as np
 
-from . import fast_ns, iso_c, pseudo_gradient
+from . import fast_ns, iso_c, pseudo_gradient, svd
 
 
 def _polar_and_sigma(x: np.ndarray, fast_steps: int):
@@ -40,9 +46,23 @@ def _polar_and_sigma(x: np.ndarray, fast_steps: int):
     return q, float(sigma)
 
 
+def clip_spectrum(x: np.ndarray, kind: int):
+    """(U diag(f(s)) V^T, sigma_bar) of one matrix, f(s) = min(s, sigma_bar) (kind 1,
+    clip_high) or max(s, sigma_bar) (kind 2, clip_low), sigma_bar = sum(s) / min(m, n)."""
+    u, s, v = svd(np.asarray(x, dtype=np.float64))
+    r = min(x.shape)
+    sbar = float(s.sum() / r)
+    smax = float(s.max()) if s.size else 0.0
+    if not smax > 0.0:
+        return np.zeros(x.shape), 0.0
+    nz = s > r * np.finfo(np.float64).eps * smax
+    f = np.where(nz, np.minimum(s, sbar) if kind == 1 else np.maximum(s, sbar), 0.0)
+    return (u * f) @ v.T, sbar
+
+
 def isoloco_outer_step_variant(table, theta, momentum, replicas, alpha=1.0, eta=0.7, mu=0.9,
                                orth_target=0, momentum_kind=0, scale_kind=0, fast_steps=0,
-                               reduce_mean=True, only=None):
+                               reduce_mean=True, only=None, spectrum_kind=0):
     """Returns dict(theta, momentum, update, sigma_bar) in fp64 (sigma_bar per table entry,
     0 for 1-D tensors); entries of parameters outside ``only`` are NaN."""
     th = np.asarray(theta, dtype=np.float64).ravel()
@@ -61,7 +81,10 @@ def isoloco_outer_step_variant(table, theta, momentum, replicas, alpha=1.0, eta=
         if orth_target:
             nb = mu * b + d
             p = d + mu * nb if momentum_kind == 0 else nb
-            if cols > 0:
+            if cols > 0 and spectrum_kind:
+                um, sig[i] = clip_spectrum(p.reshape(rows, cols), spectrum_kind)
+                u = alpha * um.ravel()
+            elif cols > 0:
                 q, sigma = _polar_and_sigma(p.reshape(rows, cols), fast_steps)
                 sig[i] = sigma
                 u = alpha * (sigma if scale_kind == 0 else np.sqrt(rows / cols)) * q.ravel()
@@ -69,7 +92,10 @@ def isoloco_outer_step_variant(table, theta, momentum, replicas, alpha=1.0, eta=
                 u = p
             to[sl] = th[sl] - eta * u
         else:
-            if cols > 0:
+            if cols > 0 and spectrum_kind:
+                um, sig[i] = clip_spectrum(d.reshape(rows, cols), spectrum_kind)
+                u = alpha * um.ravel()
+            elif cols > 0:
                 q, sigma = _polar_and_sigma(d.reshape(rows, cols), fast_steps)
                 sig[i] = sigma
                 u = alpha * (sigma if scale_kind == 0 else np.sqrt(rows / cols)) * q.ravel()

@@ -44,6 +44,15 @@ __global__ void k_reduce_p(const Chunk*, const MatDesc*, ReplicaPtrs, int, int, 
                            __nv_bfloat16*, __nv_bfloat16*, float*, uint32_t*, int, float, const float*, float*);
 __global__ void k_apply(const Chunk*, const MatDesc*, const MatState*, UpdateSrc, int, float, float, float,
                         float*, float*, const float*, float*, float*, const uint32_t*, int, int, int, const float*);
+__global__ void k_clip_q_bf16(const MatDesc*, const MatState*, __nv_bfloat16*, __nv_bfloat16*, __nv_bfloat16*,
+                              __nv_bfloat16*);
+__global__ void k_clip_form_a(const MatDesc*, const MatState*, const float*, const int64_t*, const int64_t*,
+                              const int*, const MatDesc*, const int*, __nv_bfloat16*, __nv_bfloat16*);
+__global__ void k_clip_form_p(const MatDesc*, const MatState*, __nv_bfloat16*, __nv_bfloat16*, __nv_bfloat16*,
+                              __nv_bfloat16*, float);
+__global__ void k_clip_form_s(const MatDesc*, const MatDesc*, const int*, const MatState*, const __nv_bfloat16*,
+                              const __nv_bfloat16*, __nv_bfloat16*, __nv_bfloat16*, const uint32_t*, uint32_t*);
+__global__ void k_clip_flip(MatState*, int);
 __global__ void k_diloco(ReplicaPtrs, int, int, float*, float*, int64_t, float, float, float, uint32_t*);
 __global__ void k_dare(ReplicaPtrs, int, int, float*, float*, int64_t, float, uint32_t, float, unsigned int,
                        uint64_t, float, float, uint32_t*);
@@ -137,6 +146,9 @@ struct isoloco_plan {
     int g_max_iter = -1;
     float g_tol = 0.f;
     int g_fast = -1;
+    int g_full = -1;
+    bool full_prec = false;         // every polar step with three passes and no Horner form
+                                    // (the clip variants' sign iteration)
     int fast_steps = 0;             // this call's fast-variant step count (0: exact Iso-C)
     bool skip_trace = false;        // this call needs no tr(Q^T Delta) (fast variant, spectral scale)
     float* bnew = nullptr;          // B' of the orthogonalise-P ablation (allocated on first use)
@@ -149,6 +161,15 @@ struct isoloco_plan {
     double prof_ms[ISOLOCO_NUM_PHASES] = {0};
     int64_t prof_n[ISOLOCO_NUM_PHASES] = {0};
     int64_t launches = 0;
+    // clip variants (Sec. 4.5), allocated on first use: the plan of the n x n matrices
+    // H - sigma_bar I whose polar factors are sign(H - sigma_bar I); fp32 H (split-K
+    // partials) with per-matrix offsets and split strides; aux matrix index of each matrix
+    isoloco_plan* aux = nullptr;
+    float* hbuf = nullptr;
+    int64_t* hoff_d = nullptr;
+    int64_t* hss_d = nullptr;
+    int* aux_of_d = nullptr;
+    std::vector<int64_t> hbucket_off;
     // TIES trim: per-worker radix-select histogram (K x 256), rank and chosen key prefix
     unsigned long long* ties_hist = nullptr;
     uint64_t* ties_rank = nullptr;
@@ -244,6 +265,7 @@ static int dalloc(isoloco_plan* p, T** ptr, int64_t count) {
 
 static void free_plan(isoloco_plan* p) {
     if (!p) return;
+    if (p->aux) free_plan(p->aux);
     for (void* a : p->allocs) cudaFree(a);
     for (int ph = 0; ph < ISOLOCO_NUM_PHASES; ++ph)
         for (auto& pr : p->pend[ph]) {
@@ -627,10 +649,12 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
         const bool first = (t == 0);
         // The fast variant stops after a fixed number of steps, so nothing corrects a step's
         // rounding afterwards: every step splits both operands (fp16 three passes) and the
-        // polynomial is formed from G's hi/lo planes (no single-plane Y).  The converging
-        // path keeps one operand single from iteration 1 on (its rounding only perturbs the
-        // spectrum, which later steps correct).
-        const bool full = p->fast_steps > 0;
+        // polynomial is formed from G's hi/lo planes (no single-plane Y).  So does the clip
+        // variants' sign iteration (full_prec): there a single-plane rounding perturbs the
+        // invariant subspaces the result must separate, which later steps do not undo.  The
+        // converging path keeps one operand single from iteration 1 on (its rounding only
+        // perturbs the spectrum, which later steps correct).
+        const bool full = p->fast_steps > 0 || p->full_prec;
         const Precision gram_pr = first ? Precision{0, 0, 1, 1, 0}
                                         : (full ? Precision{1, 1, 1, 1, 0} : Precision{1, 1, 1, 0, 0});
         LaunchSet tall, wide;
@@ -805,6 +829,7 @@ static int build_polar_graph(isoloco_plan* p, int max_iter, float tol) {
     p->g_max_iter = max_iter;
     p->g_tol = tol;
     p->g_fast = p->fast_steps;
+    p->g_full = p->full_prec ? 1 : 0;
     return ISOLOCO_OK;
 }
 
@@ -821,7 +846,8 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
     CUDA_TRY(cudaStreamIsCapturing(st, &cs));
     const bool use_graph = kPairMma && !p->prof && cs == cudaStreamCaptureStatusNone;
     if (use_graph) {
-        if (!p->gexec || p->g_max_iter != max_iter || p->g_tol != tol || p->g_fast != p->fast_steps)
+        if (!p->gexec || p->g_max_iter != max_iter || p->g_tol != tol || p->g_fast != p->fast_steps ||
+            p->g_full != (p->full_prec ? 1 : 0))
             if ((rc = build_polar_graph(p, max_iter, tol))) return rc;
         CUDA_TRY(cudaGraphLaunch(p->gexec, st));
     } else {
@@ -856,6 +882,214 @@ static int finish_call(isoloco_plan* p, cudaStream_t st, int sync) {
     return isoloco_last_status(p, st);
 }
 
+// ---------------------------------------------------------------- clip variants (Sec. 4.5)
+// Creates, on first use, the auxiliary plan (one n x n matrix per matrix of the plan, the
+// same n) and the fp32 buffer of H.
+static int ensure_clip(isoloco_plan* p) {
+    if (p->aux) return ISOLOCO_OK;
+    std::vector<isoloco_param_t> t(p->nmat);
+    int64_t off = 0;
+    for (int i = 0; i < p->nmat; ++i) {
+        const int n = p->mats_h[i].n;
+        t[i].offset = off;
+        t[i].rows = n;
+        t[i].cols = n;
+        off += (int64_t)n * n;
+    }
+    isoloco_plan_t a = nullptr;
+    int rc = isoloco_plan_create(&a, t.data(), (int)t.size(), off, 1, ISOLOCO_F32);
+    if (rc) return rc;
+    // aux matrix i holds aux parameter aux->mat_param[i], i.e. this plan's matrix of that index
+    std::vector<int> aux_of(p->nmat);
+    for (int j = 0; j < a->nmat; ++j) aux_of[a->mat_param[j]] = j;
+    std::vector<int64_t> hoff(p->nmat), hss(p->nmat);
+    int64_t hb = 0;
+    p->hbucket_off.clear();
+    for (const Bucket& bk : p->buckets) {
+        const int64_t g = (int64_t)bk.n * bk.ld_n;
+        p->hbucket_off.push_back(hb);
+        for (int j = 0; j < bk.count; ++j) {
+            hoff[bk.mat_base + j] = hb + j * g;
+            hss[bk.mat_base + j] = (int64_t)bk.count * g;
+        }
+        hb += round_up((int64_t)bk.splits * bk.count * g, 128);
+    }
+    if ((rc = dalloc(p, &p->hbuf, hb)) || (rc = dalloc(p, &p->hoff_d, p->nmat)) ||
+        (rc = dalloc(p, &p->hss_d, p->nmat)) || (rc = dalloc(p, &p->aux_of_d, p->nmat))) {
+        isoloco_plan_destroy(a);
+        return rc;
+    }
+    p->aux = a;
+    CUDA_TRY(cudaMemcpy(p->hoff_d, hoff.data(), sizeof(int64_t) * p->nmat, cudaMemcpyHostToDevice));
+    CUDA_TRY(cudaMemcpy(p->hss_d, hss.data(), sizeof(int64_t) * p->nmat, cudaMemcpyHostToDevice));
+    CUDA_TRY(cudaMemcpy(p->aux_of_d, aux_of.data(), sizeof(int) * p->nmat, cudaMemcpyHostToDevice));
+    return ISOLOCO_OK;
+}
+
+// After the polar iteration and the trace pass (Q and sigma_bar known): Q S' in the ping-pong
+// buffer that did not hold Q, and final_buf pointed at it, so that the apply pass forms
+// U = alpha sigma_bar Q S' (derivation in spectral.cu).  kind 1: clip_high, 2: clip_low.
+static int run_clip(isoloco_plan* p, int kind, int max_iter, float tol, cudaStream_t st) {
+    if (p->nmat == 0) return ISOLOCO_OK;
+    int rc;
+    if ((rc = ensure_clip(p))) return rc;
+    isoloco_plan* a = p->aux;
+    const CUtensorMap* maps = p->tmaps_d;
+    const dim3 grid(64, p->nmat);
+    { PhaseTimer tm(p, ISOLOCO_PHASE_CLIP, st);
+    k_clip_q_bf16<<<grid, 256, 0, st>>>(p->mats_d, p->state, p->xhi[0], p->xlo[0], p->xhi[1], p->xlo[1]); }
+    CUDA_TRY(cudaGetLastError());
+    // ---- H = Qb^T Delta (tall, MN-major operands) or Delta Qb^T (wide, K-major), fp32,
+    // upper-triangle tiles mirrored; one group per (bucket, buffer holding Q)
+    LaunchSet htall, hwide;
+    init_set(htall, kEpiF32, kGateNone, p, Precision{0, 0, 1, 1, 0});
+    init_set(hwide, kEpiF32, kGateNone, p, Precision{0, 0, 1, 1, 0});
+    htall.p.list = hwide.p.list = nullptr;
+    htall.p.cnt = hwide.p.cnt = nullptr;
+    for (size_t b = 0; b < p->buckets.size(); ++b) {
+        const Bucket& bk = p->buckets[b];
+        const CUtensorMap* m = maps + b * kMapsPerBucket;
+        for (int fb = 0; fb < 2; ++fb) {
+            const int qsrc = 1 + (1 - fb);  // the bf16 copy of Q sits in the other buffer
+            GemmGroup g{};
+            if (bk.tall) {
+                g.a_hi = m + src_map(qsrc, kRoleMN, 0);
+                g.a_lo = m + src_map(qsrc, kRoleMN, 1);
+                g.b_hi = m + src_map(0, kRoleMN, 0);
+                g.b_lo = m + src_map(0, kRoleMN, 1);
+            } else {
+                g.a_hi = m + src_map(0, kRoleKA, 0);
+                g.a_lo = m + src_map(0, kRoleKA, 1);
+                g.b_hi = m + src_map(qsrc, kRoleKB, 0);
+                g.b_lo = m + src_map(qsrc, kRoleKB, 1);
+            }
+            set_group_common(g, bk.n, bk.n, bk.tall ? bk.rows : bk.cols, bk.count, bk.splits, bk.mat_base);
+            g.bucket = (int)b;
+            g.gate_fb = fb + 1;
+            g.out_f32 = p->hbuf + p->hbucket_off[b];
+            g.f32_batch_stride = (int64_t)bk.n * bk.ld_n;
+            g.f32_split_stride = (int64_t)bk.count * bk.n * bk.ld_n;
+            g.ld_f32 = bk.ld_n;
+            set_sym(g, bk.n);
+            (bk.tall ? htall : hwide).add(g);
+        }
+    }
+    if ((rc = flush_set(p, ISOLOCO_PHASE_CLIP, htall, true, true, st)) ||
+        (rc = flush_set(p, ISOLOCO_PHASE_CLIP, hwide, false, false, st)))
+        return rc;
+    // ---- A' = H / sigma_bar - I -> the auxiliary plan; its polar factor Q_A = sign(A');
+    // P = (I -/+ Q_A) / 2; S'' = (P A') P, all in the auxiliary plan's planes
+    { PhaseTimer tm(p, ISOLOCO_PHASE_CLIP, st, 0);
+    k_reset_state<<<(std::max(1, a->nmat) + 255) / 256, 256, 0, st>>>(
+        a->state, a->nmat, a->err_d, a->mats_d, a->bucket_first_d, a->bucket_count_d, (int)a->buckets.size(),
+        a->list_gram, a->cnt_gram, a->counters, kLaunchCounters);
+    a->launches += 1;
+    a->launch_seq = 0;
+    CUDA_TRY(cudaGetLastError());
+    k_clip_form_a<<<grid, 256, 0, st>>>(p->mats_d, p->state, p->hbuf, p->hoff_d, p->hss_d, p->nsplit_d, a->mats_d,
+                                         p->aux_of_d, a->dhi, a->dlo);
+    p->launches += 1;
+    CUDA_TRY(cudaGetLastError());
+    a->fast_steps = 0;
+    a->skip_trace = true;
+    a->full_prec = true;  // sign(A') is used to first order (P A' P): no single-plane steps
+    if ((rc = run_polar(a, max_iter, tol, st))) return rc;
+    k_clip_form_p<<<dim3(64, a->nmat), 256, 0, st>>>(a->mats_d, a->state, a->xhi[0], a->xlo[0], a->xhi[1],
+                                                     a->xlo[1], kind == 1 ? -1.f : 1.f);
+    a->launches += 1;
+    CUDA_TRY(cudaGetLastError());
+    const CUtensorMap* amaps = a->tmaps_d;
+    for (int step = 0; step < 2; ++step) {
+        // step 0: T = P A' -> G planes; step 1: S'' = T P -> P planes (P and A' symmetric,
+        // so their K-major role reads them as they are); bf16, three passes
+        LaunchSet ls;
+        init_set(ls, kEpiXSplit, kGateNone, a, Precision{0, 0, 1, 1, 0});
+        ls.p.list = nullptr;
+        ls.p.cnt = nullptr;
+        for (size_t b = 0; b < a->buckets.size(); ++b) {
+            const Bucket& bk = a->buckets[b];
+            const CUtensorMap* m = amaps + b * kMapsPerBucket;
+            for (int fa = 0; fa < 2; ++fa) {
+                const int psrc = 1 + (1 - fa);  // P sits in the buffer not holding Q_A
+                GemmGroup g{};
+                if (step == 0) {
+                    g.a_hi = m + src_map(psrc, kRoleKA, 0);
+                    g.a_lo = m + src_map(psrc, kRoleKA, 1);
+                    g.b_hi = m + src_map(0, kRoleKB, 0);
+                    g.b_lo = m + src_map(0, kRoleKB, 1);
+                    g.out_hi = a->ghi + bk.gplane_off;
+                    g.out_lo = a->glo + bk.gplane_off;
+                    g.st_hi = m + st_map(2, 0);
+                    g.st_lo = m + st_map(2, 1);
+                } else {
+                    g.a_hi = m + g_map(kRoleKA, 0);
+                    g.a_lo = m + g_map(kRoleKA, 1);
+                    g.b_hi = m + src_map(psrc, kRoleKB, 0);
+                    g.b_lo = m + src_map(psrc, kRoleKB, 1);
+                    g.out_hi = a->phi + bk.gplane_off;
+                    g.out_lo = a->plo + bk.gplane_off;
+                    g.st_hi = m + st_map(3, 0);
+                    g.st_lo = m + st_map(3, 1);
+                }
+                set_group_common(g, bk.n, bk.n, bk.n, bk.count, 1, bk.mat_base);
+                g.bucket = (int)b;
+                g.gate_fb = fa + 1;
+                g.bf_batch_stride = (int64_t)bk.n * bk.ld_n;
+                g.ld_bf = bk.ld_n;
+                ls.add(g);
+            }
+        }
+        if ((rc = flush_set(a, ISOLOCO_PHASE_CLIP, ls, false, false, st))) return rc;
+    } }
+    // ---- S' = I + S'' -> this plan's P planes (fp16); X = Q S' (tall) or S' Q (wide) into
+    // the other ping-pong buffer (fp16, three passes), which then holds the result
+    { PhaseTimer tm(p, ISOLOCO_PHASE_CLIP, st);
+    k_clip_form_s<<<grid, 256, 0, st>>>(p->mats_d, a->mats_d, p->aux_of_d, a->state, a->phi, a->plo, p->phi, p->plo,
+                                         a->err_d, p->err_d); }
+    CUDA_TRY(cudaGetLastError());
+    LaunchSet ut, uw;
+    init_set(ut, kEpiXSplit, kGateNone, p, Precision{1, 1, 1, 1, 0});
+    init_set(uw, kEpiXSplit, kGateNone, p, Precision{1, 1, 1, 1, 0});
+    ut.p.list = uw.p.list = nullptr;
+    ut.p.cnt = uw.p.cnt = nullptr;
+    for (size_t b = 0; b < p->buckets.size(); ++b) {
+        const Bucket& bk = p->buckets[b];
+        const CUtensorMap* m = maps + b * kMapsPerBucket;
+        for (int fb = 0; fb < 2; ++fb) {
+            const int src = 1 + fb, dst = 1 - fb;
+            GemmGroup g{};
+            if (bk.tall) {
+                g.a_hi = m + src_map(src, kRoleKA, 0);
+                g.a_lo = m + src_map(src, kRoleKA, 1);
+                g.b_hi = m + p_map(kRoleKB, 0);
+                g.b_lo = m + p_map(kRoleKB, 1);
+            } else {
+                g.a_hi = m + p_map(kRoleKA, 0);
+                g.a_lo = m + p_map(kRoleKA, 1);
+                g.b_hi = m + src_map(src, kRoleMN, 0);
+                g.b_lo = m + src_map(src, kRoleMN, 1);
+            }
+            set_group_common(g, bk.rows, bk.cols, bk.n, bk.count, 1, bk.mat_base);
+            g.bucket = (int)b;
+            g.gate_fb = fb + 1;
+            g.out_hi = p->xhi[dst] + bk.plane_off;
+            g.out_lo = p->xlo[dst] + bk.plane_off;
+            g.st_hi = m + st_map(dst, 0);
+            g.st_lo = m + st_map(dst, 1);
+            g.bf_batch_stride = (int64_t)bk.rows * bk.ld;
+            g.ld_bf = bk.ld;
+            (bk.tall ? ut : uw).add(g);
+        }
+    }
+    if ((rc = flush_set(p, ISOLOCO_PHASE_CLIP, ut, false, false, st)) ||
+        (rc = flush_set(p, ISOLOCO_PHASE_CLIP, uw, false, true, st)))
+        return rc;
+    { PhaseTimer tm(p, ISOLOCO_PHASE_CLIP, st);
+    k_clip_flip<<<(p->nmat + 255) / 256, 256, 0, st>>>(p->state, p->nmat); }
+    CUDA_TRY(cudaGetLastError());
+    return ISOLOCO_OK;
+}
+
 static int check_opts(const isoloco_opts_t* o, isoloco_opts_t* out) {
     isoloco_opts_default(out);
     if (o) *out = *o;
@@ -869,6 +1103,11 @@ static int check_opts(const isoloco_opts_t* o, isoloco_opts_t* out) {
     if (out->aggregator < 0 || out->aggregator > 2) return fail(ISOLOCO_ERR_INVALID, "aggregator must be 0, 1 or 2");
     if (!(out->sparsity >= 0.f && out->sparsity < 1.f))
         return fail(ISOLOCO_ERR_INVALID, "sparsity must be in [0, 1)");
+    if (out->spectrum_kind < 0 || out->spectrum_kind > 2)
+        return fail(ISOLOCO_ERR_INVALID, "spectrum_kind must be 0, 1 or 2");
+    if (out->spectrum_kind && (out->fast_steps || out->scale_kind))
+        return fail(ISOLOCO_ERR_INVALID, "clip_high / clip_low need the exact polar path and sigma_bar "
+                                         "(fast_steps = 0, scale_kind = 0)");
     return ISOLOCO_OK;
 }
 
@@ -918,8 +1157,11 @@ static int run_isoc_step(isoloco_plan* p, int merge, float* theta, float* mom, c
         CUDA_TRY(cudaGetLastError());
     }
     p->fast_steps = merge ? 0 : o.fast_steps;
+    p->full_prec = !merge && o.spectrum_kind != 0;
     p->skip_trace = !merge && (o.fast_steps > 0 || o.scale_kind == 1);
     if ((rc = run_polar(p, p->fast_steps ? std::max(o.max_iter, o.fast_steps) : o.max_iter, o.tol, st))) return rc;
+    const int clip = merge ? 0 : o.spectrum_kind;
+    if (clip && (rc = run_clip(p, clip, o.max_iter, o.tol, st))) return rc;
     UpdateSrc us;
     us.qh[0] = p->xhi[0];
     us.qh[1] = p->xhi[1];
@@ -961,6 +1203,7 @@ int isoloco_opts_default(isoloco_opts_t* o) {
     o->aggregator = 0;
     o->sparsity = 0.f;
     o->seed = 0u;
+    o->spectrum_kind = 0;
     return ISOLOCO_OK;
 }
 
@@ -1173,7 +1416,7 @@ int64_t isoloco_plan_launches(isoloco_plan_t p) {
     long long runs[2] = {0, 0};
     if (p->body_launches > 0 && cudaMemcpy(runs, p->loopc, sizeof(runs), cudaMemcpyDeviceToHost) != cudaSuccess)
         runs[1] = 0;
-    return p->launches + p->body_launches * static_cast<int64_t>(runs[1]);
+    return p->launches + p->body_launches * static_cast<int64_t>(runs[1]) + (p->aux ? isoloco_plan_launches(p->aux) : 0);
 }
 
 int isoloco_read_diag(isoloco_plan_t p, void* stream, float* sigma_bar, int32_t* iters, int32_t* status,

@@ -118,6 +118,7 @@ __device__ __forceinline__ bool decode_tile(const GemmParams& p, const int* pre,
     ti.b_split = p.b_split != 0;
     ti.ca = 0.f, ti.cb = 0.f, ti.cc = 1.f, ti.xs = 1.f, ti.yb = 0.f, ti.yc = 0.f;
     ti.horner = false;
+    if (g.gate_fb && p.state[ti.mat].final_buf != g.gate_fb - 1) return false;
     if (p.gate != kGateNone) {
         const MatState& st = p.state[ti.mat];
         if (p.gate == kGateActive) {

@@ -83,6 +83,7 @@ struct GemmGroup {
     int cta_begin;  // (host bookkeeping) first tile of the group when every matrix is active
     int mat_base;   // index of the group's first matrix in the state array
     int bucket;     // shape bucket: index into the work-list counts
+    int gate_fb;    // 0: no condition; f > 0: only matrices whose Q is in buffer f - 1 (final_buf)
     // fp32 output (kEpiF32): out_f32 + split*split_stride + b*batch_stride + row*ld + col
     float* out_f32;
     int64_t f32_split_stride, f32_batch_stride;

@@ -223,6 +223,9 @@ ABLATIONS = [
     {"scale_kind": 1},                                   # Muon's spectral scale sqrt(rows / cols)
     {"scale_kind": 1, "fast_steps": 5},                  # fixed steps + spectral scale (Muon-like)
     {"orth_target": 1, "fast_steps": 5},
+    {"spectrum_kind": 1},                                # clip_high: s_i > sigma_bar -> sigma_bar
+    {"spectrum_kind": 2},                                # clip_low: s_i < sigma_bar -> sigma_bar
+    {"spectrum_kind": 1, "orth_target": 1},
 ]
 
 
@@ -244,6 +247,40 @@ def test_ablation_variants(iso, flags):
         ref["sigma_bar"] = np.asarray(ref["sigma_bar"])
     check_step(wl.table, th.double().cpu().numpy(), b.double().cpu().numpy(), upd.double().cpu().numpy(),
                sigma, ref)
+
+
+@pytest.mark.parametrize("kind", [1, 2])
+def test_clip_180m_sampled(iso, kind):
+    """clip_high / clip_low on the benchmarked configuration at full size."""
+    sampled_parity(iso, "llama_180m_k8", ("layers.0.wq", "layers.5.w_gate", "layers.11.w_down", "head"),
+                   spectrum_kind=kind)
+
+
+@pytest.mark.parametrize("kind", [1, 2])
+def test_clip_tiny_bf16_and_zero(iso, kind):
+    """bf16 replicas; then replicas equal to theta (Delta = 0): U = 0, status OK."""
+    from oracle import variants
+    spec = W.custom_spec(W.tiny_shapes(), K=2, rank=4, replica_dtype="bf16", momentum_std=1e-4)
+    wl = W.make_workload(spec, seed=21, device="cuda")
+    rc, th, b, upd, diag, plan = run_gpu(iso, wl, 1.0, 0.7, 0.9, spectrum_kind=kind)
+    assert rc == 0
+    ref = variants.isoloco_outer_step_variant(
+        wl.table, wl.theta.cpu().numpy(), wl.momentum.cpu().numpy(), W.replicas_as_numpy(wl.replicas),
+        alpha=1.0, eta=0.7, mu=0.9, spectrum_kind=kind)
+    ref["theta_in"] = wl.theta.double().cpu().numpy()
+    check_step(wl.table, th.double().cpu().numpy(), b.double().cpu().numpy(), upd.double().cpu().numpy(),
+               diag["sigma_bar"], ref)
+    same = wl.theta.to(torch.bfloat16).float().to(torch.bfloat16).expand(wl.K, -1).contiguous()
+    th0 = wl.theta.to(torch.bfloat16).float()
+    rc, th, b, upd, diag, _ = run_gpu(iso, wl, 1.0, 0.7, 0.9, reps=same, theta=th0, plan=plan, spectrum_kind=kind)
+    assert rc == 0 and float(upd.abs().max()) == 0.0
+
+
+def test_clip_options_rejected(iso):
+    wl = W.make_workload("tiny", seed=0, device="cuda")
+    for flags in ({"spectrum_kind": 3}, {"spectrum_kind": 1, "fast_steps": 5}, {"spectrum_kind": 2, "scale_kind": 1}):
+        with pytest.raises(iso.IsolocoError):
+            run_gpu(iso, wl, 1.0, 0.7, 0.9, **flags)
 
 
 def test_excluded_matrix_is_listed_as_1d(iso):
@@ -300,13 +337,14 @@ def test_host_buffer_entry_point(iso):
     assert torch.equal(th_h, th.cpu()) and torch.equal(b_h, b.cpu())
 
 
-def sampled_parity(iso, workload, pick_names, fast_steps=0):
+def sampled_parity(iso, workload, pick_names, fast_steps=0, **ablation):
     """A configuration at full size on the GPU (the launch configuration bench.py times),
     checked against the oracle on the sampled matrices plus every 1-D tensor (each matrix's
     Iso-C and each element's Nesterov step are independent of the others)."""
     wl = W.make_workload(workload, seed=0, device="cuda")
     sp = wl.spec
-    rc, th, b, upd, diag, plan = run_gpu(iso, wl, sp.alpha, sp.outer_lr, sp.momentum, fast_steps=fast_steps)
+    rc, th, b, upd, diag, plan = run_gpu(iso, wl, sp.alpha, sp.outer_lr, sp.momentum, fast_steps=fast_steps,
+                                         **ablation)
     assert rc == 0
     names = [s[0] for s in sp.shapes]
     pick = [names.index(n) for n in pick_names]
@@ -320,7 +358,13 @@ def sampled_parity(iso, workload, pick_names, fast_steps=0):
         parts.append((o, n))
         off += n
     idx = torch.cat([torch.arange(o, o + n, device="cuda") for o, n in parts])
-    if fast_steps:
+    if ablation:
+        from oracle import variants
+        ref = variants.isoloco_outer_step_variant(
+            sub_table, wl.theta[idx].cpu().numpy(), wl.momentum[idx].cpu().numpy(),
+            W.replicas_as_numpy(wl.replicas[:, idx]), alpha=sp.alpha, eta=sp.outer_lr, mu=sp.momentum,
+            fast_steps=fast_steps, **ablation)
+    elif fast_steps:
         ref = oracle_fast_step(sub_table, wl.theta[idx], wl.momentum[idx], wl.replicas[:, idx], sp.alpha,
                                sp.outer_lr, sp.momentum, fast_steps)
     else:

@@ -94,3 +94,65 @@ def test_excluding_a_matrix_is_a_table_choice():
     out = variants.isoloco_outer_step_variant(table, th, b, reps, alpha=1.0, eta=0.7, mu=0.9)
     dil = oracle.diloco_outer_step(th, b, reps, eta=0.7, mu=0.9)
     assert np.allclose(out["theta"][:24], dil["theta"][:24], rtol=1e-12, atol=1e-15)
+
+
+# ---------------------------------------------------------------- clip_high / clip_low (Sec. 4.5)
+def test_clip_diagonal_worked_example():
+    """Singular values 3, 1, 2 (mean 2): clip_high -> 2, 1, 2; clip_low -> 3, 2, 2."""
+    d = np.zeros((4, 3))
+    d[0, 0], d[1, 1], d[2, 2] = 3.0, 1.0, 2.0
+    hi, sb = variants.clip_spectrum(d, 1)
+    lo, _ = variants.clip_spectrum(d, 2)
+    assert sb == pytest.approx(2.0, rel=1e-14)
+    want_hi = np.zeros((4, 3)); want_hi[0, 0], want_hi[1, 1], want_hi[2, 2] = 2.0, 1.0, 2.0
+    want_lo = np.zeros((4, 3)); want_lo[0, 0], want_lo[1, 1], want_lo[2, 2] = 3.0, 2.0, 2.0
+    assert np.allclose(hi, want_hi, atol=1e-13) and np.allclose(lo, want_lo, atol=1e-13)
+
+
+@pytest.mark.parametrize("shape", [(7, 4), (3, 6), (5, 5)])
+def test_clip_high_plus_clip_low_is_delta_plus_iso_c(shape):
+    """min(s, m) + max(s, m) = s + m for every singular value."""
+    d = np.random.default_rng(sum(shape)).standard_normal(shape)
+    hi, _ = variants.clip_spectrum(d, 1)
+    lo, _ = variants.clip_spectrum(d, 2)
+    iso, _ = oracle.iso_c(d, 1.0)
+    assert np.allclose(hi + lo, d + iso, rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("kind", [1, 2])
+def test_clip_spectrum_against_lapack(kind):
+    d = np.random.default_rng(7 + kind).standard_normal((9, 6)) @ np.diag([5, 3, 1, 0.5, 0.2, 0.1])
+    out, sb = variants.clip_spectrum(d, kind)
+    s = np.linalg.svd(d, compute_uv=False)
+    assert sb == pytest.approx(s.mean(), rel=1e-12)
+    want = np.sort(np.minimum(s, sb) if kind == 1 else np.maximum(s, sb))
+    assert np.allclose(np.sort(np.linalg.svd(out, compute_uv=False)), want, rtol=1e-12)
+    # the singular vectors are Delta's: out^T Delta is symmetric
+    h = out.T @ d
+    assert np.allclose(h, h.T, atol=1e-12)
+
+
+@pytest.mark.parametrize("kind", [1, 2])
+def test_clip_orthogonal_equivariance_and_fixed_points(kind):
+    rng = np.random.default_rng(11)
+    d = rng.standard_normal((6, 4))
+    p, _ = np.linalg.qr(rng.standard_normal((6, 6)))
+    w, _ = np.linalg.qr(rng.standard_normal((4, 4)))
+    a, _ = variants.clip_spectrum(p @ d @ w, kind)
+    b, _ = variants.clip_spectrum(d, kind)
+    assert np.allclose(a, p @ b @ w, atol=1e-12)
+    q, _ = np.linalg.qr(rng.standard_normal((6, 4)))
+    c, _ = variants.clip_spectrum(0.3 * q, kind)          # equal singular values: unchanged
+    assert np.allclose(c, 0.3 * q, atol=1e-13)
+
+
+@pytest.mark.parametrize("kind", [1, 2])
+def test_clip_outer_step_sgd(kind):
+    th, b, reps = _inputs(5)
+    out = variants.isoloco_outer_step_variant(TABLE, th, b, reps, alpha=1.3, eta=0.7, mu=0.0, spectrum_kind=kind)
+    d = oracle.pseudo_gradient(th, reps)
+    for i, (off, r, c) in enumerate(TABLE):
+        sl = slice(off, off + r * (c or 1))
+        want = 1.3 * variants.clip_spectrum(d[sl].reshape(r, c), kind)[0].ravel() if c else d[sl]
+        assert np.allclose(out["update"][sl], want, rtol=1e-12, atol=1e-15)
+    assert np.allclose(out["theta"], th.astype(np.float64) - 0.7 * out["update"], rtol=1e-12, atol=1e-15)
