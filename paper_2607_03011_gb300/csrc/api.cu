@@ -147,6 +147,7 @@ struct isoloco_plan {
     float g_tol = 0.f;
     int g_fast = -1;
     int g_full = -1;
+    bool per_launch = false;        // polar iterations as plain launches (no graph), with early stop
     bool full_prec = false;         // every polar step with three passes and no Horner form
                                     // (the clip variants' sign iteration)
     int fast_steps = 0;             // this call's fast-variant step count (0: exact Iso-C)
@@ -844,7 +845,7 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
     if (rc) return rc;
     cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
     CUDA_TRY(cudaStreamIsCapturing(st, &cs));
-    const bool use_graph = kPairMma && !p->prof && cs == cudaStreamCaptureStatusNone;
+    const bool use_graph = kPairMma && !p->prof && !p->per_launch && cs == cudaStreamCaptureStatusNone;
     if (use_graph) {
         if (!p->gexec || p->g_max_iter != max_iter || p->g_tol != tol || p->g_fast != p->fast_steps ||
             p->g_full != (p->full_prec ? 1 : 0))
@@ -854,7 +855,7 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
         std::vector<int> cnt(p->buckets.size());
         for (int t = 1; t <= max_iter; ++t) {
             if ((rc = polar_iteration(p, t, max_iter, tol, st, 0, 0))) return rc;
-            if (p->prof && cs == cudaStreamCaptureStatusNone && !cnt.empty()) {
+            if ((p->prof || p->per_launch) && cs == cudaStreamCaptureStatusNone && !cnt.empty()) {
                 // profiling: stop, as the graph does, once no matrix is left (the wait for
                 // the count lies between the phases' events)
                 CUDA_TRY(cudaMemcpyAsync(cnt.data(), p->cnt_gram, sizeof(int) * cnt.size(), cudaMemcpyDeviceToHost, st));
@@ -993,6 +994,7 @@ static int run_clip(isoloco_plan* p, int kind, int max_iter, float tol, cudaStre
     a->fast_steps = 0;
     a->skip_trace = true;
     a->full_prec = true;  // sign(A') is used to first order (P A' P): no single-plane steps
+    a->per_launch = p->prof;  // under phase profiling, plain launches as in this plan
     if ((rc = run_polar(a, max_iter, tol, st))) return rc;
     k_clip_form_p<<<dim3(64, a->nmat), 256, 0, st>>>(a->mats_d, a->state, a->xhi[0], a->xlo[0], a->xhi[1],
                                                      a->xlo[1], kind == 1 ? -1.f : 1.f);

@@ -9,7 +9,8 @@ is the 48 square 1024 x 1024 matrices of the 180M recipe with K = 8 replicas
 `square12` a quarter of it; with --per-launch the polar iterations are launched one
 by one (phase profiling on) instead of as the library's CUDA graph, so that every
 kernel is a plain launch.  `gemm` runs the split-precision GEMM entry point on random
-inputs.
+inputs; `diloco` runs DiLoCo outer steps with a merging aggregator (Sec. 3.2), and
+`step --spectrum 1|2` the clip variants of Sec. 4.5.
 """
 from __future__ import annotations
 
@@ -30,13 +31,13 @@ EXTRA = {
 }
 
 
-def run_step(workload: str, steps: int, per_launch: bool = False) -> None:
+def run_step(workload: str, steps: int, per_launch: bool = False, spectrum_kind: int = 0) -> None:
     spec = EXTRA[workload]() if workload in EXTRA else W.SPECS[workload]
     wl = W.make_workload(spec, seed=0, device="cuda")
     plan = isoloco.Plan(wl.table, wl.N, wl.K, wl.replicas.dtype)
     if per_launch:
         plan.profile(True)
-    opts = isoloco.make_opts(spec.alpha, spec.outer_lr, spec.momentum)
+    opts = isoloco.make_opts(spec.alpha, spec.outer_lr, spec.momentum, spectrum_kind=spectrum_kind)
     th0, b0 = wl.theta.clone(), wl.momentum.clone()
     for _ in range(steps):
         wl.theta.copy_(th0)
@@ -44,6 +45,23 @@ def run_step(workload: str, steps: int, per_launch: bool = False) -> None:
         plan.outer_step(wl.theta, wl.momentum, wl.replicas, opts)
     rc = plan.last_status()
     print("status", isoloco.STATUS_NAMES.get(rc, rc), "iters", sorted(set(plan.read_diag()["iters"])))
+    if rc != 0:
+        raise SystemExit(1)
+
+
+def run_diloco(workload: str, steps: int, aggregator: int, sparsity: float) -> None:
+    spec = EXTRA[workload]() if workload in EXTRA else W.SPECS[workload]
+    wl = W.make_workload(spec, seed=0, device="cuda")
+    plan = isoloco.Plan(wl.table, wl.N, wl.K, wl.replicas.dtype)
+    opts = isoloco.make_opts(outer_lr=spec.outer_lr, momentum=spec.momentum, aggregator=aggregator,
+                             sparsity=sparsity, seed=1)
+    th0, b0 = wl.theta.clone(), wl.momentum.clone()
+    for _ in range(steps):
+        wl.theta.copy_(th0)
+        wl.momentum.copy_(b0)
+        plan.diloco_outer_step(wl.theta, wl.momentum, wl.replicas, opts)
+    rc = plan.last_status()
+    print("status", isoloco.STATUS_NAMES.get(rc, rc))
     if rc != 0:
         raise SystemExit(1)
 
@@ -65,6 +83,12 @@ def main():
     s.add_argument("--workload", default="square12")
     s.add_argument("--steps", type=int, default=2)
     s.add_argument("--per-launch", action="store_true")
+    s.add_argument("--spectrum", type=int, default=0, help="0 Iso-C, 1 clip_high, 2 clip_low")
+    dl = sub.add_parser("diloco")
+    dl.add_argument("--workload", default="llama_180m_k8")
+    dl.add_argument("--steps", type=int, default=2)
+    dl.add_argument("--aggregator", type=int, default=1, help="0 mean, 1 TIES, 2 DARE")
+    dl.add_argument("--sparsity", type=float, default=0.1)
     gm = sub.add_parser("gemm")
     gm.add_argument("--batch", type=int, default=48)
     gm.add_argument("--m", type=int, default=1024)
@@ -76,7 +100,9 @@ def main():
     gm.add_argument("--precision", type=int, default=0)
     a = ap.parse_args()
     if a.cmd == "step":
-        run_step(a.workload, a.steps, a.per_launch)
+        run_step(a.workload, a.steps, a.per_launch, a.spectrum)
+    elif a.cmd == "diloco":
+        run_diloco(a.workload, a.steps, a.aggregator, a.sparsity)
     else:
         run_gemm(a.batch, a.m, a.n, a.k, a.a_mn, a.b_mn, a.reps, a.precision)
 
