@@ -521,7 +521,10 @@ def main():
         e2e = {"value": wl.N / (statistics.median(e_ms) / 1000.0), "unit": UNIT,
                "h2d_bytes_per_step": int(wl.N * (4 + 4 + wl.K * rep_bytes)),
                "d2h_bytes_per_step": int(wl.N * 8), "ms_per_step": statistics.median(e_ms),
-               "api": "isoloco_outer_step_host"}
+               "api": "isoloco_outer_step_host",
+               "link_h2d_bytes_per_step": int(wl.N * (4 + 4 + 4 + wl.K * rep_bytes)),
+               "note": "pinned inputs: the reduce reads the replicas and theta in place over the host link, "
+                       "theta and B are copied during the polar iteration (theta crosses the link twice)"}
         del reps_h
 
     if rank != 0:

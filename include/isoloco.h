@@ -148,10 +148,15 @@ int isoloco_outer_step(isoloco_plan_t plan, float* theta, float* momentum,
                        const void* const* replicas, const isoloco_opts_t* opts, void* stream,
                        float* update_out);
 
-/* Same step with every buffer in HOST memory (pinned memory is fastest): the
- * call copies theta, momentum and the replicas to plan-owned device buffers,
- * runs the step and copies theta and momentum back, all on `stream`, and
- * synchronizes before returning the step's status. */
+/* Same step with every buffer in HOST memory: the result lands in theta_host and
+ * momentum_host, and the call synchronizes `stream` before returning the step's status.
+ * When theta, momentum and every replica are page-locked memory registered with CUDA
+ * (cudaHostAlloc, cudaHostRegister, torch's pin_memory; 16-byte aligned), the reduce pass
+ * reads them in place over the host link and theta / momentum are copied to plan-owned
+ * device buffers on a plan-owned side stream while the polar iteration runs; otherwise all
+ * of them are first copied to plan-owned device buffers on `stream`.  Either way theta and
+ * momentum are copied back at the end.  The first call allocates the device buffers (and
+ * the side stream). */
 int isoloco_outer_step_host(isoloco_plan_t plan, float* theta_host, float* momentum_host,
                             const void* const* replicas_host, const isoloco_opts_t* opts,
                             void* stream);

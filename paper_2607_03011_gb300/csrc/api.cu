@@ -175,10 +175,14 @@ struct isoloco_plan {
     unsigned long long* ties_hist = nullptr;
     uint64_t* ties_rank = nullptr;
     uint64_t* ties_prefix = nullptr;
-    // staging for the host-buffer entry point (allocated on first use)
+    // staging for the host-buffer entry point (allocated on first use); with pinned inputs
+    // the replicas are read in place and theta / B are copied on side_st during the polar
+    // iteration
     float* st_theta = nullptr;
     float* st_mom = nullptr;
     void* st_reps = nullptr;
+    cudaStream_t side_st = nullptr;
+    cudaEvent_t ev_reduced = nullptr, ev_copied = nullptr;
 };
 
 // ------------------------------------------------------------------ errors
@@ -279,6 +283,9 @@ static void free_plan(isoloco_plan* p) {
     if (p->gexec) cudaGraphExecDestroy(p->gexec);
     if (p->graph) cudaGraphDestroy(p->graph);
     if (p->cap_st) cudaStreamDestroy(p->cap_st);
+    if (p->side_st) cudaStreamDestroy(p->side_st);
+    if (p->ev_reduced) cudaEventDestroy(p->ev_reduced);
+    if (p->ev_copied) cudaEventDestroy(p->ev_copied);
     delete p;
 }
 
@@ -1124,16 +1131,25 @@ static int check_replicas(isoloco_plan* p, const void* const* reps, ReplicaPtrs&
     return ISOLOCO_OK;
 }
 
+// The host-buffer entry point with pinned inputs: the reduce reads theta (and B, for the
+// orthogonalise-P ablation) from the mapped host buffers; theta and B reach the device
+// buffers the step updates by copies on side_st after the reduce (the host link is idle
+// while the polar iteration runs), which the apply pass waits for.
+struct HostInputs {
+    const float* theta_h;
+    const float* mom_h;
+};
+
 static int run_isoc_step(isoloco_plan* p, int merge, float* theta, float* mom, const void* const* reps,
                          const isoloco_opts_t* opts_in, cudaStream_t st, float* upd_out, const float* base,
-                         float* out, float alpha_merge) {
+                         float* out, float alpha_merge, const HostInputs* hin = nullptr) {
     isoloco_opts_t o;
     int rc;
     if ((rc = check_opts(opts_in, &o))) return rc;
     ReplicaPtrs rp;
     if ((rc = check_replicas(p, reps, rp))) return rc;
     CUDA_TRY(cudaSetDevice(p->device));
-    const float* th_src = merge ? base : theta;
+    const float* th_src = hin ? hin->theta_h : (merge ? base : theta);
     const float scale = merge ? -1.f : (o.reduce_mean ? 1.f / (float)p->K : 1.f);
     // orthogonalise-P ablation: the reduce pass takes the momentum step on the raw Delta and
     // keeps B' aside, so that a non-finite Delta still leaves B untouched
@@ -1152,11 +1168,19 @@ static int run_isoc_step(isoloco_plan* p, int merge, float* theta, float* mom, c
         PhaseTimer tm(p, ISOLOCO_PHASE_REDUCE, st);
         if (pmode)
             k_reduce_p<<<p->nchunks, 256, 0, st>>>(p->chunks_d, p->mats_d, rp, p->K, p->dtype, th_src, scale,
-                                                   p->dhi, p->dlo, p->d1d, p->err_d, pmode, o.momentum, mom, p->bnew);
+                                                   p->dhi, p->dlo, p->d1d, p->err_d, pmode, o.momentum,
+                                                   hin ? hin->mom_h : mom, p->bnew);
         else
             k_reduce<<<p->nchunks, 256, 0, st>>>(p->chunks_d, p->mats_d, rp, p->K, p->dtype, th_src, scale, p->dhi,
                                                  p->dlo, p->d1d, p->err_d);
         CUDA_TRY(cudaGetLastError());
+    }
+    if (hin) {
+        CUDA_TRY(cudaEventRecord(p->ev_reduced, st));
+        CUDA_TRY(cudaStreamWaitEvent(p->side_st, p->ev_reduced, 0));
+        CUDA_TRY(cudaMemcpyAsync(theta, hin->theta_h, p->N * 4, cudaMemcpyHostToDevice, p->side_st));
+        CUDA_TRY(cudaMemcpyAsync(mom, hin->mom_h, p->N * 4, cudaMemcpyHostToDevice, p->side_st));
+        CUDA_TRY(cudaEventRecord(p->ev_copied, p->side_st));
     }
     p->fast_steps = merge ? 0 : o.fast_steps;
     p->full_prec = !merge && o.spectrum_kind != 0;
@@ -1170,6 +1194,7 @@ static int run_isoc_step(isoloco_plan* p, int merge, float* theta, float* mom, c
     us.ql[0] = p->xlo[0];
     us.ql[1] = p->xlo[1];
     us.d1d = p->d1d;
+    if (hin) CUDA_TRY(cudaStreamWaitEvent(st, p->ev_copied, 0));
     if (p->nchunks) {
         PhaseTimer tm(p, ISOLOCO_PHASE_APPLY, st);
         if (merge)
@@ -1330,6 +1355,18 @@ int diloco_outer_step(isoloco_plan_t p, float* theta, float* momentum, const voi
     return finish_call(p, st, o.sync);
 }
 
+// A host pointer the device may read in place: page-locked memory registered with CUDA.
+static bool mapped_host(const void* h, const void** dptr) {
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, h) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return false;
+    }
+    if (at.type != cudaMemoryTypeHost || !at.devicePointer) return false;
+    *dptr = at.devicePointer;
+    return true;
+}
+
 int isoloco_outer_step_host(isoloco_plan_t p, float* theta_h, float* mom_h, const void* const* reps_h,
                             const isoloco_opts_t* opts, void* stream) {
     if (!p) return fail(ISOLOCO_ERR_INVALID, "plan is NULL");
@@ -1340,26 +1377,45 @@ int isoloco_outer_step_host(isoloco_plan_t p, float* theta_h, float* mom_h, cons
     const size_t eb = p->dtype == ISOLOCO_F32 ? 4 : 2;
     const size_t rep_bytes = round_up((int64_t)(p->N * eb), 256);
     int rc;
-    if (!p->st_theta) {
-        if ((rc = dalloc(p, &p->st_theta, p->N)) || (rc = dalloc(p, &p->st_mom, p->N))) return rc;
-        uint8_t* r = nullptr;
-        if ((rc = dalloc(p, &r, (int64_t)rep_bytes * p->K))) return rc;
-        p->st_reps = r;
-    }
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    CUDA_TRY(cudaMemcpyAsync(p->st_theta, theta_h, p->N * 4, cudaMemcpyHostToDevice, st));
-    CUDA_TRY(cudaMemcpyAsync(p->st_mom, mom_h, p->N * 4, cudaMemcpyHostToDevice, st));
-    std::vector<const void*> dr(p->K);
-    for (int k = 0; k < p->K; ++k) {
-        void* d = static_cast<uint8_t*>(p->st_reps) + k * rep_bytes;
-        CUDA_TRY(cudaMemcpyAsync(d, reps_h[k], p->N * eb, cudaMemcpyHostToDevice, st));
-        dr[k] = d;
-    }
     isoloco_opts_t o;
     if ((rc = check_opts(opts, &o))) return rc;
     o.sync = 0;
-    if ((rc = run_isoc_step(p, 0, p->st_theta, p->st_mom, dr.data(), &o, st, nullptr, nullptr, nullptr, 0.f)))
-        return rc;
+    if (!p->st_theta)
+        if ((rc = dalloc(p, &p->st_theta, p->N)) || (rc = dalloc(p, &p->st_mom, p->N))) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    // pinned inputs: replicas, theta and B read in place by the reduce (no staging copy)
+    std::vector<const void*> dr(p->K);
+    const void* th_d = nullptr;
+    const void* mom_d = nullptr;
+    bool mapped = mapped_host(theta_h, &th_d) && mapped_host(mom_h, &mom_d) && ((uintptr_t)th_d & 15u) == 0 &&
+                  ((uintptr_t)mom_d & 15u) == 0;
+    for (int k = 0; mapped && k < p->K; ++k) mapped = mapped_host(reps_h[k], &dr[k]);
+    if (mapped) {
+        if (!p->side_st) {
+            CUDA_TRY(cudaStreamCreateWithFlags(&p->side_st, cudaStreamNonBlocking));
+            CUDA_TRY(cudaEventCreateWithFlags(&p->ev_reduced, cudaEventDisableTiming));
+            CUDA_TRY(cudaEventCreateWithFlags(&p->ev_copied, cudaEventDisableTiming));
+        }
+        const HostInputs hin{static_cast<const float*>(th_d), static_cast<const float*>(mom_d)};
+        if ((rc = run_isoc_step(p, 0, p->st_theta, p->st_mom, dr.data(), &o, st, nullptr, nullptr, nullptr, 0.f,
+                                &hin)))
+            return rc;
+    } else {
+        if (!p->st_reps) {
+            uint8_t* r = nullptr;
+            if ((rc = dalloc(p, &r, (int64_t)rep_bytes * p->K))) return rc;
+            p->st_reps = r;
+        }
+        CUDA_TRY(cudaMemcpyAsync(p->st_theta, theta_h, p->N * 4, cudaMemcpyHostToDevice, st));
+        CUDA_TRY(cudaMemcpyAsync(p->st_mom, mom_h, p->N * 4, cudaMemcpyHostToDevice, st));
+        for (int k = 0; k < p->K; ++k) {
+            void* d = static_cast<uint8_t*>(p->st_reps) + k * rep_bytes;
+            CUDA_TRY(cudaMemcpyAsync(d, reps_h[k], p->N * eb, cudaMemcpyHostToDevice, st));
+            dr[k] = d;
+        }
+        if ((rc = run_isoc_step(p, 0, p->st_theta, p->st_mom, dr.data(), &o, st, nullptr, nullptr, nullptr, 0.f)))
+            return rc;
+    }
     CUDA_TRY(cudaMemcpyAsync(theta_h, p->st_theta, p->N * 4, cudaMemcpyDeviceToHost, st));
     CUDA_TRY(cudaMemcpyAsync(mom_h, p->st_mom, p->N * 4, cudaMemcpyDeviceToHost, st));
     return isoloco_last_status(p, st);

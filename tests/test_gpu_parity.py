@@ -330,11 +330,24 @@ def test_host_buffer_entry_point(iso):
     plan = iso.Plan(wl.table, wl.N, wl.K)
     th, b = wl.theta.clone(), wl.momentum.clone()
     assert plan.outer_step(th, b, wl.replicas, iso.make_opts(sync=True)) == 0
+    # pinned buffers: read in place by the reduce, theta / B copied during the polar iteration
     th_h = wl.theta.cpu().pin_memory()
     b_h = wl.momentum.cpu().pin_memory()
     reps_h = [wl.replicas[k].cpu().pin_memory() for k in range(wl.K)]
     assert plan.outer_step_host(th_h, b_h, reps_h, iso.make_opts()) == 0
     assert torch.equal(th_h, th.cpu()) and torch.equal(b_h, b.cpu())
+    # pageable buffers: staged copies first
+    th_p, b_p = wl.theta.cpu().clone(), wl.momentum.cpu().clone()
+    reps_p = [wl.replicas[k].cpu().clone() for k in range(wl.K)]
+    assert not th_p.is_pinned()
+    assert plan.outer_step_host(th_p, b_p, reps_p, iso.make_opts()) == 0
+    assert torch.equal(th_p, th.cpu()) and torch.equal(b_p, b.cpu())
+    # pinned again, with the orthogonalise-P ablation (its reduce reads B in place too)
+    th2, b2 = wl.theta.clone(), wl.momentum.clone()
+    assert plan.outer_step(th2, b2, wl.replicas, iso.make_opts(sync=True, orth_target=1)) == 0
+    th_h.copy_(wl.theta.cpu()); b_h.copy_(wl.momentum.cpu())
+    assert plan.outer_step_host(th_h, b_h, reps_h, iso.make_opts(orth_target=1)) == 0
+    assert torch.equal(th_h, th2.cpu()) and torch.equal(b_h, b2.cpu())
 
 
 def sampled_parity(iso, workload, pick_names, fast_steps=0, **ablation):
