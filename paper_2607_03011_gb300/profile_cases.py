@@ -10,7 +10,8 @@ is the 48 square 1024 x 1024 matrices of the 180M recipe with K = 8 replicas
 by one (phase profiling on) instead of as the library's CUDA graph, so that every
 kernel is a plain launch.  `gemm` runs the split-precision GEMM entry point on random
 inputs; `diloco` runs DiLoCo outer steps with a merging aggregator (Sec. 3.2), and
-`step --spectrum 1|2` the clip variants of Sec. 4.5.
+`step --spectrum 1|2` the clip variants of Sec. 4.5; `hostlink` measures the host link
+(copy engines, and the host-buffer step's reduce reading pinned memory in place).
 """
 from __future__ import annotations
 
@@ -66,6 +67,58 @@ def run_diloco(workload: str, steps: int, aggregator: int, sparsity: float) -> N
         raise SystemExit(1)
 
 
+def run_hostlink(gib: int, workload: str) -> None:
+    """The host link: copy-engine transfers of a pinned buffer (one and four streams), and
+    the library's reduce pass reading pinned replicas and theta in place
+    (isoloco_outer_step_host, reduce phase timed by events)."""
+    n = gib << 28  # floats
+    h = torch.ones(n, dtype=torch.float32).pin_memory()
+    d = torch.empty(n, dtype=torch.float32, device="cuda")
+    streams = [torch.cuda.Stream() for _ in range(4)]
+
+    def timed(fn, stream):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        a.record(stream)
+        fn()
+        torch.cuda.synchronize()
+        b.record(stream)
+        b.synchronize()
+        return a.elapsed_time(b)
+
+    nbytes = n * 4
+    for _ in range(2):
+        with torch.cuda.stream(streams[0]):
+            ms = timed(lambda: d.copy_(h, non_blocking=True), streams[0])
+        print(f"H2D one stream: {nbytes / ms / 1e6:.1f} GB/s")
+        with torch.cuda.stream(streams[0]):
+            ms = timed(lambda: h.copy_(d, non_blocking=True), streams[0])
+        print(f"D2H one stream: {nbytes / ms / 1e6:.1f} GB/s")
+
+        def four():
+            q = n // 4
+            for i, s_ in enumerate(streams):
+                with torch.cuda.stream(s_):
+                    d[i * q:(i + 1) * q].copy_(h[i * q:(i + 1) * q], non_blocking=True)
+        ms = timed(four, torch.cuda.current_stream())
+        print(f"H2D four streams: {nbytes / ms / 1e6:.1f} GB/s")
+    del h, d
+    spec = EXTRA[workload]() if workload in EXTRA else W.SPECS[workload]
+    wl = W.make_workload(spec, seed=0, device="cuda")
+    plan = isoloco.Plan(wl.table, wl.N, wl.K, wl.replicas.dtype)
+    th_h, b_h = wl.theta.cpu().pin_memory(), wl.momentum.cpu().pin_memory()
+    reps_h = [wl.replicas[k].cpu().pin_memory() for k in range(wl.K)]
+    opts = isoloco.make_opts(spec.alpha, spec.outer_lr, spec.momentum)
+    plan.outer_step_host(th_h.clone().pin_memory(), b_h.clone().pin_memory(), reps_h, opts)
+    plan.profile(True)
+    for _ in range(2):
+        plan.outer_step_host(th_h.clone().pin_memory(), b_h.clone().pin_memory(), reps_h, opts)
+    ms = plan.profile_read()["reduce"][0] / 2
+    rb = wl.N * (wl.K * wl.replicas.element_size() + 4)
+    print(f"reduce pass reading pinned replicas and theta in place: {rb / 1e9:.2f} GB in {ms:.3f} ms = "
+          f"{rb / ms / 1e6:.1f} GB/s")
+
+
 def run_gemm(batch, m, n, k, a_mn, b_mn, reps, precision=0) -> None:
     g = torch.Generator(device="cuda").manual_seed(0)
     A = torch.randn((batch, k, m) if a_mn else (batch, m, k), device="cuda", generator=g)
@@ -89,6 +142,9 @@ def main():
     dl.add_argument("--steps", type=int, default=2)
     dl.add_argument("--aggregator", type=int, default=1, help="0 mean, 1 TIES, 2 DARE")
     dl.add_argument("--sparsity", type=float, default=0.1)
+    hl = sub.add_parser("hostlink")
+    hl.add_argument("--gib", type=int, default=4)
+    hl.add_argument("--workload", default="square12")
     gm = sub.add_parser("gemm")
     gm.add_argument("--batch", type=int, default=48)
     gm.add_argument("--m", type=int, default=1024)
@@ -103,6 +159,8 @@ def main():
         run_step(a.workload, a.steps, a.per_launch, a.spectrum)
     elif a.cmd == "diloco":
         run_diloco(a.workload, a.steps, a.aggregator, a.sparsity)
+    elif a.cmd == "hostlink":
+        run_hostlink(a.gib, a.workload)
     else:
         run_gemm(a.batch, a.m, a.n, a.k, a.a_mn, a.b_mn, a.reps, a.precision)
 
