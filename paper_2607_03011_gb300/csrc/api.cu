@@ -31,7 +31,7 @@ __global__ void k_gram_finalize(const MatDesc*, const int2*, const MatState*, co
                                 __nv_bfloat16*);
 __global__ void k_control(const MatDesc*, int, MatState*, const float*, int, int, float, uint32_t*, const int*,
                           const int*, int, int*, int*, int*, int*, cudaGraphConditionalHandle, int, long long*,
-                          int);
+                          int, int*);
 __global__ void k_trace_partial(const MatDesc*, const int4*, const MatState*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, double*);
@@ -477,7 +477,7 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         (rc = dalloc(p, &p->bucket_count_d, (int64_t)p->buckets.size())) ||
         (rc = dalloc(p, &p->cnt_gram, (int64_t)p->buckets.size())) ||
         (rc = dalloc(p, &p->cnt_step, (int64_t)p->buckets.size())) ||
-        (rc = dalloc(p, &p->counters, kLaunchCounters)) || (rc = dalloc(p, &p->loopc, 2)) ||
+        (rc = dalloc(p, &p->counters, kLaunchCounters + 1)) || (rc = dalloc(p, &p->loopc, 2)) ||
         (rc = dalloc(p, &p->ties_hist, (int64_t)p->K * 256)) || (rc = dalloc(p, &p->ties_rank, p->K)) ||
         (rc = dalloc(p, &p->ties_prefix, p->K)) ||
         (rc = dalloc(p, &p->tmaps_d, (int64_t)kMapsPerBucket * std::max<size_t>(1, p->buckets.size()))))
@@ -709,10 +709,10 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
             CUDA_TRY(cudaGetLastError());
         }
         { PhaseTimer tm(p, ISOLOCO_PHASE_CONTROL, st);
-        k_control<<<1, 1024, 0, st>>>(p->mats_d, p->nmat, p->state, p->fin_part, t, max_iter, tol, p->err_d,
+        k_control<<<(p->nmat + kControlThreads / 32 - 1) / (kControlThreads / 32), kControlThreads, 0, st>>>(p->mats_d, p->nmat, p->state, p->fin_part, t, max_iter, tol, p->err_d,
                                       p->bucket_first_d, p->bucket_count_d, (int)p->buckets.size(), p->list_gram,
                                       p->cnt_gram, p->list_step, p->cnt_step, cond, set_cond, p->loopc,
-                                      p->fast_steps); }
+                                      p->fast_steps, p->counters + kLaunchCounters); }
         CUDA_TRY(cudaGetLastError());
         // ---- P = a I + b G + c G^2
         LaunchSet poly;
@@ -990,7 +990,7 @@ static int run_clip(isoloco_plan* p, int kind, int max_iter, float tol, cudaStre
     { PhaseTimer tm(p, ISOLOCO_PHASE_CLIP, st, 0);
     k_reset_state<<<(std::max(1, a->nmat) + 255) / 256, 256, 0, st>>>(
         a->state, a->nmat, a->err_d, a->mats_d, a->bucket_first_d, a->bucket_count_d, (int)a->buckets.size(),
-        a->list_gram, a->cnt_gram, a->counters, kLaunchCounters);
+        a->list_gram, a->cnt_gram, a->counters, kLaunchCounters + 1);
     a->launches += 1;
     a->launch_seq = 0;
     CUDA_TRY(cudaGetLastError());
@@ -1161,7 +1161,7 @@ static int run_isoc_step(isoloco_plan* p, int merge, float* theta, float* mom, c
     { PhaseTimer tm(p, ISOLOCO_PHASE_OTHER, st);
     k_reset_state<<<(std::max(1, p->nmat) + 255) / 256, 256, 0, st>>>(
         p->state, p->nmat, p->err_d, p->mats_d, p->bucket_first_d, p->bucket_count_d, (int)p->buckets.size(),
-        p->list_gram, p->cnt_gram, p->counters, kLaunchCounters); }
+        p->list_gram, p->cnt_gram, p->counters, kLaunchCounters + 1); }
     p->launch_seq = 0;
     CUDA_TRY(cudaGetLastError());
     if (p->nchunks) {

@@ -204,6 +204,7 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
 
     const double n = static_cast<double>(md.n);
     double d, gscale = 1.0, xscale = 1.0;
+    const int st_step = st.step, st_iters = st.iters;  // one read each; st is global memory
     if (t == 0) {
         const double s2 = sqrt(sq);  // ||Delta^T Delta||_F >= sigma_max(Delta)^2
         if (!(s2 > 0.0) || !isfinite(s2)) {
@@ -223,7 +224,7 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
         // ||G/s2 - I||_F^2 = ||G||^2/s2^2 - 2 tr(G)/s2 + n, with ||G||^2/s2^2 = 1
         d = sqrt(fmax(0.0, 1.0 - 2.0 * tr * gscale + n) / n);
     } else {
-        d = sqrt(fmax(0.0, dev) / n);
+        d = sqrtf(fmaxf(0.f, devf) / static_cast<float>(md.n));  // fp32: the narrow fp64 pipe is slow
     }
     st.resid = static_cast<float>(d);
     st.xscale = static_cast<float>(xscale);
@@ -238,14 +239,14 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
         // fast variant: a fixed number of standard quintic steps, no test, no polish (steps
         // after the schedule's last repeat it); the last one leaves Q in the buffer its
         // update writes
-        const float* q = kSched[st.step < kSchedSteps ? st.step : kSchedSteps - 1];
+        const float* q = kSched[st_step < kSchedSteps ? st_step : kSchedSteps - 1];
         st.mode = 1;
         st.a = q[0];
         st.b = static_cast<float>(q[1] * gscale);
         st.c = static_cast<float>(q[2] * gscale * gscale);
-        st.step += 1;
-        st.iters += 1;
-        if (st.iters >= fast_steps) {
+        st.step = st_step + 1;
+        st.iters = st_iters + 1;
+        if (st_iters + 1 >= fast_steps) {
             st.done = 1;
             st.final_buf = (t + 1) & 1;
         }
@@ -255,65 +256,73 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
         st.a = 1.5f;
         st.b = static_cast<float>(-0.5 * gscale);
         st.c = 0.f;
-        st.iters += 1;
+        st.iters = st_iters + 1;
         st.done = 1;
         st.final_buf = (t + 1) & 1;
-    } else if (st.iters >= max_iter) {
+    } else if (st_iters >= max_iter) {
         st.mode = 0;
         st.done = 1;
         st.final_buf = t & 1;
         st.status = kErrNotConverged;
         atomicOr(err, kErrNotConverged);
     } else {
-        const float* q = sched_row(md.deep != 0, st.step);
+        const float* q = sched_row(md.deep != 0, st_step);
         st.mode = 1;
         st.a = q[0];
         st.b = static_cast<float>(q[1] * gscale);
         st.c = static_cast<float>(q[2] * gscale * gscale);
-        st.step += 1;
-        st.iters += 1;
+        st.step = st_step + 1;
+        st.iters = st_iters + 1;
         // the next Gram writes Y = b I + c G of the step after this one (X normalised by then)
-        const float* qn = sched_row(md.deep != 0, st.step);
+        const float* qn = sched_row(md.deep != 0, st_step + 1);
         st.yb = qn[1];
         st.yc = qn[2];
     }
 }
 
 
-// One block of 1024 threads.  Warp w takes the decisions of matrices w, w + 32, ...; then
-// warp b compacts, for shape bucket b, the matrices that still need a Gram (not done) and
-// those that take a step this iteration (mode != 0), in matrix order.  GEMM launches only
-// enumerate the listed matrices.  As the last kernel of the polar graph's loop body
-// (set_cond), it also sets the loop's condition: run the body again while some matrix is
-// not done, at most until the iteration count passes max_iter (loopc[0] counts body runs
-// in this call, reset at t = 0; loopc[1] counts them over the plan's life).
-__global__ void __launch_bounds__(1024) k_control(const MatDesc* __restrict__ mats, int nmat,
-                                                  MatState* __restrict__ state,
-                                                  const float* __restrict__ fin_part, int t, int max_iter,
-                                                  float tol, uint32_t* __restrict__ err,
-                                                  const int* __restrict__ bucket_first,
-                                                  const int* __restrict__ bucket_count, int nbuckets,
-                                                  int* __restrict__ list_gram, int* __restrict__ cnt_gram,
-                                                  int* __restrict__ list_step, int* __restrict__ cnt_step,
-                                                  cudaGraphConditionalHandle cond, int set_cond,
-                                                  long long* __restrict__ loopc, int fast_steps) {
+// kControlThreads-thread blocks, one warp per matrix (grid = ceil(nmat / warps per block)).
+// The last block to finish (a ticket counter; no block waits for another) compacts, per
+// shape bucket, the matrices that still need a Gram (not done) and those that take a step
+// this iteration (mode != 0), in matrix order; GEMM launches only enumerate the listed
+// matrices.  As the last kernel of the polar graph's loop body (set_cond), it also sets the
+// loop's condition: run the body again while some matrix is not done, at most until the
+// iteration count passes max_iter (loopc[0] counts body runs in this call, reset at t = 0;
+// loopc[1] counts them over the plan's life).  The ticket returns to 0 at the end.
+__global__ void __launch_bounds__(kControlThreads) k_control(const MatDesc* __restrict__ mats, int nmat,
+                                                             MatState* __restrict__ state,
+                                                             const float* __restrict__ fin_part, int t,
+                                                             int max_iter, float tol, uint32_t* __restrict__ err,
+                                                             const int* __restrict__ bucket_first,
+                                                             const int* __restrict__ bucket_count, int nbuckets,
+                                                             int* __restrict__ list_gram, int* __restrict__ cnt_gram,
+                                                             int* __restrict__ list_step, int* __restrict__ cnt_step,
+                                                             cudaGraphConditionalHandle cond, int set_cond,
+                                                             long long* __restrict__ loopc, int fast_steps,
+                                                             int* __restrict__ ticket) {
+    constexpr int kWarps = kControlThreads / 32;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (t == 0 && threadIdx.x == 0) loopc[0] = 0;
-    for (int mi = warp; mi < nmat; mi += 32) {
+    for (int mi = blockIdx.x * kWarps + warp; mi < nmat; mi += gridDim.x * kWarps) {
         control_matrix(mats, mi, state, fin_part, t, max_iter, tol, err, lane, fast_steps);
         __syncwarp();
     }
+    __threadfence();
     __syncthreads();
-    for (int bk = warp; bk < nbuckets; bk += 32) {
+    __shared__ int last;
+    if (threadIdx.x == 0) last = (atomicAdd(ticket, 1) == static_cast<int>(gridDim.x) - 1);
+    __syncthreads();
+    if (!last) return;
+    __threadfence();
+    // other blocks' decisions: read past L1
+    for (int bk = warp; bk < nbuckets; bk += kWarps) {
         const int first = bucket_first[bk], count = bucket_count[bk];
         int ng = 0, ns = 0;
         for (int j0 = 0; j0 < count; j0 += 32) {
             const int j = j0 + lane;
             bool g_on = false, s_on = false;
             if (j < count) {
-                const MatState& st = state[first + j];
-                g_on = (st.done == 0);
-                s_on = (st.mode != 0);
+                g_on = (__ldcg(&state[first + j].done) == 0);
+                s_on = (__ldcg(&state[first + j].mode) != 0);
             }
             const unsigned bg = __ballot_sync(0xffffffffu, g_on), bs = __ballot_sync(0xffffffffu, s_on);
             const unsigned below = (1u << lane) - 1u;
@@ -327,9 +336,11 @@ __global__ void __launch_bounds__(1024) k_control(const MatDesc* __restrict__ ma
             cnt_step[bk] = ns;
         }
     }
-    if (set_cond) {
-        __syncthreads();
-        if (threadIdx.x == 0) {
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        *ticket = 0;
+        if (t == 0) loopc[0] = 0;
+        if (set_cond) {
             int active = 0;
             for (int bk = 0; bk < nbuckets; ++bk) active += cnt_gram[bk];
             const long long runs = ++loopc[0];

@@ -34,6 +34,7 @@ constexpr int kPartSlots = kEpiWarps * (kPairMma ? 2 : 1);  // Gram partial sums
 constexpr int kGemmThreads = 64 + 32 * kEpiWarps;  // warp 0 TMA, warp 1 MMA, warps 2.. epilogue
 constexpr int kTmemCols = 256;     // one accumulator; the kernel double-buffers (512 columns)
 constexpr int kMaxGroups = 8;
+constexpr int kControlThreads = 256;  // k_control block: one warp per matrix
 constexpr int kFinRows = 32;  // rows of one k_gram_finalize tile (x BN columns)
 // Epilogue staging: per epilogue warp kStageBlocks blocks of 32 x 32 16-bit values (2 KB,
 // 64-byte swizzled rows), written to global memory by TMA stores.  With four, a symmetric
