@@ -224,17 +224,16 @@ def run_reference(args):
 
 # --------------------------------------------------------------------------- DiLoCo arm
 AGG_CODE = {"mean": 0, "ties": 1, "dare": 2}
-AGG_KERNELS = {"mean": "k_diloco", "ties": "k_ties_hist (4 radix-select passes) + k_ties_merge",
-               "dare": "k_dare"}
+AGG_KERNELS = {"mean": "k_diloco", "ties": "k_ties_bracket (one pass) + k_ties_merge", "dare": "k_dare"}
 
 
 def diloco_bytes(agg, N, K, eb):
     """Algorithmic HBM bytes of one DiLoCo step per phase: the streaming pass reads theta,
     B and the K replicas and writes theta and B; TIES's trim reads theta and the replicas
-    once per radix pass (4 passes)."""
+    once (the bracket pass; the sample and the candidate selection are small)."""
     out = {"diloco": (16 + K * eb) * N}
     if agg == "ties":
-        out["trim"] = 4 * (4 + K * eb) * N
+        out["trim"] = (4 + K * eb) * N
     return out
 
 
@@ -360,7 +359,7 @@ def run_diloco(args, torch, isoloco, wl, plan, world, rank, local, dist, barrier
     dom = max(phases, key=lambda k: phases[k]["ms_per_step"])
     roofline = {"bound": "hbm", "kernel": {"diloco": "k_diloco" if agg == "mean" else
                                            ("k_ties_merge" if agg == "ties" else "k_dare"),
-                                           "trim": "k_ties_hist x4 + k_ties_select x4 + k_ties_init"}[dom],
+                                           "trim": "k_ties_bracket (+ sample and candidate selection)"}[dom],
                 "achieved": phases[dom]["achieved"], "peak": hbm, "unit": "GB/s", "frac": phases[dom]["frac"],
                 "traffic": None, "peak_source": f"{peak_src} hbm_gbs",
                 "kernel_times": "per-phase CUDA events on the launch stream, in a profiled pass of the same "

@@ -56,12 +56,20 @@ __global__ void k_clip_flip(MatState*, int);
 __global__ void k_diloco(ReplicaPtrs, int, int, float*, float*, int64_t, float, float, float, uint32_t*);
 __global__ void k_dare(ReplicaPtrs, int, int, float*, float*, int64_t, float, uint32_t, float, unsigned int,
                        uint64_t, float, float, uint32_t*);
-__global__ void k_ties_init(int, uint64_t, unsigned long long*, uint64_t*, uint64_t*);
-__global__ void k_ties_hist(ReplicaPtrs, int, int, const float*, int64_t, int, const uint64_t*,
-                            unsigned long long*);
-__global__ void k_ties_select(int, int, unsigned long long*, uint64_t*, uint64_t*);
-__global__ void k_ties_merge(ReplicaPtrs, int, int, float*, float*, int64_t, const uint64_t*, float, float,
-                             uint32_t*);
+__global__ void k_ties_init(int, uint64_t, uint64_t, uint64_t, unsigned long long*, uint64_t*, uint64_t*, uint64_t*,
+                            uint64_t*, uint64_t*, uint64_t*, unsigned long long*, int*);
+__global__ void k_ties_sample(ReplicaPtrs, int, int, const float*, int64_t, int64_t, uint32_t*);
+__global__ void k_ties_hist_buf(const uint32_t*, const uint32_t*, int, int64_t, int, int, int, const uint64_t*,
+                                unsigned long long*);
+__global__ void k_ties_bracket(ReplicaPtrs, int, int, const float*, int64_t, const uint64_t*, uint32_t*, uint32_t*,
+                               int64_t, unsigned long long*);
+__global__ void k_ties_check(int, int, int64_t, uint64_t, const unsigned long long*, const uint32_t*, uint64_t*,
+                             int*);
+__global__ void k_ties_hist(ReplicaPtrs, int, int, const float*, int64_t, int, const uint64_t*, unsigned long long*,
+                            const int*);
+__global__ void k_ties_select(int, int, unsigned long long*, uint64_t*, uint64_t*, const int*);
+__global__ void k_ties_merge(ReplicaPtrs, int, int, float*, float*, int64_t, const uint64_t*, const uint64_t*,
+                             const int*, float, float, uint32_t*);
 __global__ void k_split_planes(const float*, int64_t, int, int, int, __nv_bfloat16*, __nv_bfloat16*, int);
 
 constexpr int kChunkElems = 16384;
@@ -171,10 +179,20 @@ struct isoloco_plan {
     int64_t* hss_d = nullptr;
     int* aux_of_d = nullptr;
     std::vector<int64_t> hbucket_off;
-    // TIES trim: per-worker radix-select histogram (K x 256), rank and chosen key prefix
+    // TIES trim (allocated on first use): radix-select histograms [2K][256]; ranks and key
+    // prefixes of the sample (2 per worker), candidate and fallback selections; the keys
+    // above each bracket; the fallback flag; the sample [K][S]; the candidate segments
+    // [K][ties_nseg][ties_segcap] and their counts
     unsigned long long* ties_hist = nullptr;
-    uint64_t* ties_rank = nullptr;
-    uint64_t* ties_prefix = nullptr;
+    uint64_t *ties_rank_s = nullptr, *ties_prefix_s = nullptr, *ties_rank_c = nullptr, *ties_prefix_c = nullptr;
+    uint64_t *ties_rank_f = nullptr, *ties_prefix_f = nullptr;
+    unsigned long long* ties_above = nullptr;
+    int* ties_fail = nullptr;
+    uint32_t* ties_samp = nullptr;
+    uint32_t* ties_cand = nullptr;
+    uint32_t* ties_cnt = nullptr;
+    int64_t ties_S = 0, ties_segcap = 0;
+    int ties_nseg = 0;
     // staging for the host-buffer entry point (allocated on first use); with pinned inputs
     // the replicas are read in place and theta / B are copied on side_st during the polar
     // iteration
@@ -478,15 +496,18 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         (rc = dalloc(p, &p->cnt_gram, (int64_t)p->buckets.size())) ||
         (rc = dalloc(p, &p->cnt_step, (int64_t)p->buckets.size())) ||
         (rc = dalloc(p, &p->counters, kLaunchCounters + 1)) || (rc = dalloc(p, &p->loopc, 2)) ||
-        (rc = dalloc(p, &p->ties_hist, (int64_t)p->K * 256)) || (rc = dalloc(p, &p->ties_rank, p->K)) ||
-        (rc = dalloc(p, &p->ties_prefix, p->K)) ||
         (rc = dalloc(p, &p->tmaps_d, (int64_t)kMapsPerBucket * std::max<size_t>(1, p->buckets.size()))))
         return rc;
     CUDA_TRY(cudaHostAlloc(reinterpret_cast<void**>(&p->err_h), sizeof(uint32_t), cudaHostAllocDefault));
     *p->err_h = 0;
     CUDA_TRY(cudaEventCreateWithFlags(&p->done_ev, cudaEventDisableTiming));
-    if (p->K * 256 * 4 > 48 * 1024)  // TIES histogram: K x 256 shared counters
+    if (p->K * 256 * 4 > 48 * 1024)  // TIES histograms: K (replica passes) or 2K x 256 shared counters
         CUDA_TRY(cudaFuncSetAttribute(k_ties_hist, cudaFuncAttributeMaxDynamicSharedMemorySize, p->K * 256 * 4));
+    if (p->K * 256 * 4 > 48 * 1024)  // per-thread counters of the TIES bracket pass
+        CUDA_TRY(cudaFuncSetAttribute(k_ties_bracket, cudaFuncAttributeMaxDynamicSharedMemorySize, p->K * 256 * 4));
+    if (2 * p->K * 256 * 4 > 48 * 1024)
+        CUDA_TRY(cudaFuncSetAttribute(k_ties_hist_buf, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      2 * p->K * 256 * 4));
     CUDA_TRY(cudaStreamCreateWithFlags(&p->cap_st, cudaStreamNonBlocking));
     CUDA_TRY(cudaMemset(p->loopc, 0, 2 * sizeof(long long)));
     // zero the planes once so that padding columns hold zeros
@@ -888,6 +909,34 @@ static int finish_call(isoloco_plan* p, cudaStream_t st, int sync) {
     CUDA_TRY(cudaEventRecord(p->done_ev, st));
     if (!sync) return ISOLOCO_OK;
     return isoloco_last_status(p, st);
+}
+
+// ---------------------------------------------------------------- TIES trim buffers
+// Sized once for the plan: a sample of S = min(N, 2^20) keys per worker, and candidate
+// segments (one per CTA of the bracket pass) for the widest bracket (sparsity 1/2), with 4x
+// headroom over the expected count per CTA.
+static int ensure_ties(isoloco_plan* p, int nseg) {
+    if (p->ties_hist) return ISOLOCO_OK;
+    const int K = p->K;
+    const int64_t S = std::min<int64_t>(p->N, int64_t(1) << 20);
+    const double m = 8.0 * std::sqrt((double)S * 0.25) + 16.0;
+    const double expected = (2.0 * m + 1.0) / (double)S * (double)p->N;  // candidates per worker
+    const int64_t segcap = round_up((int64_t)std::ceil(4.0 * expected / nseg) + 256, 4);
+    int rc;
+    if ((rc = dalloc(p, &p->ties_hist, (int64_t)2 * K * 256)) || (rc = dalloc(p, &p->ties_rank_s, 2 * K)) ||
+        (rc = dalloc(p, &p->ties_prefix_s, 2 * K)) || (rc = dalloc(p, &p->ties_rank_c, K)) ||
+        (rc = dalloc(p, &p->ties_prefix_c, K)) || (rc = dalloc(p, &p->ties_rank_f, K)) ||
+        (rc = dalloc(p, &p->ties_prefix_f, K)) || (rc = dalloc(p, &p->ties_above, K)) ||
+        (rc = dalloc(p, &p->ties_fail, 1)) || (rc = dalloc(p, &p->ties_samp, (int64_t)K * S)) ||
+        (rc = dalloc(p, &p->ties_cand, (int64_t)K * nseg * segcap)) ||
+        (rc = dalloc(p, &p->ties_cnt, (int64_t)K * nseg))) {
+        p->ties_hist = nullptr;
+        return rc;
+    }
+    p->ties_S = S;
+    p->ties_segcap = segcap;
+    p->ties_nseg = nseg;
+    return ISOLOCO_OK;
 }
 
 // ---------------------------------------------------------------- clip variants (Sec. 4.5)
@@ -1337,19 +1386,52 @@ int diloco_outer_step(isoloco_plan_t p, float* theta, float* momentum, const voi
         // keep the n_keep largest |Delta_k| of each worker; n_keep = N keeps all (threshold 0)
         const uint64_t n_keep = (uint64_t)(p->N - (int64_t)std::floor((double)o.sparsity * (double)p->N));
         const bool select = n_keep < (uint64_t)p->N;
+        if ((rc = ensure_ties(p, grid))) return rc;
+        const int K = p->K;
+        // sample ranks bracketing the threshold's expected rank n_keep S / N by 8 standard
+        // deviations of a sample count (and 16)
+        const double S = (double)p->ties_S, q = (double)n_keep / (double)p->N;
+        const double r_mid = q * S, m = 8.0 * std::sqrt(S * q * (1.0 - q)) + 16.0;
+        const uint64_t r_hi = (uint64_t)std::max(1.0, std::floor(r_mid - m));
+        const uint64_t r_lo = (uint64_t)std::min(S, std::ceil(r_mid + m));
         {
-            PhaseTimer tm(p, ISOLOCO_PHASE_TRIM, st, select ? 9 : 1);
-            k_ties_init<<<1, 256, 0, st>>>(p->K, n_keep, p->ties_hist, p->ties_rank, p->ties_prefix);
-            const int smem = p->K * 256 * 4;
-            for (int pass = 0; select && pass < 4; ++pass) {
-                k_ties_hist<<<grid, 256, smem, st>>>(rp, p->K, p->dtype, theta, p->N, pass, p->ties_prefix,
-                                                     p->ties_hist);
-                k_ties_select<<<1, 64, 0, st>>>(p->K, pass, p->ties_hist, p->ties_rank, p->ties_prefix);
+            PhaseTimer tm(p, ISOLOCO_PHASE_TRIM, st, select ? 29 : 1);
+            k_ties_init<<<1, 256, 0, st>>>(K, n_keep, r_hi, r_lo, p->ties_hist, p->ties_rank_s, p->ties_prefix_s,
+                                           p->ties_rank_c, p->ties_prefix_c, p->ties_rank_f, p->ties_prefix_f,
+                                           p->ties_above, p->ties_fail);
+            if (select) {
+                k_ties_sample<<<(unsigned)((p->ties_S + 255) / 256), 256, 0, st>>>(rp, K, p->dtype, theta, p->N,
+                                                                                 p->ties_S, p->ties_samp);
+                for (int pass = 0; pass < 4; ++pass) {
+                    k_ties_hist_buf<<<dim3(1, 256), 256, 2 * K * 256 * 4, st>>>(
+                        p->ties_samp, nullptr, 1, p->ties_S, 2 * K, 2, pass, p->ties_prefix_s, p->ties_hist);
+                    k_ties_select<<<(2 * K * 32 + 255) / 256, 256, 0, st>>>(2 * K, pass, p->ties_hist, p->ties_rank_s, p->ties_prefix_s,
+                                                     nullptr);
+                }
+                k_ties_bracket<<<p->ties_nseg, 256, K * 256 * 4, st>>>(rp, K, p->dtype, theta, p->N, p->ties_prefix_s,
+                                                            p->ties_cand, p->ties_cnt, p->ties_segcap, p->ties_above);
+                k_ties_check<<<K, 256, 0, st>>>(K, p->ties_nseg, p->ties_segcap, n_keep, p->ties_above, p->ties_cnt,
+                                               p->ties_rank_c, p->ties_fail);
+                for (int pass = 0; pass < 4; ++pass) {
+                    k_ties_hist_buf<<<dim3(p->ties_nseg, 1), 256, K * 256 * 4, st>>>(
+                        p->ties_cand, p->ties_cnt, p->ties_nseg, p->ties_segcap, K, 1, pass, p->ties_prefix_c,
+                        p->ties_hist);
+                    k_ties_select<<<(K * 32 + 255) / 256, 256, 0, st>>>(K, pass, p->ties_hist, p->ties_rank_c, p->ties_prefix_c,
+                                                    nullptr);
+                }
+                // fallback, only when some bracket missed: the four passes over the replicas
+                const int smem = K * 256 * 4;
+                for (int pass = 0; pass < 4; ++pass) {
+                    k_ties_hist<<<grid, 256, smem, st>>>(rp, K, p->dtype, theta, p->N, pass, p->ties_prefix_f,
+                                                         p->ties_hist, p->ties_fail);
+                    k_ties_select<<<(K * 32 + 255) / 256, 256, 0, st>>>(K, pass, p->ties_hist, p->ties_rank_f, p->ties_prefix_f,
+                                                    p->ties_fail);
+                }
             }
         }
         PhaseTimer tm(p, ISOLOCO_PHASE_DILOCO, st);
-        k_ties_merge<<<grid, 256, 0, st>>>(rp, p->K, p->dtype, theta, momentum, p->N, p->ties_prefix, o.outer_lr,
-                                           o.momentum, p->err_d);
+        k_ties_merge<<<grid, 256, 0, st>>>(rp, p->K, p->dtype, theta, momentum, p->N, p->ties_prefix_c,
+                                           p->ties_prefix_f, p->ties_fail, o.outer_lr, o.momentum, p->err_d);
     }
     CUDA_TRY(cudaGetLastError());
     return finish_call(p, st, o.sync);

@@ -402,15 +402,29 @@ __global__ void __launch_bounds__(kStreamThreads) k_dare(ReplicaPtrs reps, int K
 }
 
 // TIES trim: per worker k, the key (fp32 bits of |Delta_k|, ordered like the magnitudes) of
-// the rank-th largest magnitude over all N entries, by four radix passes over the 31 key
-// bits: [30:23], [22:15], [14:7], [6:0].  prefix[k] collects the chosen digits; rank[k]
-// starts at the number of entries kept, N - floor(sparsity * N).
+// the n_keep-th largest magnitude over all N entries, n_keep = N - floor(sparsity * N).
+// Radix select over the 31 key bits in four digits, [30:23], [22:15], [14:7], [6:0]: a
+// pass histograms one digit of the keys whose higher digits match the prefix chosen so far,
+// and k_ties_select appends the digit holding the wanted rank.  To avoid four passes over
+// the replicas, the library brackets the threshold first:
+//   1. k_ties_sample: S keys per worker at jittered strided positions;
+//   2. radix select on the sample for two ranks per worker, the expected rank of the
+//      threshold -/+ 8 standard deviations (and 16): keys hi >= lo;
+//   3. k_ties_bracket, one pass over the replicas: A = #(key > hi) and the keys in [lo, hi]
+//      collected per CTA (its own segment of the candidate buffer);
+//   4. k_ties_check: if A < n_keep <= A + #candidates and no segment overflowed, the
+//      threshold is the (n_keep - A)-th largest candidate, found by radix select on them;
+//   5. otherwise (a flag) the four passes over the replicas run and give it directly.
+// Either way the threshold is exact.
 __host__ __device__ constexpr int ties_shift(int pass) { return pass == 0 ? 23 : pass == 1 ? 15 : pass == 2 ? 7 : 0; }
 __host__ __device__ constexpr int ties_bins(int pass) { return pass == 3 ? 128 : 256; }
 
+__device__ __forceinline__ uint32_t ties_key(float d) { return __float_as_uint(fabsf(d)); }
+constexpr int kLoadBatch = 8;  // replicas whose loads are issued together in the TIES passes
+
 // Counts, per worker, the digit of this pass of every key whose higher digits equal the
-// prefix chosen so far.  Shared histogram K x 256; keys sharing a bin within a warp are
-// counted by one atomic (most magnitudes fall in a few exponent bins).
+// prefix chosen so far.  Shared histogram [workers][256]; keys sharing a bin within a warp
+// are counted by one atomic (most magnitudes fall in a few exponent bins).
 __device__ __forceinline__ void ties_count(uint32_t* sh, int k, uint32_t key, bool valid, int hs, uint32_t phi,
                                            int shift, uint32_t mask) {
     const bool m = valid && (key >> hs) == phi;
@@ -419,10 +433,13 @@ __device__ __forceinline__ void ties_count(uint32_t* sh, int k, uint32_t key, bo
     if (m && (threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&sh[k * 256 + bin], static_cast<uint32_t>(__popc(peers)));
 }
 
+// A radix pass over the replicas (the fallback).  Runs only when *fail != 0.
 __global__ void __launch_bounds__(kStreamThreads) k_ties_hist(ReplicaPtrs reps, int K, int dtype,
                                                               const float* __restrict__ theta, int64_t N, int pass,
                                                               const uint64_t* __restrict__ prefix,
-                                                              unsigned long long* __restrict__ hist) {
+                                                              unsigned long long* __restrict__ hist,
+                                                              const int* __restrict__ fail) {
+    if (*fail == 0) return;
     extern __shared__ uint32_t sh[];
     __shared__ uint32_t phi_s[kMaxK];
     const int shift = ties_shift(pass);
@@ -444,10 +461,10 @@ __global__ void __launch_bounds__(kStreamThreads) k_ties_hist(ReplicaPtrs reps, 
         for (int k = 0; k < K; ++k) {
             const float4 r = ld_rep4(reps.p[k], dtype, i);
             const uint32_t ph = phi_s[k];
-            ties_count(sh, k, __float_as_uint(fabsf(th.x - r.x)), valid, hs, ph, shift, mask);
-            ties_count(sh, k, __float_as_uint(fabsf(th.y - r.y)), valid, hs, ph, shift, mask);
-            ties_count(sh, k, __float_as_uint(fabsf(th.z - r.z)), valid, hs, ph, shift, mask);
-            ties_count(sh, k, __float_as_uint(fabsf(th.w - r.w)), valid, hs, ph, shift, mask);
+            ties_count(sh, k, ties_key(th.x - r.x), valid, hs, ph, shift, mask);
+            ties_count(sh, k, ties_key(th.y - r.y), valid, hs, ph, shift, mask);
+            ties_count(sh, k, ties_key(th.z - r.z), valid, hs, ph, shift, mask);
+            ties_count(sh, k, ties_key(th.w - r.w), valid, hs, ph, shift, mask);
         }
     }
     if (blockIdx.x == 0 && threadIdx.x < 32) {
@@ -456,7 +473,7 @@ __global__ void __launch_bounds__(kStreamThreads) k_ties_hist(ReplicaPtrs reps, 
         const float th = valid ? __ldg(theta + i) : 0.f;
         for (int k = 0; k < K; ++k) {
             const float r = valid ? ld_rep1(reps.p[k], dtype, i) : 0.f;
-            ties_count(sh, k, __float_as_uint(fabsf(th - r)), valid, hs, phi_s[k], shift, mask);
+            ties_count(sh, k, ties_key(th - r), valid, hs, phi_s[k], shift, mask);
         }
     }
     __syncthreads();
@@ -464,39 +481,234 @@ __global__ void __launch_bounds__(kStreamThreads) k_ties_hist(ReplicaPtrs reps, 
         if (sh[j]) atomicAdd(&hist[j], static_cast<unsigned long long>(sh[j]));
 }
 
-// rank[k] = n_keep, prefix[k] = 0, histogram cleared.  One CTA.
-__global__ void k_ties_init(int K, uint64_t n_keep, unsigned long long* __restrict__ hist,
-                            uint64_t* __restrict__ rank, uint64_t* __restrict__ prefix) {
-    for (int j = threadIdx.x; j < K * 256; j += blockDim.x) hist[j] = 0ull;
+// A radix pass over keys already in a buffer [K][nseg][segcap] (counts[k][seg] valid keys,
+// clamped to segcap; all segcap when counts is null), for nw selections: selection v reads
+// worker v / vdiv.  grid = (nseg, splits of a segment).
+__global__ void __launch_bounds__(kStreamThreads) k_ties_hist_buf(const uint32_t* __restrict__ keys,
+                                                                  const uint32_t* __restrict__ counts, int nseg,
+                                                                  int64_t segcap, int nw, int vdiv, int pass,
+                                                                  const uint64_t* __restrict__ prefix,
+                                                                  unsigned long long* __restrict__ hist) {
+    extern __shared__ uint32_t sh[];
+    const int shift = ties_shift(pass);
+    const int hs = pass == 0 ? 31 : ties_shift(pass - 1);
+    const uint32_t mask = static_cast<uint32_t>(ties_bins(pass) - 1);
+    for (int j = threadIdx.x; j < nw * 256; j += blockDim.x) sh[j] = 0u;
+    __syncthreads();
+    const int seg = blockIdx.x;
+    const int lane = threadIdx.x & 31;
+    for (int v = 0; v < nw; ++v) {
+        const int k = v / vdiv;
+        const int64_t n = counts ? min(static_cast<int64_t>(counts[static_cast<int64_t>(k) * nseg + seg]), segcap)
+                                 : segcap;
+        const int64_t chunk = (n + gridDim.y - 1) / gridDim.y;
+        const int64_t lo = blockIdx.y * chunk, hi = min(n, lo + chunk);
+        const uint32_t* src = keys + (static_cast<int64_t>(k) * nseg + seg) * segcap;
+        const uint32_t phi = static_cast<uint32_t>(prefix[v]) >> hs;
+        for (int64_t jb = lo + (threadIdx.x & ~31); jb < hi; jb += blockDim.x) {
+            const int64_t j = jb + lane;
+            const bool valid = j < hi;
+            ties_count(sh, v, valid ? src[j] : 0u, valid, hs, phi, shift, mask);
+        }
+    }
+    __syncthreads();
+    for (int j = threadIdx.x; j < nw * 256; j += blockDim.x)
+        if (sh[j]) atomicAdd(&hist[j], static_cast<unsigned long long>(sh[j]));
+}
+
+// Clears the histogram and sets the ranks: sample selections 2k (hi) and 2k + 1 (lo) want
+// ranks r_hi and r_lo; the fallback wants n_keep; the candidate selection's rank is set by
+// k_ties_check.  One CTA.
+__global__ void k_ties_init(int K, uint64_t n_keep, uint64_t r_hi, uint64_t r_lo,
+                            unsigned long long* __restrict__ hist, uint64_t* __restrict__ rank_s,
+                            uint64_t* __restrict__ prefix_s, uint64_t* __restrict__ rank_c,
+                            uint64_t* __restrict__ prefix_c, uint64_t* __restrict__ rank_f,
+                            uint64_t* __restrict__ prefix_f, unsigned long long* __restrict__ above,
+                            int* __restrict__ fail) {
+    for (int j = threadIdx.x; j < 2 * K * 256; j += blockDim.x) hist[j] = 0ull;
     for (int k = threadIdx.x; k < K; k += blockDim.x) {
-        rank[k] = n_keep;
-        prefix[k] = 0ull;
+        rank_s[2 * k] = r_hi;
+        rank_s[2 * k + 1] = r_lo;
+        prefix_s[2 * k] = prefix_s[2 * k + 1] = 0ull;
+        rank_c[k] = 1;
+        prefix_c[k] = 0ull;
+        rank_f[k] = n_keep;
+        prefix_f[k] = 0ull;
+        above[k] = 0ull;
+    }
+    if (threadIdx.x == 0) *fail = 0;
+}
+
+// Sample j of worker k: the key at position floor(j N / S) + h(j) mod floor(N / S), h a
+// SplitMix64-type mix of j (one position in each of S equal strata).
+__global__ void __launch_bounds__(kStreamThreads) k_ties_sample(ReplicaPtrs reps, int K, int dtype,
+                                                                const float* __restrict__ theta, int64_t N, int64_t S,
+                                                                uint32_t* __restrict__ samp) {
+    const int64_t j = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
+    if (j >= S) return;
+    const uint64_t width = static_cast<uint64_t>(N / S);
+    const uint64_t base = static_cast<uint64_t>(j) * static_cast<uint64_t>(N) / static_cast<uint64_t>(S);
+    const int64_t i = static_cast<int64_t>(base + splitmix64_top24(static_cast<uint64_t>(j + 1) * kSmGamma) % width);
+    const float th = __ldg(theta + i);
+    for (int k = 0; k < K; ++k) samp[static_cast<int64_t>(k) * S + j] = ties_key(th - ld_rep1(reps.p[k], dtype, i));
+}
+
+// One pass over theta and the replicas: per worker, the keys above the bracket [lo, hi] are
+// counted and those inside it collected into this CTA's segment of cand [K][gridDim.x][segcap];
+// cnt[k][cta] may exceed segcap (overflow: k_ties_check then fails).  Each thread counts in
+// its own shared slots up_s[k][thread] (no atomics, no warp votes in the loop); the rare keys
+// inside a bracket take a shared atomic for their position.  Dynamic shared memory:
+// K x blockDim.x counters.
+__global__ void __launch_bounds__(kStreamThreads) k_ties_bracket(ReplicaPtrs reps, int K, int dtype,
+                                                                 const float* __restrict__ theta, int64_t N,
+                                                                 const uint64_t* __restrict__ prefix_s,
+                                                                 uint32_t* __restrict__ cand,
+                                                                 uint32_t* __restrict__ cnt, int64_t segcap,
+                                                                 unsigned long long* __restrict__ above) {
+    extern __shared__ uint32_t up_s[];
+    __shared__ uint32_t hi_s[kMaxK], lo_s[kMaxK], cnt_s[kMaxK];
+    for (int k = threadIdx.x; k < K; k += blockDim.x) {
+        hi_s[k] = static_cast<uint32_t>(prefix_s[2 * k]);
+        lo_s[k] = static_cast<uint32_t>(prefix_s[2 * k + 1]);
+        cnt_s[k] = 0u;
+    }
+    for (int j = threadIdx.x; j < K * static_cast<int>(blockDim.x); j += blockDim.x) up_s[j] = 0u;
+    __syncthreads();
+    const int64_t G = gridDim.x;
+    const int64_t nv = N >> 2;
+    const int64_t stride = G * blockDim.x;
+    uint32_t* mine = up_s + threadIdx.x;
+    auto one = [&](uint32_t key, int k) -> uint32_t {
+        if (key > hi_s[k]) return 1u;
+        if (key >= lo_s[k]) {
+            const uint32_t pos = atomicAdd(&cnt_s[k], 1u);
+            if (pos < segcap) cand[(static_cast<int64_t>(k) * G + blockIdx.x) * segcap + pos] = key;
+        }
+        return 0u;
+    };
+    for (int64_t v = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; v < nv; v += stride) {
+        const int64_t i = 4 * v;
+        const float4 th = __ldg(reinterpret_cast<const float4*>(theta + i));
+        for (int k0 = 0; k0 < K; k0 += 4) {
+            float4 r[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+                if (k0 + q < K) r[q] = ld_rep4(reps.p[k0 + q], dtype, i);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int k = k0 + q;
+                if (k >= K) break;
+                const uint32_t c = one(ties_key(th.x - r[q].x), k) + one(ties_key(th.y - r[q].y), k) +
+                                   one(ties_key(th.z - r[q].z), k) + one(ties_key(th.w - r[q].w), k);
+                if (c) mine[k * blockDim.x] += c;
+            }
+        }
+    }
+    if (blockIdx.x == 0) {
+        for (int64_t i = 4 * nv + threadIdx.x; i < N; i += blockDim.x) {
+            const float th = __ldg(theta + i);
+            for (int k = 0; k < K; ++k) mine[k * blockDim.x] += one(ties_key(th - ld_rep1(reps.p[k], dtype, i)), k);
+        }
+    }
+    __syncthreads();
+    // per worker: the block's sum of the thread counters (one warp per worker)
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
+    for (int k = warp; k < K; k += nwarps) {
+        uint32_t t = 0;
+        for (int j = lane; j < static_cast<int>(blockDim.x); j += 32) t += up_s[k * blockDim.x + j];
+        t = __reduce_add_sync(0xffffffffu, t);
+        if (lane == 0) {
+            cnt[static_cast<int64_t>(k) * G + blockIdx.x] = cnt_s[k];
+            if (t) atomicAdd(&above[k], static_cast<unsigned long long>(t));
+        }
     }
 }
 
-// One thread per worker: the bin holding the rank-th largest key (counting from the top),
-// appended to the prefix; the histogram is cleared for the next pass.
-__global__ void k_ties_select(int K, int pass, unsigned long long* __restrict__ hist, uint64_t* __restrict__ rank,
-                              uint64_t* __restrict__ prefix) {
-    const int k = blockIdx.x * blockDim.x + threadIdx.x;
-    if (k >= K) return;
-    unsigned long long* h = hist + static_cast<int64_t>(k) * 256;
-    uint64_t r = rank[k];
-    int digit = 0;
-    for (int b = ties_bins(pass) - 1; b >= 0; --b) {
-        const uint64_t c = h[b];
-        if (r <= c) {
-            digit = b;
+// One CTA per worker: does the bracket hold the threshold (A < n_keep <= A + candidates, no
+// segment overflowed)?  Then the candidate selection wants rank n_keep - A; else *fail is set.
+__global__ void __launch_bounds__(256) k_ties_check(int K, int nseg, int64_t segcap, uint64_t n_keep,
+                                                    const unsigned long long* __restrict__ above,
+                                                    const uint32_t* __restrict__ cnt, uint64_t* __restrict__ rank_c,
+                                                    int* __restrict__ fail) {
+    const int k = blockIdx.x;
+    __shared__ unsigned long long tot_s[256 / 32];
+    __shared__ int over_s;
+    if (threadIdx.x == 0) over_s = 0;
+    __syncthreads();
+    unsigned long long total = 0;
+    bool over = false;
+    for (int b = threadIdx.x; b < nseg; b += blockDim.x) {
+        const uint32_t c = cnt[static_cast<int64_t>(k) * nseg + b];
+        over |= c > segcap;
+        total += static_cast<unsigned long long>(min(static_cast<int64_t>(c), segcap));
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) total += __shfl_xor_sync(0xffffffffu, total, o);
+    if (__any_sync(0xffffffffu, over) && (threadIdx.x & 31) == 0) over_s = 1;
+    if ((threadIdx.x & 31) == 0) tot_s[threadIdx.x >> 5] = total;
+    __syncthreads();
+    if (threadIdx.x != 0) return;
+    unsigned long long t = 0;
+    for (int w = 0; w < 256 / 32; ++w) t += tot_s[w];
+    const uint64_t a = above[k];
+    const bool ok = !over_s && a < n_keep && n_keep <= a + t;
+    rank_c[k] = ok ? n_keep - a : 1;
+    if (!ok) atomicOr(fail, 1);
+}
+
+// One warp per selection: the bin holding the rank-th largest key (counting from the top),
+// appended to the prefix; the histogram row is cleared for the next pass.  Lane l holds bins
+// 8 l .. 8 l + 7; a suffix sum over the warp finds the bin.  With only_if_fail it runs only
+// when *only_if_fail != 0 (the fallback passes).
+__global__ void __launch_bounds__(256) k_ties_select(int nw, int pass, unsigned long long* __restrict__ hist,
+                                                     uint64_t* __restrict__ rank, uint64_t* __restrict__ prefix,
+                                                     const int* __restrict__ only_if_fail) {
+    if (only_if_fail && *only_if_fail == 0) return;
+    const int w = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+    if (w >= nw) return;
+    unsigned long long* h = hist + static_cast<int64_t>(w) * 256;
+    const int nb = ties_bins(pass);
+    unsigned long long c[8], mine = 0;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+        const int b = 8 * lane + q;
+        c[q] = b < nb ? h[b] : 0ull;
+        mine += c[q];
+        h[b] = 0ull;
+    }
+    // above = keys in the bins of the lanes above this one
+    unsigned long long incl = mine;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const unsigned long long t = __shfl_down_sync(0xffffffffu, incl, o);
+        if (lane + o < 32) incl += t;
+    }
+    const unsigned long long above = incl - mine;
+    const uint64_t r = rank[w];
+    // the lane whose bins hold rank r: above < r <= above + mine
+    const bool here = above < r && r <= above + mine;
+    const unsigned who = __ballot_sync(0xffffffffu, here);
+    if (!here) {
+        if (who == 0 && lane == 0) {  // not found (a count mismatch): keep the old behaviour, digit 0
+            rank[w] = r;
+        }
+        return;
+    }
+    unsigned long long rr = r - above;
+    int digit = 8 * lane;
+#pragma unroll
+    for (int q = 7; q >= 0; --q) {
+        if (rr <= c[q]) {
+            digit = 8 * lane + q;
             break;
         }
-        r -= c;
+        rr -= c[q];
     }
-    rank[k] = r;
-    prefix[k] |= static_cast<uint64_t>(digit) << ties_shift(pass);
-    for (int b = 0; b < 256; ++b) h[b] = 0ull;
+    rank[w] = rr;
+    prefix[w] |= static_cast<uint64_t>(digit) << ties_shift(pass);
 }
 
-// TIES elect and disjoint merge.  Entry kept when its key >= thr[k] (ties kept).  P and N
+// TIES elect and disjoint merge.  Entry kept when its key >= the threshold (ties kept).  P and N
 // are the fp32 sums, in worker order, of the kept positive and negative values; the elected
 // sign is that of P + N, and U the mean of the kept values of that sign (0 if P + N = 0).
 __device__ __forceinline__ float ties_u(float P, float Nn, int cp, int cn) {
@@ -513,9 +725,12 @@ __device__ __forceinline__ void ties_acc(float d, uint32_t t, float& P, float& N
 
 __global__ void __launch_bounds__(kStreamThreads) k_ties_merge(ReplicaPtrs reps, int K, int dtype,
                                                                float* __restrict__ theta, float* __restrict__ mom,
-                                                               int64_t N, const uint64_t* __restrict__ thr,
-                                                               float eta, float mu, uint32_t* __restrict__ err) {
+                                                               int64_t N, const uint64_t* __restrict__ thr_c,
+                                                               const uint64_t* __restrict__ thr_f,
+                                                               const int* __restrict__ fail, float eta, float mu,
+                                                               uint32_t* __restrict__ err) {
     __shared__ uint32_t thr_s[kMaxK];
+    const uint64_t* thr = *fail ? thr_f : thr_c;  // the bracket's result, or the fallback's
     for (int k = threadIdx.x; k < K; k += blockDim.x) thr_s[k] = static_cast<uint32_t>(thr[k]);
     __syncthreads();
     bool bad = false;
@@ -527,14 +742,21 @@ __global__ void __launch_bounds__(kStreamThreads) k_ties_merge(ReplicaPtrs reps,
         float4 bb = *reinterpret_cast<const float4*>(mom + i);
         float P[4] = {0.f, 0.f, 0.f, 0.f}, Nn[4] = {0.f, 0.f, 0.f, 0.f}, T = 0.f;
         int cp[4] = {0, 0, 0, 0}, cn[4] = {0, 0, 0, 0};
-        for (int k = 0; k < K; ++k) {
-            const float4 r = ld_rep4(reps.p[k], dtype, i);
-            const uint32_t t = thr_s[k];
-            const float d[4] = {th.x - r.x, th.y - r.y, th.z - r.z, th.w - r.w};
+        for (int k0 = 0; k0 < K; k0 += kLoadBatch) {
+            float4 r[kLoadBatch];
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                T += d[j];
-                ties_acc(d[j], t, P[j], Nn[j], cp[j], cn[j]);
+            for (int q = 0; q < kLoadBatch; ++q)
+                if (k0 + q < K) r[q] = ld_rep4(reps.p[k0 + q], dtype, i);
+#pragma unroll
+            for (int q = 0; q < kLoadBatch; ++q) {
+                if (k0 + q >= K) break;
+                const uint32_t t = thr_s[k0 + q];
+                const float d[4] = {th.x - r[q].x, th.y - r[q].y, th.z - r[q].z, th.w - r[q].w};
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    T += d[j];
+                    ties_acc(d[j], t, P[j], Nn[j], cp[j], cn[j]);
+                }
             }
         }
         bad |= !isfinite(T);

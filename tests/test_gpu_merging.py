@@ -213,3 +213,26 @@ def test_dare_mask_at_k8_with_64bit_draw_numbers(iso):
     assert np.array_equal(got, code)
     rate = [float(((bits >> k) & 1).float().mean()) for k in range(K)]
     assert all(abs(r - 0.5) < 5 * 0.5 / np.sqrt(n) for r in rate), rate
+
+
+def test_ties_bracket_fallback_on_tied_magnitudes(iso):
+    """|Delta_k| takes two values only, so the sampled bracket around the threshold holds
+    about half of all entries and overflows its candidate segments: the trim falls back to
+    the radix passes over the replicas, and the result is still the exact threshold's."""
+    n, K = (1 << 22) + 5, 3
+    g = torch.Generator(device="cuda").manual_seed(5)
+    theta = torch.randn(n, device="cuda", generator=g) * 0.02
+    npad = (n + 63) // 64 * 64
+    reps = torch.empty((K, npad), device="cuda")[:, :n]
+    for k in range(K):
+        mag = torch.where(torch.rand(n, device="cuda", generator=g) < 0.5, 1e-3, 2e-3)
+        sign = torch.where(torch.rand(n, device="cuda", generator=g) < 0.5, -1.0, 1.0)
+        reps[k] = theta - sign * mag
+    plan = iso.Plan([], n, K)
+    th, b = theta.clone(), torch.zeros_like(theta)
+    opts = iso.make_opts(outer_lr=0.7, momentum=0.9, sync=True, aggregator=1, sparsity=0.5)
+    assert plan.diloco_outer_step(th, b, reps, opts) == 0
+    th_in = theta.cpu().numpy()
+    ref = merging.merged_outer_step(th_in, np.zeros(n, np.float32), [r.cpu().numpy() for r in reps], "ties",
+                                    sparsity=0.5, eta=0.7, mu=0.9)
+    check(th, b, ref, th_in.astype(np.float64), "ties")
