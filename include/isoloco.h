@@ -164,8 +164,10 @@ int isoloco_outer_step_host(isoloco_plan_t plan, float* theta_host, float* momen
 /* DiLoCo outer step, Alg. 1 with Nesterov SGD: one streaming pass over every
  * parameter (no Iso-C).  Elementwise, so a non-finite input only affects its own
  * element; the step's status reports it.  opts->aggregator selects the merging rule of
- * Sec. 3.2 that replaces the mean (TIES: 4 extra read passes over the replicas for the
- * trim, then one pass; DARE: one pass).  The table is not used: every entry of
+ * Sec. 3.2 that replaces the mean (TIES: one extra read pass over the replicas for the
+ * trim, four if the sampled bracket of its threshold misses, then one pass; DARE: one
+ * pass); TIES's first call allocates its trim buffers (~K x 4 MB of samples and candidate
+ * segments sized from n_total).  The table is not used: every entry of
  * [0, n_total) is updated.  Errors: INVALID for a bad aggregator or sparsity. */
 int diloco_outer_step(isoloco_plan_t plan, float* theta, float* momentum,
                       const void* const* replicas, const isoloco_opts_t* opts, void* stream);

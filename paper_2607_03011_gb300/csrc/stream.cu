@@ -13,9 +13,10 @@
 //                   Mode 1: Iso-C merge output base + alpha IsoC(T) / base + alpha T (Eq. 1).
 //  k_dare         : Alg. 1 with DARE aggregation (Sec. 3.2): random drop and rescale of
 //                   each Delta_k, then the mean and the outer step, one pass.
-//  k_ties_*       : Alg. 1 with TIES aggregation (Sec. 3.2): per-worker magnitude trim by
-//                   radix select over all N entries (4 histogram passes), then sign
-//                   election, disjoint mean and the outer step in one pass.
+//  k_ties_*       : Alg. 1 with TIES aggregation (Sec. 3.2): per-worker magnitude trim, an
+//                   exact radix select of the threshold over all N entries bracketed from a
+//                   sample (one pass over the replicas), then sign election, disjoint mean
+//                   and the outer step in one pass.
 //  k_split_planes : fp32 -> bf16 hi/lo planes (tests of the split-precision GEMM).
 #include "common.cuh"
 #include "types.h"
