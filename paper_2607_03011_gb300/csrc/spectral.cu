@@ -20,19 +20,32 @@
 
 namespace isoloco {
 
-__device__ __forceinline__ float ld16pair(const __nv_bfloat16* hi, const __nv_bfloat16* lo, int64_t o, bool f16) {
-    return dec16(__bfloat16_as_ushort(hi[o]), f16) + dec16(__bfloat16_as_ushort(lo[o]), f16);
+// Eight 16-bit values of a hi/lo plane pair as floats (16-byte loads).
+__device__ __forceinline__ void ld16x8(const __nv_bfloat16* hi, const __nv_bfloat16* lo, int64_t o, bool f16,
+                                       float (&v)[8]) {
+    const uint4 h = *reinterpret_cast<const uint4*>(hi + o);
+    const uint4 l = *reinterpret_cast<const uint4*>(lo + o);
+    const uint32_t hw[4] = {h.x, h.y, h.z, h.w}, lw[4] = {l.x, l.y, l.z, l.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        v[2 * q] = dec16(hw[q] & 0xFFFFu, f16) + dec16(lw[q] & 0xFFFFu, f16);
+        v[2 * q + 1] = dec16(hw[q] >> 16, f16) + dec16(lw[q] >> 16, f16);
+    }
 }
 
-__device__ __forceinline__ void st16pair(__nv_bfloat16* hi, __nv_bfloat16* lo, int64_t o, float v) {
-    uint16_t h, l;
-    split16(v, false, h, l);
-    hi[o] = __ushort_as_bfloat16(h);
-    lo[o] = __ushort_as_bfloat16(l);
+// Eight floats as a hi/lo plane pair of 16-bit values (16-byte stores).
+__device__ __forceinline__ void st16x8(__nv_bfloat16* hi, __nv_bfloat16* lo, int64_t o, bool f16,
+                                       const float (&v)[8]) {
+    uint32_t hw[4], lw[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) split16x2(v[2 * q], v[2 * q + 1], f16, hw[q], lw[q]);
+    *reinterpret_cast<uint4*>(hi + o) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+    *reinterpret_cast<uint4*>(lo + o) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
 }
 
 // Q (fp16 hi/lo planes in buffer final_buf) -> bf16 hi/lo planes in the other buffer, the
-// operand type of Delta's planes (one MMA never mixes fp16 and bf16).
+// operand type of Delta's planes (one MMA never mixes fp16 and bf16).  Eight elements per
+// thread over the padded rows (ld is a multiple of 8; padding columns are never read as data).
 __global__ void __launch_bounds__(256) k_clip_q_bf16(const MatDesc* __restrict__ mats,
                                                      const MatState* __restrict__ state,
                                                      __nv_bfloat16* xh0, __nv_bfloat16* xl0,
@@ -45,12 +58,17 @@ __global__ void __launch_bounds__(256) k_clip_q_bf16(const MatDesc* __restrict__
     const __nv_bfloat16* sl = fb ? xl1 : xl0;
     __nv_bfloat16* dh = fb ? xh0 : xh1;
     __nv_bfloat16* dl = fb ? xl0 : xl1;
-    const int64_t total = static_cast<int64_t>(md.rows) * md.cols;
-    for (int64_t e = blockIdx.x * 256 + threadIdx.x; e < total; e += static_cast<int64_t>(gridDim.x) * 256) {
-        const int64_t o = md.slot + (e / md.cols) * md.ld + e % md.cols;
-        st16pair(dh, dl, o, ld16pair(sh, sl, o, true));
+    const int64_t groups = static_cast<int64_t>(md.rows) * md.ld / 8;
+    for (int64_t g = blockIdx.x * 256 + threadIdx.x; g < groups; g += static_cast<int64_t>(gridDim.x) * 256) {
+        const int64_t o = md.slot + 8 * g;
+        float v[8];
+        ld16x8(sh, sl, o, true, v);
+        st16x8(dh, dl, o, false, v);
     }
 }
+
+// The n x n kernels below run eight consecutive columns per thread over rows padded to a
+// multiple of 8 (ld_n); padding columns are never read as data.
 
 // A' = H / sigma_bar - I into the auxiliary plan's input planes (bf16 hi/lo), H summed from
 // the fp32 split-K partials of the H GEMM; a matrix whose Q is 0 (Delta = 0) gets A' = 0.
@@ -70,20 +88,25 @@ __global__ void __launch_bounds__(256) k_clip_form_a(const MatDesc* __restrict__
     const float sbar = state[mi].sigma_bar;
     const bool zero = state[mi].final_buf > 1 || !(sbar > 0.f);
     const float inv = zero ? 0.f : 1.f / sbar;
-    const int n = md.n, splits = nsplit[mi];
+    const int ld = md.ld_n, splits = nsplit[mi];
     const float* h0 = hbuf + hoff[mi];
     const int64_t ss = hsstride[mi];
-    const int64_t total = static_cast<int64_t>(n) * n;
-    for (int64_t e = blockIdx.x * 256 + threadIdx.x; e < total; e += static_cast<int64_t>(gridDim.x) * 256) {
-        const int r = static_cast<int>(e / n), c = static_cast<int>(e % n);
-        float a = 0.f;
+    const int64_t groups = static_cast<int64_t>(md.n) * ld / 8;
+    for (int64_t g = blockIdx.x * 256 + threadIdx.x; g < groups; g += static_cast<int64_t>(gridDim.x) * 256) {
+        const int64_t e = 8 * g;
+        const int r = static_cast<int>(e / ld), c = static_cast<int>(e % ld);
+        float v[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
         if (!zero) {
-            const int64_t o = static_cast<int64_t>(r) * md.ld_n + c;
-            for (int sp = 0; sp < splits; ++sp) a += h0[sp * ss + o];
-            a *= inv;
-            if (r == c) a -= 1.f;
+            for (int sp = 0; sp < splits; ++sp) {
+                const float4 x = *reinterpret_cast<const float4*>(h0 + sp * ss + e);
+                const float4 y = *reinterpret_cast<const float4*>(h0 + sp * ss + e + 4);
+                v[0] += x.x; v[1] += x.y; v[2] += x.z; v[3] += x.w;
+                v[4] += y.x; v[5] += y.y; v[6] += y.z; v[7] += y.w;
+            }
+#pragma unroll
+            for (int q = 0; q < 8; ++q) v[q] = v[q] * inv - (c + q == r ? 1.f : 0.f);
         }
-        st16pair(ah, al, amd.slot + static_cast<int64_t>(r) * amd.ld + c, a);
+        st16x8(ah, al, amd.slot + static_cast<int64_t>(r) * amd.ld + c, false, v);
     }
 }
 
@@ -102,12 +125,16 @@ __global__ void __launch_bounds__(256) k_clip_form_p(const MatDesc* __restrict__
     const __nv_bfloat16* ql = fa ? axl1 : axl0;
     __nv_bfloat16* ph = fa ? axh0 : axh1;
     __nv_bfloat16* pl = fa ? axl0 : axl1;
-    const int n = amd.n;
-    const int64_t total = static_cast<int64_t>(n) * n;
-    for (int64_t e = blockIdx.x * 256 + threadIdx.x; e < total; e += static_cast<int64_t>(gridDim.x) * 256) {
-        const int r = static_cast<int>(e / n), c = static_cast<int>(e % n);
-        const int64_t o = amd.slot + static_cast<int64_t>(r) * amd.ld + c;
-        st16pair(ph, pl, o, 0.5f * ((r == c ? 1.f : 0.f) + sgn * ld16pair(qh, ql, o, true)));
+    const int ld = amd.ld;
+    const int64_t groups = static_cast<int64_t>(amd.n) * ld / 8;
+    for (int64_t g = blockIdx.x * 256 + threadIdx.x; g < groups; g += static_cast<int64_t>(gridDim.x) * 256) {
+        const int64_t e = 8 * g;
+        const int r = static_cast<int>(e / ld), c = static_cast<int>(e % ld);
+        float v[8];
+        ld16x8(qh, ql, amd.slot + e, true, v);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) v[q] = 0.5f * ((c + q == r ? 1.f : 0.f) + sgn * v[q]);
+        st16x8(ph, pl, amd.slot + e, false, v);
     }
 }
 
@@ -131,17 +158,16 @@ __global__ void __launch_bounds__(256) k_clip_form_s(const MatDesc* __restrict__
     const int ai = aux_of[mi];
     const MatDesc amd = amats[ai];
     const bool ident = astate[ai].final_buf > 1;
-    const int n = md.n;
-    const int64_t total = static_cast<int64_t>(n) * n;
-    for (int64_t e = blockIdx.x * 256 + threadIdx.x; e < total; e += static_cast<int64_t>(gridDim.x) * 256) {
-        const int r = static_cast<int>(e / n), c = static_cast<int>(e % n);
-        float v = (r == c) ? 1.f : 0.f;
-        if (!ident) v += ld16pair(aph, apl, amd.gslot + static_cast<int64_t>(r) * amd.ld_n + c, false);
-        uint16_t h, l;
-        split16(v, true, h, l);
-        const int64_t o = md.gslot + static_cast<int64_t>(r) * md.ld_n + c;
-        ph[o] = __ushort_as_bfloat16(h);
-        pl[o] = __ushort_as_bfloat16(l);
+    const int ld = md.ld_n;
+    const int64_t groups = static_cast<int64_t>(md.n) * ld / 8;
+    for (int64_t g = blockIdx.x * 256 + threadIdx.x; g < groups; g += static_cast<int64_t>(gridDim.x) * 256) {
+        const int64_t e = 8 * g;
+        const int r = static_cast<int>(e / ld), c = static_cast<int>(e % ld);
+        float v[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        if (!ident) ld16x8(aph, apl, amd.gslot + e, false, v);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) v[q] += (c + q == r ? 1.f : 0.f);
+        st16x8(ph, pl, md.gslot + e, true, v);
     }
 }
 

@@ -62,3 +62,33 @@ def test_validation_without_gpu(lib):
     assert lib.diloco_outer_step(None, None, None, None, None, None) == isoloco.ERR_INVALID
     assert lib.isoloco_debug_gemm(0, 0, 0, 0, 1, 1, 1, None, None, None, None) == isoloco.ERR_INVALID
     assert lib.isoloco_debug_gemm(0, 0, 9, 1, 1, 1, 1, None, None, None, None) == isoloco.ERR_INVALID
+
+
+def test_opts_layout_matches_the_header(tmp_path, lib):
+    """The binding's ctypes mirror of isoloco_opts_t has the header's size and field offsets
+    (checked by a C program compiled against include/isoloco.h), and the new fields default
+    to the paper's method (mean aggregation, Iso-C spectrum)."""
+    import shutil
+    import subprocess
+    from paper_2607_03011_gb300 import isoloco
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no C compiler")
+    fields = [f for f, _ in isoloco.Opts._fields_]
+    src = tmp_path / "layout.c"
+    lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "isoloco.h"', "int main(void) {",
+             '  printf("size %zu\\n", sizeof(isoloco_opts_t));']
+    lines += [f'  printf("{f} %zu\\n", offsetof(isoloco_opts_t, {f}));' for f in fields]
+    lines += ["  return 0;", "}"]
+    src.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "layout"
+    subprocess.run([gcc, "-std=c11", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)], check=True)
+    out = dict(line.split() for line in subprocess.run([str(exe)], capture_output=True, text=True,
+                                                       check=True).stdout.splitlines())
+    assert int(out["size"]) == ctypes.sizeof(isoloco.Opts)
+    for f in fields:
+        assert int(out[f]) == getattr(isoloco.Opts, f).offset, f
+    o = isoloco.Opts()
+    assert lib.isoloco_opts_default(ctypes.byref(o)) == 0
+    assert (o.fast_steps, o.orth_target, o.momentum_kind, o.scale_kind, o.aggregator, o.sparsity, o.seed,
+            o.spectrum_kind) == (0, 0, 0, 0, 0, 0.0, 0, 0)
