@@ -90,6 +90,22 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
+# --------------------------------------------------------------------------- multi-rank timing
+def max_over_ranks(total_ms: float, dist, device) -> float:
+    """The slowest rank's timed total (ms); the local value without a process group."""
+    if dist is None:
+        return total_ms
+    import torch
+    t = torch.tensor([total_ms], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_value(world: int, params: int, steps: int, total_ms: float) -> float:
+    """Whole-job throughput: every rank's parameters, every step, over the slowest rank's time."""
+    return world * params * steps / (total_ms / 1000.0)
+
+
 # --------------------------------------------------------------------------- accounting
 def gemm_flops(table, diag, fast=False):
     """Algorithmic (single-pass) FLOPs of the polar GEMMs of one step, per phase, from
@@ -305,12 +321,9 @@ def run_diloco(args, torch, isoloco, wl, plan, world, rank, local, dist, barrier
     torch.cuda.synchronize()
     prof = plan.profile_read()
     plan.profile(False)
-    if dist is not None:
-        t = torch.tensor([total_ms], device="cuda", dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, dist, "cuda")
     ms_per_step = total_ms / args.steps
-    value = world * wl.N * args.steps / (total_ms / 1000.0)
+    value = job_value(world, wl.N, args.steps, total_ms)
 
     # end to end: pinned host buffers copied in and out on the stream around the call
     e2e = None
@@ -491,12 +504,9 @@ def main():
     torch.cuda.synchronize()
     prof = plan.profile_read()
     plan.profile(False)
-    if dist is not None:
-        t = torch.tensor([total_ms], device="cuda", dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, dist, "cuda")
     ms_per_step = total_ms / args.steps
-    value = world * wl.N * args.steps / (total_ms / 1000.0)
+    value = job_value(world, wl.N, args.steps, total_ms)
 
     # ---- end-to-end through the host-buffer entry point (pinned host memory)
     e2e = None
