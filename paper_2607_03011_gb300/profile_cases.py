@@ -6,7 +6,8 @@
 `step` runs IsoLoCo outer steps through the C ABI on a named workload; `square48`
 is the 48 square 1024 x 1024 matrices of the 180M recipe with K = 8 replicas
 (1.6 GB of replicas: larger than L2, small enough for a full ncu capture), and
-`square12` a quarter of it; with --per-launch the polar iterations are launched one
+`square12` a quarter of it; `wide12` / `tall12` the 12 w_down-shaped 1024 x 2816 matrices and
+their transposes; with --per-launch the polar iterations are launched one
 by one (phase profiling on) instead of as the library's CUDA graph, so that every
 kernel is a plain launch.  `gemm` runs the split-precision GEMM entry point on random
 inputs; `diloco` runs DiLoCo outer steps with a merging aggregator (Sec. 3.2), and
@@ -27,6 +28,10 @@ EXTRA = {
                                       shared_std=2e-5, noise_std=2e-5, momentum_std=2e-5, name="square48"),
     "square12": lambda: W.custom_spec([(f"w{i}", 1024, 1024) for i in range(12)], K=8, rank=32,
                                       shared_std=2e-5, noise_std=2e-5, momentum_std=2e-5, name="square12"),
+    "wide12": lambda: W.custom_spec([(f"d{i}", 1024, 2816) for i in range(12)], K=8, rank=32, shared_std=2e-5,
+                                    noise_std=2e-5, momentum_std=2e-5, name="wide12"),
+    "tall12": lambda: W.custom_spec([(f"g{i}", 2816, 1024) for i in range(12)], K=8, rank=32, shared_std=2e-5,
+                                    noise_std=2e-5, momentum_std=2e-5, name="tall12"),
     "tall4": lambda: W.custom_spec([("e", 32000, 1024), ("d0", 2816, 1024), ("d1", 2816, 1024), ("g", 1024, 2816)],
                                    K=8, rank=32, shared_std=2e-5, noise_std=2e-5, momentum_std=2e-5, name="tall4"),
 }
