@@ -32,6 +32,35 @@ METRIC = "IsoLoCo outer-step ms & params/s at ~180M shapes, K=8; % HBM / TC roof
 UNIT = "params/s"
 
 
+def cpu_model() -> str:
+    """The host CPU's model string (x86 `model name`, or the Arm implementer / part ids)."""
+    try:
+        with open("/proc/cpuinfo") as f:
+            info = f.read()
+    except OSError:
+        return "unknown"
+    for line in info.splitlines():
+        if line.lower().startswith("model name"):
+            return line.split(":", 1)[1].strip()
+    impl = part = None
+    for line in info.splitlines():
+        if line.startswith("CPU implementer") and impl is None:
+            impl = line.split(":", 1)[1].strip()
+        if line.startswith("CPU part") and part is None:
+            part = line.split(":", 1)[1].strip()
+    return f"arm implementer {impl} part {part}" if impl else "unknown"
+
+
+def iters_by_shape(table, iters):
+    """Polar iteration counts per matrix shape: {"rows x cols": {count: matrices}}."""
+    out = {}
+    mats = [(r, c) for (_, r, c) in table if c > 0]
+    for (r, c), it in zip(mats, iters):
+        d = out.setdefault(f"{r}x{c}", {})
+        d[str(it)] = d.get(str(it), 0) + 1
+    return out
+
+
 def load_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -231,7 +260,7 @@ def run_reference(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": args.workload, "sample": desc, "sample_params": nparams},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "cpu_model": cpu_model(),
                              "sample": f"oracle outer step on {desc} ({nparams} params) per step"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
@@ -383,7 +412,7 @@ def run_diloco(args, torch, isoloco, wl, plan, world, rank, local, dist, barrier
         import oracle
         oracle.build()
         nparams, dt, desc = oracle_merging_sample(args.workload, CPU_SAMPLE, agg, args.sparsity)
-        cpu = {"value": nparams / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+        cpu = {"value": nparams / dt, "unit": UNIT, "cores": 1, "kind": "oracle", "cpu_model": cpu_model(),
                "sample": f"oracle DiLoCo step ({agg}) on {desc} ({nparams} params, {dt:.1f} s), "
                          "same generator recipe"}
     line = {
@@ -594,6 +623,7 @@ def main():
         oracle.build()
         nparams, dt, desc = oracle_sample_run(args.workload, CPU_SAMPLE)
         cpu = {"value": nparams / dt, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+               "cpu_model": cpu_model(),
                "sample": f"fp64 oracle outer step on {desc} ({nparams} params, {dt:.1f} s), "
                          "same generator recipe"}
 
@@ -614,7 +644,9 @@ def main():
                              f"fast variant: {args.fast_steps} fixed polar steps, sigma_bar = ||Delta||_F/sqrt(r)"),
                    "spectrum": args.spectrum},
         "status": isoloco.STATUS_NAMES.get(status, status),
-        "polar_iters": {"min": min(iters), "max": max(iters), "mean": sum(iters) / len(iters)},
+        "polar_iters": {"min": min(iters), "max": max(iters), "mean": sum(iters) / len(iters),
+                        "by_shape": iters_by_shape(wl.table, iters)},
+        "ms_step_median": statistics.median(step_ms), "ms_step_best": min(step_ms),
         "phases_ms_per_step": phases_ms, "phases_algorithmic_tflops": phases_tflops,
         "phases_executed_tflops": phases_exec,
         "roofline": roofline, "roofline_hbm": roofline_hbm,

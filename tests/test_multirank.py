@@ -68,3 +68,12 @@ def test_reference_arm_prints_on_rank_0_only(monkeypatch, capsys):
 
     assert bench.run_reference(Args()) == 0
     assert capsys.readouterr().out == ""
+
+
+def test_bench_report_helpers():
+    import sys
+    sys.path.insert(0, ROOT)
+    import bench
+    table = [(0, 4, 4), (16, 3, 0), (19, 2, 8), (35, 4, 4)]
+    assert bench.iters_by_shape(table, [7, 12, 9]) == {"4x4": {"7": 1, "9": 1}, "2x8": {"12": 1}}
+    assert isinstance(bench.cpu_model(), str) and bench.cpu_model()
