@@ -6,8 +6,8 @@
 `step` runs IsoLoCo outer steps through the C ABI on a named workload; `square48`
 is the 48 square 1024 x 1024 matrices of the 180M recipe with K = 8 replicas
 (1.6 GB of replicas: larger than L2, small enough for a full ncu capture), and
-`square12` a quarter of it; `wide12` / `tall12` the 12 w_down-shaped 1024 x 2816 matrices and
-their transposes; with --per-launch the polar iterations are launched one
+`square12` a quarter of it; `wide12` / `tall12` twelve 1024 x 2816 matrices (the shape of
+w_gate and w_up) and twelve 2816 x 1024 ones (w_down); with --per-launch the polar iterations are launched one
 by one (phase profiling on) instead of as the library's CUDA graph, so that every
 kernel is a plain launch.  `gemm` runs the split-precision GEMM entry point on random
 inputs; `diloco` runs DiLoCo outer steps with a merging aggregator (Sec. 3.2), and
