@@ -25,7 +25,7 @@
 namespace isoloco {
 
 // kernels defined in the other translation units
-cudaError_t launch_gemm(const GemmParams& p, bool a_mn, bool b_mn, int max_ctas, cudaStream_t stream);
+cudaError_t launch_gemm(const GemmParams& p, int max_ctas, cudaStream_t stream);
 __global__ void k_gram_finalize(const MatDesc*, const int2*, const MatState*, const float*, const int64_t*,
                                 const int64_t*, const int*, __nv_bfloat16*, __nv_bfloat16*, float*, int,
                                 __nv_bfloat16*);
@@ -611,7 +611,12 @@ static int group_tiles(const GemmGroup& g) { return g.sym ? g.tiles_sym : g.tile
 struct LaunchSet {
     GemmParams p;
     std::vector<GemmGroup> groups;
-    void add(const GemmGroup& g) { groups.push_back(g); }
+    // a_mn / b_mn: the operands' layouts in this group (MN-major or K-major)
+    void add(GemmGroup g, bool a_mn, bool b_mn) {
+        g.a_mn = a_mn ? 1 : 0;
+        g.b_mn = b_mn ? 1 : 0;
+        groups.push_back(g);
+    }
 };
 
 // Precision of a GEMM launch: operand and output plane types and which operands carry
@@ -641,7 +646,7 @@ static void init_set(LaunchSet& s, int epi, int gate, isoloco_plan* pl, Precisio
     s.p.err = pl->err_d;
 }
 
-static int flush_set(isoloco_plan* pl, int phase, LaunchSet& s, bool a_mn, bool b_mn, cudaStream_t st) {
+static int flush_set(isoloco_plan* pl, int phase, LaunchSet& s, cudaStream_t st) {
     if (s.groups.empty()) return ISOLOCO_OK;
     // longest CTAs first, so that short tiles fill in behind them (less tail)
     std::stable_sort(s.groups.begin(), s.groups.end(), [](const GemmGroup& x, const GemmGroup& y) {
@@ -660,7 +665,7 @@ static int flush_set(isoloco_plan* pl, int phase, LaunchSet& s, bool a_mn, bool 
         }
         p.total_tiles = cta;
         p.counter = pl->counters + (pl->launch_seq++ % kLaunchCounters);
-        CUDA_TRY(launch_gemm(p, a_mn, b_mn, pl->num_sms, st));
+        CUDA_TRY(launch_gemm(p, pl->num_sms, st));
     }
     return ISOLOCO_OK;
 }
@@ -686,10 +691,10 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
         const bool full = p->fast_steps > 0 || p->full_prec;
         const Precision gram_pr = first ? Precision{0, 0, 1, 1, 0}
                                         : (full ? Precision{1, 1, 1, 1, 0} : Precision{1, 1, 1, 0, 0});
-        LaunchSet tall, wide;
-        init_set(tall, kEpiGram, kGateActive, p, gram_pr);
-        init_set(wide, kEpiGram, kGateActive, p, gram_pr);
-        tall.p.gram_y = wide.p.gram_y = (first || full) ? 0 : 1;
+        // Tall and wide matrices share one launch (their tiles pack into fewer waves).
+        LaunchSet gram;
+        init_set(gram, kEpiGram, kGateActive, p, gram_pr);
+        gram.p.gram_y = (first || full) ? 0 : 1;
         for (size_t b = 0; b < p->buckets.size(); ++b) {
             const Bucket& bk = p->buckets[b];
             const CUtensorMap* m = maps + b * kMapsPerBucket;
@@ -716,12 +721,10 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
             g.part = p->fin_part;
             g.part_base = p->mats_h[bk.mat_base].gpart_slot;
             set_sym(g, bk.n);
-            (bk.tall ? tall : wide).add(g);
+            gram.add(g, bk.tall, bk.tall);
         }
         int rc;
-        if ((rc = flush_set(p, ISOLOCO_PHASE_GRAM, tall, true, true, st)) ||
-            (rc = flush_set(p, ISOLOCO_PHASE_GRAM, wide, false, false, st)))
-            return rc;
+        if ((rc = flush_set(p, ISOLOCO_PHASE_GRAM, gram, st))) return rc;
         if (p->nftiles) {
             PhaseTimer tm(p, ISOLOCO_PHASE_FINALIZE, st);
             k_gram_finalize<<<p->nftiles, 256, 0, st>>>(p->mats_d, p->ftiles, p->state, p->gpart, p->gpart_off_d,
@@ -759,9 +762,9 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
             g.g_hi = p->ghi + bk.gplane_off;
             g.g_lo = p->glo + bk.gplane_off;
             set_sym(g, bk.n);
-            poly.add(g);
+            poly.add(g, false, false);
         }
-        if ((rc = flush_set(p, ISOLOCO_PHASE_POLY, poly, false, false, st))) return rc;
+        if ((rc = flush_set(p, ISOLOCO_PHASE_POLY, poly, st))) return rc;
         // ---- X_{t+1} = xscale * X_t P (tall) or P X_t (wide)
         // X_{t+1} is always written as fp16 planes; X is the split operand (A when tall,
         // B when wide), P the single one except in the polish step (3 passes)
@@ -793,10 +796,13 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
             g.st_lo = m + st_map(dst, 1);
             g.bf_batch_stride = (int64_t)bk.rows * bk.ld;
             g.ld_bf = bk.ld;
-            (bk.tall ? utall : uwide).add(g);
+            if (bk.tall)
+                utall.add(g, false, false);
+            else
+                uwide.add(g, false, true);
         }
-        if ((rc = flush_set(p, ISOLOCO_PHASE_UPDATE, utall, false, false, st)) ||
-            (rc = flush_set(p, ISOLOCO_PHASE_UPDATE, uwide, false, true, st)))
+        if ((rc = flush_set(p, ISOLOCO_PHASE_UPDATE, utall, st)) ||
+            (rc = flush_set(p, ISOLOCO_PHASE_UPDATE, uwide, st)))
             return rc;
     }
     return ISOLOCO_OK;
@@ -997,12 +1003,11 @@ static int run_clip(isoloco_plan* p, int kind, int max_iter, float tol, cudaStre
     k_clip_q_bf16<<<grid, 256, 0, st>>>(p->mats_d, p->state, p->xhi[0], p->xlo[0], p->xhi[1], p->xlo[1]); }
     CUDA_TRY(cudaGetLastError());
     // ---- H = Qb^T Delta (tall, MN-major operands) or Delta Qb^T (wide, K-major), fp32,
-    // upper-triangle tiles mirrored; one group per (bucket, buffer holding Q)
-    LaunchSet htall, hwide;
-    init_set(htall, kEpiF32, kGateNone, p, Precision{0, 0, 1, 1, 0});
-    init_set(hwide, kEpiF32, kGateNone, p, Precision{0, 0, 1, 1, 0});
-    htall.p.list = hwide.p.list = nullptr;
-    htall.p.cnt = hwide.p.cnt = nullptr;
+    // upper-triangle tiles mirrored; one group per (bucket, buffer holding Q), one launch
+    LaunchSet hs;
+    init_set(hs, kEpiF32, kGateNone, p, Precision{0, 0, 1, 1, 0});
+    hs.p.list = nullptr;
+    hs.p.cnt = nullptr;
     for (size_t b = 0; b < p->buckets.size(); ++b) {
         const Bucket& bk = p->buckets[b];
         const CUtensorMap* m = maps + b * kMapsPerBucket;
@@ -1028,12 +1033,10 @@ static int run_clip(isoloco_plan* p, int kind, int max_iter, float tol, cudaStre
             g.f32_split_stride = (int64_t)bk.count * bk.n * bk.ld_n;
             g.ld_f32 = bk.ld_n;
             set_sym(g, bk.n);
-            (bk.tall ? htall : hwide).add(g);
+            hs.add(g, bk.tall, bk.tall);
         }
     }
-    if ((rc = flush_set(p, ISOLOCO_PHASE_CLIP, htall, true, true, st)) ||
-        (rc = flush_set(p, ISOLOCO_PHASE_CLIP, hwide, false, false, st)))
-        return rc;
+    if ((rc = flush_set(p, ISOLOCO_PHASE_CLIP, hs, st))) return rc;
     // ---- A' = H / sigma_bar - I -> the auxiliary plan; its polar factor Q_A = sign(A');
     // P = (I -/+ Q_A) / 2; S'' = (P A') P, all in the auxiliary plan's planes
     { PhaseTimer tm(p, ISOLOCO_PHASE_CLIP, st, 0);
@@ -1094,10 +1097,10 @@ static int run_clip(isoloco_plan* p, int kind, int max_iter, float tol, cudaStre
                 g.gate_fb = fa + 1;
                 g.bf_batch_stride = (int64_t)bk.n * bk.ld_n;
                 g.ld_bf = bk.ld_n;
-                ls.add(g);
+                ls.add(g, false, false);
             }
         }
-        if ((rc = flush_set(a, ISOLOCO_PHASE_CLIP, ls, false, false, st))) return rc;
+        if ((rc = flush_set(a, ISOLOCO_PHASE_CLIP, ls, st))) return rc;
     } }
     // ---- S' = I + S'' -> this plan's P planes (fp16); X = Q S' (tall) or S' Q (wide) into
     // the other ping-pong buffer (fp16, three passes), which then holds the result
@@ -1105,11 +1108,10 @@ static int run_clip(isoloco_plan* p, int kind, int max_iter, float tol, cudaStre
     k_clip_form_s<<<grid, 256, 0, st>>>(p->mats_d, a->mats_d, p->aux_of_d, a->state, a->phi, a->plo, p->phi, p->plo,
                                          a->err_d, p->err_d); }
     CUDA_TRY(cudaGetLastError());
-    LaunchSet ut, uw;
-    init_set(ut, kEpiXSplit, kGateNone, p, Precision{1, 1, 1, 1, 0});
-    init_set(uw, kEpiXSplit, kGateNone, p, Precision{1, 1, 1, 1, 0});
-    ut.p.list = uw.p.list = nullptr;
-    ut.p.cnt = uw.p.cnt = nullptr;
+    LaunchSet us;
+    init_set(us, kEpiXSplit, kGateNone, p, Precision{1, 1, 1, 1, 0});
+    us.p.list = nullptr;
+    us.p.cnt = nullptr;
     for (size_t b = 0; b < p->buckets.size(); ++b) {
         const Bucket& bk = p->buckets[b];
         const CUtensorMap* m = maps + b * kMapsPerBucket;
@@ -1136,12 +1138,10 @@ static int run_clip(isoloco_plan* p, int kind, int max_iter, float tol, cudaStre
             g.st_lo = m + st_map(dst, 1);
             g.bf_batch_stride = (int64_t)bk.rows * bk.ld;
             g.ld_bf = bk.ld;
-            (bk.tall ? ut : uw).add(g);
+            us.add(g, false, !bk.tall);
         }
     }
-    if ((rc = flush_set(p, ISOLOCO_PHASE_CLIP, ut, false, false, st)) ||
-        (rc = flush_set(p, ISOLOCO_PHASE_CLIP, uw, false, true, st)))
-        return rc;
+    if ((rc = flush_set(p, ISOLOCO_PHASE_CLIP, us, st))) return rc;
     { PhaseTimer tm(p, ISOLOCO_PHASE_CLIP, st);
     k_clip_flip<<<(p->nmat + 255) / 256, 256, 0, st>>>(p->state, p->nmat); }
     CUDA_TRY(cudaGetLastError());
@@ -1626,6 +1626,8 @@ int isoloco_debug_gemm(int a_mn, int b_mn, int precision, int batch, int M, int 
     gp.err = err;
     GemmGroup& g = gp.g[0];
     g.a_hi = maps_d; g.a_lo = maps_d + 1; g.b_hi = maps_d + 2; g.b_lo = maps_d + 3;
+    g.a_mn = a_mn != 0 ? 1 : 0;
+    g.b_mn = b_mn != 0 ? 1 : 0;
     set_group_common(g, M, N, K, batch, 1, 0);
     g.cta_begin = 0;
     g.out_f32 = D;
@@ -1638,7 +1640,7 @@ int isoloco_debug_gemm(int a_mn, int b_mn, int precision, int batch, int M, int 
     int dev = 0, sms = 148;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    cudaError_t e = launch_gemm(gp, a_mn != 0, b_mn != 0, sms, st);
+    cudaError_t e = launch_gemm(gp, sms, st);
     uint32_t herr = 0;
     if (e == cudaSuccess) e = cudaMemcpyAsync(&herr, err, 4, cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
@@ -1742,6 +1744,8 @@ int isoloco_debug_gemm_noalloc(int a_mn, int b_mn, int precision, int batch, int
     gp.err = err;
     GemmGroup& g = gp.g[0];
     g.a_hi = maps_d; g.a_lo = maps_d + 1; g.b_hi = maps_d + 2; g.b_lo = maps_d + 3;
+    g.a_mn = a_mn != 0 ? 1 : 0;
+    g.b_mn = b_mn != 0 ? 1 : 0;
     set_group_common(g, M, N, K, batch, 1, 0);
     g.cta_begin = 0;
     g.out_f32 = D;
@@ -1754,7 +1758,7 @@ int isoloco_debug_gemm_noalloc(int a_mn, int b_mn, int precision, int batch, int
     int dev = 0, sms = 148;
     CUDA_TRY(cudaGetDevice(&dev));
     CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
-    CUDA_TRY(launch_gemm(gp, a_mn != 0, b_mn != 0, sms, st));
+    CUDA_TRY(launch_gemm(gp, sms, st));
     uint32_t herr = 0;
     CUDA_TRY(cudaMemcpyAsync(&herr, err, 4, cudaMemcpyDeviceToHost, st));
     CUDA_TRY(cudaStreamSynchronize(st));

@@ -20,7 +20,9 @@
 // Operand layouts: K-major operands (K contiguous in global memory) use swizzled
 // tiles BK deep; MN-major operands (M or N contiguous) use 128-byte swizzled tiles of
 // 64 MN-elements x BK rows, two (A) or four (B) boxes per stage.  This lets X^T X,
-// X P and P X all read the row-major iterate without transposes.
+// X P and P X all read the row-major iterate without transposes.  The layout is a
+// property of each group, so one launch can mix them (the Grams X^T X of tall and
+// X X^T of wide matrices share a launch).
 #include <cstdio>
 
 #include "common.cuh"
@@ -390,7 +392,6 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
 // `tempty`.  The TMA ring runs continuously across tile boundaries, and the accumulator
 // is double buffered in tensor memory (2 x 256 columns): the epilogue of one tile
 // overlaps the MMAs of the next.
-template <bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_constant__ GemmParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = align1024(smem_raw);
@@ -515,7 +516,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                             tma_load_3d(dst, map, &full[stage], c0, c1, ti.b);
                     };
                     const int k0 = kb * BK;
-                    if (A_MN) {
+                    if (g.a_mn) {
 #pragma unroll
                         for (int c = 0; c < BM / 64; ++c) {
                             load(sa_hi + c * (BK * 128), g.a_hi, ti.m0 + 64 * c, k0);
@@ -525,7 +526,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                         load(sa_hi, g.a_hi, k0, ti.m0);
                         if (ti.a_split) load(sa_lo, g.a_lo, k0, ti.m0);
                     }
-                    if (B_MN) {
+                    if (g.b_mn) {
 #pragma unroll
                         for (int c = 0; c < kBRows / 64; ++c) {
                             load(sb_hi + c * (BK * 128), g.b_hi, nb0 + 64 * c, k0);
@@ -578,12 +579,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                 if (tile < 0) break;
             }
         } else if (lane == 0) {
-            const uint32_t idesc = make_idesc_16bit(kTileM, BN, A_MN, B_MN, p.in_f16 != 0);
-            const uint64_t desc_a0 = operand_desc<A_MN>(smem_u32(smem), 0);
-            const uint64_t desc_b0 = operand_desc<B_MN>(smem_u32(smem), 0);
-            // start-address step of one 16-deep K slice: 2048 bytes MN-major, 32 bytes K-major
-            constexpr uint64_t kDescStepA = A_MN ? (2048 >> 4) : (32 >> 4);
-            constexpr uint64_t kDescStepB = B_MN ? (2048 >> 4) : (32 >> 4);
+            const uint32_t sbase = smem_u32(smem);
             int stage = 0;
             uint32_t phase = 0;
             uint32_t n = 0;  // active tiles processed
@@ -614,6 +610,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                 tc_fence_after();
                 const uint32_t tacc = tmem_base + buf * kTmemCols;
                 if (ti.run_mma) {
+                    // instruction and operand descriptors for the layouts of this tile's group
+                    const bool a_mn = p.g[ti.gi].a_mn != 0, b_mn = p.g[ti.gi].b_mn != 0;
+                    const uint32_t idesc = make_idesc_16bit(kTileM, BN, a_mn, b_mn, p.in_f16 != 0);
+                    const uint64_t desc_a0 = a_mn ? operand_desc<true>(sbase, 0) : operand_desc<false>(sbase, 0);
+                    const uint64_t desc_b0 = b_mn ? operand_desc<true>(sbase, 0) : operand_desc<false>(sbase, 0);
+                    // start-address step of one 16-deep K slice: 2048 bytes MN-major, 32 bytes K-major
+                    const uint64_t step_a = a_mn ? (2048 >> 4) : (32 >> 4);
+                    const uint64_t step_b = b_mn ? (2048 >> 4) : (32 >> 4);
                     // descriptors of this tile's planes in stage 0; a stage or a 16-deep K
                     // slice only moves the start address (14-bit field in 16-byte units; every
                     // shared address is below 256 KB, so the sum never carries out of it)
@@ -633,7 +637,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
                         const uint64_t so = static_cast<uint64_t>(stage) * (stage_stride >> 4);
 #pragma unroll
                         for (int ks = 0; ks < BK / 16; ++ks) {
-                            const uint64_t da = so + ks * kDescStepA, db = so + ks * kDescStepB;
+                            const uint64_t da = so + ks * step_a, db = so + ks * step_b;
                             if (kPairMma) {
                                 umma_16bit_pair(tacc, a_hi0 + da, b_hi0 + db, idesc, acc);
                                 if (bs) umma_16bit_pair(tacc, a_hi0 + da, b_lo0 + db, idesc, 1u);
@@ -741,12 +745,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_split(const __grid_con
 }
 
 // ------------------------------------------------------------------ host launcher
-template <bool A_MN, bool B_MN>
-static cudaError_t launch_gemm_t(const GemmParams& p, int max_ctas, cudaStream_t stream) {
+// Launches one persistent GEMM over the groups of `p` (p.total_tiles output tiles) on at
+// most `max_ctas` CTAs (one per SM; with kPairMma, clusters of two CTAs per tile).
+cudaError_t launch_gemm(const GemmParams& p, int max_ctas, cudaStream_t stream) {
+    if (p.total_tiles <= 0) return cudaSuccess;
     static int max_clusters = 0;  // clusters of two that can be resident at once
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(k_gemm_split<A_MN, B_MN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaError_t e = cudaFuncSetAttribute(k_gemm_split, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              kGemmSmemBytes);
         if (e != cudaSuccess) return e;
         if (kPairMma) {
@@ -762,7 +768,7 @@ static cudaError_t launch_gemm_t(const GemmParams& p, int max_ctas, cudaStream_t
             cfg.attrs = at;
             cfg.numAttrs = 1;
             int n = 0;
-            e = cudaOccupancyMaxActiveClusters(&n, k_gemm_split<A_MN, B_MN>, &cfg);
+            e = cudaOccupancyMaxActiveClusters(&n, k_gemm_split, &cfg);
             if (e != cudaSuccess) return e;
             max_clusters = n > 0 ? n : 1;
         }
@@ -770,7 +776,7 @@ static cudaError_t launch_gemm_t(const GemmParams& p, int max_ctas, cudaStream_t
     }
     if (!kPairMma) {
         const int grid = p.total_tiles < max_ctas ? p.total_tiles : max_ctas;
-        k_gemm_split<A_MN, B_MN><<<grid, kGemmThreads, kGemmSmemBytes, stream>>>(p);
+        k_gemm_split<<<grid, kGemmThreads, kGemmSmemBytes, stream>>>(p);
         return cudaGetLastError();
     }
     int clusters = p.total_tiles;
@@ -788,17 +794,7 @@ static cudaError_t launch_gemm_t(const GemmParams& p, int max_ctas, cudaStream_t
     cfg.stream = stream;
     cfg.attrs = at;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, k_gemm_split<A_MN, B_MN>, p);
-}
-
-// Launches one persistent GEMM over the groups of `p` (p.total_tiles output tiles) on at
-// most `max_ctas` CTAs (one per SM; with kPairMma, clusters of two CTAs per tile).
-cudaError_t launch_gemm(const GemmParams& p, bool a_mn, bool b_mn, int max_ctas, cudaStream_t stream) {
-    if (p.total_tiles <= 0) return cudaSuccess;
-    if (!a_mn && !b_mn) return launch_gemm_t<false, false>(p, max_ctas, stream);
-    if (a_mn && b_mn) return launch_gemm_t<true, true>(p, max_ctas, stream);
-    if (!a_mn && b_mn) return launch_gemm_t<false, true>(p, max_ctas, stream);
-    return launch_gemm_t<true, false>(p, max_ctas, stream);
+    return cudaLaunchKernelEx(&cfg, k_gemm_split, p);
 }
 
 }  // namespace isoloco

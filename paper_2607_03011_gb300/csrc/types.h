@@ -85,6 +85,7 @@ struct GemmGroup {
     int mat_base;   // index of the group's first matrix in the state array
     int bucket;     // shape bucket: index into the work-list counts
     int gate_fb;    // 0: no condition; f > 0: only matrices whose Q is in buffer f - 1 (final_buf)
+    int a_mn, b_mn; // operand layout: 1 MN-major (M or N index contiguous), 0 K-major
     // fp32 output (kEpiF32): out_f32 + split*split_stride + b*batch_stride + row*ld + col
     float* out_f32;
     int64_t f32_split_stride, f32_batch_stride;
