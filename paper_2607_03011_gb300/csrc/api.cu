@@ -611,10 +611,17 @@ static int group_tiles(const GemmGroup& g) { return g.sym ? g.tiles_sym : g.tile
 struct LaunchSet {
     GemmParams p;
     std::vector<GemmGroup> groups;
-    // a_mn / b_mn: the operands' layouts in this group (MN-major or K-major)
-    void add(GemmGroup g, bool a_mn, bool b_mn) {
+    // a_mn / b_mn: the operands' layouts in this group (MN-major or K-major); the operands
+    // carry lo planes as the set's precision says
+    void add(GemmGroup g, bool a_mn, bool b_mn) { add(g, a_mn, b_mn, p.a_split != 0, p.b_split != 0); }
+    // ... or as given for this group (the launch's stages take room for either)
+    void add(GemmGroup g, bool a_mn, bool b_mn, bool a_split, bool b_split) {
         g.a_mn = a_mn ? 1 : 0;
         g.b_mn = b_mn ? 1 : 0;
+        g.a_split = a_split ? 1 : 0;
+        g.b_split = b_split ? 1 : 0;
+        p.a_split |= g.a_split;
+        p.b_split |= g.b_split;
         groups.push_back(g);
     }
 };
@@ -765,14 +772,14 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
             poly.add(g, false, false);
         }
         if ((rc = flush_set(p, ISOLOCO_PHASE_POLY, poly, st))) return rc;
-        // ---- X_{t+1} = xscale * X_t P (tall) or P X_t (wide)
+        // ---- X_{t+1} = xscale * X_t P (tall) or P X_t (wide), one launch
         // X_{t+1} is always written as fp16 planes; X is the split operand (A when tall,
-        // B when wide), P the single one except in the polish step (3 passes)
-        LaunchSet utall, uwide;
-        init_set(utall, kEpiXSplit, kGateStep, p,
-                 first ? Precision{0, 1, 1, 1, 0} : (full ? Precision{1, 1, 1, 1, 0} : Precision{1, 1, 1, 0, 1}));
-        init_set(uwide, kEpiXSplit, kGateStep, p,
-                 first ? Precision{0, 1, 1, 1, 0} : (full ? Precision{1, 1, 1, 1, 0} : Precision{1, 1, 0, 1, 1}));
+        // B when wide), P the single one except in the polish step (3 passes) and in
+        // iteration 0 and the full-precision paths (both split)
+        LaunchSet upd;
+        init_set(upd, kEpiXSplit, kGateStep, p,
+                 first ? Precision{0, 1, 0, 0, 0} : (full ? Precision{1, 1, 0, 0, 0} : Precision{1, 1, 0, 0, 1}));
+        const bool p_split = first || full;
         for (size_t b = 0; b < p->buckets.size(); ++b) {
             const Bucket& bk = p->buckets[b];
             const CUtensorMap* m = maps + b * kMapsPerBucket;
@@ -797,12 +804,11 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
             g.bf_batch_stride = (int64_t)bk.rows * bk.ld;
             g.ld_bf = bk.ld;
             if (bk.tall)
-                utall.add(g, false, false);
+                upd.add(g, false, false, true, p_split);
             else
-                uwide.add(g, false, true);
+                upd.add(g, false, true, p_split, true);
         }
-        if ((rc = flush_set(p, ISOLOCO_PHASE_UPDATE, utall, st)) ||
-            (rc = flush_set(p, ISOLOCO_PHASE_UPDATE, uwide, st)))
+        if ((rc = flush_set(p, ISOLOCO_PHASE_UPDATE, upd, st)))
             return rc;
     }
     return ISOLOCO_OK;
@@ -1628,6 +1634,8 @@ int isoloco_debug_gemm(int a_mn, int b_mn, int precision, int batch, int M, int 
     g.a_hi = maps_d; g.a_lo = maps_d + 1; g.b_hi = maps_d + 2; g.b_lo = maps_d + 3;
     g.a_mn = a_mn != 0 ? 1 : 0;
     g.b_mn = b_mn != 0 ? 1 : 0;
+    g.a_split = gp.a_split;
+    g.b_split = gp.b_split;
     set_group_common(g, M, N, K, batch, 1, 0);
     g.cta_begin = 0;
     g.out_f32 = D;
@@ -1746,6 +1754,8 @@ int isoloco_debug_gemm_noalloc(int a_mn, int b_mn, int precision, int batch, int
     g.a_hi = maps_d; g.a_lo = maps_d + 1; g.b_hi = maps_d + 2; g.b_lo = maps_d + 3;
     g.a_mn = a_mn != 0 ? 1 : 0;
     g.b_mn = b_mn != 0 ? 1 : 0;
+    g.a_split = gp.a_split;
+    g.b_split = gp.b_split;
     set_group_common(g, M, N, K, batch, 1, 0);
     g.cta_begin = 0;
     g.out_f32 = D;

@@ -116,8 +116,8 @@ __device__ __forceinline__ bool decode_tile(const GemmParams& p, const int* pre,
     ti.n0 = tn * BN;
     ti.mat = g.mat_base + ti.b;
     ti.run_mma = true;
-    ti.a_split = p.a_split != 0;
-    ti.b_split = p.b_split != 0;
+    ti.a_split = g.a_split != 0;
+    ti.b_split = g.b_split != 0;
     ti.ca = 0.f, ti.cb = 0.f, ti.cc = 1.f, ti.xs = 1.f, ti.yb = 0.f, ti.yc = 0.f;
     ti.horner = false;
     if (g.gate_fb && p.state[ti.mat].final_buf != g.gate_fb - 1) return false;

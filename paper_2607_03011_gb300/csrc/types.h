@@ -86,6 +86,7 @@ struct GemmGroup {
     int bucket;     // shape bucket: index into the work-list counts
     int gate_fb;    // 0: no condition; f > 0: only matrices whose Q is in buffer f - 1 (final_buf)
     int a_mn, b_mn; // operand layout: 1 MN-major (M or N index contiguous), 0 K-major
+    int a_split, b_split;  // operand carries a lo plane in this group (one tensor pass each)
     // fp32 output (kEpiF32): out_f32 + split*split_stride + b*batch_stride + row*ld + col
     float* out_f32;
     int64_t f32_split_stride, f32_batch_stride;
@@ -136,7 +137,7 @@ struct GemmParams {
     int gate;
     int in_f16;           // operand planes are fp16 (else bf16); also the G planes of kEpiPoly
     int out_f16;          // hi/lo output planes are fp16 (else bf16)
-    int a_split, b_split; // operand carries a lo plane (adds one tensor pass each)
+    int a_split, b_split; // some group's operand carries a lo plane (sizes the ring's stages)
     int split_on_polish;  // matrices in the polish step use both lo planes
     int gram_y;           // kEpiGram: also write Y = b I + c G for the next quintic step
     int poly_horner;      // kEpiPoly: B is Y, so P = G Y + a I (quintic steps)
