@@ -590,7 +590,8 @@ def main():
                 "achieved": achieved_tf, "peak": tc_peak, "unit": "TFLOP/s",
                 "frac": achieved_tf / tc_peak if tc_peak else None, "traffic": None,
                 "peak_source": f"{peak_src} bf16_tflops_sustained (dense 16-bit tensor rate; the kernel "
-                               "runs inside a ~20 ms step)",
+                               "runs inside a 10-30 ms step, repeated)",
+                "frac_of_burst": achieved_tf / peaks["bf16_tflops"] if peaks.get("bf16_tflops") else None,
                 "counts": "executed 16-bit tensor-pass FLOPs of the computed tiles",
                 "kernel_times": "per-phase CUDA events on the launch stream, in a profiled pass of the "
                                 "same steps right after the timed region",
