@@ -200,7 +200,7 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
     trf = warp_sum_f(trf);
     devf = warp_sum_f(devf);
     if (lane != 0) return;
-    const double sq = sqf, tr = trf, dev = devf;
+    const double sq = sqf, tr = trf;
 
     const double n = static_cast<double>(md.n);
     double d, gscale = 1.0, xscale = 1.0;
