@@ -174,10 +174,11 @@ def _sym_tiles(n):
     return c
 
 
-def gemm_exec_flops(table, diag, fast=False):
+def gemm_exec_flops(table, diag, fast=False, full=False):
     """Tensor-core FLOPs the GEMM launches execute per phase: 2*BM*BN*K_padded per
     computed tile and per 16-bit pass (3 passes at iteration 0 and in the final polish
-    update, 2 elsewhere), symmetric Grams/G^2 on their upper-triangle tiles only."""
+    update, 2 elsewhere; 3 everywhere with `full`, the clip variants' main iteration),
+    symmetric Grams/G^2 on their upper-triangle tiles only."""
     out = {"gram": 0.0, "poly": 0.0, "update": 0.0}
     mats = [(r, c) for (_, r, c) in table if c > 0]
     for (r, c), it, st in zip(mats, diag["iters"], diag["status"]):
@@ -197,12 +198,13 @@ def gemm_exec_flops(table, diag, fast=False):
         converged = (st == 0)
         grams = it + (0 if converged else 1)
         quintic = it - (1 if converged else 0)
-        out["gram"] += 3 * gram1 + 2 * gram1 * (grams - 1)
-        out["poly"] += (3 * poly1 + 2 * poly1 * (quintic - 1)) if quintic >= 1 else 0.0
+        p = 3 if full else 2   # passes after iteration 0
+        out["gram"] += 3 * gram1 + p * gram1 * (grams - 1)
+        out["poly"] += (3 * poly1 + p * poly1 * (quintic - 1)) if quintic >= 1 else 0.0
         if converged:
-            out["update"] += 3 * upd1 * (1 if it == 1 else 2) + 2 * upd1 * max(0, it - 2)
+            out["update"] += 3 * upd1 * (1 if it == 1 else 2) + p * upd1 * max(0, it - 2)
         else:
-            out["update"] += 3 * upd1 + 2 * upd1 * (it - 1)
+            out["update"] += 3 * upd1 + p * upd1 * (it - 1)
     return out
 
 
@@ -572,7 +574,7 @@ def main():
 
     peaks, peak_src = load_peaks()
     fl = gemm_flops(wl.table, diag, fast=args.fast_steps > 0)
-    fx = gemm_exec_flops(wl.table, diag, fast=args.fast_steps > 0)
+    fx = gemm_exec_flops(wl.table, diag, fast=args.fast_steps > 0, full=spectrum_kind != 0)
     flops = sum(fl.values()) * args.steps
     xflops = sum(fx.values()) * args.steps
     gemm_ms = prof["gram"][0] + prof["poly"][0] + prof["update"][0]
