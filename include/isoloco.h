@@ -244,6 +244,16 @@ int isoloco_debug_gemm_noalloc(int a_mn_major, int b_mn_major, int precision, in
                                int N, int K, const float* A, const float* B, float* D,
                                void* stream);
 
+/* Test of the timeout path of the pipelined kernels (no counterpart in the paper): one
+ * thread waits, with the bounded mbarrier wait every pipeline stage of the GEMM uses, on a
+ * barrier that nothing arrives on, and gives up after limit_ns nanoseconds of the GPU's
+ * global timer, as a kernel whose wait runs out does (it raises the TIMEOUT flag and
+ * returns; the context stays usable).  limit_ns must lie in 1e6 .. 1e9 (1 ms .. 1 s), else
+ * ISOLOCO_ERR_INVALID before any launch.  Returns ISOLOCO_ERR_TIMEOUT when the wait gave up
+ * (the expected outcome), ISOLOCO_OK if the barrier completed.  elapsed_ns (may be NULL)
+ * receives how long the wait took.  Allocates 12 bytes of scratch and synchronizes `stream`. */
+int isoloco_debug_wait_timeout(int64_t limit_ns, int64_t* elapsed_ns, void* stream);
+
 /* Phases of the launch sequence, for isoloco_profile_read. */
 enum {
     ISOLOCO_PHASE_REDUCE = 0,   /* pseudo-gradient reduction (HBM stream) */
@@ -257,7 +267,7 @@ enum {
     ISOLOCO_PHASE_DILOCO = 8,   /* fused DiLoCo pass (mean, DARE, or TIES's merge pass) */
     ISOLOCO_PHASE_OTHER = 9,
     ISOLOCO_PHASE_TRIM = 10,    /* TIES trim: per-worker radix select of the threshold */
-    ISOLOCO_PHASE_CLIP = 11,    /* clip_high / clip_low: H, sign(H - sigma_bar I), E P_sel */
+    ISOLOCO_PHASE_CLIP = 11,    /* clip_high / clip_low: H, sign(H / sigma_bar - I), P A' P, Q S' */
     ISOLOCO_NUM_PHASES = 12
 };
 

@@ -71,6 +71,7 @@ __global__ void k_ties_select(int, int, unsigned long long*, uint64_t*, uint64_t
 __global__ void k_ties_merge(ReplicaPtrs, int, int, float*, float*, int64_t, const uint64_t*, const uint64_t*,
                              const int*, float, float, uint32_t*);
 __global__ void k_split_planes(const float*, int64_t, int, int, int, __nv_bfloat16*, __nv_bfloat16*, int);
+__global__ void k_debug_wait(uint32_t*, uint64_t, unsigned long long*);
 
 constexpr int kChunkElems = 16384;
 constexpr int kTraceChunkElems = 16384;
@@ -1583,6 +1584,33 @@ int isoloco_read_diag(isoloco_plan_t p, void* stream, float* sigma_bar, int32_t*
         if (status) status[j] = m.status ? ISOLOCO_ERR_NOT_CONVERGED : ISOLOCO_OK;
         if (resid) resid[j] = m.resid;
     }
+    return ISOLOCO_OK;
+}
+
+int isoloco_debug_wait_timeout(int64_t limit_ns, int64_t* elapsed_ns, void* stream) {
+    if (limit_ns < 1000000 || limit_ns > 1000000000) return fail(ISOLOCO_ERR_INVALID, "limit_ns outside 1 ms .. 1 s");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    uint32_t* err = nullptr;
+    unsigned long long* el = nullptr;
+    if (cudaMalloc(&err, 4) != cudaSuccess || cudaMalloc(&el, 8) != cudaSuccess) {
+        cudaFree(err);
+        return fail(ISOLOCO_ERR_OOM, "debug_wait_timeout scratch allocation failed");
+    }
+    uint32_t herr = 0;
+    unsigned long long hel = 0;
+    cudaError_t e = cudaMemsetAsync(err, 0, 4, st);
+    if (e == cudaSuccess) {
+        k_debug_wait<<<1, 32, 0, st>>>(err, static_cast<uint64_t>(limit_ns), el);
+        e = cudaGetLastError();
+    }
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&herr, err, 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&hel, el, 8, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    cudaFree(err);
+    cudaFree(el);
+    if (e != cudaSuccess) return fail(ISOLOCO_ERR_CUDA, std::string("debug_wait_timeout: ") + cudaGetErrorString(e));
+    if (elapsed_ns) *elapsed_ns = static_cast<int64_t>(hel);
+    if (herr & kErrTimeout) return fail(ISOLOCO_ERR_TIMEOUT, "debug_wait_timeout: the wait gave up");
     return ISOLOCO_OK;
 }
 

@@ -18,6 +18,7 @@
 //                   sample (one pass over the replicas), then sign election, disjoint mean
 //                   and the outer step in one pass.
 //  k_split_planes : fp32 -> bf16 hi/lo planes (tests of the split-precision GEMM).
+//  k_debug_wait   : the bounded mbarrier wait running out (tests of the timeout path).
 #include "common.cuh"
 #include "types.h"
 
@@ -801,6 +802,21 @@ __global__ void k_split_planes(const float* __restrict__ x, int64_t total, int r
         reinterpret_cast<uint16_t*>(hi)[o] = h;
         reinterpret_cast<uint16_t*>(lo)[o] = l;
     }
+}
+
+// One thread waits, with the bounded wait of the GEMM's pipeline, on a fresh mbarrier that
+// nothing arrives on (its phase 0 never completes) and gives up after limit_ns; it then
+// raises kErrTimeout and returns, as a pipelined kernel does.  elapsed[0]: the wait's
+// duration (ns).
+__global__ void k_debug_wait(uint32_t* __restrict__ err, uint64_t limit_ns, unsigned long long* __restrict__ elapsed) {
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x != 0) return;
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+    const uint64_t t0 = globaltimer_ns();
+    const bool ok = mbar_wait(&bar, 0u, limit_ns);
+    elapsed[0] = globaltimer_ns() - t0;
+    if (!ok) atomicOr(err, kErrTimeout);
 }
 
 }  // namespace isoloco

@@ -84,6 +84,7 @@ def lib():
             L.isoloco_debug_gemm.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                              ctypes.c_int, ctypes.c_int, _vp, _vp, _vp, _vp]
             L.isoloco_debug_gemm_noalloc.argtypes = L.isoloco_debug_gemm.argtypes
+            L.isoloco_debug_wait_timeout.argtypes = [ctypes.c_int64, ctypes.POINTER(ctypes.c_int64), _vp]
             _lib = L
     return _lib
 
@@ -269,3 +270,13 @@ def debug_gemm_noalloc(A: torch.Tensor, B: torch.Tensor, D: torch.Tensor, a_mn_m
     rc = lib().isoloco_debug_gemm_noalloc(int(a_mn_major), int(b_mn_major), int(precision), A.shape[0], M, N, K,
                                           A.data_ptr(), B.data_ptr(), D.data_ptr(), _stream(stream))
     return _check(rc, "isoloco_debug_gemm_noalloc", hard_only=False)
+
+
+def debug_wait_timeout(limit_ns: int, stream=None):
+    """A bounded device wait that nothing ends runs out after limit_ns (see
+    isoloco_debug_wait_timeout in include/isoloco.h).  Returns (status, elapsed_ns)."""
+    el = ctypes.c_int64(0)
+    rc = lib().isoloco_debug_wait_timeout(int(limit_ns), ctypes.byref(el), _stream(stream))
+    if rc not in (OK, ERR_TIMEOUT):
+        raise IsolocoError(rc, f"isoloco_debug_wait_timeout: {last_error()}")
+    return rc, el.value

@@ -62,6 +62,8 @@ def test_validation_without_gpu(lib):
     assert lib.diloco_outer_step(None, None, None, None, None, None) == isoloco.ERR_INVALID
     assert lib.isoloco_debug_gemm(0, 0, 0, 0, 1, 1, 1, None, None, None, None) == isoloco.ERR_INVALID
     assert lib.isoloco_debug_gemm(0, 0, 9, 1, 1, 1, 1, None, None, None, None) == isoloco.ERR_INVALID
+    assert lib.isoloco_debug_wait_timeout(1_000, None, None) == isoloco.ERR_INVALID          # below 1 ms
+    assert lib.isoloco_debug_wait_timeout(2_000_000_000, None, None) == isoloco.ERR_INVALID  # above 1 s
 
 
 def test_opts_layout_matches_the_header(tmp_path, lib):

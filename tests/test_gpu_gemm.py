@@ -80,3 +80,22 @@ def test_debug_gemm_deterministic(iso):
     D1 = iso.debug_gemm(A, B, 0, 1, 256, 512, 512)
     D2 = iso.debug_gemm(A, B, 0, 1, 256, 512, 512)
     assert torch.equal(D1, D2)
+
+
+def test_bounded_wait_runs_out_and_the_context_survives(iso):
+    """The pipeline's bounded mbarrier wait on a barrier that nothing arrives on gives up
+    after its limit and reports TIMEOUT; the GPU context stays usable (a GEMM right after
+    is exact).  Limits outside 1 ms .. 1 s are refused before any launch."""
+    rc, elapsed = iso.debug_wait_timeout(20_000_000)
+    assert rc == iso.ERR_TIMEOUT
+    assert 20_000_000 <= elapsed < 1_000_000_000
+    with pytest.raises(iso.IsolocoError):
+        iso.debug_wait_timeout(1_000)
+    with pytest.raises(iso.IsolocoError):
+        iso.debug_wait_timeout(2_000_000_000)
+    g = torch.Generator(device="cuda").manual_seed(9)
+    A = torch.randn((1, 256, 512), device="cuda", generator=g)
+    B = torch.randn((1, 256, 512), device="cuda", generator=g)
+    D = iso.debug_gemm(A, B, 0, 0, 256, 256, 512)
+    ref = _ref(A, B, 0, 0)
+    assert ((D.double() - ref).norm() / ref.norm()).item() < 3e-5
