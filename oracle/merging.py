@@ -8,9 +8,10 @@ direction U with the outer optimiser (Nesterov; mu = 0 is the SGD step of Sec. 5
   - trim: each worker keeps its n_keep = N - floor(sparsity * N) largest magnitudes
     |Delta_k| over all N entries of its task vector; entries equal to the n_keep-th largest
     are kept too (ties kept);
-  - elect: the sign of the total mass of the kept values; here sign(P + Nn), P and Nn the
-    sums, in worker order, of an entry's kept positive and kept negative values, taken in
-    fp32 (the precision of the library's decision);
+  - elect: the sign of the total mass of the kept values, sign(sum_k kept_k), taken
+    exactly: an fp64 sum decides every entry whose sum clears that sum's own rounding
+    bound, and the few that do not are summed as exact rationals, so the election depends
+    on neither the order of the workers nor a working precision;
   - merge: U = mean of the kept values whose sign is the elected one (fp64), 0 if the
     elected sign is 0.
 * DARE (drop and rescale; Yu et al. 2024): each entry of each Delta_k is dropped with
@@ -31,6 +32,7 @@ at sparsity 0, DARE's drop rate and unbiasedness).
 from __future__ import annotations
 
 import math
+from fractions import Fraction
 
 import numpy as np
 
@@ -89,23 +91,43 @@ def ties_trim(d: np.ndarray, sparsity: float):
     return np.abs(d) >= thr[:, None], thr
 
 
-def ties_merge(d: np.ndarray, sparsity: float, thr: np.ndarray | None = None) -> np.ndarray:
+def ties_elect(kept: np.ndarray) -> np.ndarray:
+    """Elected sign per entry (-1, 0 or 1): the sign of the exact sum over workers of the
+    kept fp32 values kept [K, N].  The fp64 sum of K fp32 values is within
+    K * 2^-53 * sum|kept| of the exact one, so its sign is exact wherever it clears that
+    bound; the remaining entries (exact or near-exact cancellations) are summed as
+    rationals."""
+    k64 = kept.astype(np.float64)
+    s = k64.sum(axis=0)
+    bound = kept.shape[0] * 2.0 ** -53 * np.abs(k64).sum(axis=0)
+    gamma = np.sign(s)
+    for i in np.nonzero((np.abs(s) <= bound) & (bound > 0))[0]:
+        gamma[i] = np.sign(sum((Fraction(float(x)) for x in kept[:, i]), Fraction(0)))
+    return gamma
+
+
+def ties_merge(d: np.ndarray, sparsity: float, thr: np.ndarray | None = None, parts: bool = False):
     """TIES direction U in fp64 from fp32 task vectors d [K, N]; thr (per worker) given when
-    d holds only some entries of the task vectors."""
+    d holds only some entries of the task vectors.  With parts=True also returns the
+    disjoint means of the kept positive and kept negative values (the two values U can
+    take), the kept mass sum_k kept_k and sum_k |kept_k| (fp64), for callers that check an
+    election taken in a narrower precision."""
     if thr is None:
         thr = ties_thresholds(d, sparsity)
     kept = np.where(np.abs(d) >= np.asarray(thr, np.float32)[:, None], d, np.float32(0.0)).astype(np.float32)
-    P = np.zeros(d.shape[1], np.float32)
-    Nn = np.zeros(d.shape[1], np.float32)
-    for k in range(d.shape[0]):                      # fp32, worker order
-        P = P + np.where(kept[k] > 0, kept[k], np.float32(0.0))
-        Nn = Nn + np.where(kept[k] < 0, kept[k], np.float32(0.0))
-    gamma = np.sign(P + Nn)                          # fp32 sum, then its sign
+    gamma = ties_elect(kept)
     k64 = kept.astype(np.float64)
     agree = (np.sign(k64) == gamma[None, :]) & (k64 != 0)
     cnt = agree.sum(axis=0)
     tot = np.where(agree, k64, 0.0).sum(axis=0)
-    return np.where(cnt > 0, tot / np.maximum(cnt, 1), 0.0)
+    u = np.where(cnt > 0, tot / np.maximum(cnt, 1), 0.0)
+    if not parts:
+        return u
+    pos, neg = k64 > 0, k64 < 0
+    u_pos = np.where(pos, k64, 0.0).sum(axis=0) / np.maximum(pos.sum(axis=0), 1)
+    u_neg = np.where(neg, k64, 0.0).sum(axis=0) / np.maximum(neg.sum(axis=0), 1)
+    return {"update": u, "u_pos": u_pos, "u_neg": u_neg, "mass": k64.sum(axis=0),
+            "abs_mass": np.abs(k64).sum(axis=0)}
 
 
 def dare_mask(K: int, n: int, sparsity: float, seed: int, idx: np.ndarray | None = None) -> np.ndarray:
@@ -132,10 +154,13 @@ def dare_merge(d: np.ndarray, sparsity: float, seed: int, reduce_mean: bool = Tr
 def merged_outer_step(theta, momentum, replicas, aggregator: str, sparsity: float = 0.0,
                       seed: int = 0, eta: float = 0.7, mu: float = 0.9, reduce_mean: bool = True):
     """Alg. 1's outer step with a merging aggregator ("ties" or "dare") in place of the
-    mean.  Returns dict(theta, momentum, update) in fp64."""
+    mean.  Returns dict(theta, momentum, update) in fp64; for TIES also "ties_parts", the
+    election's candidates and mass (``ties_merge(parts=True)``)."""
     d = task_vectors(theta, replicas)
+    parts = None
     if aggregator == "ties":
-        u = ties_merge(d, sparsity)
+        parts = ties_merge(d, sparsity, parts=True)
+        u = parts["update"]
     elif aggregator == "dare":
         u = dare_merge(d, sparsity, seed, reduce_mean)
     else:
@@ -143,4 +168,7 @@ def merged_outer_step(theta, momentum, replicas, aggregator: str, sparsity: floa
     th = np.asarray(theta, dtype=np.float32).astype(np.float64).ravel()
     b = np.asarray(momentum, dtype=np.float32).astype(np.float64).ravel()
     to, bo = nesterov(u, th, b, eta, mu)
-    return {"theta": to, "momentum": bo, "update": u}
+    out = {"theta": to, "momentum": bo, "update": u}
+    if parts is not None:
+        out["ties_parts"] = parts
+    return out

@@ -9,6 +9,13 @@ at K > 1 is a sum of mixed signs that can cancel to 0 on one side only; a wrong 
 there moves U by |Delta_k| / K, far outside the value tolerance).  U = B' elementwise to
 a relative 1e-5 (fp32 sums of at most K terms against fp64), and theta' to its own fp32
 rounding plus 1e-5 of the update.
+
+The oracle elects TIES's sign from the exact kept mass; the library sums in fp32, whose
+result is within K 2^-24 sum_k |kept_k| of the exact mass.  Entries whose exact mass lies
+inside that bound may elect either sign there: they are exempt from the sign check, and
+their U must equal one of the two candidates the oracle gives (the disjoint mean of the
+kept positive or of the kept negative values) or 0.  Every other entry is compared bit
+for bit; the exempt count is printed.
 """
 import numpy as np
 import pytest
@@ -43,12 +50,41 @@ def run(iso, wl, agg, s, seed=1234, eta=0.7, mu=0.9, reduce_mean=True, plan=None
     return rc, th, b
 
 
-def check(th, b, ref, theta_in, agg):
+def ties_exempt(parts, K):
+    """Entries whose exact kept mass lies within the fp32 election's rounding bound
+    K 2^-24 sum_k |kept_k| of 0 (and that keep something)."""
+    return (np.abs(parts["mass"]) <= K * 2.0 ** -24 * parts["abs_mass"]) & (parts["abs_mass"] > 0)
+
+
+def ties_check(u_gpu, parts, K, where=""):
+    """TIES's U against the oracle's exact election (module docstring); returns the number
+    of entries exempt from the sign check."""
+    u_ref = parts["update"]
+    amb = ties_exempt(parts, K)
+    ok = ~amb
+    assert np.array_equal(u_gpu[ok] == 0, u_ref[ok] == 0), f"trim decisions differ{where}"
+    assert np.array_equal(np.sign(u_gpu[ok]), np.sign(u_ref[ok])), f"elected signs differ{where}"
+    assert elementwise_rel(u_gpu[ok], u_ref[ok]) < 1e-5
+    if amb.any():
+        ua = u_gpu[amb]
+        rms = np.sqrt(np.mean(u_ref ** 2)) if u_ref.size else 0.0
+        best = np.min(np.stack([np.abs(ua - parts["u_pos"][amb]) / np.maximum(np.abs(parts["u_pos"][amb]), rms),
+                                np.abs(ua - parts["u_neg"][amb]) / np.maximum(np.abs(parts["u_neg"][amb]), rms),
+                                np.abs(ua) / max(rms, 1e-300)]), axis=0)
+        assert np.max(best) < 1e-5, f"an exempt entry is none of the election's candidates{where}"
+    return int(amb.sum())
+
+
+def check(th, b, ref, theta_in, agg, K):
     u_gpu = b.double().cpu().numpy()
     u_ref = ref["update"]
     if agg == "ties":
-        assert np.array_equal(u_gpu == 0, u_ref == 0), "trim decisions differ"
-        assert np.array_equal(np.sign(u_gpu), np.sign(u_ref)), "elected signs differ"
+        nex = ties_check(u_gpu, ref["ties_parts"], K)
+        print(f"TIES: {nex} of {u_gpu.size} entries within the fp32 election bound (exempt from the sign check)")
+        # theta' follows U: compare it where the election is decided
+        ok = ~ties_exempt(ref["ties_parts"], K)
+        check_theta(th.double().cpu().numpy()[ok], ref["theta"][ok], theta_in[ok])
+        return
     assert elementwise_rel(u_gpu, u_ref) < 1e-5
     check_theta(th.double().cpu().numpy(), ref["theta"], theta_in)
 
@@ -75,7 +111,7 @@ def test_ragged(iso, agg, s, dtype):
     th_in = wl.theta.cpu().numpy()
     ref = merging.merged_outer_step(th_in, np.zeros(wl.N, np.float32), W.replicas_as_numpy(wl.replicas),
                                     agg, sparsity=s, seed=1234, eta=0.7, mu=0.9)
-    check(th, b, ref, th_in.astype(np.float64), agg)
+    check(th, b, ref, th_in.astype(np.float64), agg, K=wl.K)
 
 
 @pytest.mark.parametrize("agg,s", [("ties", 0.3), ("dare", 0.3)])
@@ -106,7 +142,7 @@ def test_sum_reduction_and_sgd(iso):
         assert rc == 0
         ref = merging.merged_outer_step(th_in, np.zeros(wl.N, np.float32), reps, agg, sparsity=0.2, seed=5,
                                         eta=0.7, mu=mu, reduce_mean=mean)
-        check(th, b, ref, th_in.astype(np.float64), agg)
+        check(th, b, ref, th_in.astype(np.float64), agg, K=wl.K)
 
 
 @pytest.mark.parametrize("agg", ["ties", "dare"])
@@ -120,7 +156,7 @@ def test_mid_size_many_grid_strides(iso, agg):
     th_in = wl.theta.cpu().numpy()
     ref = merging.merged_outer_step(th_in, np.zeros(wl.N, np.float32), W.replicas_as_numpy(wl.replicas),
                                     agg, sparsity=0.1, seed=3, eta=0.7, mu=0.9)
-    check(th, b, ref, th_in.astype(np.float64), agg)
+    check(th, b, ref, th_in.astype(np.float64), agg, K=wl.K)
 
 
 def test_bad_options_rejected(iso):
@@ -165,21 +201,25 @@ def test_llama_180m_k8_full(iso, agg):
             thr[k] = merging.ties_thresholds(dk, s)[0]
             del dk
     step = 1 << 24
+    exempt = 0
     for c0 in range(0, n, step):
         c1 = min(n, c0 + step)
         d = merging.task_vectors(th_in[c0:c1], W.replicas_as_numpy(wl.replicas[:, c0:c1]))
+        ug = u_gpu[c0:c1].astype(np.float64)
+        t_in = th_in[c0:c1].astype(np.float64)
+        sel = slice(None)
         if agg == "ties":
-            u_ref = merging.ties_merge(d, s, thr=thr)
+            parts = merging.ties_merge(d, s, thr=thr, parts=True)
+            u_ref = parts["update"]
+            exempt += ties_check(ug, parts, K, where=f" in [{c0}, {c1})")
+            sel = ~ties_exempt(parts, K)
         else:
             u_ref = merging.dare_merge(d, s, seed, n_total=n, idx=np.arange(c0, c1))
-        ug = u_gpu[c0:c1].astype(np.float64)
-        if agg == "ties":
-            assert np.array_equal(ug == 0, u_ref == 0), f"trim decisions differ in [{c0}, {c1})"
-            assert np.array_equal(np.sign(ug), np.sign(u_ref))
-        assert elementwise_rel(ug, u_ref) < 1e-5
-        t_in = th_in[c0:c1].astype(np.float64)
+            assert elementwise_rel(ug, u_ref) < 1e-5
         t_ref = t_in - wl.spec.outer_lr * (u_ref + wl.spec.momentum * u_ref)
-        check_theta(th_gpu[c0:c1].astype(np.float64), t_ref, t_in)
+        check_theta(th_gpu[c0:c1].astype(np.float64)[sel], t_ref[sel], t_in[sel])
+    if agg == "ties":
+        print(f"TIES at 180M K=8: {exempt} of {n} entries within the fp32 election bound (exempt from the sign check)")
     del wl
     torch.cuda.empty_cache()
 
@@ -235,4 +275,4 @@ def test_ties_bracket_fallback_on_tied_magnitudes(iso):
     th_in = theta.cpu().numpy()
     ref = merging.merged_outer_step(th_in, np.zeros(n, np.float32), [r.cpu().numpy() for r in reps], "ties",
                                     sparsity=0.5, eta=0.7, mu=0.9)
-    check(th, b, ref, th_in.astype(np.float64), "ties")
+    check(th, b, ref, th_in.astype(np.float64), "ties", K=K)

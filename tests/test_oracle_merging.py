@@ -61,6 +61,34 @@ def test_ties_exact_cancellation_gives_zero():
     assert list(merging.ties_merge(d, 0.0)) == [0.0, 1.0]
 
 
+def test_ties_election_is_exact_and_order_free():
+    """The election is the sign of the exact kept mass.  [2^60, 1, -2^60] sums to 1 > 0,
+    which an fp64 sum in this order misses (2^60 + 1 rounds to 2^60) and an fp32 running
+    sum misses too; [1, 2^-30, -1] sums to 2^-30 > 0, lost by an fp32 running sum.  Every
+    worker order gives the same sign and the same disjoint mean."""
+    import itertools
+    for col, want_sign in (([2.0 ** 60, 1.0, -(2.0 ** 60)], 1.0), ([1.0, 2.0 ** -30, -1.0], 1.0),
+                           ([-(2.0 ** 60), -1.0, 2.0 ** 60], -1.0), ([3.0, -1.0, -2.0], 0.0)):
+        for perm in itertools.permutations(col):
+            kept = np.array(perm, np.float32)[:, None]
+            assert merging.ties_elect(kept)[0] == want_sign
+            u = merging.ties_merge(kept, 0.0)[0]
+            pos = [x for x in col if x > 0]
+            neg = [x for x in col if x < 0]
+            want = np.mean(pos) if want_sign > 0 else (np.mean(neg) if want_sign < 0 else 0.0)
+            assert u == want
+    # fp32 running sums in worker order would elect 0 for the second column
+    assert np.float32(np.float32(1.0) + np.float32(2.0 ** -30)) - np.float32(1.0) == 0.0
+
+
+def test_ties_parts_hold_both_candidates():
+    d = np.array([[1.0, -2.0, 0.5], [3.0, 1.0, -0.5], [-1.0, -4.0, 0.0]], np.float32)
+    p = merging.ties_merge(d, 0.0, parts=True)
+    assert np.allclose(p["u_pos"], [2.0, 1.0, 0.5]) and np.allclose(p["u_neg"], [-1.0, -3.0, -0.5])
+    assert np.allclose(p["mass"], [3.0, -5.0, 0.0]) and np.allclose(p["abs_mass"], [5.0, 7.0, 1.0])
+    assert list(p["update"]) == [2.0, -3.0, 0.0]
+
+
 def test_ties_keeps_ties_at_threshold():
     """n_keep = 3 of [2, -2, 1, -1]: the 3rd largest magnitude is 1, so all four stay."""
     d = merging.task_vectors(*_reps_from_deltas([[2.0, -2.0, 1.0, -1.0]]))
