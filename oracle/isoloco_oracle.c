@@ -118,16 +118,20 @@ void orc_nesterov(int64_t n, const double* U, double mu, double eta,
 /*   W_in V = W_out  with orthogonal columns,  sigma_i = ||w_i||.              */
 /* Pairs are visited in round-robin (tournament) order, so the n/2 pairs of a  */
 /* round touch disjoint columns and may be rotated concurrently.               */
+/* A column whose squared norm is at most `neg2` = n (eps ||W||_F)^2 is below  */
+/* Iso-C's zero cut r eps sigma_max (||W||_F <= sqrt(n) sigma_max, r = n): it  */
+/* is not rotated.  Without this the rounding-level columns of an exactly      */
+/* rank-deficient W keep rotating among themselves and the sweeps never end.   */
 /* ------------------------------------------------------------------------- */
 static int rotate_pair(int m, int n, double* wp, double* wq, double* vp, double* vq,
-                       double tol) {
+                       double tol, double neg2) {
     double a = 0.0, b = 0.0, c = 0.0;
     for (int i = 0; i < m; ++i) {
         a += wp[i] * wp[i];
         b += wq[i] * wq[i];
         c += wp[i] * wq[i];
     }
-    if (a == 0.0 || b == 0.0) return 0;
+    if (a <= neg2 || b <= neg2) return 0;
     if (fabs(c) <= tol * sqrt(a) * sqrt(b)) return 0;
     /* Choose the rotation angle that zeroes the off-diagonal entry of the 2x2
      * Gram [[a, c], [c, b]]: t = tan(angle) is the smaller root of
@@ -158,6 +162,9 @@ static int jacobi_svd_cols(int m, int n, double* W, double* V, int max_sweeps,
     for (int j = 0; j < n; ++j)
         for (int i = 0; i < n; ++i) V[(size_t)j * n + i] = (i == j) ? 1.0 : 0.0;
     double tol = (double)(m > 1 ? m : 1) * DBL_EPSILON;
+    double fro2 = 0.0;
+    for (size_t i = 0; i < (size_t)m * n; ++i) fro2 += W[i] * W[i];
+    double neg2 = (double)n * DBL_EPSILON * DBL_EPSILON * fro2;
     int sweep = 0, converged = (n < 2);
     while (!converged && sweep < max_sweeps) {
         long rotated = 0;
@@ -169,7 +176,7 @@ static int jacobi_svd_cols(int m, int n, double* W, double* V, int max_sweeps,
                 if (p >= n || q >= n) continue;
                 if (p > q) { int tmp = p; p = q; q = tmp; }
                 rotated += rotate_pair(m, n, W + (size_t)p * m, W + (size_t)q * m,
-                                       V + (size_t)p * n, V + (size_t)q * n, tol);
+                                       V + (size_t)p * n, V + (size_t)q * n, tol, neg2);
             }
             /* tournament schedule: keep order[0], cycle the rest by one seat */
             int last = order[n2 - 1];

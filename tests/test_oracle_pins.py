@@ -199,6 +199,47 @@ def test_rank_deficient_is_partial_isometry():
     assert s_out.sum() == pytest.approx(nuc * rho / n, rel=1e-10)
 
 
+def _np_partial_isometry(d, alpha=1.0):
+    """Iso-C of a rank-deficient matrix from LAPACK's SVD: alpha * mean(sigma) * U_rho V_rho^T
+    with rho the singular values above r * eps * sigma_max (reading C3)."""
+    u, s, vt = np.linalg.svd(d, full_matrices=False)
+    rho = int(np.sum(s > min(d.shape) * np.finfo(float).eps * s[0]))
+    return alpha * s.mean() * (u[:, :rho] @ vt[:rho]), s.mean(), rho
+
+
+@pytest.mark.parametrize("m,n,zero", [(128, 64, ("rows", 5)), (64, 128, ("cols", 7)), (96, 40, ("cols", 25)),
+                                      (256, 256, ("rows", 240)), (200, 200, ("both", 150))])
+def test_structurally_rank_deficient(m, n, zero):
+    """Zero rows or columns (entries no worker touched) give an exactly rank-deficient
+    matrix; rounding-level columns must not keep the Jacobi sweeps going, and the result
+    is LAPACK's partial isometry with rho = the number of nonzero rows (columns)."""
+    rng = np.random.default_rng(m * 1000 + n)
+    D = rng.standard_normal((m, n))
+    kind, keep = zero
+    if kind in ("rows", "both"):
+        D[keep:, :] = 0.0
+    if kind in ("cols", "both"):
+        D[:, keep:] = 0.0
+    out, sb = oracle.iso_c(D, 0.5)
+    ref, sb_ref, rho = _np_partial_isometry(D, 0.5)
+    assert rho == keep
+    assert sb == pytest.approx(sb_ref, rel=1e-12)
+    assert np.linalg.norm(out - ref) / np.linalg.norm(ref) < 1e-11
+    s_out = np.linalg.svd(out, compute_uv=False)
+    assert np.all(np.abs(s_out[:rho] / (0.5 * sb) - 1.0) < 1e-11) and np.all(s_out[rho:] < 1e-12 * s_out[0])
+
+
+def test_low_rank_product_is_partial_isometry():
+    """A generic rank-12 product (no zero rows) of a 300 x 200 matrix."""
+    rng = np.random.default_rng(7)
+    D = rng.standard_normal((300, 12)) @ rng.standard_normal((12, 200))
+    out, sb = oracle.iso_c(D)
+    ref, sb_ref, rho = _np_partial_isometry(D)
+    assert rho == 12
+    assert sb == pytest.approx(sb_ref, rel=1e-10)
+    assert np.linalg.norm(out - ref) / np.linalg.norm(ref) < 1e-9
+
+
 def test_zero_matrix():
     out, sb = oracle.iso_c(np.zeros((8, 5)), 1.0)
     assert sb == 0.0 and not out.any()
