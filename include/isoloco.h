@@ -116,6 +116,16 @@ typedef struct {
                         * max(s_i, sigma_bar).  1 and 2 need fast_steps = 0 and scale_kind = 0;
                         * their first call allocates an auxiliary plan (the n x n matrices
                         * H - sigma_bar I, H = Q^T Delta) and its buffers. */
+    int full_precision; /* 0: the polar steps after the first keep one GEMM operand at 11 bits
+                         * (two 16-bit passes; its rounding only perturbs the spectrum of a
+                         * full-rank iterate, which later steps correct).  1: every step splits
+                         * both operands (three passes, ~22 bits each; ~1.5x the GEMM work).
+                         * For an exactly rank-deficient Delta (Iso-C's partial isometry
+                         * U_rho V_rho^T) whose zero directions are not whole rows of a wide or
+                         * whole columns of a tall matrix (e.g. many zero rows of a tall or
+                         * square one), the 11-bit operand turns the iterate's row space toward
+                         * the zero directions by ~2^-11 per step; 1 keeps the result within
+                         * the Iso-C tolerance there. */
 } isoloco_opts_t;
 
 /* Fills *opts with alpha = 1, outer_lr = 0.7, momentum = 0.9 (the paper's DiLoCo

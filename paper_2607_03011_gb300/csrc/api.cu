@@ -1170,6 +1170,8 @@ static int check_opts(const isoloco_opts_t* o, isoloco_opts_t* out) {
         return fail(ISOLOCO_ERR_INVALID, "sparsity must be in [0, 1)");
     if (out->spectrum_kind < 0 || out->spectrum_kind > 2)
         return fail(ISOLOCO_ERR_INVALID, "spectrum_kind must be 0, 1 or 2");
+    if (out->full_precision < 0 || out->full_precision > 1)
+        return fail(ISOLOCO_ERR_INVALID, "full_precision must be 0 or 1");
     if (out->spectrum_kind && (out->fast_steps || out->scale_kind))
         return fail(ISOLOCO_ERR_INVALID, "clip_high / clip_low need the exact polar path and sigma_bar "
                                          "(fast_steps = 0, scale_kind = 0)");
@@ -1239,7 +1241,7 @@ static int run_isoc_step(isoloco_plan* p, int merge, float* theta, float* mom, c
         CUDA_TRY(cudaEventRecord(p->ev_copied, p->side_st));
     }
     p->fast_steps = merge ? 0 : o.fast_steps;
-    p->full_prec = !merge && o.spectrum_kind != 0;
+    p->full_prec = !merge && (o.spectrum_kind != 0 || o.full_precision != 0);
     p->skip_trace = !merge && (o.fast_steps > 0 || o.scale_kind == 1);
     if ((rc = run_polar(p, p->fast_steps ? std::max(o.max_iter, o.fast_steps) : o.max_iter, o.tol, st))) return rc;
     const int clip = merge ? 0 : o.spectrum_kind;
@@ -1287,6 +1289,7 @@ int isoloco_opts_default(isoloco_opts_t* o) {
     o->sparsity = 0.f;
     o->seed = 0u;
     o->spectrum_kind = 0;
+    o->full_precision = 0;
     return ISOLOCO_OK;
 }
 

@@ -5,8 +5,9 @@
 //                    convergence test (the Gram GEMM's epilogue does this otherwise).
 //  k_control       : one warp per matrix; sums the partials in a fixed order,
 //                    normalises at t = 0 (s^2 = ||Delta^T Delta||_F >= sigma_max^2),
-//                    tests ||X^T X - I||_F / sqrt(n) < tol and picks this
-//                    iteration's polynomial: the next quintic of the schedule, the
+//                    tests ||X^T X - I||_F / sqrt(n) < tol (or, for an exactly
+//                    rank-deficient Delta, the partial-isometry test below) and picks
+//                    this iteration's polynomial: the next quintic of the schedule, the
 //                    final cubic polish, or stop.
 //  k_trace_partial / k_trace_final : sigma_bar = tr(Q^T Delta) / n (Alg. 2's mean
 //                    singular value: for the polar factor Q, Q^T Delta = V S V^T).
@@ -157,6 +158,44 @@ __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict
 // any later round, and every round of the other matrices, is the full standard schedule.
 // (Singular values under 1e-8 of s are below what the split arithmetic resolves.)
 constexpr int kDeepRestart = 2;  // first standard step after the deep round
+
+// Partial isometries (Alg. 2's Iso-C of a rank-deficient Delta: Q = U_rho V_rho^T).  A
+// direction whose singular value is exactly 0 stays at 0 under every odd polynomial step,
+// so ||X^T X - I||_F^2 keeps one unit per such direction and the full-rank test never
+// passes.  The iteration cannot tell such a direction from a tiny nonzero one still being
+// lifted, so singular values below kZeroFloor of the normalisation (under what the
+// split-precision arithmetic resolves) are the ones taken as zero, and the test waits for
+// the end of a round that started with every value at or above kZeroFloor inside the
+// round's design interval (lift_round * kZeroFloor >= the round's first lower bound): the
+// schedule then guarantees all of them in [0.998, 1.002], and what is left near 0 is zero.
+// With rho = round(tr X^T X) < n directions at 1, the residual of the converged part,
+// (||X^T X - I||_F^2 - (n - rho)) / rho (each zero direction adds ~1 to the first term),
+// must be below tol^2; the matrix then takes the cubic polish, which keeps zeros at zero.
+constexpr float kZeroFloor = 1e-8f;
+
+// Rounds of the schedule (sched_row): a near-square matrix takes the deep round (steps
+// 0 .. kSchedDeepSteps - 1), the restart round (kSchedSteps - kDeepRestart steps from the
+// standard schedule's step kDeepRestart) and then standard rounds; any other matrix takes
+// standard rounds.  True when `steps` quintic steps end a round; *lo is then the lower end
+// of the design interval that round started from.
+__device__ __forceinline__ bool round_end(bool deep, int steps, float* lo) {
+    if (steps <= 0) return false;
+    if (!deep) {
+        *lo = kSchedLo[0];
+        return steps % kSchedSteps == 0;
+    }
+    const int restart_end = kSchedDeepSteps + kSchedSteps - kDeepRestart;
+    if (steps == kSchedDeepSteps) {
+        *lo = kSchedDeepLo[0];
+        return true;
+    }
+    if (steps == restart_end) {
+        *lo = kSchedLo[kDeepRestart];
+        return true;
+    }
+    *lo = kSchedLo[0];
+    return steps > restart_end && (steps - restart_end) % kSchedSteps == 0;
+}
 __device__ __forceinline__ const float* sched_row(bool deep, int step) {
     if (!deep) return kSched[step % kSchedSteps];
     if (step < kSchedDeepSteps) return kSchedDeep[step];
@@ -235,6 +274,16 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
         st.final_buf = 2;
         return;
     }
+    // partial-isometry test at the end of a round (see kZeroFloor)
+    const float lift = st.lift, lift_round = st.lift_round;
+    float round_lo = 1.f;
+    const bool at_round_end = round_end(md.deep != 0, st_step, &round_lo);
+    bool partial = false;
+    if (t > 0 && !fast_steps && at_round_end && lift_round * kZeroFloor >= round_lo) {
+        const float rho = rintf(trf);
+        const float ext = static_cast<float>(md.n) - rho;  // directions taken as zero
+        if (rho >= 1.f && ext >= 1.f) partial = (devf - ext) / rho < tol * tol;
+    }
     if (fast_steps) {
         // fast variant: a fixed number of standard quintic steps, no test, no polish (steps
         // after the schedule's last repeat it); the last one leaves Q in the buffer its
@@ -250,8 +299,8 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
             st.done = 1;
             st.final_buf = (t + 1) & 1;
         }
-    } else if (d < tol) {
-        // Cubic polish p(x) = 1.5 x - 0.5 x^3 on singular values already near 1.
+    } else if (d < tol || partial) {
+        // Cubic polish p(x) = 1.5 x - 0.5 x^3 on singular values already near 1 (or 0).
         st.mode = 2;
         st.a = 1.5f;
         st.b = static_cast<float>(-0.5 * gscale);
@@ -268,6 +317,8 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
     } else {
         const float* q = sched_row(md.deep != 0, st_step);
         st.mode = 1;
+        if (st_step == 0 || at_round_end) st.lift_round = lift;  // this step starts a round
+        st.lift = lift * q[0];
         st.a = q[0];
         st.b = static_cast<float>(q[1] * gscale);
         st.c = static_cast<float>(q[2] * gscale * gscale);
@@ -460,6 +511,8 @@ __global__ void k_reset_state(MatState* state, int nmat, uint32_t* err, const Ma
     s.final_buf = 2;
     s.yb = s.yc = 0.f;
     s.status = 0;
+    s.lift = 1.f;
+    s.lift_round = 1.f;
     s.trace = 0.0;
     state[i] = s;
 }

@@ -121,6 +121,9 @@ struct MatState {
     int final_buf;    // ping-pong buffer holding Q (0/1), or 2 when Q = 0
     float yb, yc;     // Y = yb I + yc G for the quintic step the next Gram leads to
     int status;       // 0, or kErrNotConverged
+    float lift;       // product of the linear coefficients of the steps taken: the factor
+                      // by which a singular value near 0 (relative to the normalisation) has grown
+    float lift_round; // lift when the current round of the schedule started
     double trace;     // tr(Q^T Delta)
 };
 

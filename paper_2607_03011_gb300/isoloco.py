@@ -47,7 +47,8 @@ class Opts(ctypes.Structure):
                 ("reduce_mean", ctypes.c_int), ("max_iter", ctypes.c_int), ("tol", ctypes.c_float),
                 ("sync", ctypes.c_int), ("fast_steps", ctypes.c_int), ("orth_target", ctypes.c_int),
                 ("momentum_kind", ctypes.c_int), ("scale_kind", ctypes.c_int), ("aggregator", ctypes.c_int),
-                ("sparsity", ctypes.c_float), ("seed", ctypes.c_uint), ("spectrum_kind", ctypes.c_int)]
+                ("sparsity", ctypes.c_float), ("seed", ctypes.c_uint), ("spectrum_kind", ctypes.c_int),
+                ("full_precision", ctypes.c_int)]
 
 
 _lib = None
@@ -111,11 +112,12 @@ def _stream(stream=None) -> int:
 
 def make_opts(alpha=1.0, outer_lr=0.7, momentum=0.9, reduce_mean=True, max_iter=0, tol=0.0,
               sync=False, fast_steps=0, orth_target=0, momentum_kind=0, scale_kind=0, aggregator=0,
-              sparsity=0.0, seed=0, spectrum_kind=0) -> Opts:
+              sparsity=0.0, seed=0, spectrum_kind=0, full_precision=0) -> Opts:
     """Options of an outer step; fast_steps > 0 selects the fixed-step variant of Sec. 4.3,
     orth_target / momentum_kind / scale_kind / spectrum_kind (1 clip_high, 2 clip_low) the
     ablations of Sec. 4.5 / App. B, and aggregator / sparsity / seed the merging rule of
-    diloco_outer_step (Sec. 3.2: 0 mean, 1 TIES, 2 DARE); see include/isoloco.h."""
+    diloco_outer_step (Sec. 3.2: 0 mean, 1 TIES, 2 DARE); full_precision = 1 splits both
+    operands of every polar step; see include/isoloco.h."""
     o = Opts()
     lib().isoloco_opts_default(ctypes.byref(o))
     o.alpha, o.outer_lr, o.momentum = float(alpha), float(outer_lr), float(momentum)
@@ -124,6 +126,7 @@ def make_opts(alpha=1.0, outer_lr=0.7, momentum=0.9, reduce_mean=True, max_iter=
     o.orth_target, o.momentum_kind, o.scale_kind = int(orth_target), int(momentum_kind), int(scale_kind)
     o.aggregator, o.sparsity, o.seed = int(aggregator), float(sparsity), int(seed) & 0xFFFFFFFF
     o.spectrum_kind = int(spectrum_kind)
+    o.full_precision = int(full_precision)
     return o
 
 

@@ -134,6 +134,73 @@ def test_zero_pseudo_gradient(iso):
     assert diag["sigma_bar"] == [0.0]
 
 
+def _zero_region(reps, theta, off, rows, cols, r0, r1, c0, c1):
+    """Makes Delta_k = theta - theta_k exactly 0 on rows [r0, r1) x cols [c0, c1) of the
+    matrix at `off`, for every worker k."""
+    th = theta[off:off + rows * cols].view(rows, cols)
+    for k in range(reps.shape[0]):
+        reps[k, off:off + rows * cols].view(rows, cols)[r0:r1, c0:c1] = th[r0:r1, c0:c1].to(reps.dtype)
+
+
+def _rank_deficient_case(iso, shapes, zeros, seed, **opts):
+    """Runs a workload whose pseudo-gradients are exactly zero on the given regions
+    (name -> rows [r0, r1) x cols [c0, c1)); returns (worst, per-matrix error, diag)."""
+    spec = W.custom_spec(shapes, K=2, rank=4, momentum_std=1e-4)
+    wl = W.make_workload(spec, seed=seed, device="cuda")
+    # a copy with the generator's row padding (every replica 16-byte aligned)
+    npad = (wl.N + 63) // 64 * 64
+    reps = torch.empty((wl.K, npad), dtype=wl.replicas.dtype, device="cuda")[:, :wl.N]
+    reps.copy_(wl.replicas)
+    t = {name: wl.table[i] for i, (name, _, _) in enumerate(shapes)}
+    for name, (r0, r1, c0, c1) in zeros.items():
+        o, r, c = t[name]
+        _zero_region(reps, wl.theta, o, r, c, r0, r1, c0, c1)
+    rc, th, b, upd, diag, _ = run_gpu(iso, wl, 1.0, 0.7, 0.9, reps=reps, **opts)
+    assert rc == 0, iso.STATUS_NAMES.get(rc, rc)
+    assert all(s == 0 for s in diag["status"])
+    worst, ref = compare(wl, rc, th, b, upd, diag, 1.0, 0.7, 0.9, reps=reps)
+    # the output is the partial isometry: exactly rho singular values, all alpha * sigma_bar
+    u = upd.double().cpu().numpy()
+    mats = [n for n, _, cc in shapes if cc > 0]
+    for name, (r0, r1, c0, c1) in zeros.items():
+        o, r, c = t[name]
+        rank = min(r - (r1 - r0) if (c0, c1) == (0, c) else r, c - (c1 - c0) if (r0, r1) == (0, r) else c)
+        sv = np.linalg.svd(u[o:o + r * c].reshape(r, c), compute_uv=False)
+        assert np.all(np.abs(sv[:rank] / diag["sigma_bar"][mats.index(name)] - 1.0) < 5e-3), name
+        assert np.all(sv[rank:] < 1e-6 * sv[0]), name
+    return worst, diag
+
+
+def test_rank_deficient_partial_isometry(iso):
+    """Exactly rank-deficient pseudo-gradients (Alg. 2 / reading C3: Iso-C returns the
+    partial isometry U_rho V_rho^T), with status OK.  The zeros are structural, as for
+    embedding rows or input features that no worker's data touched, so the deficiency is
+    exact on both sides.  Default precision where the zero lines lie on the side the Gram
+    is formed over (columns of a tall or square matrix, rows of a wide one: they stay
+    exactly zero), or are few: a tall matrix with 24 of 64 columns zero, a wide one with
+    24 of 64 rows zero, 1024 x 1024 ones with 24 zero columns and with 24 zero rows (deep
+    schedule), beside a full-rank matrix and a vector."""
+    shapes = [("c40", 192, 64), ("wr", 64, 128), ("sqc", 1024, 1024), ("sq24", 1024, 1024), ("full", 96, 80),
+              ("v", 33, 0)]
+    zeros = {"c40": (0, 192, 40, 64), "wr": (40, 64, 0, 128), "sqc": (0, 1024, 1000, 1024),
+             "sq24": (1000, 1024, 0, 1024)}
+    worst, diag = _rank_deficient_case(iso, shapes, zeros, seed=21)
+    print("rank-deficient (default precision) worst errors", worst, "iterations", diag["iters"])
+
+
+def test_rank_deficient_many_zero_rows_full_precision(iso):
+    """Zero lines on the long side in large numbers (a tall matrix with 5 nonzero rows, a
+    wide one with 7 nonzero columns, a 1024 x 1024 one with 512 zero rows): with the
+    two-pass steps the 11-bit operand turns the iterate's row space toward the zero
+    directions (~2^-11 per step, up to ~1e-2 here), so these take full_precision = 1 (every
+    step three passes), which meets the Iso-C tolerance."""
+    shapes = [("r5", 128, 64), ("w7", 64, 128), ("sq512", 1024, 1024), ("c40", 192, 64), ("v", 17, 0)]
+    zeros = {"r5": (5, 128, 0, 64), "w7": (0, 64, 7, 128), "sq512": (512, 1024, 0, 1024),
+             "c40": (0, 192, 40, 64)}
+    worst, diag = _rank_deficient_case(iso, shapes, zeros, seed=22, full_precision=1)
+    print("rank-deficient (full precision) worst errors", worst, "iterations", diag["iters"])
+
+
 def test_nonfinite_leaves_state_untouched(iso):
     spec = W.custom_spec([("m", 64, 48), ("v", 16, 0)], K=2, momentum_std=1e-3)
     wl = W.make_workload(spec, seed=1, device="cuda")
@@ -395,13 +462,49 @@ def sampled_parity(iso, workload, pick_names, fast_steps=0, **ablation):
     torch.cuda.empty_cache()
 
 
-def test_llama_180m_k8_sampled(iso):
-    """The benchmarked configuration (180M shapes, K = 8): one matrix of each shape bucket."""
-    sampled_parity(iso, "llama_180m_k8", ("layers.0.wq", "layers.5.w_gate", "layers.11.w_down", "head"))
+def test_llama_180m_k8_every_matrix(iso):
+    """The benchmarked configuration (180M shapes, K = 8) in the launch configuration the
+    bench times, checked against the oracle on every tensor: all 86 matrices (including the
+    1024 x 1024 ones that need the most polar iterations) and every vector."""
+    wl = W.make_workload("llama_180m_k8", seed=0, device="cuda")
+    sp = wl.spec
+    rc, th, b, upd, diag, plan = run_gpu(iso, wl, sp.alpha, sp.outer_lr, sp.momentum)
+    assert rc == 0
+    assert all(s == 0 for s in diag["status"])
+    ref = oracle.isoloco_outer_step(wl.table, wl.theta.cpu().numpy(), wl.momentum.cpu().numpy(),
+                                    W.replicas_as_numpy(wl.replicas), alpha=sp.alpha, eta=sp.outer_lr,
+                                    mu=sp.momentum)
+    ref["theta_in"] = wl.theta.double().cpu().numpy()
+    u = upd.double().cpu().numpy()
+    worst = check_step(wl.table, th.double().cpu().numpy(), b.double().cpu().numpy(), u, diag["sigma_bar"], ref)
+    rows, mi = [], 0
+    for pi, (o, r, c) in enumerate(wl.table):
+        if not c:
+            continue
+        sl = slice(o, o + r * c)
+        rows.append((rel_fro(u[sl], ref["update"][sl]), sp.shapes[pi][0], f"{r}x{c}", diag["iters"][mi]))
+        mi += 1
+    assert len(rows) == 86
+    rows.sort(reverse=True)
+    print("180M K=8, all 86 matrices: worst", worst)
+    for e, name, shape, it in rows[:8]:
+        print(f"  {name:18s} {shape:10s} iterations {it:2d}  Iso-C rel. Frobenius error {e:.3e}")
+    # the matrices that need a second schedule round are among those checked
+    slow = [x for x in rows if x[3] > 12]
+    print("  matrices with more than 12 iterations:", [(x[1], x[3], f"{x[0]:.2e}") for x in slow])
+    assert slow, "expected some 1024 x 1024 matrices to need a second schedule round"
+    del wl, th, b, upd, plan
+    torch.cuda.empty_cache()
+
+
+def test_llama_180m_k16_every_square(iso):
+    """180M shapes with K = 16: every 1024 x 1024 matrix (the ill-conditioned bucket) and
+    one matrix of each other shape, plus every vector."""
+    names = [s[0] for s in W.SPECS["llama_180m_k16"].shapes if s[1] == s[2]]
+    sampled_parity(iso, "llama_180m_k16", tuple(names) + ("layers.7.w_up", "layers.0.w_down", "embed"))
 
 
 @pytest.mark.parametrize("workload,pick", [
-    ("llama_180m_k16", ("layers.3.wk", "layers.7.w_up", "layers.0.w_down")),
     ("llama_1b_k8", ("layers.0.wq", "layers.11.w_gate", "layers.23.w_down")),
     ("llama_3b_k4", ("layers.0.wv",)),   # bf16 replicas; 3072-wide matrices keep the oracle sample small
 ])
