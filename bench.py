@@ -174,11 +174,20 @@ def _sym_tiles(n):
     return c
 
 
-def gemm_exec_flops(table, diag, fast=False, full=False):
+# The library's default precision schedule (the quintic steps whose GEMMs run one pass),
+# as the library defines it: per schedule kind, [from, to) for the Gram and polynomial and
+# for the update.  Standard schedule: rectangular matrices; deep: near-square ones.
+DEFAULT_SCHEDULE = {"std": {"gp": (1, 6), "upd": (2, 6)}, "deep": {"gp": (9, 11), "upd": (10, 11)}}
+NO_DEMOTION = {"std": {"gp": (0, 0), "upd": (0, 0)}, "deep": {"gp": (0, 0), "upd": (0, 0)}}
+
+
+def gemm_exec_flops(table, diag, fast=False, full=False, sched=None):
     """Tensor-core FLOPs the GEMM launches execute per phase: 2*BM*BN*K_padded per
-    computed tile and per 16-bit pass (3 passes at iteration 0 and in the final polish
-    update, 2 elsewhere; 3 everywhere with `full`, the clip variants' main iteration),
-    symmetric Grams/G^2 on their upper-triangle tiles only."""
+    computed tile and per 16-bit pass, symmetric Grams/G^2 on their upper-triangle tiles
+    only.  Passes: 3 at iteration 0 and in the polish update; elsewhere 2, or 1 for the
+    steps the precision schedule `sched` (default: the library's) runs single-pass; 3
+    everywhere with `full` (full precision, the clip variants) and in the fast variant."""
+    sched = DEFAULT_SCHEDULE if sched is None else sched
     out = {"gram": 0.0, "poly": 0.0, "update": 0.0}
     mats = [(r, c) for (_, r, c) in table if c > 0]
     for (r, c), it, st in zip(mats, diag["iters"], diag["status"]):
@@ -195,16 +204,22 @@ def gemm_exec_flops(table, diag, fast=False, full=False):
         if it == 0:
             out["gram"] += 3 * gram1
             continue
+        kind = sched["deep" if abs(r - c) * 16 < n else "std"]
         converged = (st == 0)
-        grams = it + (0 if converged else 1)
-        quintic = it - (1 if converged else 0)
-        p = 3 if full else 2   # passes after iteration 0
-        out["gram"] += 3 * gram1 + p * gram1 * (grams - 1)
-        out["poly"] += (3 * poly1 + p * poly1 * (quintic - 1)) if quintic >= 1 else 0.0
+        quintic = it - (1 if converged else 0)   # steps 0 .. quintic - 1, then the polish
+
+        def passes(k, rng):
+            if k == 0 or full:
+                return 3
+            return 1 if rng[0] <= k < rng[1] else 2
+        # the Gram of iteration t leads to step t (t quintic steps taken before it)
+        for t in range(it + (0 if converged else 1)):
+            out["gram"] += passes(t, kind["gp"]) * gram1
+        for k in range(quintic):
+            out["poly"] += passes(k, kind["gp"]) * poly1
+            out["update"] += passes(k, kind["upd"]) * upd1
         if converged:
-            out["update"] += 3 * upd1 * (1 if it == 1 else 2) + p * upd1 * max(0, it - 2)
-        else:
-            out["update"] += 3 * upd1 + p * upd1 * (it - 1)
+            out["update"] += 3 * upd1          # the polish
     return out
 
 

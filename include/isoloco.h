@@ -126,6 +126,14 @@ typedef struct {
                          * square one), the 11-bit operand turns the iterate's row space toward
                          * the zero directions by ~2^-11 per step; 1 keeps the result within
                          * the Iso-C tolerance there. */
+    long long precision_schedule; /* which quintic polar steps run a single 16-bit pass instead of
+                         * two (full_precision = 0 only).  0: the library's default schedule;
+                         * -1: none.  Otherwise eight 5-bit step indices, field i at bits
+                         * 5i .. 5i + 4: [f0, f1) the steps whose Gram and polynomial GEMMs and
+                         * [f2, f3) those whose update runs one pass, for the standard schedule
+                         * (rectangular matrices); f4 .. f7 the same for the deep schedule
+                         * (near-square ones).  Step k is the matrix's k-th quintic step
+                         * (0-based); the polish and iteration 0's GEMMs keep their passes. */
 } isoloco_opts_t;
 
 /* Fills *opts with alpha = 1, outer_lr = 0.7, momentum = 0.9 (the paper's DiLoCo

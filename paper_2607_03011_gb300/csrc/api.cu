@@ -156,6 +156,12 @@ struct isoloco_plan {
     float g_tol = 0.f;
     int g_fast = -1;
     int g_full = -1;
+    long long g_prec = -2;
+    // precision schedule of this call (isoloco_opts_t::precision_schedule, decoded): per
+    // schedule kind (0 standard, 1 deep) the quintic steps [from, to) whose Gram and
+    // polynomial, and those whose update, run a single pass
+    long long prec_code = 0;
+    int gp_from[2] = {0, 0}, gp_to[2] = {0, 0}, up_from[2] = {0, 0}, up_to[2] = {0, 0};
     bool per_launch = false;        // polar iterations as plain launches (no graph), with early stop
     bool full_prec = false;         // every polar step with three passes and no Horner form
                                     // (the clip variants' sign iteration)
@@ -678,6 +684,40 @@ static int flush_set(isoloco_plan* pl, int phase, LaunchSet& s, cudaStream_t st)
     return ISOLOCO_OK;
 }
 
+// The library's default precision schedule (isoloco_opts_t::precision_schedule = 0), chosen
+// by measuring each bucket's Iso-C error against the oracle at 180M K = 8 (every matrix):
+// standard schedule (steps 0 .. 5 quintic): Gram and polynomial of steps 1 .. 5 and the
+// update of steps 2 .. 5 single-pass; deep schedule (0 .. 10): Gram and polynomial of steps
+// 9, 10 and the update of step 10.  Symmetric (Gram, polynomial) roundings only perturb the
+// spectrum, which later steps correct; a single-pass update rounds X itself, which turns
+// singular vectors for good, so it is kept to the steps where the singular values are
+// already clustered near 1.
+constexpr long long kDefaultPrecisionSchedule =
+    (1ll << 0) | (6ll << 5) | (2ll << 10) | (6ll << 15) | (9ll << 20) | (11ll << 25) | (10ll << 30) | (11ll << 35);
+
+// Decodes a precision schedule code into the plan's per-kind step ranges.
+static void set_precision_schedule(isoloco_plan* p, long long code) {
+    if (code == 0) code = kDefaultPrecisionSchedule;
+    for (int kind = 0; kind < 2; ++kind) {
+        int f[4] = {0, 0, 0, 0};
+        if (code > 0)
+            for (int i = 0; i < 4; ++i) f[i] = static_cast<int>((code >> (5 * (4 * kind + i))) & 31);
+        p->gp_from[kind] = f[0];
+        p->gp_to[kind] = f[1];
+        p->up_from[kind] = f[2];
+        p->up_to[kind] = f[3];
+    }
+    p->prec_code = code;
+}
+
+// Single-pass step range of a group (precision schedule; none in the full-precision paths).
+static void set_one_pass(const isoloco_plan* p, GemmGroup& g, const Bucket& bk, bool update) {
+    const int kind = (std::abs(bk.rows - bk.cols) * 16 < bk.n) ? 1 : 0;  // deep schedule (as MatDesc::deep)
+    const bool full = p->fast_steps > 0 || p->full_prec;
+    g.one_from = full ? 0 : (update ? p->up_from[kind] : p->gp_from[kind]);
+    g.one_to = full ? 0 : (update ? p->up_to[kind] : p->gp_to[kind]);
+}
+
 // Iteration t of the polar loop for every matrix still active: Gram, convergence test
 // and choice of the step (k_control), polynomial, update.  With set_cond, k_control also
 // sets the graph condition `cond` (graph body only).
@@ -729,6 +769,7 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
             g.part = p->fin_part;
             g.part_base = p->mats_h[bk.mat_base].gpart_slot;
             set_sym(g, bk.n);
+            set_one_pass(p, g, bk, false);
             gram.add(g, bk.tall, bk.tall);
         }
         int rc;
@@ -770,6 +811,7 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
             g.g_hi = p->ghi + bk.gplane_off;
             g.g_lo = p->glo + bk.gplane_off;
             set_sym(g, bk.n);
+            set_one_pass(p, g, bk, false);
             poly.add(g, false, false);
         }
         if ((rc = flush_set(p, ISOLOCO_PHASE_POLY, poly, st))) return rc;
@@ -804,6 +846,7 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
             g.st_lo = m + st_map(dst, 1);
             g.bf_batch_stride = (int64_t)bk.rows * bk.ld;
             g.ld_bf = bk.ld;
+            set_one_pass(p, g, bk, true);
             if (bk.tall)
                 upd.add(g, false, false, true, p_split);
             else
@@ -872,6 +915,7 @@ static int build_polar_graph(isoloco_plan* p, int max_iter, float tol) {
     p->g_tol = tol;
     p->g_fast = p->fast_steps;
     p->g_full = p->full_prec ? 1 : 0;
+    p->g_prec = p->prec_code;
     return ISOLOCO_OK;
 }
 
@@ -889,7 +933,7 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
     const bool use_graph = kPairMma && !p->prof && !p->per_launch && cs == cudaStreamCaptureStatusNone;
     if (use_graph) {
         if (!p->gexec || p->g_max_iter != max_iter || p->g_tol != tol || p->g_fast != p->fast_steps ||
-            p->g_full != (p->full_prec ? 1 : 0))
+            p->g_full != (p->full_prec ? 1 : 0) || p->g_prec != p->prec_code)
             if ((rc = build_polar_graph(p, max_iter, tol))) return rc;
         CUDA_TRY(cudaGraphLaunch(p->gexec, st));
     } else {
@@ -1172,6 +1216,8 @@ static int check_opts(const isoloco_opts_t* o, isoloco_opts_t* out) {
         return fail(ISOLOCO_ERR_INVALID, "spectrum_kind must be 0, 1 or 2");
     if (out->full_precision < 0 || out->full_precision > 1)
         return fail(ISOLOCO_ERR_INVALID, "full_precision must be 0 or 1");
+    if (out->precision_schedule < -1 || out->precision_schedule >= (1ll << 40))
+        return fail(ISOLOCO_ERR_INVALID, "precision_schedule must be -1, 0 or a 40-bit code");
     if (out->spectrum_kind && (out->fast_steps || out->scale_kind))
         return fail(ISOLOCO_ERR_INVALID, "clip_high / clip_low need the exact polar path and sigma_bar "
                                          "(fast_steps = 0, scale_kind = 0)");
@@ -1242,6 +1288,7 @@ static int run_isoc_step(isoloco_plan* p, int merge, float* theta, float* mom, c
     }
     p->fast_steps = merge ? 0 : o.fast_steps;
     p->full_prec = !merge && (o.spectrum_kind != 0 || o.full_precision != 0);
+    set_precision_schedule(p, merge ? -1 : o.precision_schedule);
     p->skip_trace = !merge && (o.fast_steps > 0 || o.scale_kind == 1);
     if ((rc = run_polar(p, p->fast_steps ? std::max(o.max_iter, o.fast_steps) : o.max_iter, o.tol, st))) return rc;
     const int clip = merge ? 0 : o.spectrum_kind;
@@ -1290,6 +1337,7 @@ int isoloco_opts_default(isoloco_opts_t* o) {
     o->seed = 0u;
     o->spectrum_kind = 0;
     o->full_precision = 0;
+    o->precision_schedule = 0;
     return ISOLOCO_OK;
 }
 

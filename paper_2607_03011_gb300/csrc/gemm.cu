@@ -137,6 +137,11 @@ __device__ __forceinline__ bool decode_tile(const GemmParams& p, const int* pre,
             ti.horner = (p.epi == kEpiPoly && p.poly_horner && st.mode == 1);
             if (p.split_on_polish && st.mode == 2) ti.a_split = ti.b_split = true;  // final step: 3 passes
         }
+        // precision schedule: single-pass steps (a Gram only after iteration 0's)
+        const int k = (p.epi == kEpiGram) ? st.step : st.step - 1;
+        if (k >= g.one_from && k < g.one_to &&
+            ((p.epi == kEpiGram) ? st.step > 0 : st.mode == 1))
+            ti.a_split = ti.b_split = false;
         ti.ca = st.a;
         ti.cb = st.b;
         ti.cc = st.c;

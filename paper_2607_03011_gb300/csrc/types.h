@@ -87,6 +87,10 @@ struct GemmGroup {
     int gate_fb;    // 0: no condition; f > 0: only matrices whose Q is in buffer f - 1 (final_buf)
     int a_mn, b_mn; // operand layout: 1 MN-major (M or N index contiguous), 0 K-major
     int a_split, b_split;  // operand carries a lo plane in this group (one tensor pass each)
+    // quintic steps whose index k lies in [one_from, one_to) run a single pass (no lo planes);
+    // k = the matrix's step count for a Gram (the step it leads to), the step count - 1 for
+    // the polynomial and the update (the step they form)
+    int one_from, one_to;
     // fp32 output (kEpiF32): out_f32 + split*split_stride + b*batch_stride + row*ld + col
     float* out_f32;
     int64_t f32_split_stride, f32_batch_stride;

@@ -48,7 +48,7 @@ class Opts(ctypes.Structure):
                 ("sync", ctypes.c_int), ("fast_steps", ctypes.c_int), ("orth_target", ctypes.c_int),
                 ("momentum_kind", ctypes.c_int), ("scale_kind", ctypes.c_int), ("aggregator", ctypes.c_int),
                 ("sparsity", ctypes.c_float), ("seed", ctypes.c_uint), ("spectrum_kind", ctypes.c_int),
-                ("full_precision", ctypes.c_int)]
+                ("full_precision", ctypes.c_int), ("precision_schedule", ctypes.c_longlong)]
 
 
 _lib = None
@@ -112,7 +112,7 @@ def _stream(stream=None) -> int:
 
 def make_opts(alpha=1.0, outer_lr=0.7, momentum=0.9, reduce_mean=True, max_iter=0, tol=0.0,
               sync=False, fast_steps=0, orth_target=0, momentum_kind=0, scale_kind=0, aggregator=0,
-              sparsity=0.0, seed=0, spectrum_kind=0, full_precision=0) -> Opts:
+              sparsity=0.0, seed=0, spectrum_kind=0, full_precision=0, precision_schedule=0) -> Opts:
     """Options of an outer step; fast_steps > 0 selects the fixed-step variant of Sec. 4.3,
     orth_target / momentum_kind / scale_kind / spectrum_kind (1 clip_high, 2 clip_low) the
     ablations of Sec. 4.5 / App. B, and aggregator / sparsity / seed the merging rule of
@@ -127,7 +127,17 @@ def make_opts(alpha=1.0, outer_lr=0.7, momentum=0.9, reduce_mean=True, max_iter=
     o.aggregator, o.sparsity, o.seed = int(aggregator), float(sparsity), int(seed) & 0xFFFFFFFF
     o.spectrum_kind = int(spectrum_kind)
     o.full_precision = int(full_precision)
+    o.precision_schedule = int(precision_schedule)
     return o
+
+
+def precision_code(std_gp=(0, 0), std_upd=(0, 0), deep_gp=(0, 0), deep_upd=(0, 0)) -> int:
+    """Packs a precision schedule (isoloco_opts_t::precision_schedule): per schedule kind,
+    the quintic step ranges [from, to) whose Gram and polynomial, and whose update, run one
+    pass."""
+    f = list(std_gp) + list(std_upd) + list(deep_gp) + list(deep_upd)
+    assert all(0 <= v < 32 for v in f)
+    return sum(v << (5 * i) for i, v in enumerate(f))
 
 
 def _ptr_array(tensors) -> ctypes.Array:

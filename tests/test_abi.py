@@ -93,4 +93,4 @@ def test_opts_layout_matches_the_header(tmp_path, lib):
     o = isoloco.Opts()
     assert lib.isoloco_opts_default(ctypes.byref(o)) == 0
     assert (o.fast_steps, o.orth_target, o.momentum_kind, o.scale_kind, o.aggregator, o.sparsity, o.seed,
-            o.spectrum_kind, o.full_precision) == (0, 0, 0, 0, 0, 0.0, 0, 0, 0)
+            o.spectrum_kind, o.full_precision, o.precision_schedule) == (0, 0, 0, 0, 0, 0.0, 0, 0, 0, 0)

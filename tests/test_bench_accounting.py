@@ -58,8 +58,14 @@ def test_executed_flops_square():
     Iteration 0 and the polish update take three passes, the rest two; with `full` three."""
     g1 = 10 * 256 * 256 * 2.0 * 1024
     u1 = 16 * 256 * 256 * 2.0 * 1024
-    fx = bench.gemm_exec_flops([("w", 1024, 1024)], _diag([12]))
+    fx = bench.gemm_exec_flops([("w", 1024, 1024)], _diag([12]), sched=bench.NO_DEMOTION)
     assert fx == {"gram": (3 + 2 * 11) * g1, "poly": (3 + 2 * 10) * g1, "update": (3 + 3 + 2 * 10) * u1}
+    # the default schedule: a 1024 x 1024 matrix is near-square (deep schedule, quintic steps
+    # 0 .. 10): Grams leading to steps 9, 10 and G^2 of steps 9, 10 single-pass, the update of
+    # step 10 too
+    fx = bench.gemm_exec_flops([("w", 1024, 1024)], _diag([12]))
+    assert fx == {"gram": (3 + 2 * 9 + 1 * 2) * g1, "poly": (3 + 2 * 8 + 1 * 2) * g1,
+                  "update": (3 + 2 * 9 + 1 + 3) * u1}
     fx = bench.gemm_exec_flops([("w", 1024, 1024)], _diag([12]), full=True)
     assert fx == {"gram": 36 * g1, "poly": 33 * g1, "update": 36 * u1}
     fx = bench.gemm_exec_flops([("w", 1024, 1024)], _diag([5]), fast=True)
@@ -75,8 +81,34 @@ def test_executed_flops_ragged_padding():
     fx = bench.gemm_exec_flops([("w", 300, 257)], _diag([1]))
     # one iteration: iteration 0 is also the polish (three passes, no G^2)
     assert fx == {"gram": 3 * g1, "poly": 0.0, "update": 3 * u1}
-    fx = bench.gemm_exec_flops([("w", 300, 257)], _diag([2]))
+    fx = bench.gemm_exec_flops([("w", 300, 257)], _diag([2]), sched=bench.NO_DEMOTION)
     assert fx == {"gram": (3 + 2) * g1, "poly": 3 * p1, "update": 6 * u1}
+    # default schedule (standard kind): the Gram of iteration 1 leads to step 1, single-pass
+    fx = bench.gemm_exec_flops([("w", 300, 257)], _diag([2]))
+    assert fx == {"gram": (3 + 1) * g1, "poly": 3 * p1, "update": 6 * u1}
+
+
+def test_executed_flops_standard_schedule_default():
+    """2816 x 1024 (standard schedule), 7 iterations: quintic steps 0 .. 5, polish at 6.
+    Grams leading to steps 1 .. 5 and G^2 of steps 1 .. 5 single-pass (the Gram before the
+    polish keeps two), updates of steps 2 .. 5 single-pass, step 1's two, the polish three."""
+    n, m = 1024, 2816
+    kp = 2816  # 2816 = 44 k-blocks of 64
+    g1 = 10 * 256 * 256 * 2.0 * kp
+    p1 = 10 * 256 * 256 * 2.0 * 1024
+    u1 = 11 * 4 * 256 * 256 * 2.0 * 1024
+    fx = bench.gemm_exec_flops([("w", m, n)], _diag([7]))
+    assert fx == {"gram": (3 + 5 * 1 + 2) * g1, "poly": (3 + 5 * 1) * p1, "update": (3 + 2 + 4 * 1 + 3) * u1}
+
+
+def test_default_schedule_matches_the_library():
+    """bench's mirror of the default precision schedule is the library's constant."""
+    src = open(os.path.join(ROOT, "paper_2607_03011_gb300", "csrc", "api.cu")).read()
+    body = src.split("constexpr long long kDefaultPrecisionSchedule =")[1].split(";")[0]
+    fields = [int(v) for v, _ in re.findall(r"\((\d+)ll << (\d+)\)", body)]
+    d = bench.DEFAULT_SCHEDULE
+    assert fields == [d["std"]["gp"][0], d["std"]["gp"][1], d["std"]["upd"][0], d["std"]["upd"][1],
+                      d["deep"]["gp"][0], d["deep"]["gp"][1], d["deep"]["upd"][0], d["deep"]["upd"][1]]
 
 
 def test_stream_bytes():
