@@ -186,7 +186,10 @@ def gemm_exec_flops(table, diag, fast=False, full=False, sched=None):
     computed tile and per 16-bit pass, symmetric Grams/G^2 on their upper-triangle tiles
     only.  Passes: 3 at iteration 0 and in the polish update; elsewhere 2, or 1 for the
     steps the precision schedule `sched` (default: the library's) runs single-pass; 3
-    everywhere with `full` (full precision, the clip variants) and in the fast variant."""
+    everywhere with `full` (full precision, the clip variants) and in the fast variant.
+    A Gram in the single-pass range runs one pass only while the matrix's previous residual
+    is large (the library's rule); this count takes every such Gram as single-pass, a lower
+    bound on the executed FLOPs."""
     sched = DEFAULT_SCHEDULE if sched is None else sched
     out = {"gram": 0.0, "poly": 0.0, "update": 0.0}
     mats = [(r, c) for (_, r, c) in table if c > 0]
@@ -480,9 +483,10 @@ def main():
                     help="iso_c: the IsoLoCo step (Alg. 2, default); mean / ties / dare: the DiLoCo step "
                          "(Alg. 1) with that merging rule (Sec. 3.2)")
     ap.add_argument("--sparsity", type=float, default=0.1, help="TIES / DARE sparsity (0.1: Sec. 5.1's best)")
-    ap.add_argument("--spectrum", default="iso_c", choices=["iso_c", "clip_high", "clip_low"],
+    ap.add_argument("--spectrum", default="iso_c", choices=["iso_c", "clip_high", "clip_low", "svd"],
                     help="the IsoLoCo step's spectrum map (Sec. 4.5): every singular value to the mean (Iso-C), "
-                         "or only those above (clip_high) / below (clip_low) it")
+                         "or only those above (clip_high) / below (clip_low) it; svd: Iso-C with every singular "
+                         "value computed (Alg. 2's SVD form)")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     if args.impl == "reference":
@@ -511,7 +515,7 @@ def main():
     plan = isoloco.Plan(wl.table, wl.N, wl.K, wl.replicas.dtype)
     if args.aggregator != "iso_c":
         return run_diloco(args, torch, isoloco, wl, plan, world, rank, local, dist, barrier)
-    spectrum_kind = {"iso_c": 0, "clip_high": 1, "clip_low": 2}[args.spectrum]
+    spectrum_kind = {"iso_c": 0, "clip_high": 1, "clip_low": 2, "svd": 3}[args.spectrum]
     opts = isoloco.make_opts(spec.alpha, spec.outer_lr, spec.momentum, fast_steps=args.fast_steps,
                              spectrum_kind=spectrum_kind)
     theta0, mom0 = wl.theta.clone(), wl.momentum.clone()

@@ -115,7 +115,16 @@ typedef struct {
                         * diag(min(s_i, sigma_bar)) V_D^T.  2: clip_low, only those below,
                         * max(s_i, sigma_bar).  1 and 2 need fast_steps = 0 and scale_kind = 0;
                         * their first call allocates an auxiliary plan (the n x n matrices
-                        * H - sigma_bar I, H = Q^T Delta) and its buffers. */
+                        * H - sigma_bar I, H = Q^T Delta) and its buffers.  3: Iso-C from the
+                        * singular values (Alg. 2's SVD form): every sigma_i of every matrix is
+                        * computed, as the eigenvalues of H = Q^T Delta (Delta Q^T when wide;
+                        * Householder tridiagonalization in fp32 and bisection), sigma_bar is
+                        * their mean, and U = alpha sigma_bar Q as for 0 (the polar iteration
+                        * then runs three passes at every step, as for 1 and 2, so that Q's
+                        * singular values are 1 to ~1e-6); the sigma_i are read
+                        * with isoloco_read_singular_values.  Its first call allocates the
+                        * n x n fp32 H of every matrix; the reduction is BLAS-2 bound (about
+                        * n^3 / 3 fp32 elements read and written per matrix). */
     int full_precision; /* 0: the polar steps after the first keep one GEMM operand at 11 bits
                          * (two 16-bit passes; its rounding only perturbs the spectrum of a
                          * full-rank iterate, which later steps correct).  1: every step splits
@@ -204,6 +213,14 @@ int isoloco_last_status(isoloco_plan_t plan, void* stream);
  * only (n_matrices entries each; any pointer may be NULL).  Synchronizes `stream`.
  *   sigma_bar: tr(Q^T Delta) / min(m, n);  iters: polar iterations used;
  *   status: 0 or NOT_CONVERGED;  residual: last ||X^T X - I||_F / sqrt(n). */
+/* Singular values of 2-D tensor `matrix` (table order over the 2-D tensors) from the
+ * plan's last call with spectrum_kind = 3 (Alg. 2: Delta = U S V^T; here sigma_i of the
+ * reduced pseudo-gradient), in descending order, copied to host memory out[0 .. r-1],
+ * r = min(rows, cols) <= capacity.  Synchronizes `stream`.  Returns r, or INVALID (no such
+ * call yet, bad index, buffer too small) or CUDA.  A zero pseudo-gradient gives zeros. */
+int isoloco_read_singular_values(isoloco_plan_t plan, void* stream, int matrix, float* out_host,
+                                 int capacity);
+
 int isoloco_read_diag(isoloco_plan_t plan, void* stream, float* sigma_bar_host,
                       int32_t* iters_host, int32_t* status_host, float* residual_host);
 

@@ -31,7 +31,7 @@ __global__ void k_gram_finalize(const MatDesc*, const int2*, const MatState*, co
                                 __nv_bfloat16*);
 __global__ void k_control(const MatDesc*, int, MatState*, const float*, int, int, float, uint32_t*, const int*,
                           const int*, int, int*, int*, int*, int*, cudaGraphConditionalHandle, int, long long*,
-                          int, int*);
+                          int, int*, int4);
 __global__ void k_trace_partial(const MatDesc*, const int4*, const MatState*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, double*);
@@ -53,6 +53,10 @@ __global__ void k_clip_form_p(const MatDesc*, const MatState*, __nv_bfloat16*, _
 __global__ void k_clip_form_s(const MatDesc*, const MatDesc*, const int*, const MatState*, const __nv_bfloat16*,
                               const __nv_bfloat16*, __nv_bfloat16*, __nv_bfloat16*, const uint32_t*, uint32_t*);
 __global__ void k_clip_flip(MatState*, int);
+__global__ void k_svd_tridiag(const MatDesc*, const MatState*, float*, const int64_t*, const int64_t*, const int*,
+                              float*, const int64_t*);
+__global__ void k_svd_bisect(const MatDesc*, const float*, const int64_t*, float*, const int64_t*);
+__global__ void k_svd_sigma_bar(const MatDesc*, int, MatState*, const float*, const int64_t*);
 __global__ void k_diloco(ReplicaPtrs, int, int, float*, float*, int64_t, float, float, float, uint32_t*);
 __global__ void k_dare(ReplicaPtrs, int, int, float*, float*, int64_t, float, uint32_t, float, unsigned int,
                        uint64_t, float, float, uint32_t*);
@@ -186,6 +190,12 @@ struct isoloco_plan {
     int64_t* hss_d = nullptr;
     int* aux_of_d = nullptr;
     std::vector<int64_t> hbucket_off;
+    // exact singular values (spectrum_kind 3): tridiagonal (d, e) and sigma_i per matrix
+    float* tri = nullptr;
+    int64_t* tri_off_d = nullptr;
+    float* sv = nullptr;
+    int64_t* sv_off_d = nullptr;
+    std::vector<int64_t> sv_off_h;  // by matrix index (plan order)
     // TIES trim (allocated on first use): radix-select histograms [2K][256]; ranks and key
     // prefixes of the sample (2 per worker), candidate and fallback selections; the keys
     // above each bracket; the fallback flag; the sample [K][S]; the candidate segments
@@ -710,6 +720,13 @@ static void set_precision_schedule(isoloco_plan* p, long long code) {
     p->prec_code = code;
 }
 
+// Bound `end` (0 from, 1 to) of the single-pass Gram / polynomial steps of a schedule kind
+// (0 standard, 1 deep); an empty range in the full-precision paths.
+static int gp_one(const isoloco_plan* p, int kind, int end) {
+    if (p->fast_steps > 0 || p->full_prec) return 0;
+    return end ? p->gp_to[kind] : p->gp_from[kind];
+}
+
 // Single-pass step range of a group (precision schedule; none in the full-precision paths).
 static void set_one_pass(const isoloco_plan* p, GemmGroup& g, const Bucket& bk, bool update) {
     const int kind = (std::abs(bk.rows - bk.cols) * 16 < bk.n) ? 1 : 0;  // deep schedule (as MatDesc::deep)
@@ -785,7 +802,8 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
         k_control<<<(p->nmat + kControlThreads / 32 - 1) / (kControlThreads / 32), kControlThreads, 0, st>>>(p->mats_d, p->nmat, p->state, p->fin_part, t, max_iter, tol, p->err_d,
                                       p->bucket_first_d, p->bucket_count_d, (int)p->buckets.size(), p->list_gram,
                                       p->cnt_gram, p->list_step, p->cnt_step, cond, set_cond, p->loopc,
-                                      p->fast_steps, p->counters + kLaunchCounters); }
+                                      p->fast_steps, p->counters + kLaunchCounters,
+                                      make_int4(gp_one(p, 0, 0), gp_one(p, 0, 1), gp_one(p, 1, 0), gp_one(p, 1, 1))); }
         CUDA_TRY(cudaGetLastError());
         // ---- P = a I + b G + c G^2
         LaunchSet poly;
@@ -999,8 +1017,33 @@ static int ensure_ties(isoloco_plan* p, int nseg) {
 // ---------------------------------------------------------------- clip variants (Sec. 4.5)
 // Creates, on first use, the auxiliary plan (one n x n matrix per matrix of the plan, the
 // same n) and the fp32 buffer of H.
+// The fp32 n x n matrices H = Q^T Delta (per split for split-K buckets) and their offsets.
+static int ensure_hbuf(isoloco_plan* p) {
+    if (p->hbuf) return ISOLOCO_OK;
+    std::vector<int64_t> hoff(p->nmat), hss(p->nmat);
+    int64_t hb = 0;
+    p->hbucket_off.clear();
+    for (const Bucket& bk : p->buckets) {
+        const int64_t g = (int64_t)bk.n * bk.ld_n;
+        p->hbucket_off.push_back(hb);
+        for (int j = 0; j < bk.count; ++j) {
+            hoff[bk.mat_base + j] = hb + j * g;
+            hss[bk.mat_base + j] = (int64_t)bk.count * g;
+        }
+        hb += round_up((int64_t)bk.splits * bk.count * g, 128);
+    }
+    int rc;
+    if ((rc = dalloc(p, &p->hbuf, hb)) || (rc = dalloc(p, &p->hoff_d, p->nmat)) || (rc = dalloc(p, &p->hss_d, p->nmat)))
+        return rc;
+    CUDA_TRY(cudaMemcpy(p->hoff_d, hoff.data(), sizeof(int64_t) * p->nmat, cudaMemcpyHostToDevice));
+    CUDA_TRY(cudaMemcpy(p->hss_d, hss.data(), sizeof(int64_t) * p->nmat, cudaMemcpyHostToDevice));
+    return ISOLOCO_OK;
+}
+
 static int ensure_clip(isoloco_plan* p) {
     if (p->aux) return ISOLOCO_OK;
+    int rc0 = ensure_hbuf(p);
+    if (rc0) return rc0;
     std::vector<isoloco_param_t> t(p->nmat);
     int64_t off = 0;
     for (int i = 0; i < p->nmat; ++i) {
@@ -1016,45 +1059,24 @@ static int ensure_clip(isoloco_plan* p) {
     // aux matrix i holds aux parameter aux->mat_param[i], i.e. this plan's matrix of that index
     std::vector<int> aux_of(p->nmat);
     for (int j = 0; j < a->nmat; ++j) aux_of[a->mat_param[j]] = j;
-    std::vector<int64_t> hoff(p->nmat), hss(p->nmat);
-    int64_t hb = 0;
-    p->hbucket_off.clear();
-    for (const Bucket& bk : p->buckets) {
-        const int64_t g = (int64_t)bk.n * bk.ld_n;
-        p->hbucket_off.push_back(hb);
-        for (int j = 0; j < bk.count; ++j) {
-            hoff[bk.mat_base + j] = hb + j * g;
-            hss[bk.mat_base + j] = (int64_t)bk.count * g;
-        }
-        hb += round_up((int64_t)bk.splits * bk.count * g, 128);
-    }
-    if ((rc = dalloc(p, &p->hbuf, hb)) || (rc = dalloc(p, &p->hoff_d, p->nmat)) ||
-        (rc = dalloc(p, &p->hss_d, p->nmat)) || (rc = dalloc(p, &p->aux_of_d, p->nmat))) {
+    if ((rc = dalloc(p, &p->aux_of_d, p->nmat))) {
         isoloco_plan_destroy(a);
         return rc;
     }
     p->aux = a;
-    CUDA_TRY(cudaMemcpy(p->hoff_d, hoff.data(), sizeof(int64_t) * p->nmat, cudaMemcpyHostToDevice));
-    CUDA_TRY(cudaMemcpy(p->hss_d, hss.data(), sizeof(int64_t) * p->nmat, cudaMemcpyHostToDevice));
     CUDA_TRY(cudaMemcpy(p->aux_of_d, aux_of.data(), sizeof(int) * p->nmat, cudaMemcpyHostToDevice));
     return ISOLOCO_OK;
 }
 
-// After the polar iteration and the trace pass (Q and sigma_bar known): Q S' in the ping-pong
-// buffer that did not hold Q, and final_buf pointed at it, so that the apply pass forms
-// U = alpha sigma_bar Q S' (derivation in spectral.cu).  kind 1: clip_high, 2: clip_low.
-static int run_clip(isoloco_plan* p, int kind, int max_iter, float tol, cudaStream_t st) {
-    if (p->nmat == 0) return ISOLOCO_OK;
-    int rc;
-    if ((rc = ensure_clip(p))) return rc;
-    isoloco_plan* a = p->aux;
+// H = Qb^T Delta (tall, MN-major operands) or Delta Qb^T (wide, K-major), fp32, upper-triangle
+// tiles mirrored, split-K partials for split buckets; Qb is Q converted to bf16 (the type of
+// Delta's planes) in the ping-pong buffer that does not hold Q.  One GEMM launch per set.
+static int form_h(isoloco_plan* p, cudaStream_t st) {
     const CUtensorMap* maps = p->tmaps_d;
     const dim3 grid(64, p->nmat);
     { PhaseTimer tm(p, ISOLOCO_PHASE_CLIP, st);
     k_clip_q_bf16<<<grid, 256, 0, st>>>(p->mats_d, p->state, p->xhi[0], p->xlo[0], p->xhi[1], p->xlo[1]); }
     CUDA_TRY(cudaGetLastError());
-    // ---- H = Qb^T Delta (tall, MN-major operands) or Delta Qb^T (wide, K-major), fp32,
-    // upper-triangle tiles mirrored; one group per (bucket, buffer holding Q), one launch
     LaunchSet hs;
     init_set(hs, kEpiF32, kGateNone, p, Precision{0, 0, 1, 1, 0});
     hs.p.list = nullptr;
@@ -1087,7 +1109,70 @@ static int run_clip(isoloco_plan* p, int kind, int max_iter, float tol, cudaStre
             hs.add(g, bk.tall, bk.tall);
         }
     }
-    if ((rc = flush_set(p, ISOLOCO_PHASE_CLIP, hs, st))) return rc;
+    return flush_set(p, ISOLOCO_PHASE_CLIP, hs, st);
+}
+
+// Buffers of the exact singular values: per matrix the tridiagonal (2 n floats) and sigma_i.
+static int ensure_svd(isoloco_plan* p) {
+    if (p->sv) return ISOLOCO_OK;
+    int rc = ensure_hbuf(p);
+    if (rc) return rc;
+    std::vector<int64_t> toff(p->nmat), soff(p->nmat);
+    int64_t t = 0, v = 0;
+    for (int i = 0; i < p->nmat; ++i) {
+        toff[i] = t;
+        soff[i] = v;
+        t += 2 * (int64_t)p->mats_h[i].n;
+        v += p->mats_h[i].n;
+    }
+    if ((rc = dalloc(p, &p->tri, std::max<int64_t>(t, 1))) || (rc = dalloc(p, &p->tri_off_d, p->nmat)) ||
+        (rc = dalloc(p, &p->sv, std::max<int64_t>(v, 1))) || (rc = dalloc(p, &p->sv_off_d, p->nmat)))
+        return rc;
+    CUDA_TRY(cudaMemcpy(p->tri_off_d, toff.data(), sizeof(int64_t) * p->nmat, cudaMemcpyHostToDevice));
+    CUDA_TRY(cudaMemcpy(p->sv_off_d, soff.data(), sizeof(int64_t) * p->nmat, cudaMemcpyHostToDevice));
+    p->sv_off_h = soff;
+    return ISOLOCO_OK;
+}
+
+// After the polar iteration and the trace (Q known): sigma_i of every matrix as the
+// eigenvalues of H (svd.cu), and sigma_bar = their mean in place of the trace's.
+static int run_svd(isoloco_plan* p, cudaStream_t st) {
+    if (p->nmat == 0) return ISOLOCO_OK;
+    int rc;
+    if ((rc = ensure_svd(p)) || (rc = form_h(p, st))) return rc;
+    int nmax = 1;
+    for (int i = 0; i < p->nmat; ++i) nmax = std::max(nmax, p->mats_h[i].n);
+    const size_t smem = sizeof(float) * (4 * (size_t)nmax + 32);
+    static bool attr = false;
+    if (!attr) {
+        CUDA_TRY(cudaFuncSetAttribute(k_svd_tridiag, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024));
+        attr = true;
+    }
+    if (smem > 200 * 1024) return fail(ISOLOCO_ERR_INVALID, "exact singular values: matrices up to 12,792 wide");
+    PhaseTimer tm(p, ISOLOCO_PHASE_CLIP, st);
+    k_svd_tridiag<<<p->nmat, kSvdThreads, smem, st>>>(p->mats_d, p->state, p->hbuf, p->hoff_d, p->hss_d, p->nsplit_d,
+                                                      p->tri, p->tri_off_d);
+    CUDA_TRY(cudaGetLastError());
+    k_svd_bisect<<<dim3((nmax + 255) / 256, p->nmat), 256, 0, st>>>(p->mats_d, p->tri, p->tri_off_d, p->sv,
+                                                                     p->sv_off_d);
+    CUDA_TRY(cudaGetLastError());
+    k_svd_sigma_bar<<<(p->nmat + 7) / 8, 256, 0, st>>>(p->mats_d, p->nmat, p->state, p->sv, p->sv_off_d);
+    CUDA_TRY(cudaGetLastError());
+    p->launches += 4;
+    return ISOLOCO_OK;
+}
+
+// After the polar iteration and the trace pass (Q and sigma_bar known): Q S' in the ping-pong
+// buffer that did not hold Q, and final_buf pointed at it, so that the apply pass forms
+// U = alpha sigma_bar Q S' (derivation in spectral.cu).  kind 1: clip_high, 2: clip_low.
+static int run_clip(isoloco_plan* p, int kind, int max_iter, float tol, cudaStream_t st) {
+    if (p->nmat == 0) return ISOLOCO_OK;
+    int rc;
+    if ((rc = ensure_clip(p))) return rc;
+    isoloco_plan* a = p->aux;
+    const CUtensorMap* maps = p->tmaps_d;
+    const dim3 grid(64, p->nmat);
+    if ((rc = form_h(p, st))) return rc;
     // ---- A' = H / sigma_bar - I -> the auxiliary plan; its polar factor Q_A = sign(A');
     // P = (I -/+ Q_A) / 2; S'' = (P A') P, all in the auxiliary plan's planes
     { PhaseTimer tm(p, ISOLOCO_PHASE_CLIP, st, 0);
@@ -1212,8 +1297,8 @@ static int check_opts(const isoloco_opts_t* o, isoloco_opts_t* out) {
     if (out->aggregator < 0 || out->aggregator > 2) return fail(ISOLOCO_ERR_INVALID, "aggregator must be 0, 1 or 2");
     if (!(out->sparsity >= 0.f && out->sparsity < 1.f))
         return fail(ISOLOCO_ERR_INVALID, "sparsity must be in [0, 1)");
-    if (out->spectrum_kind < 0 || out->spectrum_kind > 2)
-        return fail(ISOLOCO_ERR_INVALID, "spectrum_kind must be 0, 1 or 2");
+    if (out->spectrum_kind < 0 || out->spectrum_kind > 3)
+        return fail(ISOLOCO_ERR_INVALID, "spectrum_kind must be 0, 1, 2 or 3");
     if (out->full_precision < 0 || out->full_precision > 1)
         return fail(ISOLOCO_ERR_INVALID, "full_precision must be 0 or 1");
     if (out->precision_schedule < -1 || out->precision_schedule >= (1ll << 40))
@@ -1287,12 +1372,15 @@ static int run_isoc_step(isoloco_plan* p, int merge, float* theta, float* mom, c
         CUDA_TRY(cudaEventRecord(p->ev_copied, p->side_st));
     }
     p->fast_steps = merge ? 0 : o.fast_steps;
+    // the spectrum variants need Q's singular values at 1 to ~2^-20: three passes throughout
+    // (a two-pass Gram feeding the polish leaves ~1e-4 in them)
     p->full_prec = !merge && (o.spectrum_kind != 0 || o.full_precision != 0);
     set_precision_schedule(p, merge ? -1 : o.precision_schedule);
     p->skip_trace = !merge && (o.fast_steps > 0 || o.scale_kind == 1);
     if ((rc = run_polar(p, p->fast_steps ? std::max(o.max_iter, o.fast_steps) : o.max_iter, o.tol, st))) return rc;
     const int clip = merge ? 0 : o.spectrum_kind;
-    if (clip && (rc = run_clip(p, clip, o.max_iter, o.tol, st))) return rc;
+    if ((clip == 1 || clip == 2) && (rc = run_clip(p, clip, o.max_iter, o.tol, st))) return rc;
+    if (clip == 3 && (rc = run_svd(p, st))) return rc;
     UpdateSrc us;
     us.qh[0] = p->xhi[0];
     us.qh[1] = p->xhi[1];
@@ -1636,6 +1724,22 @@ int isoloco_read_diag(isoloco_plan_t p, void* stream, float* sigma_bar, int32_t*
         if (resid) resid[j] = m.resid;
     }
     return ISOLOCO_OK;
+}
+
+int isoloco_read_singular_values(isoloco_plan_t p, void* stream, int matrix, float* out, int capacity) {
+    if (!p) return fail(ISOLOCO_ERR_INVALID, "plan is NULL");
+    if (matrix < 0 || matrix >= p->nmat) return fail(ISOLOCO_ERR_INVALID, "matrix index out of range");
+    if (!p->sv) return fail(ISOLOCO_ERR_INVALID, "no singular values: run a step with spectrum_kind = 3 first");
+    // table order of the 2-D tensors -> plan order
+    std::vector<int> order(p->nmat);
+    for (int i = 0; i < p->nmat; ++i) order[i] = i;
+    std::sort(order.begin(), order.end(), [&](int a, int b) { return p->mat_param[a] < p->mat_param[b]; });
+    const int mi = order[matrix];
+    const int n = p->mats_h[mi].n;
+    if (!out || capacity < n) return fail(ISOLOCO_ERR_INVALID, "output buffer smaller than min(rows, cols)");
+    CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+    CUDA_TRY(cudaMemcpy(out, p->sv + p->sv_off_h[mi], sizeof(float) * n, cudaMemcpyDeviceToHost));
+    return n;
 }
 
 int isoloco_debug_wait_timeout(int64_t limit_ns, int64_t* elapsed_ns, void* stream) {

@@ -137,10 +137,12 @@ __device__ __forceinline__ bool decode_tile(const GemmParams& p, const int* pre,
             ti.horner = (p.epi == kEpiPoly && p.poly_horner && st.mode == 1);
             if (p.split_on_polish && st.mode == 2) ti.a_split = ti.b_split = true;  // final step: 3 passes
         }
-        // precision schedule: single-pass steps (a Gram only after iteration 0's)
+        // precision schedule: single-pass steps.  A Gram only after iteration 0's and only
+        // while the last residual is large (>= kOnePassGramResid): a Gram whose test can pass
+        // feeds the final polish, which nothing corrects afterwards, so it keeps its passes.
         const int k = (p.epi == kEpiGram) ? st.step : st.step - 1;
         if (k >= g.one_from && k < g.one_to &&
-            ((p.epi == kEpiGram) ? st.step > 0 : st.mode == 1))
+            ((p.epi == kEpiGram) ? (st.step > 0 && st.resid >= kOnePassGramResid) : st.mode == 1))
             ti.a_split = ti.b_split = false;
         ti.ca = st.a;
         ti.cb = st.b;

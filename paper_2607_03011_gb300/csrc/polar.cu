@@ -207,7 +207,7 @@ __device__ __forceinline__ const float* sched_row(bool deep, int step) {
 // Decision for matrix mi, taken by one warp.  t: iteration index (0 = first Gram of Delta).
 __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatState* __restrict__ state,
                                const float* __restrict__ fin_part, int t, int max_iter, float tol,
-                               uint32_t* __restrict__ err, int lane, int fast_steps) {
+                               uint32_t* __restrict__ err, int lane, int fast_steps, int4 gram_one) {
     MatState& st = state[mi];
     if (st.done) {
         if (lane == 0) st.mode = 0;
@@ -244,6 +244,10 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
     const double n = static_cast<double>(md.n);
     double d, gscale = 1.0, xscale = 1.0;
     const int st_step = st.step, st_iters = st.iters;  // one read each; st is global memory
+    // this Gram ran a single pass (precision schedule: the step range of the matrix's kind,
+    // gram_one = (standard from, to, deep from, to), and a large previous residual)
+    const int g_from = md.deep ? gram_one.z : gram_one.x, g_to = md.deep ? gram_one.w : gram_one.y;
+    const bool gram_single = t > 0 && st_step >= g_from && st_step < g_to && st.resid >= kOnePassGramResid;
     if (t == 0) {
         const double s2 = sqrt(sq);  // ||Delta^T Delta||_F >= sigma_max(Delta)^2
         if (!(s2 > 0.0) || !isfinite(s2)) {
@@ -299,8 +303,10 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
             st.done = 1;
             st.final_buf = (t + 1) & 1;
         }
-    } else if (d < tol || partial) {
+    } else if ((d < tol || partial) && !gram_single) {
         // Cubic polish p(x) = 1.5 x - 0.5 x^3 on singular values already near 1 (or 0).
+        // (Not from a single-pass Gram: the matrix then takes one more quintic step, and the
+        // Gram after it, with a small residual, keeps its passes.)
         st.mode = 2;
         st.a = 1.5f;
         st.b = static_cast<float>(-0.5 * gscale);
@@ -350,11 +356,11 @@ __global__ void __launch_bounds__(kControlThreads) k_control(const MatDesc* __re
                                                              int* __restrict__ list_step, int* __restrict__ cnt_step,
                                                              cudaGraphConditionalHandle cond, int set_cond,
                                                              long long* __restrict__ loopc, int fast_steps,
-                                                             int* __restrict__ ticket) {
+                                                             int* __restrict__ ticket, int4 gram_one) {
     constexpr int kWarps = kControlThreads / 32;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     for (int mi = blockIdx.x * kWarps + warp; mi < nmat; mi += gridDim.x * kWarps) {
-        control_matrix(mats, mi, state, fin_part, t, max_iter, tol, err, lane, fast_steps);
+        control_matrix(mats, mi, state, fin_part, t, max_iter, tol, err, lane, fast_steps, gram_one);
         __syncwarp();
     }
     __threadfence();

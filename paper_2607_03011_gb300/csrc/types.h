@@ -36,6 +36,11 @@ constexpr int kTmemCols = 256;     // one accumulator; the kernel double-buffers
 constexpr int kMaxGroups = 8;
 constexpr int kControlThreads = 256;  // k_control block: one warp per matrix
 constexpr int kFinRows = 32;  // rows of one k_gram_finalize tile (x BN columns)
+constexpr int kSvdThreads = 1024;  // k_svd_tridiag block: one CTA per matrix
+// A Gram of the precision schedule's single-pass steps runs one pass only when the previous
+// residual ||X^T X - I||_F / sqrt(n) is at least this: one quintic step cannot bring such a
+// residual below the convergence tolerance, so the Gram cannot be the one the polish uses.
+constexpr float kOnePassGramResid = 0.5f;
 // Epilogue staging: per epilogue warp kStageBlocks blocks of 32 x 32 16-bit values (2 KB,
 // 64-byte swizzled rows), written to global memory by TMA stores.  With four, a symmetric
 // output uses them as two (direct, transposed) pairs and anything else as four single

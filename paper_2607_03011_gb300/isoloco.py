@@ -78,6 +78,7 @@ def lib():
             L.iso_c_merge.argtypes = [_vp, _vp, ctypes.POINTER(_vp), ctypes.c_float, _vp, _vp]
             L.isoloco_last_status.argtypes = [_vp, _vp]
             L.isoloco_read_diag.argtypes = [_vp, _vp, _vp, _vp, _vp, _vp]
+            L.isoloco_read_singular_values.argtypes = [_vp, _vp, ctypes.c_int, _vp, ctypes.c_int]
             L.isoloco_profile_enable.argtypes = [_vp, ctypes.c_int]
             L.isoloco_profile_read.argtypes = [_vp, _vp, _vp, _vp, ctypes.c_int]
             L.isoloco_plan_launches.argtypes = [_vp]
@@ -114,7 +115,8 @@ def make_opts(alpha=1.0, outer_lr=0.7, momentum=0.9, reduce_mean=True, max_iter=
               sync=False, fast_steps=0, orth_target=0, momentum_kind=0, scale_kind=0, aggregator=0,
               sparsity=0.0, seed=0, spectrum_kind=0, full_precision=0, precision_schedule=0) -> Opts:
     """Options of an outer step; fast_steps > 0 selects the fixed-step variant of Sec. 4.3,
-    orth_target / momentum_kind / scale_kind / spectrum_kind (1 clip_high, 2 clip_low) the
+    orth_target / momentum_kind / scale_kind / spectrum_kind (1 clip_high, 2 clip_low, 3 Iso-C
+    from the exact singular values) the
     ablations of Sec. 4.5 / App. B, and aggregator / sparsity / seed the merging rule of
     diloco_outer_step (Sec. 3.2: 0 mean, 1 TIES, 2 DARE); full_precision = 1 splits both
     operands of every polar step; see include/isoloco.h."""
@@ -261,6 +263,16 @@ class Plan:
         _check(self._L.isoloco_read_diag(self._h, _stream(stream), sb, it, st, rs), "isoloco_read_diag")
         return {"sigma_bar": list(sb)[:n], "iters": list(it)[:n], "status": list(st)[:n],
                 "residual": list(rs)[:n]}
+
+    def singular_values(self, matrix: int, stream=None) -> list:
+        """Descending singular values of 2-D tensor `matrix` (table order over the 2-D
+        tensors) from the last step with spectrum_kind = 3."""
+        cap = 1 << 16
+        buf = (ctypes.c_float * cap)()
+        n = self._L.isoloco_read_singular_values(self._h, _stream(stream), int(matrix), buf, cap)
+        if n < 0:
+            _check(n, "isoloco_read_singular_values")
+        return list(buf)[:n]
 
 
 def debug_gemm(A: torch.Tensor, B: torch.Tensor, a_mn_major: bool, b_mn_major: bool, M: int, N: int, K: int,

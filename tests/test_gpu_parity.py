@@ -345,7 +345,8 @@ def test_clip_tiny_bf16_and_zero(iso, kind):
 
 def test_clip_options_rejected(iso):
     wl = W.make_workload("tiny", seed=0, device="cuda")
-    for flags in ({"spectrum_kind": 3}, {"spectrum_kind": 1, "fast_steps": 5}, {"spectrum_kind": 2, "scale_kind": 1}):
+    for flags in ({"spectrum_kind": 4}, {"spectrum_kind": -1}, {"spectrum_kind": 1, "fast_steps": 5},
+                  {"spectrum_kind": 2, "scale_kind": 1}, {"spectrum_kind": 3, "fast_steps": 5}):
         with pytest.raises(iso.IsolocoError):
             run_gpu(iso, wl, 1.0, 0.7, 0.9, **flags)
 
