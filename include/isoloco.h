@@ -64,7 +64,8 @@ typedef enum {
     ISOLOCO_ERR_NOT_CONVERGED = -4, /* a polar iteration hit max_iter (update still applied) */
     ISOLOCO_ERR_CUDA = -5,          /* a CUDA runtime call failed */
     ISOLOCO_ERR_OOM = -6,           /* workspace allocation failed */
-    ISOLOCO_ERR_TIMEOUT = -7        /* a device-side wait gave up (kernel returned early) */
+    ISOLOCO_ERR_TIMEOUT = -7,       /* a device-side wait gave up (kernel returned early) */
+    ISOLOCO_ERR_GUARD = -8          /* isoloco_check_guards: a workspace guard byte was overwritten */
 } isoloco_status_t;
 
 /* Options of one outer step (Alg. 2's hyperparameters plus solver controls). */
@@ -213,6 +214,18 @@ int isoloco_last_status(isoloco_plan_t plan, void* stream);
  * only (n_matrices entries each; any pointer may be NULL).  Synchronizes `stream`.
  *   sigma_bar: tr(Q^T Delta) / min(m, n);  iters: polar iterations used;
  *   status: 0 or NOT_CONVERGED;  residual: last ||X^T X - I||_F / sqrt(n). */
+/* Bounds check of the plan's device workspace (no counterpart in the paper; it stands in
+ * for a memory checker).  Every workspace region the plan (and its auxiliary plan) owns
+ * sits between 256 guard bytes before it and its padding plus 256 guard bytes after it,
+ * filled with 0xA5 when allocated; this synchronizes `stream` and compares them.  Returns OK,
+ * GUARD (the message names the region, the side and the distance) or CUDA. */
+int isoloco_check_guards(isoloco_plan_t plan, void* stream);
+
+/* Test support for isoloco_check_guards: sets the guard byte right before (after = 0) or
+ * right after (after = 1) workspace region `region` of the plan to a value other than the
+ * fill, with cudaMemset inside the region's own allocation.  Returns OK or INVALID. */
+int isoloco_debug_touch_guard(isoloco_plan_t plan, int region, int after);
+
 /* Singular values of 2-D tensor `matrix` (table order over the 2-D tensors) from the
  * plan's last call with spectrum_kind = 3 (Alg. 2: Delta = U S V^T; here sigma_i of the
  * reduced pseudo-gradient), in descending order, copied to host memory out[0 .. r-1],

@@ -24,6 +24,11 @@
 
 namespace isoloco {
 
+// Guard bytes around each workspace region (the plan's bounds check: a kernel that writes
+// past either end of its region changes them; isoloco_check_guards compares them).
+constexpr size_t kGuardBytes = 256;
+constexpr int kGuardByte = 0xA5;
+
 // kernels defined in the other translation units
 cudaError_t launch_gemm(const GemmParams& p, int max_ctas, cudaStream_t stream);
 __global__ void k_gram_finalize(const MatDesc*, const int2*, const MatState*, const float*, const int64_t*,
@@ -122,6 +127,8 @@ struct isoloco_plan {
     int64_t plane_elems = 0, gplane_elems = 0, gpart_elems = 0, n1d = 0;
     // device workspace
     std::vector<void*> allocs;
+    // every workspace region sits between guard bytes (dalloc): allocation base, region bytes
+    std::vector<std::pair<uint8_t*, size_t>> guards;
     int64_t ws_bytes = 0;
     __nv_bfloat16 *dhi = nullptr, *dlo = nullptr, *xhi[2] = {nullptr, nullptr}, *xlo[2] = {nullptr, nullptr};
     __nv_bfloat16 *ghi = nullptr, *glo = nullptr, *phi = nullptr, *plo = nullptr;
@@ -293,13 +300,23 @@ static int dalloc(isoloco_plan* p, T** ptr, int64_t count) {
     *ptr = nullptr;
     if (count <= 0) count = 1;
     const size_t bytes = static_cast<size_t>(count) * sizeof(T);
-    cudaError_t e = cudaMalloc(reinterpret_cast<void**>(ptr), bytes);
+    // [guard | region | pad to 256 | guard]: the region keeps cudaMalloc's 256-byte alignment
+    const size_t body = (bytes + kGuardBytes - 1) / kGuardBytes * kGuardBytes;
+    uint8_t* base = nullptr;
+    cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&base), body + 2 * kGuardBytes);
     if (e != cudaSuccess) {
         (void)cudaGetLastError();
         return fail(ISOLOCO_ERR_OOM, std::string("cudaMalloc of ") + std::to_string(bytes) + " bytes failed");
     }
-    p->allocs.push_back(*ptr);
-    p->ws_bytes += static_cast<int64_t>(bytes);
+    if (cudaMemset(base, kGuardByte, kGuardBytes) != cudaSuccess ||
+        cudaMemset(base + kGuardBytes + bytes, kGuardByte, body - bytes + kGuardBytes) != cudaSuccess) {
+        cudaFree(base);
+        return fail(ISOLOCO_ERR_CUDA, "guard fill failed");
+    }
+    *ptr = reinterpret_cast<T*>(base + kGuardBytes);
+    p->allocs.push_back(base);
+    p->guards.push_back({base, bytes});
+    p->ws_bytes += static_cast<int64_t>(body + 2 * kGuardBytes);
     return ISOLOCO_OK;
 }
 
@@ -1723,6 +1740,43 @@ int isoloco_read_diag(isoloco_plan_t p, void* stream, float* sigma_bar, int32_t*
         if (status) status[j] = m.status ? ISOLOCO_ERR_NOT_CONVERGED : ISOLOCO_OK;
         if (resid) resid[j] = m.resid;
     }
+    return ISOLOCO_OK;
+}
+
+int isoloco_check_guards(isoloco_plan_t p, void* stream) {
+    if (!p) return fail(ISOLOCO_ERR_INVALID, "plan is NULL");
+    CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+    std::vector<uint8_t> h;
+    for (isoloco_plan* q = p; q; q = q->aux) {
+        for (size_t r = 0; r < q->guards.size(); ++r) {
+            uint8_t* base = q->guards[r].first;
+            const size_t bytes = q->guards[r].second;
+            const size_t body = (bytes + kGuardBytes - 1) / kGuardBytes * kGuardBytes;
+            const size_t tail = body - bytes + kGuardBytes;
+            h.resize(kGuardBytes + tail);
+            CUDA_TRY(cudaMemcpy(h.data(), base, kGuardBytes, cudaMemcpyDeviceToHost));
+            CUDA_TRY(cudaMemcpy(h.data() + kGuardBytes, base + kGuardBytes + bytes, tail, cudaMemcpyDeviceToHost));
+            for (size_t i = 0; i < h.size(); ++i)
+                if (h[i] != static_cast<uint8_t>(kGuardByte)) {
+                    const bool front = i < kGuardBytes;
+                    return fail(ISOLOCO_ERR_GUARD, std::string("workspace region ") + std::to_string(r) + " of " +
+                                                       (q == p ? "the plan" : "its auxiliary plan") + ": byte " +
+                                                       std::to_string(front ? kGuardBytes - i : i - kGuardBytes + 1) +
+                                                       (front ? " before its start" : " past its end") +
+                                                       " overwritten");
+                }
+        }
+    }
+    return ISOLOCO_OK;
+}
+
+int isoloco_debug_touch_guard(isoloco_plan_t p, int region, int after) {
+    if (!p) return fail(ISOLOCO_ERR_INVALID, "plan is NULL");
+    if (region < 0 || region >= static_cast<int>(p->guards.size()))
+        return fail(ISOLOCO_ERR_INVALID, "no such workspace region");
+    uint8_t* base = p->guards[region].first;
+    uint8_t* at = after ? base + kGuardBytes + p->guards[region].second : base + kGuardBytes - 1;
+    CUDA_TRY(cudaMemset(at, 0x5A, 1));  // one guard byte, inside the allocation
     return ISOLOCO_OK;
 }
 

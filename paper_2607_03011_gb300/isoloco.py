@@ -27,8 +27,9 @@ ERR_NOT_CONVERGED = -4
 ERR_CUDA = -5
 ERR_OOM = -6
 ERR_TIMEOUT = -7
+ERR_GUARD = -8
 STATUS_NAMES = {0: "OK", -1: "INVALID", -2: "ALIGN", -3: "NONFINITE", -4: "NOT_CONVERGED",
-                -5: "CUDA", -6: "OOM", -7: "TIMEOUT"}
+                -5: "CUDA", -6: "OOM", -7: "TIMEOUT", -8: "GUARD"}
 _HARD_ERRORS = {ERR_INVALID, ERR_ALIGN, ERR_CUDA, ERR_OOM}
 
 
@@ -79,6 +80,8 @@ def lib():
             L.isoloco_last_status.argtypes = [_vp, _vp]
             L.isoloco_read_diag.argtypes = [_vp, _vp, _vp, _vp, _vp, _vp]
             L.isoloco_read_singular_values.argtypes = [_vp, _vp, ctypes.c_int, _vp, ctypes.c_int]
+            L.isoloco_check_guards.argtypes = [_vp, _vp]
+            L.isoloco_debug_touch_guard.argtypes = [_vp, ctypes.c_int, ctypes.c_int]
             L.isoloco_profile_enable.argtypes = [_vp, ctypes.c_int]
             L.isoloco_profile_read.argtypes = [_vp, _vp, _vp, _vp, ctypes.c_int]
             L.isoloco_plan_launches.argtypes = [_vp]
@@ -263,6 +266,11 @@ class Plan:
         _check(self._L.isoloco_read_diag(self._h, _stream(stream), sb, it, st, rs), "isoloco_read_diag")
         return {"sigma_bar": list(sb)[:n], "iters": list(it)[:n], "status": list(st)[:n],
                 "residual": list(rs)[:n]}
+
+    def check_guards(self, stream=None) -> int:
+        """Compares the guard bytes around every workspace region (isoloco_check_guards):
+        0, or ERR_GUARD with last_error() naming the region."""
+        return self._L.isoloco_check_guards(self._h, _stream(stream))
 
     def singular_values(self, matrix: int, stream=None) -> list:
         """Descending singular values of 2-D tensor `matrix` (table order over the 2-D

@@ -63,6 +63,7 @@ def test_validation_without_gpu(lib):
     assert lib.isoloco_debug_gemm(0, 0, 0, 0, 1, 1, 1, None, None, None, None) == isoloco.ERR_INVALID
     assert lib.isoloco_debug_gemm(0, 0, 9, 1, 1, 1, 1, None, None, None, None) == isoloco.ERR_INVALID
     assert lib.isoloco_read_singular_values(None, None, 0, None, 0) == isoloco.ERR_INVALID
+    assert lib.isoloco_check_guards(None, None) == isoloco.ERR_INVALID
     assert lib.isoloco_debug_wait_timeout(1_000, None, None) == isoloco.ERR_INVALID          # below 1 ms
     assert lib.isoloco_debug_wait_timeout(2_000_000_000, None, None) == isoloco.ERR_INVALID  # above 1 s
 
