@@ -241,9 +241,16 @@ def stream_bytes(table, K, replica_bytes):
 # tensor-core passes over hi/lo splits of fp32 operands with fp32 accumulation.
 DTYPE_ISO = "f32 streaming; polar GEMMs as bf16/fp16 hi+lo split passes, f32 accumulate"
 
-# DRAM bytes (read + write) of all k_gemm_split launches of one step, from an ncu capture of
-# the current kernel (workload, fast_steps, spectrum_kind) -> figure; see profiles/.
-GEMM_TRAFFIC = {}
+# DRAM bytes (read + write) of all k_gemm_split launches of one step, from ncu captures of
+# the current kernel, (workload, fast_steps, spectrum_kind) -> figure: the 180M step's four
+# shape buckets captured one at a time and summed (profiles/k_gemm_split_dram_llama_180m_buckets.md).
+GEMM_TRAFFIC = {
+    ("llama_180m_k8", 0, 0): {
+        "bytes_per_step": 28.30e9,
+        "note": "dram__bytes_read.sum + dram__bytes_write.sum of every k_gemm_split launch of one step, "
+                "captured per shape bucket (square48, tall12, wide24, embed2) and summed; same unit as "
+                "achieved (per step over all GEMM launches)"},
+}
 
 
 # --------------------------------------------------------------------------- CPU oracle arm

@@ -7,7 +7,9 @@
 is the 48 square 1024 x 1024 matrices of the 180M recipe with K = 8 replicas
 (1.6 GB of replicas: larger than L2, small enough for a full ncu capture), and
 `square12` a quarter of it; `wide12` / `tall12` twelve 1024 x 2816 matrices (the shape of
-w_gate and w_up) and twelve 2816 x 1024 ones (w_down); with --per-launch the polar iterations are launched one
+w_gate and w_up) and twelve 2816 x 1024 ones (w_down); `wide24` the 24 w_gate / w_up matrices
+and `embed2` the 32000 x 1024 embedding and head (with `square48` and `tall12`, the 180M
+recipe's four shape buckets one at a time); with --per-launch the polar iterations are launched one
 by one (phase profiling on) instead of as the library's CUDA graph, so that every
 kernel is a plain launch.  `gemm` runs the split-precision GEMM entry point on random
 inputs; `diloco` runs DiLoCo outer steps with a merging aggregator (Sec. 3.2), and
@@ -32,6 +34,10 @@ EXTRA = {
                                     noise_std=2e-5, momentum_std=2e-5, name="wide12"),
     "tall12": lambda: W.custom_spec([(f"g{i}", 2816, 1024) for i in range(12)], K=8, rank=32, shared_std=2e-5,
                                     noise_std=2e-5, momentum_std=2e-5, name="tall12"),
+    "wide24": lambda: W.custom_spec([(f"u{i}", 1024, 2816) for i in range(24)], K=8, rank=32, shared_std=2e-5,
+                                    noise_std=2e-5, momentum_std=2e-5, name="wide24"),
+    "embed2": lambda: W.custom_spec([("embed", 32000, 1024), ("head", 32000, 1024)], K=8, rank=32, shared_std=2e-5,
+                                    noise_std=2e-5, momentum_std=2e-5, name="embed2"),
     "tall4": lambda: W.custom_spec([("e", 32000, 1024), ("d0", 2816, 1024), ("d1", 2816, 1024), ("g", 1024, 2816)],
                                    K=8, rank=32, shared_std=2e-5, noise_std=2e-5, momentum_std=2e-5, name="tall4"),
 }
