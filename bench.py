@@ -136,7 +136,15 @@ def job_value(world: int, params: int, steps: int, total_ms: float) -> float:
 
 
 # --------------------------------------------------------------------------- accounting
-def gemm_flops(table, diag, fast=False):
+GRAM_SIDE_RATIO = 8   # tall matrices with rows >= 8 * cols iterate on n x n matrices (the library's rule)
+
+
+def gram_side(r, c, fast=False, full=False):
+    """Whether the library runs this matrix's polar iteration on the Gram side."""
+    return r >= GRAM_SIDE_RATIO * c and r >= 2 * BK and not fast and not full
+
+
+def gemm_flops(table, diag, fast=False, full=False):
     """Algorithmic (single-pass) FLOPs of the polar GEMMs of one step, per phase, from
     the per-matrix iteration counts: a full Gram 2*r*n^2 per iteration (symmetry not
     discounted), G^2 = 2*n^3 per quintic step, an update 2*r*n^2 per iteration
@@ -147,6 +155,16 @@ def gemm_flops(table, diag, fast=False):
     for (r, c), it, st in zip(mats, diag["iters"], diag["status"]):
         big, small = max(r, c), min(r, c)
         gram1, sq1 = 2.0 * big * small * small, 2.0 * small ** 3
+        if it > 0 and gram_side(r, c, fast, full):
+            # iteration 0's Gram (2 m n^2) and P_0; then per iteration W = A Z and G = Z^T W
+            # (2 n^3 each), P (quintic steps) and Z P (2 n^3); finally Q = Delta Z (2 m n^2)
+            converged = (st == 0)
+            grams = it + (0 if converged else 1)
+            quintic = it - (1 if converged else 0)
+            out["gram"] += gram1 + (grams - 1) * 2 * sq1
+            out["poly"] += quintic * sq1
+            out["update"] += (it - 1) * sq1 + gram1
+            continue
         if fast:
             out["gram"] += it * gram1
             out["poly"] += it * sq1
@@ -199,6 +217,17 @@ def gemm_exec_flops(table, diag, fast=False, full=False, sched=None):
         gram1 = _sym_tiles(n) * BM * BN * 2.0 * kpad_big
         poly1 = _sym_tiles(n) * BM * BN * 2.0 * kpad_n
         upd1 = (-(-r // BM)) * (-(-c // BN)) * BM * BN * 2.0 * kpad_n
+        if it > 0 and gram_side(r, c, fast, full):
+            sq_all = (-(-n // BM)) * (-(-n // BN)) * BM * BN * 2.0 * kpad_n   # every tile of an n x n product
+            converged = (st == 0)
+            grams = it + (0 if converged else 1)
+            quintic = it - (1 if converged else 0)
+            # iteration 0: Gram and P_0 three passes; later W and G three passes, P two,
+            # Z P two (three in the polish); the final Delta Z three
+            out["gram"] += 3 * gram1 + (grams - 1) * 3 * (sq_all + poly1)
+            out["poly"] += (3 * poly1 + 2 * poly1 * (quintic - 1)) if quintic >= 1 else 0.0
+            out["update"] += 2 * sq_all * max(0, quintic - 1) + (3 * sq_all if converged and it > 1 else 0.0) + 3 * upd1
+            continue
         if fast:   # `it` quintic steps, every one with three passes; no polish
             out["gram"] += 3 * gram1 * it
             out["poly"] += 3 * poly1 * it
@@ -608,7 +637,8 @@ def main():
         return 0
 
     peaks, peak_src = load_peaks()
-    fl = gemm_flops(wl.table, diag, fast=args.fast_steps > 0)
+    fl = gemm_flops(wl.table, diag, fast=args.fast_steps > 0, full=spectrum_kind != 0)
+    fl_rc = gemm_flops(wl.table, diag, fast=True if args.fast_steps > 0 else False, full=True)
     fx = gemm_exec_flops(wl.table, diag, fast=args.fast_steps > 0, full=spectrum_kind != 0)
     flops = sum(fl.values()) * args.steps
     xflops = sum(fx.values()) * args.steps
@@ -640,6 +670,10 @@ def main():
                 "kernel_times": "per-phase CUDA events on the launch stream, in a profiled pass of the "
                                 "same steps right after the timed region",
                 "algorithmic_tflop_per_step": flops / args.steps / 1e12,
+                "rows_cols_tflop_per_step": sum(fl_rc.values()) / 1e12,
+                "rows_cols_note": "the same iteration counts priced as if every matrix iterated on its rows x cols "
+                                  "side (4mn^2 + 2n^3 per quintic step); the Gram-side matrices (rows >= 8 cols) do "
+                                  "less work, which `algorithmic_tflop_per_step` counts",
                 "executed_tensor_tflop_per_step": xflops / args.steps / 1e12,
                 "executed_tflops": executed_tf,
                 "frac_executed": executed_tf / tc_peak if tc_peak else None,

@@ -18,7 +18,7 @@ BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libisoloco.so")
 INCLUDE = os.path.join(ROOT, "include")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["api.cu", "gemm.cu", "polar.cu", "stream.cu", "spectral.cu", "svd.cu"]
+SOURCES = ["api.cu", "gemm.cu", "polar.cu", "stream.cu", "spectral.cu", "svd.cu", "gramside.cu"]
 
 
 def _nvcc() -> str:

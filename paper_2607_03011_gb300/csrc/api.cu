@@ -33,7 +33,13 @@ constexpr int kGuardByte = 0xA5;
 cudaError_t launch_gemm(const GemmParams& p, int max_ctas, cudaStream_t stream);
 __global__ void k_gram_finalize(const MatDesc*, const int2*, const MatState*, const float*, const int64_t*,
                                 const int64_t*, const int*, __nv_bfloat16*, __nv_bfloat16*, float*, int,
-                                __nv_bfloat16*);
+                                __nv_bfloat16*, int);
+__global__ void k_gs_init(const MatDesc*, MatState*, const int*, const float*, const int64_t*, const int64_t*,
+                          const int*, __nv_bfloat16*, __nv_bfloat16*, __nv_bfloat16*, __nv_bfloat16*,
+                          const __nv_bfloat16*, const __nv_bfloat16*);
+__global__ void k_gs_final_prep(const MatDesc*, const MatState*, const int*, const __nv_bfloat16*, const __nv_bfloat16*,
+                                const __nv_bfloat16*, const __nv_bfloat16*, __nv_bfloat16*, __nv_bfloat16*);
+__global__ void k_gs_final_flip(MatState*, const int*, int);
 __global__ void k_control(const MatDesc*, int, MatState*, const float*, int, int, float, uint32_t*, const int*,
                           const int*, int, int*, int*, int*, int*, cudaGraphConditionalHandle, int, long long*,
                           int, int*, int4);
@@ -92,12 +98,19 @@ constexpr float kDefaultTol = 4e-3f;
 enum MapRole { kRoleKA = 0, kRoleKB = 1, kRoleMN = 2, kRoleST = 3 };
 // 3 sources x 3 roles x 2 planes + G (2x2) + P (2x2) + store maps (X0, X1, G, P) x 2 planes
 // + Y (operand KB, store)
-constexpr int kMapsPerBucket = 36;
+// + Gram-side buckets: Z in the first n rows of X0 / X1 (operand K-major A, MN-major, store)
+// x 2 planes, A (K-major A), W (MN-major, store) x 2 planes
+constexpr int kMapsPerBucket = 54;
 inline int src_map(int src, int role, int plane) { return (src * 3 + role) * 2 + plane; }
 inline int g_map(int role, int plane) { return 18 + role * 2 + plane; }
 inline int p_map(int role, int plane) { return 22 + role * 2 + plane; }
 // store maps (32 x 32 boxes): which 0 = X0, 1 = X1, 2 = G, 3 = P
 inline int st_map(int which, int plane) { return 26 + which * 2 + plane; }
+// Gram-side maps; Z's roles: 0 K-major A, 1 MN-major, 2 store
+inline int z_map(int buf, int role, int plane) { return 36 + buf * 6 + role * 2 + plane; }
+inline int an_map(int plane) { return 48 + plane; }
+inline int w_mn_map(int plane) { return 50 + plane; }
+inline int w_st_map(int plane) { return 52 + plane; }
 inline int y_map() { return 34; }     // Y as the B operand (K-major, 256 rows)
 inline int y_st_map() { return 35; }  // Y store map
 
@@ -107,6 +120,8 @@ struct Bucket {
     int mat_base;
     int64_t plane_off, gplane_off, gpart_off;
     int splits;
+    bool gs;         // Gram-side iteration (gramside.cu)
+    int64_t gs_off;  // offset of the bucket in the Gram-side n x n planes (A, W)
 };
 
 }  // namespace isoloco
@@ -133,6 +148,11 @@ struct isoloco_plan {
     __nv_bfloat16 *dhi = nullptr, *dlo = nullptr, *xhi[2] = {nullptr, nullptr}, *xlo[2] = {nullptr, nullptr};
     __nv_bfloat16 *ghi = nullptr, *glo = nullptr, *phi = nullptr, *plo = nullptr;
     __nv_bfloat16* ypl = nullptr;  // Y = b I + c G of the next quintic step (hi plane only)
+    // Gram-side buckets: A = Delta_n^T Delta_n and W = A Z (n x n, hi/lo), their matrices' list
+    __nv_bfloat16 *anhi = nullptr, *anlo = nullptr, *whi = nullptr, *wlo = nullptr;
+    int* gs_list = nullptr;
+    int n_gs = 0;
+    int64_t gs_slot_first = 0, gs_slot_count = 0;  // Gram partial slots of the Gram-side matrices
     float* gpart = nullptr;
     float* d1d = nullptr;
     float* fin_part = nullptr;
@@ -260,12 +280,15 @@ static EncodeTiledFn encode_fn() {
     return fn;
 }
 
-// 3-D bf16 map over [count][rows][ld] with logical extent cols x rows x count.
-static bool make_map(CUtensorMap* m, const void* base, int cols, int rows, int count, int ld, int role) {
+// 3-D bf16 map over [count][rows][ld] with logical extent cols x rows x count; batch_elems > 0
+// gives a batch stride other than rows * ld (an n x n matrix in the first rows of a taller slot).
+static bool make_map(CUtensorMap* m, const void* base, int cols, int rows, int count, int ld, int role,
+                     int64_t batch_elems = -1) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[3] = {(cuuint64_t)cols, (cuuint64_t)rows, (cuuint64_t)count};
-    cuuint64_t strides[2] = {(cuuint64_t)ld * 2, (cuuint64_t)rows * ld * 2};
+    cuuint64_t strides[2] = {(cuuint64_t)ld * 2,
+                             (cuuint64_t)(batch_elems > 0 ? batch_elems : (int64_t)rows * ld) * 2};
     cuuint32_t box[3];
     CUtensorMapSwizzle sw;
     if (role == kRoleMN) {
@@ -398,6 +421,8 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
                 bk.n = std::min(t.rows, t.cols);
                 bk.ld_n = (int)round_up(bk.n, 8);
                 bk.tall = t.rows >= t.cols;
+                bk.gs = bk.tall && t.rows >= kGramSideRatio * t.cols && t.rows >= 2 * BK;
+                bk.gs_off = 0;
                 p->buckets.push_back(bk);
                 members.emplace_back();
             } else {
@@ -413,6 +438,9 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
     std::vector<int4> tchunks;
     std::vector<int64_t> gpoff, gpss;
     std::vector<int> nsp;
+    std::vector<int> gs_mats;
+    int64_t gs_elems = 0;
+    auto g_elems_of = [](const Bucket& b) { return (int64_t)b.n * b.ld_n; };
     for (size_t b = 0; b < p->buckets.size(); ++b) {
         Bucket& bk = p->buckets[b];
         bk.count = (int)members[b].size();
@@ -430,6 +458,7 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         const int slots = 2 * p->num_sms / (kPairMma ? 2 : 1);
         int splits = std::max(1, (kblocks + 255) / 256);
         if (tiles * splits < slots) splits = std::max(splits, std::min(slots / std::max(1, tiles), kblocks / 32));
+        if (bk.gs) splits = std::max(splits, 2);  // iteration 0's Gram stays in fp32 partials (k_gs_init)
         int kper = (kblocks + splits - 1) / splits;
         splits = (kblocks + kper - 1) / kper;  // no empty split
         bk.splits = splits;
@@ -439,7 +468,15 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         // Gram tile (upper-triangle tiles) when the Gram's epilogue produces them; with
         // split-K one slot per finalize tile, packed, the rest of the last group zero
         const int nft = splits > 1 ? ((bk.n + kFinRows - 1) / kFinRows) * ((bk.n + BN - 1) / BN) : 0;
-        const int gtiles = splits > 1 ? (nft + kPartSlots - 1) / kPartSlots : sym_tiles(bk.n);
+        int gtiles = splits > 1 ? (nft + kPartSlots - 1) / kPartSlots : sym_tiles(bk.n);
+        // Gram-side: later Grams are n x n products with one slot group per upper tile
+        if (bk.gs) gtiles = std::max(gtiles, sym_tiles(bk.n));
+        if (bk.gs) {
+            bk.gs_off = gs_elems;
+            gs_elems += round_up((int64_t)bk.count * g_elems_of(bk), 128);
+            if (gs_mats.empty()) p->gs_slot_first = fin;
+            p->gs_slot_count = fin + (int64_t)bk.count * gtiles - p->gs_slot_first;
+        }
         for (int j = 0; j < bk.count; ++j) {
             const int pi = members[b][j];
             MatDesc md{};
@@ -456,6 +493,9 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
             md.n_gtiles = gtiles;
             // near-square (|rows - cols| < min / 16): the deep polar schedule
             md.deep = (std::abs(bk.rows - bk.cols) * 16 < bk.n) ? 1 : 0;
+            md.gs = bk.gs ? 1 : 0;
+            md.gsslot = bk.gs_off + j * g_elems;
+            if (bk.gs) gs_mats.push_back((int)p->mats_h.size());
             md.trace_part = tr;
             const int rows_per = std::max(1, kTraceChunkElems / bk.cols);
             md.n_tchunks = (bk.rows + rows_per - 1) / rows_per;
@@ -480,6 +520,7 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         gpart += round_up((int64_t)splits * bk.count * g_elems, 128);
     }
     p->nmat = (int)p->mats_h.size();
+    p->n_gs = (int)gs_mats.size();
     p->plane_elems = plane;
     p->gplane_elems = gplane;
     p->gpart_elems = gpart;
@@ -530,8 +571,13 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         (rc = dalloc(p, &p->cnt_gram, (int64_t)p->buckets.size())) ||
         (rc = dalloc(p, &p->cnt_step, (int64_t)p->buckets.size())) ||
         (rc = dalloc(p, &p->counters, kLaunchCounters + 1)) || (rc = dalloc(p, &p->loopc, 2)) ||
-        (rc = dalloc(p, &p->tmaps_d, (int64_t)kMapsPerBucket * std::max<size_t>(1, p->buckets.size()))))
+        (rc = dalloc(p, &p->tmaps_d, (int64_t)kMapsPerBucket * std::max<size_t>(1, p->buckets.size()))) ||
+        (rc = dalloc(p, &p->anhi, gs_elems)) || (rc = dalloc(p, &p->anlo, gs_elems)) ||
+        (rc = dalloc(p, &p->whi, gs_elems)) || (rc = dalloc(p, &p->wlo, gs_elems)) ||
+        (rc = dalloc(p, &p->gs_list, (int64_t)gs_mats.size())))
         return rc;
+    if (!gs_mats.empty())
+        CUDA_TRY(cudaMemcpy(p->gs_list, gs_mats.data(), sizeof(int) * gs_mats.size(), cudaMemcpyHostToDevice));
     CUDA_TRY(cudaHostAlloc(reinterpret_cast<void**>(&p->err_h), sizeof(uint32_t), cudaHostAllocDefault));
     *p->err_h = 0;
     CUDA_TRY(cudaEventCreateWithFlags(&p->done_ev, cudaEventDisableTiming));
@@ -612,6 +658,24 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
             if (!make_map(&m[y_map()], p->ypl + bk.gplane_off, bk.n, bk.n, bk.count, bk.ld_n, kRoleKB) ||
                 !make_map(&m[y_st_map()], p->ypl + bk.gplane_off, bk.n, bk.n, bk.count, bk.ld_n, kRoleST))
                 return fail(ISOLOCO_ERR_CUDA, "cuTensorMapEncodeTiled failed (Y maps)");
+            if (bk.gs) {
+                // Z in the first n rows of each matrix's slot of X0 / X1 (tall: ld = ld_n)
+                const int zroles[3] = {kRoleKA, kRoleMN, kRoleST};
+                for (int buf = 0; buf < 2; ++buf)
+                    for (int r = 0; r < 3; ++r)
+                        for (int pl = 0; pl < 2; ++pl)
+                            if (!make_map(&m[z_map(buf, r, pl)], (pl == 0 ? p->xhi[buf] : p->xlo[buf]) + bk.plane_off,
+                                          bk.n, bk.n, bk.count, bk.ld, zroles[r], (int64_t)bk.rows * bk.ld))
+                                return fail(ISOLOCO_ERR_CUDA, "cuTensorMapEncodeTiled failed (Gram-side Z maps)");
+                for (int pl = 0; pl < 2; ++pl) {
+                    const __nv_bfloat16* a = (pl == 0 ? p->anhi : p->anlo) + bk.gs_off;
+                    const __nv_bfloat16* w = (pl == 0 ? p->whi : p->wlo) + bk.gs_off;
+                    if (!make_map(&m[an_map(pl)], a, bk.n, bk.n, bk.count, bk.ld_n, kRoleKA) ||
+                        !make_map(&m[w_mn_map(pl)], w, bk.n, bk.n, bk.count, bk.ld_n, kRoleMN) ||
+                        !make_map(&m[w_st_map(pl)], w, bk.n, bk.n, bk.count, bk.ld_n, kRoleST))
+                        return fail(ISOLOCO_ERR_CUDA, "cuTensorMapEncodeTiled failed (Gram-side A / W maps)");
+                }
+            }
         }
         CUDA_TRY(cudaMemcpy(p->tmaps_d, maps.data(), sizeof(CUtensorMap) * maps.size(), cudaMemcpyHostToDevice));
     }
@@ -747,7 +811,7 @@ static int gp_one(const isoloco_plan* p, int kind, int end) {
 // Single-pass step range of a group (precision schedule; none in the full-precision paths).
 static void set_one_pass(const isoloco_plan* p, GemmGroup& g, const Bucket& bk, bool update) {
     const int kind = (std::abs(bk.rows - bk.cols) * 16 < bk.n) ? 1 : 0;  // deep schedule (as MatDesc::deep)
-    const bool full = p->fast_steps > 0 || p->full_prec;
+    const bool full = p->fast_steps > 0 || p->full_prec || bk.gs;  // Gram-side steps keep their passes
     g.one_from = full ? 0 : (update ? p->up_from[kind] : p->gp_from[kind]);
     g.one_to = full ? 0 : (update ? p->up_to[kind] : p->gp_to[kind]);
 }
@@ -771,16 +835,62 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
         // converging path keeps one operand single from iteration 1 on (its rounding only
         // perturbs the spectrum, which later steps correct).
         const bool full = p->fast_steps > 0 || p->full_prec;
+        const bool gs_on = p->n_gs > 0 && !full;  // Gram-side buckets iterate on n x n matrices
         const Precision gram_pr = first ? Precision{0, 0, 1, 1, 0}
                                         : (full ? Precision{1, 1, 1, 1, 0} : Precision{1, 1, 1, 0, 0});
         // Tall and wide matrices share one launch (their tiles pack into fewer waves).
         LaunchSet gram;
         init_set(gram, kEpiGram, kGateActive, p, gram_pr);
         gram.p.gram_y = (first || full) ? 0 : 1;
+        // Gram-side buckets after iteration 0 (gramside.cu): W = A Z, then G = Z^T W, both with
+        // three passes in launches of their own (a split B operand would thin the main Gram's ring)
+        const bool gs_iter = gs_on && !first;
+        LaunchSet wset, gsg;
+        if (gs_iter) {
+            init_set(wset, kEpiXSplit, kGateActive, p, Precision{1, 1, 1, 1, 0});
+            wset.p.unit_scale = 1;
+            init_set(gsg, kEpiGram, kGateActive, p, Precision{1, 1, 1, 1, 0});
+            gsg.p.gram_y = 1;
+        }
         for (size_t b = 0; b < p->buckets.size(); ++b) {
             const Bucket& bk = p->buckets[b];
             const CUtensorMap* m = maps + b * kMapsPerBucket;
             GemmGroup g{};
+            if (gs_iter && bk.gs) {
+                const int zb = t & 1;  // ping-pong buffer holding Z_t
+                GemmGroup w{};
+                w.a_hi = m + an_map(0);
+                w.a_lo = m + an_map(1);
+                w.b_hi = m + z_map(zb, 1, 0);
+                w.b_lo = m + z_map(zb, 1, 1);
+                set_group_common(w, bk.n, bk.n, bk.n, bk.count, 1, bk.mat_base);
+                w.bucket = (int)b;
+                w.out_hi = p->whi + bk.gs_off;
+                w.out_lo = p->wlo + bk.gs_off;
+                w.st_hi = m + w_st_map(0);
+                w.st_lo = m + w_st_map(1);
+                w.bf_batch_stride = (int64_t)bk.n * bk.ld_n;
+                w.ld_bf = bk.ld_n;
+                wset.add(w, false, true);
+                g.a_hi = m + z_map(zb, 1, 0);
+                g.a_lo = m + z_map(zb, 1, 1);
+                g.b_hi = m + w_mn_map(0);
+                g.b_lo = m + w_mn_map(1);
+                set_group_common(g, bk.n, bk.n, bk.n, bk.count, 1, bk.mat_base);
+                g.bucket = (int)b;
+                g.out_hi = p->ghi + bk.gplane_off;
+                g.out_lo = p->glo + bk.gplane_off;
+                g.st_hi = m + st_map(2, 0);
+                g.st_lo = m + st_map(2, 1);
+                g.st_y = m + y_st_map();
+                g.bf_batch_stride = (int64_t)bk.n * bk.ld_n;
+                g.ld_bf = bk.ld_n;
+                g.part = p->fin_part;
+                g.part_base = p->mats_h[bk.mat_base].gpart_slot;
+                set_sym(g, bk.n);
+                gsg.add(g, true, true);
+                continue;
+            }
             const int role_a = bk.tall ? kRoleMN : kRoleKA;
             const int role_b = bk.tall ? kRoleMN : kRoleKB;
             g.a_hi = m + src_map(src, role_a, 0);
@@ -807,12 +917,16 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
             gram.add(g, bk.tall, bk.tall);
         }
         int rc;
+        if (gs_iter && ((rc = flush_set(p, ISOLOCO_PHASE_GRAM, wset, st)) ||
+                        (rc = flush_set(p, ISOLOCO_PHASE_GRAM, gsg, st))))
+            return rc;
         if ((rc = flush_set(p, ISOLOCO_PHASE_GRAM, gram, st))) return rc;
         if (p->nftiles) {
             PhaseTimer tm(p, ISOLOCO_PHASE_FINALIZE, st);
             k_gram_finalize<<<p->nftiles, 256, 0, st>>>(p->mats_d, p->ftiles, p->state, p->gpart, p->gpart_off_d,
                                                         p->gpart_sstride_d, p->nsplit_d, p->ghi, p->glo,
-                                                        p->fin_part, first ? 0 : 1, (first || full) ? nullptr : p->ypl);
+                                                        p->fin_part, first ? 0 : 1, (first || full) ? nullptr : p->ypl,
+                                                        (!first && gs_on) ? 1 : 0);
             CUDA_TRY(cudaGetLastError());
         }
         { PhaseTimer tm(p, ISOLOCO_PHASE_CONTROL, st);
@@ -862,6 +976,24 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
             const Bucket& bk = p->buckets[b];
             const CUtensorMap* m = maps + b * kMapsPerBucket;
             GemmGroup g{};
+            if (gs_on && bk.gs) {
+                if (first) continue;  // Z_1 = P_0: k_gs_init below
+                // Z_{t+1} = Z_t P_t in the first n rows of the other buffer
+                g.a_hi = m + z_map(t & 1, 0, 0);
+                g.a_lo = m + z_map(t & 1, 0, 1);
+                g.b_hi = m + p_map(kRoleKB, 0);
+                g.b_lo = m + p_map(kRoleKB, 1);
+                set_group_common(g, bk.n, bk.n, bk.n, bk.count, 1, bk.mat_base);
+                g.bucket = (int)b;
+                g.out_hi = p->xhi[dst] + bk.plane_off;
+                g.out_lo = p->xlo[dst] + bk.plane_off;
+                g.st_hi = m + z_map(dst, 2, 0);
+                g.st_lo = m + z_map(dst, 2, 1);
+                g.bf_batch_stride = (int64_t)bk.rows * bk.ld;
+                g.ld_bf = bk.ld;
+                upd.add(g, false, false, true, p_split);
+                continue;
+            }
             if (bk.tall) {
                 g.a_hi = m + src_map(src, kRoleKA, 0);
                 g.a_lo = m + src_map(src, kRoleKA, 1);
@@ -889,6 +1021,14 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
         }
         if ((rc = flush_set(p, ISOLOCO_PHASE_UPDATE, upd, st)))
             return rc;
+        if (gs_on && first) {
+            // Gram-side: A = Delta^T Delta / s^2 from the fp32 partials, Z_1 = P_0
+            PhaseTimer tm(p, ISOLOCO_PHASE_UPDATE, st);
+            k_gs_init<<<dim3(64, p->n_gs), 256, 0, st>>>(p->mats_d, p->state, p->gs_list, p->gpart, p->gpart_off_d,
+                                                         p->gpart_sstride_d, p->nsplit_d, p->anhi, p->anlo,
+                                                         p->xhi[1], p->xlo[1], p->phi, p->plo);
+            CUDA_TRY(cudaGetLastError());
+        }
     }
     return ISOLOCO_OK;
 }
@@ -959,8 +1099,55 @@ static int build_polar_graph(isoloco_plan* p, int max_iter, float tol) {
 // as every matrix is done.  With phase profiling on (events cannot sit inside the graph
 // body), or when `st` is itself being captured, iterations 1 .. max_iter are launched one
 // by one instead (empty launches once every matrix is done).
+// Gram-side matrices after the loop: Q = Delta (Z_T / s) into the ping-pong buffer that
+// does not hold Z_T (bf16 operands, three passes), and final_buf pointed at it.
+static int gs_final(isoloco_plan* p, cudaStream_t st) {
+    const CUtensorMap* maps = p->tmaps_d;
+    { PhaseTimer tm(p, ISOLOCO_PHASE_UPDATE, st);
+    k_gs_final_prep<<<dim3(64, p->n_gs), 256, 0, st>>>(p->mats_d, p->state, p->gs_list, p->xhi[0], p->xlo[0],
+                                                       p->xhi[1], p->xlo[1], p->whi, p->wlo); }
+    CUDA_TRY(cudaGetLastError());
+    LaunchSet fq;
+    init_set(fq, kEpiXSplit, kGateNone, p, Precision{0, 1, 1, 1, 0});
+    fq.p.list = nullptr;
+    fq.p.cnt = nullptr;
+    for (size_t b = 0; b < p->buckets.size(); ++b) {
+        const Bucket& bk = p->buckets[b];
+        if (!bk.gs) continue;
+        const CUtensorMap* m = maps + b * kMapsPerBucket;
+        for (int fb = 0; fb < 2; ++fb) {
+            GemmGroup g{};
+            g.a_hi = m + src_map(0, kRoleKA, 0);
+            g.a_lo = m + src_map(0, kRoleKA, 1);
+            g.b_hi = m + w_mn_map(0);
+            g.b_lo = m + w_mn_map(1);
+            set_group_common(g, bk.rows, bk.cols, bk.n, bk.count, 1, bk.mat_base);
+            g.bucket = (int)b;
+            g.gate_fb = fb + 1;
+            g.out_hi = p->xhi[1 - fb] + bk.plane_off;
+            g.out_lo = p->xlo[1 - fb] + bk.plane_off;
+            g.st_hi = m + st_map(1 - fb, 0);
+            g.st_lo = m + st_map(1 - fb, 1);
+            g.bf_batch_stride = (int64_t)bk.rows * bk.ld;
+            g.ld_bf = bk.ld;
+            fq.add(g, false, true);
+        }
+    }
+    int rc = flush_set(p, ISOLOCO_PHASE_UPDATE, fq, st);
+    if (rc) return rc;
+    { PhaseTimer tm(p, ISOLOCO_PHASE_UPDATE, st);
+    k_gs_final_flip<<<(p->n_gs + 255) / 256, 256, 0, st>>>(p->state, p->gs_list, p->n_gs); }
+    CUDA_TRY(cudaGetLastError());
+    return ISOLOCO_OK;
+}
+
 static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) {
     if (p->nmat == 0) return ISOLOCO_OK;
+    // the Gram partial slots of Gram-side matrices: iteration 0's finalize fills fewer of them
+    // than the later n x n Grams do, and the control step sums them all
+    if (p->n_gs)
+        CUDA_TRY(cudaMemsetAsync(p->fin_part + p->gs_slot_first * kPartSlots * 3, 0,
+                                 sizeof(float) * p->gs_slot_count * kPartSlots * 3, st));
     int rc = polar_iteration(p, 0, max_iter, tol, st, 0, 0);
     if (rc) return rc;
     cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
@@ -986,6 +1173,7 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
             }
         }
     }
+    if (p->n_gs && !(p->fast_steps > 0 || p->full_prec) && (rc = gs_final(p, st))) return rc;
     if (p->skip_trace) return ISOLOCO_OK;  // sigma_bar from ||Delta||_F (fast) or not used (spectral)
     { PhaseTimer tm(p, ISOLOCO_PHASE_TRACE, st, 2);
     k_trace_partial<<<p->ntchunks, 256, 0, st>>>(p->mats_d, p->tchunks, p->state, p->dhi, p->dlo, p->xhi[0],

@@ -147,7 +147,7 @@ __device__ __forceinline__ bool decode_tile(const GemmParams& p, const int* pre,
         ti.ca = st.a;
         ti.cb = st.b;
         ti.cc = st.c;
-        ti.xs = st.xscale;
+        ti.xs = p.unit_scale ? 1.f : st.xscale;
     }
     const int total_kb = (g.K + BK - 1) / BK;
     ti.kb_begin = ti.split * g.kblocks_per_split;

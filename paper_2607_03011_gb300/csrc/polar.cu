@@ -47,10 +47,11 @@ __global__ void __launch_bounds__(256) k_gram_finalize(const MatDesc* __restrict
                                                        __nv_bfloat16* __restrict__ ghi,
                                                        __nv_bfloat16* __restrict__ glo,
                                                        float* __restrict__ fin_part, int out_f16,
-                                                       __nv_bfloat16* __restrict__ ypl) {
+                                                       __nv_bfloat16* __restrict__ ypl, int skip_gs) {
     const int2 ft = ftiles[blockIdx.x];
     const int mi = ft.x;
     if (state[mi].done) return;
+    if (skip_gs && mats[mi].gs) return;  // Gram-side matrices: their later Grams are n x n products
     // ypl != null: also write Y = yb I + yc G (hi plane) for the quintic step that may follow
     const float yb = state[mi].yb, yc = state[mi].yc;
     const MatDesc md = mats[mi];
@@ -247,7 +248,8 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
     // this Gram ran a single pass (precision schedule: the step range of the matrix's kind,
     // gram_one = (standard from, to, deep from, to), and a large previous residual)
     const int g_from = md.deep ? gram_one.z : gram_one.x, g_to = md.deep ? gram_one.w : gram_one.y;
-    const bool gram_single = t > 0 && st_step >= g_from && st_step < g_to && st.resid >= kOnePassGramResid;
+    const bool gram_single =
+        !md.gs && t > 0 && st_step >= g_from && st_step < g_to && st.resid >= kOnePassGramResid;
     if (t == 0) {
         const double s2 = sqrt(sq);  // ||Delta^T Delta||_F >= sigma_max(Delta)^2
         if (!(s2 > 0.0) || !isfinite(s2)) {
@@ -519,6 +521,7 @@ __global__ void k_reset_state(MatState* state, int nmat, uint32_t* err, const Ma
     s.status = 0;
     s.lift = 1.f;
     s.lift_round = 1.f;
+    s.xs0 = 1.f;
     s.trace = 0.0;
     state[i] = s;
 }

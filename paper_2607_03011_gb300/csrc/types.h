@@ -37,6 +37,10 @@ constexpr int kMaxGroups = 8;
 constexpr int kControlThreads = 256;  // k_control block: one warp per matrix
 constexpr int kFinRows = 32;  // rows of one k_gram_finalize tile (x BN columns)
 constexpr int kSvdThreads = 1024;  // k_svd_tridiag block: one CTA per matrix
+// Tall matrices with rows >= kGramSideRatio * cols iterate on n x n matrices (Gram side):
+// X_t = Delta_n Z_t with G_t = Z_t A Z_t, A = Delta_n^T Delta_n, instead of on the rows x cols
+// iterate; a step then costs ~8 n^3 instead of 4 rows n^2 + 2 n^3.
+constexpr int kGramSideRatio = 8;
 // A Gram of the precision schedule's single-pass steps runs one pass only when the previous
 // residual ||X^T X - I||_F / sqrt(n) is at least this: one quintic step cannot bring such a
 // residual below the convergence tolerance, so the Gram cannot be the one the polish uses.
@@ -133,6 +137,7 @@ struct MatState {
     float lift;       // product of the linear coefficients of the steps taken: the factor
                       // by which a singular value near 0 (relative to the normalisation) has grown
     float lift_round; // lift when the current round of the schedule started
+    float xs0;        // 1 / s at iteration 0 (Gram-side matrices: Q = xs0 Delta Z at the end)
     double trace;     // tr(Q^T Delta)
 };
 
@@ -153,6 +158,8 @@ struct GemmParams {
     int split_on_polish;  // matrices in the polish step use both lo planes
     int gram_y;           // kEpiGram: also write Y = b I + c G for the next quintic step
     int poly_horner;      // kEpiPoly: B is Y, so P = G Y + a I (quintic steps)
+    int unit_scale;       // kEpiXSplit: no xscale (the Gram-side W = A Z, launched before the
+                          // iteration's control step has reset xscale to 1)
     MatState* state;
     uint32_t* err;
 };
@@ -171,6 +178,8 @@ struct MatDesc {
     int n_gtiles;          // groups of kPartSlots Gram partial sums of this matrix
     int deep;              // 1: near-square, polar steps from the deep schedule
     int n_tchunks;         // trace chunks of this matrix
+    int gs;                // 1: Gram-side iteration (tall with rows >= kGramSideRatio * cols)
+    int64_t gsslot;        // element offset of the matrix in the Gram-side n x n planes
 };
 
 // A contiguous range of one parameter handled by one streaming CTA.

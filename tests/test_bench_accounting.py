@@ -121,3 +121,27 @@ def test_stream_bytes():
                   "algorithmic_step": 48 * 17 + 8 * 12}
     sb = bench.stream_bytes(table, K=4, replica_bytes=2)
     assert sb["reduce"] == (4 * 2 + 4) * 17 + 4 * 17
+
+
+def test_gram_side_rule_matches_the_library():
+    """bench's Gram-side rule (rows >= ratio * cols, rows >= 2 k-blocks) is the library's."""
+    src = open(os.path.join(ROOT, "paper_2607_03011_gb300", "csrc", "types.h")).read()
+    assert int(re.search(r"constexpr int kGramSideRatio = (\d+);", src).group(1)) == bench.GRAM_SIDE_RATIO
+    api = open(os.path.join(ROOT, "paper_2607_03011_gb300", "csrc", "api.cu")).read()
+    assert "bk.tall && t.rows >= kGramSideRatio * t.cols && t.rows >= 2 * BK" in api
+    assert bench.gram_side(32000, 1024) and not bench.gram_side(2816, 1024) and not bench.gram_side(1024, 1024)
+    assert not bench.gram_side(32000, 1024, full=True) and not bench.gram_side(32000, 1024, fast=True)
+
+
+def test_algorithmic_flops_gram_side():
+    """32000 x 1024, 7 iterations, converged (quintic steps 0 .. 5, polish at 6): iteration 0's
+    Gram 2 m n^2 and six more Grams on the n x n side (W = A Z and G = Z^T W, 2 n^3 each),
+    six G^2 products, six Z P products and the final Q = Delta Z (2 m n^2)."""
+    m, n = 32000, 1024
+    fl = bench.gemm_flops([("e", m, n)], _diag([7]))
+    assert fl["gram"] == 2.0 * m * n * n + 6 * 2 * 2.0 * n ** 3
+    assert fl["poly"] == 6 * 2.0 * n ** 3
+    assert fl["update"] == 6 * 2.0 * n ** 3 + 2.0 * m * n * n
+    # the same matrix on the full-precision path iterates on the rows x cols side
+    fl = bench.gemm_flops([("e", m, n)], _diag([7]), full=True)
+    assert fl["update"] == 7 * 2.0 * m * n * n

@@ -91,6 +91,31 @@ def test_ragged_shapes_and_tails(iso):
     compare(wl, rc, th, b, upd, diag, 1.0, 0.7, 0.9)
 
 
+def test_gram_side_shapes(iso):
+    """Tall matrices with rows >= 8 cols iterate on the Gram side (n x n matrices Z with
+    G = Z^T A Z, then Q = Delta Z): odd and small n, several matrices in one bucket, a long
+    4100 x 72, a 32000 x 256, bf16 replicas, and a zero pseudo-gradient in the bucket; the
+    same inputs on the rows x cols path (full_precision = 1) as a cross-check."""
+    shapes = [("a", 200, 3), ("b", 256, 16), ("c", 1024, 48), ("c2", 1024, 48), ("d", 2048, 33), ("e", 4100, 72),
+              ("f", 32000, 256), ("z", 1024, 48), ("v", 17, 0)]
+    for dtype in ("f32", "bf16"):
+        spec = W.custom_spec(shapes, K=3, rank=2, replica_dtype=dtype, momentum_std=1e-4)
+        wl = W.make_workload(spec, seed=51, device="cuda")
+        npad = (wl.N + 63) // 64 * 64
+        reps = torch.empty((wl.K, npad), dtype=wl.replicas.dtype, device="cuda")[:, :wl.N]
+        reps.copy_(wl.replicas)
+        o, r, c = wl.table[7]
+        # Delta = 0 in the bucket (theta there made representable in the replicas' type first)
+        wl.theta[o:o + r * c] = wl.theta[o:o + r * c].to(reps.dtype).float()
+        reps[:, o:o + r * c] = wl.theta[o:o + r * c].to(reps.dtype)
+        for fp in (0, 1):
+            rc, th, b, upd, diag, _ = run_gpu(iso, wl, 1.0, 0.7, 0.9, reps=reps, full_precision=fp)
+            worst, _ = compare(wl, rc, th, b, upd, diag, 1.0, 0.7, 0.9, reps=reps)
+            o, r, c = wl.table[7]
+            assert torch.count_nonzero(upd[o:o + r * c]) == 0
+            print("Gram-side shapes", dtype, "rows x cols path" if fp else "Gram side", worst)
+
+
 def test_split_k_gram(iso):
     """Tall-skinny matrices whose Gram takes several split-K passes."""
     spec = W.custom_spec([("t", 6000, 64), ("u", 64, 5000), ("v", 100, 0)], K=2, rank=3)
