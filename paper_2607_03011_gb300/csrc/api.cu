@@ -139,6 +139,7 @@ struct isoloco_plan {
     std::vector<MatDesc> mats_h;
     std::vector<Bucket> buckets;
     int nmat = 0, nchunks = 0, nftiles = 0, ntchunks = 0;
+    int nftiles_reg = 0;  // finalize tiles of matrices that are not Gram-side
     int64_t plane_elems = 0, gplane_elems = 0, gpart_elems = 0, n1d = 0;
     // device workspace
     std::vector<void*> allocs;
@@ -525,6 +526,7 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
     p->gplane_elems = gplane;
     p->gpart_elems = gpart;
     p->nftiles = (int)ftiles.size();
+    for (const int2& f : ftiles) p->nftiles_reg += p->mats_h[f.x].gs ? 0 : 1;
     p->ntchunks = (int)tchunks.size();
 
     // --- streaming chunks (table order) and the 1-D workspace
@@ -921,7 +923,8 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
                         (rc = flush_set(p, ISOLOCO_PHASE_GRAM, gsg, st))))
             return rc;
         if ((rc = flush_set(p, ISOLOCO_PHASE_GRAM, gram, st))) return rc;
-        if (p->nftiles) {
+        // after iteration 0 the Gram-side matrices need no finalize: skip an empty launch
+        if (p->nftiles && (first || !gs_on || p->nftiles_reg > 0)) {
             PhaseTimer tm(p, ISOLOCO_PHASE_FINALIZE, st);
             k_gram_finalize<<<p->nftiles, 256, 0, st>>>(p->mats_d, p->ftiles, p->state, p->gpart, p->gpart_off_d,
                                                         p->gpart_sstride_d, p->nsplit_d, p->ghi, p->glo,
