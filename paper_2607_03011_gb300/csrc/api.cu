@@ -153,6 +153,7 @@ struct isoloco_plan {
     __nv_bfloat16 *anhi = nullptr, *anlo = nullptr, *whi = nullptr, *wlo = nullptr;
     int* gs_list = nullptr;
     int n_gs = 0;
+    int gs_blocks = 1;  // 256-thread blocks per Gram-side matrix in k_gs_init / k_gs_final_prep (one per 256 elements)
     int64_t gs_slot_first = 0, gs_slot_count = 0;  // Gram partial slots of the Gram-side matrices
     float* gpart = nullptr;
     float* d1d = nullptr;
@@ -522,6 +523,8 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
     }
     p->nmat = (int)p->mats_h.size();
     p->n_gs = (int)gs_mats.size();
+    for (int mi : gs_mats)
+        p->gs_blocks = std::max<int>(p->gs_blocks, (int)std::min<int64_t>(65535, ((int64_t)p->mats_h[mi].n * p->mats_h[mi].n + 255) / 256));
     p->plane_elems = plane;
     p->gplane_elems = gplane;
     p->gpart_elems = gpart;
@@ -1027,7 +1030,7 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
         if (gs_on && first) {
             // Gram-side: A = Delta^T Delta / s^2 from the fp32 partials, Z_1 = P_0
             PhaseTimer tm(p, ISOLOCO_PHASE_UPDATE, st);
-            k_gs_init<<<dim3(64, p->n_gs), 256, 0, st>>>(p->mats_d, p->state, p->gs_list, p->gpart, p->gpart_off_d,
+            k_gs_init<<<dim3(p->gs_blocks, p->n_gs), 256, 0, st>>>(p->mats_d, p->state, p->gs_list, p->gpart, p->gpart_off_d,
                                                          p->gpart_sstride_d, p->nsplit_d, p->anhi, p->anlo,
                                                          p->xhi[1], p->xlo[1], p->phi, p->plo);
             CUDA_TRY(cudaGetLastError());
@@ -1107,7 +1110,7 @@ static int build_polar_graph(isoloco_plan* p, int max_iter, float tol) {
 static int gs_final(isoloco_plan* p, cudaStream_t st) {
     const CUtensorMap* maps = p->tmaps_d;
     { PhaseTimer tm(p, ISOLOCO_PHASE_UPDATE, st);
-    k_gs_final_prep<<<dim3(64, p->n_gs), 256, 0, st>>>(p->mats_d, p->state, p->gs_list, p->xhi[0], p->xlo[0],
+    k_gs_final_prep<<<dim3(p->gs_blocks, p->n_gs), 256, 0, st>>>(p->mats_d, p->state, p->gs_list, p->xhi[0], p->xlo[0],
                                                        p->xhi[1], p->xlo[1], p->whi, p->wlo); }
     CUDA_TRY(cudaGetLastError());
     LaunchSet fq;

@@ -19,7 +19,8 @@
 
 namespace isoloco {
 
-// grid (x: blocks over the n x n elements, y: Gram-side matrices listed in gs_list).
+// grid (x: 256-element blocks of the n x n matrix, grid-stride beyond 65535 blocks; y: the
+// Gram-side matrices listed in gs_list).
 __global__ void __launch_bounds__(256) k_gs_init(const MatDesc* __restrict__ mats, MatState* __restrict__ state,
                                                  const int* __restrict__ gs_list,
                                                  const float* __restrict__ gpart,
