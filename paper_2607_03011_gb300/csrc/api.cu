@@ -42,7 +42,7 @@ __global__ void k_gs_final_prep(const MatDesc*, const MatState*, const int*, con
 __global__ void k_gs_final_flip(MatState*, const int*, int);
 __global__ void k_control(const MatDesc*, int, MatState*, const float*, int, int, float, uint32_t*, const int*,
                           const int*, int, int*, int*, int*, int*, cudaGraphConditionalHandle, int, long long*,
-                          int, int*, int4);
+                          int, int*, int4, int4);
 __global__ void k_trace_partial(const MatDesc*, const int4*, const MatState*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, double*);
@@ -813,6 +813,12 @@ static int gp_one(const isoloco_plan* p, int kind, int end) {
     return end ? p->gp_to[kind] : p->gp_from[kind];
 }
 
+// The same for the update's single-pass steps.
+static int up_one(const isoloco_plan* p, int kind, int end) {
+    if (p->fast_steps > 0 || p->full_prec) return 0;
+    return end ? p->up_to[kind] : p->up_from[kind];
+}
+
 // Single-pass step range of a group (precision schedule; none in the full-precision paths).
 static void set_one_pass(const isoloco_plan* p, GemmGroup& g, const Bucket& bk, bool update) {
     const int kind = (std::abs(bk.rows - bk.cols) * 16 < bk.n) ? 1 : 0;  // deep schedule (as MatDesc::deep)
@@ -940,7 +946,8 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
                                       p->bucket_first_d, p->bucket_count_d, (int)p->buckets.size(), p->list_gram,
                                       p->cnt_gram, p->list_step, p->cnt_step, cond, set_cond, p->loopc,
                                       p->fast_steps, p->counters + kLaunchCounters,
-                                      make_int4(gp_one(p, 0, 0), gp_one(p, 0, 1), gp_one(p, 1, 0), gp_one(p, 1, 1))); }
+                                      make_int4(gp_one(p, 0, 0), gp_one(p, 0, 1), gp_one(p, 1, 0), gp_one(p, 1, 1)),
+                                      make_int4(up_one(p, 0, 0), up_one(p, 0, 1), up_one(p, 1, 0), up_one(p, 1, 1))); }
         CUDA_TRY(cudaGetLastError());
         // ---- P = a I + b G + c G^2
         LaunchSet poly;

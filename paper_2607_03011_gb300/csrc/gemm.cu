@@ -75,6 +75,8 @@ struct TileInfo {
     int gi, b, tile, split, m0, n0, mat, kb_begin, kb_end;
     bool run_mma, a_split, b_split;
     bool horner;     // kEpiPoly: P = acc + a I (the MMA computed G Y); else P = a I + b G + c acc
+    bool hi_only;    // write the hi plane only (a single-pass Gram's G; an update's X whose lo
+                     // plane no later step reads)
     float ca, cb, cc, xs;
     float yb, yc;    // kEpiGram with p.gram_y: Y = yb I + yc G for the next quintic step
 };
@@ -120,6 +122,7 @@ __device__ __forceinline__ bool decode_tile(const GemmParams& p, const int* pre,
     ti.b_split = g.b_split != 0;
     ti.ca = 0.f, ti.cb = 0.f, ti.cc = 1.f, ti.xs = 1.f, ti.yb = 0.f, ti.yc = 0.f;
     ti.horner = false;
+    ti.hi_only = false;
     if (g.gate_fb && p.state[ti.mat].final_buf != g.gate_fb - 1) return false;
     if (p.gate != kGateNone) {
         const MatState& st = p.state[ti.mat];
@@ -142,8 +145,12 @@ __device__ __forceinline__ bool decode_tile(const GemmParams& p, const int* pre,
         // feeds the final polish, which nothing corrects afterwards, so it keeps its passes.
         const int k = (p.epi == kEpiGram) ? st.step : st.step - 1;
         if (k >= g.one_from && k < g.one_to &&
-            ((p.epi == kEpiGram) ? (st.step > 0 && st.resid >= kOnePassGramResid) : st.mode == 1))
+            ((p.epi == kEpiGram) ? (st.step > 0 && st.resid >= kOnePassGramResid) : st.mode == 1)) {
             ti.a_split = ti.b_split = false;
+            // a single-pass Gram never feeds the polish and its polynomial reads G's hi only
+            if (p.epi == kEpiGram) ti.hi_only = true;
+        }
+        if (p.epi == kEpiXSplit && p.gate == kGateStep && st.mode == 1 && st.x_hi_only) ti.hi_only = true;
         ti.ca = st.a;
         ti.cb = st.b;
         ti.cc = st.c;
@@ -252,7 +259,7 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
     // planes written: hi, lo (if kept; not for a Horner-form P, whose lo plane nobody reads),
     // and for the Gram with p.gram_y the plane Y = yb I + yc G (hi only)
     const bool write_y = (p.epi == kEpiGram && p.gram_y);
-    const int nplanes = (ti.horner || g.st_lo == nullptr) ? 1 : 2;
+    const int nplanes = (ti.horner || ti.hi_only || g.st_lo == nullptr) ? 1 : 2;
     float s_sq = 0.f, s_tr = 0.f, s_dev = 0.f;
     for (int c32 = half * (BN / 64); c32 < (half + 1) * (BN / 64); ++c32) {
         const int col0 = n0 + c32 * 32;

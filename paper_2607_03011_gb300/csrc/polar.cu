@@ -208,7 +208,8 @@ __device__ __forceinline__ const float* sched_row(bool deep, int step) {
 // Decision for matrix mi, taken by one warp.  t: iteration index (0 = first Gram of Delta).
 __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatState* __restrict__ state,
                                const float* __restrict__ fin_part, int t, int max_iter, float tol,
-                               uint32_t* __restrict__ err, int lane, int fast_steps, int4 gram_one) {
+                               uint32_t* __restrict__ err, int lane, int fast_steps, int4 gram_one,
+                               int4 upd_one) {
     MatState& st = state[mi];
     if (st.done) {
         if (lane == 0) st.mode = 0;
@@ -325,6 +326,13 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
     } else {
         const float* q = sched_row(md.deep != 0, st_step);
         st.mode = 1;
+        // the X this step writes needs no lo plane when the next Gram and update run single-pass
+        // (next step in both ranges, this residual large: the next test cannot pass, no
+        // polish) and the next iteration cannot hit max_iter (Q = X would be final)
+        const int kn = st_step + 1;
+        const int u_from = md.deep ? upd_one.z : upd_one.x, u_to = md.deep ? upd_one.w : upd_one.y;
+        st.x_hi_only = (!md.gs && kn >= g_from && kn < g_to && kn >= u_from && kn < u_to &&
+                        d >= kOnePassGramResid && st_iters + 2 <= max_iter) ? 1 : 0;
         if (st_step == 0 || at_round_end) st.lift_round = lift;  // this step starts a round
         st.lift = lift * q[0];
         st.a = q[0];
@@ -358,11 +366,12 @@ __global__ void __launch_bounds__(kControlThreads) k_control(const MatDesc* __re
                                                              int* __restrict__ list_step, int* __restrict__ cnt_step,
                                                              cudaGraphConditionalHandle cond, int set_cond,
                                                              long long* __restrict__ loopc, int fast_steps,
-                                                             int* __restrict__ ticket, int4 gram_one) {
+                                                             int* __restrict__ ticket, int4 gram_one,
+                                                             int4 upd_one) {
     constexpr int kWarps = kControlThreads / 32;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     for (int mi = blockIdx.x * kWarps + warp; mi < nmat; mi += gridDim.x * kWarps) {
-        control_matrix(mats, mi, state, fin_part, t, max_iter, tol, err, lane, fast_steps, gram_one);
+        control_matrix(mats, mi, state, fin_part, t, max_iter, tol, err, lane, fast_steps, gram_one, upd_one);
         __syncwarp();
     }
     __threadfence();
@@ -522,6 +531,7 @@ __global__ void k_reset_state(MatState* state, int nmat, uint32_t* err, const Ma
     s.lift = 1.f;
     s.lift_round = 1.f;
     s.xs0 = 1.f;
+    s.x_hi_only = 0;
     s.trace = 0.0;
     state[i] = s;
 }

@@ -138,6 +138,8 @@ struct MatState {
                       // by which a singular value near 0 (relative to the normalisation) has grown
     float lift_round; // lift when the current round of the schedule started
     float xs0;        // 1 / s at iteration 0 (Gram-side matrices: Q = xs0 Delta Z at the end)
+    int x_hi_only;    // this step's update writes X's hi plane only: the next Gram and update
+                      // run single-pass and the next iteration cannot end the polar loop
     double trace;     // tr(Q^T Delta)
 };
 
