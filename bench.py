@@ -275,7 +275,7 @@ DTYPE_ISO = "f32 streaming; polar GEMMs as bf16/fp16 hi+lo split passes, f32 acc
 # shape buckets captured one at a time and summed (profiles/k_gemm_split_dram_llama_180m_buckets.md).
 GEMM_TRAFFIC = {
     ("llama_180m_k8", 0, 0): {
-        "bytes_per_step": 24.95e9,
+        "bytes_per_step": 23.67e9,
         "note": "dram__bytes_read.sum + dram__bytes_write.sum of every k_gemm_split launch of one step, "
                 "captured per shape bucket (square48, tall12, wide24, embed2) and summed; same unit as "
                 "achieved (per step over all GEMM launches)"},
