@@ -275,7 +275,7 @@ DTYPE_ISO = "f32 streaming; polar GEMMs as bf16/fp16 hi+lo split passes, f32 acc
 # shape buckets captured one at a time and summed (profiles/k_gemm_split_dram_llama_180m_buckets.md).
 GEMM_TRAFFIC = {
     ("llama_180m_k8", 0, 0): {
-        "bytes_per_step": 23.67e9,
+        "bytes_per_step": 24.45e9,
         "note": "dram__bytes_read.sum + dram__bytes_write.sum of every k_gemm_split launch of one step, "
                 "captured per shape bucket (square48, tall12, wide24, embed2) and summed; same unit as "
                 "achieved (per step over all GEMM launches)"},
@@ -687,9 +687,11 @@ def main():
         "apply": {"achieved": gbs("apply", sb["apply"]), "peak": hbm, "unit": "GB/s",
                   "frac": gbs("apply", sb["apply"]) / hbm, "bytes_per_launch": sb["apply"],
                   "ms_per_step": prof["apply"][0] / args.steps},
-        "trace": {"achieved": gbs("trace", sb["trace"]), "peak": hbm, "unit": "GB/s",
-                  "frac": gbs("trace", sb["trace"]) / hbm, "bytes_per_launch": sb["trace"],
-                  "ms_per_step": prof["trace"][0] / args.steps},
+        "trace": {"ms_per_step": prof["trace"][0] / args.steps, "fused": True,
+                  "note": "tr(Q^T Delta) is summed in the epilogue of the GEMM that writes each matrix's final "
+                          "Q (the polish update; the Gram side's Q = Delta Z), which reads Delta's planes "
+                          "(4 B per matrix element) there; the trace pass itself only covers matrices with no "
+                          "such GEMM (not converged) and is launch cost otherwise"},
         "peak_source": f"{peak_src} hbm_gbs",
     }
     phases_ms = {k: round(v[0] / args.steps, 4) for k, v in prof.items() if v[1]}

@@ -37,16 +37,16 @@ __global__ void k_gram_finalize(const MatDesc*, const int2*, const MatState*, co
 __global__ void k_gs_init(const MatDesc*, MatState*, const int*, const float*, const int64_t*, const int64_t*,
                           const int*, __nv_bfloat16*, __nv_bfloat16*, __nv_bfloat16*, __nv_bfloat16*,
                           const __nv_bfloat16*, const __nv_bfloat16*);
-__global__ void k_gs_final_prep(const MatDesc*, const MatState*, const int*, const __nv_bfloat16*, const __nv_bfloat16*,
+__global__ void k_gs_final_prep(const MatDesc*, MatState*, const int*, const __nv_bfloat16*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, __nv_bfloat16*, __nv_bfloat16*);
 __global__ void k_gs_final_flip(MatState*, const int*, int);
 __global__ void k_control(const MatDesc*, int, MatState*, const float*, int, int, float, uint32_t*, const int*,
                           const int*, int, int*, int*, int*, int*, cudaGraphConditionalHandle, int, long long*,
                           int, int*, int4, int4);
-__global__ void k_trace_partial(const MatDesc*, const int4*, const MatState*, const __nv_bfloat16*,
+__global__ void k_trace_partial(const MatDesc*, const int4*, int, const MatState*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, double*);
-__global__ void k_trace_final(const MatDesc*, int, MatState*, const double*);
+__global__ void k_trace_final(const MatDesc*, int, MatState*, const double*, const double*);
 __global__ void k_reset_state(MatState*, int, uint32_t*, const MatDesc*, const int*, const int*, int, int*, int*,
                               int*, int);
 __global__ void k_reduce(const Chunk*, const MatDesc*, ReplicaPtrs, int, int, const float*, float,
@@ -122,6 +122,8 @@ struct Bucket {
     int splits;
     bool gs;         // Gram-side iteration (gramside.cu)
     int64_t gs_off;  // offset of the bucket in the Gram-side n x n planes (A, W)
+    int64_t tf_base; // first fused-trace slot of the bucket (GemmGroup::tf_part)
+    int tf_tiles;    // output tiles of one matrix (rows x cols)
 };
 
 }  // namespace isoloco
@@ -160,6 +162,8 @@ struct isoloco_plan {
     float* fin_part = nullptr;
     int2* ftiles = nullptr;
     double* tpart = nullptr;
+    double* tfpart = nullptr;  // fused-trace slots (GemmGroup::tf_part), tf_slots doubles
+    int64_t tf_slots = 0;
     int4* tchunks = nullptr;
     MatState* state = nullptr;
     MatDesc* mats_d = nullptr;
@@ -435,7 +439,7 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
     }
     // matrices ordered bucket by bucket so each bucket's slots are contiguous
     std::vector<int> mat_of_param(n_params, -1);
-    int64_t plane = 0, gplane = 0, gpart = 0, fin = 0, tr = 0;
+    int64_t plane = 0, gplane = 0, gpart = 0, fin = 0, tr = 0, tf = 0;
     std::vector<int2> ftiles;
     std::vector<int4> tchunks;
     std::vector<int64_t> gpoff, gpss;
@@ -450,6 +454,8 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         bk.plane_off = plane;
         bk.gplane_off = gplane;
         bk.gpart_off = gpart;
+        bk.tf_base = tf;
+        bk.tf_tiles = ((bk.rows + kTileM - 1) / kTileM) * ((bk.cols + BN - 1) / BN);
         // split-K for the Gram when the bucket has few output tiles
         const int tiles = sym_tiles(bk.n) * bk.count;
         const int kdim = bk.tall ? bk.rows : bk.cols;
@@ -499,6 +505,9 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
             md.gsslot = bk.gs_off + j * g_elems;
             if (bk.gs) gs_mats.push_back((int)p->mats_h.size());
             md.trace_part = tr;
+            md.tf_part = tf;
+            md.tf_slots = bk.tf_tiles * kPartSlots;
+            tf += md.tf_slots;
             const int rows_per = std::max(1, kTraceChunkElems / bk.cols);
             md.n_tchunks = (bk.rows + rows_per - 1) / rows_per;
             const int mi = (int)p->mats_h.size();
@@ -531,6 +540,7 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
     p->nftiles = (int)ftiles.size();
     for (const int2& f : ftiles) p->nftiles_reg += p->mats_h[f.x].gs ? 0 : 1;
     p->ntchunks = (int)tchunks.size();
+    p->tf_slots = tf;
 
     // --- streaming chunks (table order) and the 1-D workspace
     std::vector<Chunk> chunks;
@@ -566,6 +576,7 @@ static int build_plan(isoloco_plan* p, const isoloco_param_t* table, int n_param
         (rc = dalloc(p, &p->plo, gplane)) || (rc = dalloc(p, &p->ypl, gplane)) || (rc = dalloc(p, &p->gpart, gpart)) || (rc = dalloc(p, &p->d1d, d1)) ||
         (rc = dalloc(p, &p->fin_part, 3 * kPartSlots * fin)) || (rc = dalloc(p, &p->ftiles, (int64_t)ftiles.size())) ||
         (rc = dalloc(p, &p->tpart, tr)) || (rc = dalloc(p, &p->tchunks, tr)) ||
+        (rc = dalloc(p, &p->tfpart, std::max<int64_t>(1, tf))) ||
         (rc = dalloc(p, &p->state, p->nmat)) || (rc = dalloc(p, &p->mats_d, p->nmat)) ||
         (rc = dalloc(p, &p->gpart_off_d, p->nmat)) || (rc = dalloc(p, &p->gpart_sstride_d, p->nmat)) ||
         (rc = dalloc(p, &p->nsplit_d, p->nmat)) || (rc = dalloc(p, &p->chunks_d, p->nchunks)) ||
@@ -1027,6 +1038,10 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
             g.bf_batch_stride = (int64_t)bk.rows * bk.ld;
             g.ld_bf = bk.ld;
             set_one_pass(p, g, bk, true);
+            // the polish writes the final Q: its epilogue also sums tr(Q^T Delta)
+            g.d_hi = p->dhi + bk.plane_off;
+            g.d_lo = p->dlo + bk.plane_off;
+            g.tf_part = p->tfpart + bk.tf_base;
             if (bk.tall)
                 upd.add(g, false, false, true, p_split);
             else
@@ -1143,6 +1158,9 @@ static int gs_final(isoloco_plan* p, cudaStream_t st) {
             g.st_lo = m + st_map(1 - fb, 1);
             g.bf_batch_stride = (int64_t)bk.rows * bk.ld;
             g.ld_bf = bk.ld;
+            g.d_hi = p->dhi + bk.plane_off;  // Q is final: tr(Q^T Delta) in the epilogue
+            g.d_lo = p->dlo + bk.plane_off;
+            g.tf_part = p->tfpart + bk.tf_base;
             fq.add(g, false, true);
         }
     }
@@ -1189,10 +1207,13 @@ static int run_polar(isoloco_plan* p, int max_iter, float tol, cudaStream_t st) 
     if (p->n_gs && !(p->fast_steps > 0 || p->full_prec) && (rc = gs_final(p, st))) return rc;
     if (p->skip_trace) return ISOLOCO_OK;  // sigma_bar from ||Delta||_F (fast) or not used (spectral)
     { PhaseTimer tm(p, ISOLOCO_PHASE_TRACE, st, 2);
-    k_trace_partial<<<p->ntchunks, 256, 0, st>>>(p->mats_d, p->tchunks, p->state, p->dhi, p->dlo, p->xhi[0],
+    // windows of 32 chunks: converged matrices' chunks (summed in their GEMM epilogue) cost a
+    // flag read each
+    k_trace_partial<<<std::max(1, std::min((p->ntchunks + 31) / 32, 4 * p->num_sms)), 256, 0, st>>>(
+        p->mats_d, p->tchunks, p->ntchunks, p->state, p->dhi, p->dlo, p->xhi[0],
                                                  p->xlo[0], p->xhi[1], p->xlo[1], p->tpart);
     CUDA_TRY(cudaGetLastError());
-    k_trace_final<<<(p->nmat + 7) / 8, 256, 0, st>>>(p->mats_d, p->nmat, p->state, p->tpart); }
+    k_trace_final<<<p->nmat, 256, 0, st>>>(p->mats_d, p->nmat, p->state, p->tpart, p->tfpart); }
     CUDA_TRY(cudaGetLastError());
     return ISOLOCO_OK;
 }

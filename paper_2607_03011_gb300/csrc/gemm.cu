@@ -77,6 +77,7 @@ struct TileInfo {
     bool horner;     // kEpiPoly: P = acc + a I (the MMA computed G Y); else P = a I + b G + c acc
     bool hi_only;    // write the hi plane only (a single-pass Gram's G; an update's X whose lo
                      // plane no later step reads)
+    bool trace;      // the output is a matrix's final Q: also sum Q o Delta (GemmGroup::d_hi)
     float ca, cb, cc, xs;
     float yb, yc;    // kEpiGram with p.gram_y: Y = yb I + yc G for the next quintic step
 };
@@ -123,6 +124,9 @@ __device__ __forceinline__ bool decode_tile(const GemmParams& p, const int* pre,
     ti.ca = 0.f, ti.cb = 0.f, ti.cc = 1.f, ti.xs = 1.f, ti.yb = 0.f, ti.yc = 0.f;
     ti.horner = false;
     ti.hi_only = false;
+    // the final Q of a matrix: the polish update, or an ungated launch (the Gram side's
+    // Q = Delta Z, which writes only matrices that have a Q)
+    ti.trace = p.epi == kEpiXSplit && g.d_hi != nullptr && p.gate == kGateNone;
     if (g.gate_fb && p.state[ti.mat].final_buf != g.gate_fb - 1) return false;
     if (p.gate != kGateNone) {
         const MatState& st = p.state[ti.mat];
@@ -139,6 +143,7 @@ __device__ __forceinline__ bool decode_tile(const GemmParams& p, const int* pre,
             if (p.epi == kEpiPoly && st.mode == 2) ti.run_mma = false;  // cubic polish: no G^2
             ti.horner = (p.epi == kEpiPoly && p.poly_horner && st.mode == 1);
             if (p.split_on_polish && st.mode == 2) ti.a_split = ti.b_split = true;  // final step: 3 passes
+            ti.trace = p.epi == kEpiXSplit && g.d_hi != nullptr && p.gate == kGateStep && st.mode == 2;
         }
         // precision schedule: single-pass steps.  A Gram only after iteration 0's and only
         // while the last residual is large (>= kOnePassGramResid): a Gram whose test can pass
@@ -261,6 +266,7 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
     const bool write_y = (p.epi == kEpiGram && p.gram_y);
     const int nplanes = (ti.horner || ti.hi_only || g.st_lo == nullptr) ? 1 : 2;
     float s_sq = 0.f, s_tr = 0.f, s_dev = 0.f;
+    float s_tq = 0.f;  // share of tr(Q^T Delta) (ti.trace)
     for (int c32 = half * (BN / 64); c32 < (half + 1) * (BN / 64); ++c32) {
         const int col0 = n0 + c32 * 32;
         if (col0 >= g.N) break;
@@ -316,6 +322,36 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
         } else if (p.epi == kEpiXSplit) {
 #pragma unroll
             for (int j = 0; j < 32; ++j) v[j] *= xs;
+            if (ti.trace && row_ok) {
+                // this row's share of tr(Q^T Delta): Q in fp32 as stored (before its split
+                // into planes), Delta from its bf16 hi/lo planes
+                const int64_t doff = b * g.bf_batch_stride + static_cast<int64_t>(row) * g.ld_bf + col0;
+                const uint16_t* dh = reinterpret_cast<const uint16_t*>(g.d_hi) + doff;
+                const uint16_t* dl = reinterpret_cast<const uint16_t*>(g.d_lo) + doff;
+                if (nvalid == 32) {
+                    const uint4* h4 = reinterpret_cast<const uint4*>(dh);
+                    const uint4* l4 = reinterpret_cast<const uint4*>(dl);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const uint4 hh = h4[q], ll = l4[q];
+                        const uint32_t hw[4] = {hh.x, hh.y, hh.z, hh.w};
+                        const uint32_t lw[4] = {ll.x, ll.y, ll.z, ll.w};
+#pragma unroll
+                        for (int w = 0; w < 4; ++w) {
+                            const float d0 = __uint_as_float(hw[w] << 16) + __uint_as_float(lw[w] << 16);
+                            const float d1 = __uint_as_float(hw[w] & 0xFFFF0000u) + __uint_as_float(lw[w] & 0xFFFF0000u);
+                            s_tq = fmaf(v[8 * q + 2 * w], d0, s_tq);
+                            s_tq = fmaf(v[8 * q + 2 * w + 1], d1, s_tq);
+                        }
+                    }
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        if (j < nvalid)
+                            s_tq = fmaf(v[j], __uint_as_float(static_cast<uint32_t>(dh[j]) << 16) +
+                                                  __uint_as_float(static_cast<uint32_t>(dl[j]) << 16), s_tq);
+                }
+            }
         }
         if (gram_fused && row_ok && sym && !diag && nvalid == 32) {
             // block strictly above the diagonal: every entry counts twice and (G - I) = G
@@ -376,6 +412,15 @@ __device__ __forceinline__ void tile_epilogue(const GemmParams& p, const TileInf
             }
             stage_store_block(lw, g.st_y, stg, sseq, diag, sym, lane, col0, row_base, b);
         }
+    }
+    if (ti.trace) {
+        // fixed-order warp reduction into this warp's slot of the tile (every slot of every
+        // tile of the matrix is written by the launch that writes its Q)
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) s_tq += __shfl_xor_sync(0xffffffffu, s_tq, o);
+        if (lane == 0)
+            g.tf_part[(static_cast<int64_t>(b) * (g.tiles_m * g.tiles_n) + ti.tile) * kPartSlots +
+                      static_cast<int>(crank) * kEpiWarps + half * 4 + eg] = static_cast<double>(s_tq);
     }
     if (gram_fused) {
         // fixed-order warp reduction; each epilogue warp owns one of the tile's kEpiWarps slots

@@ -61,7 +61,7 @@ __global__ void __launch_bounds__(256) k_gs_init(const MatDesc* __restrict__ mat
 // (1 / s) Z_T (Z_T: fp16 hi/lo in the first n rows of ping-pong buffer final_buf) -> bf16
 // hi/lo planes w, the B operand of the final product.
 __global__ void __launch_bounds__(256) k_gs_final_prep(const MatDesc* __restrict__ mats,
-                                                       const MatState* __restrict__ state,
+                                                       MatState* __restrict__ state,
                                                        const int* __restrict__ gs_list,
                                                        const __nv_bfloat16* __restrict__ xh0,
                                                        const __nv_bfloat16* __restrict__ xl0,
@@ -71,6 +71,8 @@ __global__ void __launch_bounds__(256) k_gs_final_prep(const MatDesc* __restrict
     const int mi = gs_list[blockIdx.y];
     const int fb = state[mi].final_buf;
     if (fb > 1) return;
+    // the final product Q = Delta (Z / s) sums tr(Q^T Delta) in its epilogue
+    if (blockIdx.x == 0 && threadIdx.x == 0) state[mi].trace_fused = 1;
     const MatDesc md = mats[mi];
     const int n = md.n;
     const float xs0 = state[mi].xs0;

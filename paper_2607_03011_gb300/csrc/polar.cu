@@ -311,6 +311,7 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
         // (Not from a single-pass Gram: the matrix then takes one more quintic step, and the
         // Gram after it, with a small residual, keeps its passes.)
         st.mode = 2;
+        st.trace_fused = md.gs ? 0 : 1;  // the polish update's epilogue sums tr(Q^T Delta)
         st.a = 1.5f;
         st.b = static_cast<float>(-0.5 * gscale);
         st.c = 0.f;
@@ -419,10 +420,13 @@ __global__ void __launch_bounds__(kControlThreads) k_control(const MatDesc* __re
     }
 }
 
-// grid: one block (256 threads) per (matrix, row chunk) listed in `tchunks`
-// (x = matrix, y = first row, z = rows, w = chunk index within the matrix).  Q comes from the final ping-pong buffer.
+// Blocks of 256 threads take windows of 32 (matrix, row chunk) entries of `tchunks` (x =
+// matrix, y = first row, z = rows, w = chunk index within the matrix): the first warp checks
+// one entry per lane, and the block then sums the window's chunks whose matrix still needs its
+// trace (no GEMM epilogue summed it: trace_fused), one chunk at a time.  Q comes from the final ping-pong
+// buffer.
 __global__ void __launch_bounds__(256) k_trace_partial(const MatDesc* __restrict__ mats,
-                                                       const int4* __restrict__ tchunks,
+                                                       const int4* __restrict__ tchunks, int ntchunks,
                                                        const MatState* __restrict__ state,
                                                        const __nv_bfloat16* __restrict__ dhi,
                                                        const __nv_bfloat16* __restrict__ dlo,
@@ -431,76 +435,112 @@ __global__ void __launch_bounds__(256) k_trace_partial(const MatDesc* __restrict
                                                        const __nv_bfloat16* __restrict__ x1hi,
                                                        const __nv_bfloat16* __restrict__ x1lo,
                                                        double* __restrict__ tpart) {
-    const int4 tc = tchunks[blockIdx.x];
-    const MatDesc md = mats[tc.x];
-    const int fb = state[tc.x].final_buf;
-    double acc = 0.0;
-    if (fb == 0 || fb == 1) {
-        const __nv_bfloat16* qh = (fb == 0 ? x0hi : x1hi) + md.slot;
-        const __nv_bfloat16* ql = (fb == 0 ? x0lo : x1lo) + md.slot;
-        const __nv_bfloat16* dh = dhi + md.slot;
-        const __nv_bfloat16* dl = dlo + md.slot;
-        float part = 0.f;
-        if (md.ld == md.cols && (md.cols & 7) == 0) {
-            // contiguous rows: 8 elements per 16-byte load of each plane
-            const int64_t base = static_cast<int64_t>(tc.y) * md.cols;
-            const int nv = tc.z * md.cols / 8;
-            const uint4* a4 = reinterpret_cast<const uint4*>(qh + base);
-            const uint4* b4 = reinterpret_cast<const uint4*>(ql + base);
-            const uint4* c4 = reinterpret_cast<const uint4*>(dh + base);
-            const uint4* d4 = reinterpret_cast<const uint4*>(dl + base);
-            for (int v = threadIdx.x; v < nv; v += blockDim.x) {
-                const uint4 a = a4[v], bq = b4[v], c = c4[v], d = d4[v];
-                const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, bw[4] = {bq.x, bq.y, bq.z, bq.w};
-                const uint32_t cw[4] = {c.x, c.y, c.z, c.w}, dw[4] = {d.x, d.y, d.z, d.w};
-#pragma unroll
-                for (int w = 0; w < 4; ++w) {
-                    const float q0 = dec16(aw[w] & 0xFFFFu, true) + dec16(bw[w] & 0xFFFFu, true);
-                    const float q1 = dec16(aw[w] >> 16, true) + dec16(bw[w] >> 16, true);
-                    const float d0 = __uint_as_float(cw[w] << 16) + __uint_as_float(dw[w] << 16);
-                    const float d1 = __uint_as_float(cw[w] & 0xFFFF0000u) + __uint_as_float(dw[w] & 0xFFFF0000u);
-                    part = fmaf(q0, d0, part);
-                    part = fmaf(q1, d1, part);
-                }
-            }
-        } else {
-            for (int r = tc.y; r < tc.y + tc.z; ++r) {
-                for (int c = threadIdx.x; c < md.cols; c += blockDim.x) {
-                    const int64_t idx = static_cast<int64_t>(r) * md.ld + c;
-                    const float q = dec16(__bfloat16_as_ushort(qh[idx]), true) +
-                                    dec16(__bfloat16_as_ushort(ql[idx]), true);
-                    const float dv = __bfloat162float(dh[idx]) + __bfloat162float(dl[idx]);
-                    part = fmaf(q, dv, part);
-                }
-            }
-        }
-        acc = static_cast<double>(part);
-    }
     __shared__ double red[8];
-    acc = warp_sum_d(acc);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        double s = 0.0;
-        for (int i = 0; i < (int)(blockDim.x >> 5); ++i) s += red[i];
-        tpart[md.trace_part + tc.w] = s;
+    __shared__ int todo[32];
+    __shared__ int ntodo;
+    for (int base = blockIdx.x * 32; base < ntchunks; base += gridDim.x * 32) {
+        if (threadIdx.x < 32) {
+            const int mine = base + static_cast<int>(threadIdx.x);
+            const bool need = mine < ntchunks && !state[tchunks[mine].x].trace_fused;
+            const uint32_t m = __ballot_sync(0xffffffffu, need);
+            if (need) todo[__popc(m & ((1u << threadIdx.x) - 1u))] = mine;
+            if (threadIdx.x == 0) ntodo = __popc(m);
+        }
+        __syncthreads();
+        const int cnt = ntodo;
+        for (int k = 0; k < cnt; ++k) {
+            const int4 tc = tchunks[todo[k]];
+            const MatDesc md = mats[tc.x];
+            const int fb = state[tc.x].final_buf;
+            double acc = 0.0;
+            if (fb == 0 || fb == 1) {
+                const __nv_bfloat16* qh = (fb == 0 ? x0hi : x1hi) + md.slot;
+                const __nv_bfloat16* ql = (fb == 0 ? x0lo : x1lo) + md.slot;
+                const __nv_bfloat16* dh = dhi + md.slot;
+                const __nv_bfloat16* dl = dlo + md.slot;
+                float part = 0.f;
+                if (md.ld == md.cols && (md.cols & 7) == 0) {
+                    // contiguous rows: 8 elements per 16-byte load of each plane
+                    const int64_t base = static_cast<int64_t>(tc.y) * md.cols;
+                    const int nv = tc.z * md.cols / 8;
+                    const uint4* a4 = reinterpret_cast<const uint4*>(qh + base);
+                    const uint4* b4 = reinterpret_cast<const uint4*>(ql + base);
+                    const uint4* c4 = reinterpret_cast<const uint4*>(dh + base);
+                    const uint4* d4 = reinterpret_cast<const uint4*>(dl + base);
+                    for (int v = threadIdx.x; v < nv; v += blockDim.x) {
+                        const uint4 a = a4[v], bq = b4[v], c = c4[v], d = d4[v];
+                        const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, bw[4] = {bq.x, bq.y, bq.z, bq.w};
+                        const uint32_t cw[4] = {c.x, c.y, c.z, c.w}, dw[4] = {d.x, d.y, d.z, d.w};
+    #pragma unroll
+                        for (int w = 0; w < 4; ++w) {
+                            const float q0 = dec16(aw[w] & 0xFFFFu, true) + dec16(bw[w] & 0xFFFFu, true);
+                            const float q1 = dec16(aw[w] >> 16, true) + dec16(bw[w] >> 16, true);
+                            const float d0 = __uint_as_float(cw[w] << 16) + __uint_as_float(dw[w] << 16);
+                            const float d1 = __uint_as_float(cw[w] & 0xFFFF0000u) + __uint_as_float(dw[w] & 0xFFFF0000u);
+                            part = fmaf(q0, d0, part);
+                            part = fmaf(q1, d1, part);
+                        }
+                    }
+                } else {
+                    for (int r = tc.y; r < tc.y + tc.z; ++r) {
+                        for (int c = threadIdx.x; c < md.cols; c += blockDim.x) {
+                            const int64_t idx = static_cast<int64_t>(r) * md.ld + c;
+                            const float q = dec16(__bfloat16_as_ushort(qh[idx]), true) +
+                                            dec16(__bfloat16_as_ushort(ql[idx]), true);
+                            const float dv = __bfloat162float(dh[idx]) + __bfloat162float(dl[idx]);
+                            part = fmaf(q, dv, part);
+                        }
+                    }
+                }
+                acc = static_cast<double>(part);
+            }
+            acc = warp_sum_d(acc);
+            if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                double s = 0.0;
+                for (int i = 0; i < (int)(blockDim.x >> 5); ++i) s += red[i];
+                tpart[md.trace_part + tc.w] = s;
+            }
+            __syncthreads();  // red is reused by the next chunk
+        }
+        __syncthreads();  // todo and ntodo are rewritten by the next window
     }
 }
 
-// One warp per matrix: sigma_bar = (sum of the trace partials) / n.
-__global__ void k_trace_final(const MatDesc* __restrict__ mats, int nmat, MatState* __restrict__ state,
-                              const double* __restrict__ tpart) {
-    const int mi = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    const int lane = threadIdx.x & 31;
+// One block of 256 threads per matrix: sigma_bar = (sum of the trace partials) / n, the
+// partials from k_trace_partial's row chunks or, for a matrix whose Q-writing GEMM summed them,
+// from that GEMM's tile slots.  Fixed order: four strided accumulators per thread, then a fixed
+// tree over the threads.
+__global__ void __launch_bounds__(256) k_trace_final(const MatDesc* __restrict__ mats, int nmat,
+                                                     MatState* __restrict__ state,
+                                                     const double* __restrict__ tpart,
+                                                     const double* __restrict__ tfpart) {
+    const int mi = blockIdx.x;
     if (mi >= nmat) return;
     const MatDesc md = mats[mi];
-    double s = 0.0;
-    for (int i = lane; i < md.n_tchunks; i += 32) s += tpart[md.trace_part + i];
+    const bool fused = state[mi].trace_fused != 0;
+    const double* src = fused ? tfpart + md.tf_part : tpart + md.trace_part;
+    const int cnt = fused ? md.tf_slots : md.n_tchunks;
+    double a[4] = {0.0, 0.0, 0.0, 0.0};
+    for (int i0 = threadIdx.x; i0 < cnt; i0 += 4 * 256) {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int i = i0 + 256 * u;
+            if (i < cnt) a[u] += src[i];
+        }
+    }
+    double s = (a[0] + a[1]) + (a[2] + a[3]);
+    __shared__ double red[8];
     s = warp_sum_d(s);
-    if (lane == 0) {
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double t = 0.0;
+        for (int w = 0; w < 8; ++w) t += red[w];
         MatState& st = state[mi];
-        st.trace = s;
-        st.sigma_bar = (st.final_buf == 2) ? 0.f : static_cast<float>(s / md.n);
+        st.trace = t;
+        st.sigma_bar = (st.final_buf == 2) ? 0.f : static_cast<float>(t / md.n);
     }
 }
 
@@ -533,6 +573,7 @@ __global__ void k_reset_state(MatState* state, int nmat, uint32_t* err, const Ma
     s.xs0 = 1.f;
     s.x_hi_only = 0;
     s.trace = 0.0;
+    s.trace_fused = 0;
     state[i] = s;
 }
 

@@ -119,6 +119,13 @@ struct GemmGroup {
     // kEpiGram: per-tile partial sums, 3 floats at part[(part_base + b * tiles + tile) * 3]
     float* part;
     int64_t part_base;
+    // kEpiXSplit: when the tile writes a matrix's final Q (the polish update, the Gram side's
+    // Q = Delta Z), the tile's share of tr(Q^T Delta) = sum of Q o Delta, with Delta's bf16
+    // hi/lo planes indexed like the output; one double per epilogue warp and CTA at
+    // tf_part[(b * tiles + tile) * kPartSlots + slot].  Null d_hi: no trace here.
+    const __nv_bfloat16* d_hi;
+    const __nv_bfloat16* d_lo;
+    double* tf_part;
 };
 
 // Per-matrix state of the polar iteration (device memory, one per 2-D tensor).
@@ -141,6 +148,7 @@ struct MatState {
     int x_hi_only;    // this step's update writes X's hi plane only: the next Gram and update
                       // run single-pass and the next iteration cannot end the polar loop
     double trace;     // tr(Q^T Delta)
+    int trace_fused;  // 1: the GEMM that wrote Q also summed tr(Q^T Delta) (its tf_part slots)
 };
 
 struct GemmParams {
@@ -182,6 +190,8 @@ struct MatDesc {
     int n_tchunks;         // trace chunks of this matrix
     int gs;                // 1: Gram-side iteration (tall with rows >= kGramSideRatio * cols)
     int64_t gsslot;        // element offset of the matrix in the Gram-side n x n planes
+    int64_t tf_part;       // first of the matrix's fused-trace slots (GemmGroup::tf_part)
+    int tf_slots;          // their number: output tiles x kPartSlots
 };
 
 // A contiguous range of one parameter handled by one streaming CTA.

@@ -243,6 +243,36 @@ def test_max_iter_reports_not_converged(iso):
     assert any(s == iso.ERR_NOT_CONVERGED for s in diag["status"])
 
 
+@pytest.mark.parametrize("name, max_iter", [("tiny", 0), ("tiny", 1), ("gram_side_small", 0)])
+def test_trace_is_tr_q_delta(iso, name, max_iter):
+    """sigma_bar = tr(Q^T Delta) / r on both of its paths: summed in the epilogue of the GEMM that
+    writes a converged matrix's Q (the polish update; the Gram side's Q = Delta Z), and by the
+    separate trace pass for a matrix left unconverged (max_iter = 1).  Checked against the step's
+    own output U = alpha sigma_bar Q: sigma_bar^2 = tr(U^T Delta) / (alpha r), Delta in fp64."""
+    if name == "gram_side_small":
+        spec = W.custom_spec([("e", 1024, 96), ("d", 600, 40), ("w", 200, 200)], K=2, rank=4,
+                             shared_std=1e-3, noise_std=5e-4, momentum_std=0.0, name=name)
+        wl = W.make_workload(spec, seed=3, device="cuda")
+    else:
+        wl = W.make_workload(name, seed=0, device="cuda")
+    alpha = 0.5
+    rc, th, b, upd, diag, _ = run_gpu(iso, wl, alpha, 0.7, 0.9, max_iter=max_iter)
+    assert rc in (0, iso.ERR_NOT_CONVERGED)
+    delta = (wl.theta.double() - wl.replicas.double().mean(0)).cpu().numpy()
+    u = upd.double().cpu().numpy()
+    mats = [(o, r, c) for (o, r, c) in wl.table if c > 0]
+    checked = 0
+    for k, (o, r, c) in enumerate(mats):
+        dm = delta[o:o + r * c].reshape(r, c)
+        um = u[o:o + r * c].reshape(r, c)
+        sb = float(diag["sigma_bar"][k])
+        assert sb > 0.0, (name, max_iter, o, r, c)
+        est = np.sqrt(max(0.0, float(np.sum(um * dm))) / (alpha * min(r, c)))
+        assert abs(est / sb - 1.0) < 2e-4, (name, max_iter, r, c, est, sb)
+        checked += 1
+    assert checked == len(mats)
+
+
 def test_deterministic(iso):
     wl = W.make_workload("tiny", seed=5, device="cuda")
     plan = iso.Plan(wl.table, wl.N, wl.K)
