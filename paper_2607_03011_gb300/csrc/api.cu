@@ -864,15 +864,15 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
         LaunchSet gram;
         init_set(gram, kEpiGram, kGateActive, p, gram_pr);
         gram.p.gram_y = (first || full) ? 0 : 1;
-        // Gram-side buckets after iteration 0 (gramside.cu): W = A Z in a launch of its own, then
-        // G = Z^T W, with three passes, as groups of the main Gram launch (their split B operand
-        // sizes that launch's ring stages for three planes; its one- and two-pass tiles lose
-        // under 1 % to the shallower ring, against a launch per iteration saved)
+        // Gram-side buckets after iteration 0 (gramside.cu): W = A Z, then G = Z^T W, both with
+        // three passes in launches of their own (a split B operand would thin the main Gram's ring)
         const bool gs_iter = gs_on && !first;
-        LaunchSet wset;
+        LaunchSet wset, gsg;
         if (gs_iter) {
             init_set(wset, kEpiXSplit, kGateActive, p, Precision{1, 1, 1, 1, 0});
             wset.p.unit_scale = 1;
+            init_set(gsg, kEpiGram, kGateActive, p, Precision{1, 1, 1, 1, 0});
+            gsg.p.gram_y = 1;
         }
         for (size_t b = 0; b < p->buckets.size(); ++b) {
             const Bucket& bk = p->buckets[b];
@@ -910,7 +910,7 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
                 g.part = p->fin_part;
                 g.part_base = p->mats_h[bk.mat_base].gpart_slot;
                 set_sym(g, bk.n);
-                gram.add(g, true, true, true, true);
+                gsg.add(g, true, true);
                 continue;
             }
             const int role_a = bk.tall ? kRoleMN : kRoleKA;
@@ -939,7 +939,9 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
             gram.add(g, bk.tall, bk.tall);
         }
         int rc;
-        if (gs_iter && (rc = flush_set(p, ISOLOCO_PHASE_GRAM, wset, st))) return rc;
+        if (gs_iter && ((rc = flush_set(p, ISOLOCO_PHASE_GRAM, wset, st)) ||
+                        (rc = flush_set(p, ISOLOCO_PHASE_GRAM, gsg, st))))
+            return rc;
         if ((rc = flush_set(p, ISOLOCO_PHASE_GRAM, gram, st))) return rc;
         // after iteration 0 the Gram-side matrices need no finalize: skip an empty launch
         if (p->nftiles && (first || !gs_on || p->nftiles_reg > 0)) {
