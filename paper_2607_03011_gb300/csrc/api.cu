@@ -5,8 +5,10 @@
 //   k_reset_state -> k_reduce (Delta, all tensors)
 //   for t = 0..max_iter:   Gram X^T X (tcgen05) -> k_gram_finalize -> k_control
 //                          -> G^2 with P = a I + b G + c G^2 epilogue (tcgen05)
-//                          -> X P (tcgen05)  [matrices that finished exit at once]
-//   k_trace_partial -> k_trace_final (sigma_bar) -> k_apply (Nesterov) -> status copy
+//                          -> X P (tcgen05)  [matrices that finished exit at once; the
+//                             polish's epilogue also sums tr(Q^T Delta)]
+//   k_trace_partial (matrices left unconverged) -> k_trace_final (sigma_bar)
+//   -> k_apply (Nesterov) -> status copy
 // Every kernel reads its per-matrix decisions from device memory: the host never
 // waits inside a step.
 #include <algorithm>
@@ -1401,7 +1403,7 @@ static int run_svd(isoloco_plan* p, cudaStream_t st) {
     return ISOLOCO_OK;
 }
 
-// After the polar iteration and the trace pass (Q and sigma_bar known): Q S' in the ping-pong
+// After the polar iteration and sigma_bar's trace (Q and sigma_bar known): Q S' in the ping-pong
 // buffer that did not hold Q, and final_buf pointed at it, so that the apply pass forms
 // U = alpha sigma_bar Q S' (derivation in spectral.cu).  kind 1: clip_high, 2: clip_low.
 static int run_clip(isoloco_plan* p, int kind, int max_iter, float tol, cudaStream_t st) {

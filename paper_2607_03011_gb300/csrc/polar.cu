@@ -10,8 +10,10 @@
 //                    this iteration's polynomial: the next quintic of the schedule, the
 //                    final cubic polish, or stop.
 //  k_trace_partial / k_trace_final : sigma_bar = tr(Q^T Delta) / n (Alg. 2's mean
-//                    singular value: for the polar factor Q, Q^T Delta = V S V^T).
-//                    Q planes hold fp16 hi/lo bits, Delta planes bf16 hi/lo.
+//                    singular value: for the polar factor Q, Q^T Delta = V S V^T).  The
+//                    GEMM that writes a matrix's final Q sums its share in the epilogue
+//                    (trace_fused); the partial pass covers the other matrices, reading Q's
+//                    fp16 hi/lo planes and Delta's bf16 hi/lo planes.
 //
 // All reductions use fixed assignments and fixed shuffle trees: two runs on the same
 // inputs give bitwise-identical results.
