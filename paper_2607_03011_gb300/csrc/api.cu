@@ -53,6 +53,8 @@ __global__ void k_reset_state(MatState*, int, uint32_t*, const MatDesc*, const i
                               int*, int);
 __global__ void k_reduce(const Chunk*, const MatDesc*, ReplicaPtrs, int, int, const float*, float,
                          __nv_bfloat16*, __nv_bfloat16*, float*, uint32_t*);
+__global__ void k_reduce_f32(const Chunk*, const MatDesc*, ReplicaPtrs, int, const float*, float, __nv_bfloat16*,
+                             __nv_bfloat16*, float*, uint32_t*);
 __global__ void k_reduce_p(const Chunk*, const MatDesc*, ReplicaPtrs, int, int, const float*, float,
                            __nv_bfloat16*, __nv_bfloat16*, float*, uint32_t*, int, float, const float*, float*);
 __global__ void k_apply(const Chunk*, const MatDesc*, const MatState*, UpdateSrc, int, float, float, float,
@@ -1600,6 +1602,9 @@ static int run_isoc_step(isoloco_plan* p, int merge, float* theta, float* mom, c
             k_reduce_p<<<p->nchunks, 256, 0, st>>>(p->chunks_d, p->mats_d, rp, p->K, p->dtype, th_src, scale,
                                                    p->dhi, p->dlo, p->d1d, p->err_d, pmode, o.momentum,
                                                    hin ? hin->mom_h : mom, p->bnew);
+        else if (p->dtype == ISOLOCO_F32)
+            k_reduce_f32<<<p->nchunks, 256, 0, st>>>(p->chunks_d, p->mats_d, rp, p->K, th_src, scale, p->dhi,
+                                                     p->dlo, p->d1d, p->err_d);
         else
             k_reduce<<<p->nchunks, 256, 0, st>>>(p->chunks_d, p->mats_d, rp, p->K, p->dtype, th_src, scale, p->dhi,
                                                  p->dlo, p->d1d, p->err_d);
