@@ -272,7 +272,7 @@ DTYPE_ISO = "f32 streaming; polar GEMMs as bf16/fp16 hi+lo split passes, f32 acc
 
 # DRAM bytes (read + write) of all k_gemm_split launches of one step, from ncu captures of
 # the current kernel, (workload, fast_steps, spectrum_kind) -> figure: the 180M step's four
-# shape buckets captured one at a time and summed (profiles/k_gemm_split_dram_llama_180m_buckets.md).
+# shape buckets captured one at a time with ncu (dram__bytes_read.sum + dram__bytes_write.sum) and summed.
 GEMM_TRAFFIC = {
     ("llama_180m_k8", 0, 0): {
         "bytes_per_step": 24.45e9,
