@@ -44,7 +44,7 @@ __global__ void k_gs_final_prep(const MatDesc*, MatState*, const int*, const __n
 __global__ void k_gs_final_flip(MatState*, const int*, int);
 __global__ void k_control(const MatDesc*, int, MatState*, const float*, int, int, float, uint32_t*, const int*,
                           const int*, int, int*, int*, int*, int*, cudaGraphConditionalHandle, int, long long*,
-                          int, int*, int4, int4);
+                          int, int*, int4, int4, int);
 __global__ void k_trace_partial(const MatDesc*, const int4*, int, const MatState*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, const __nv_bfloat16*,
                                 const __nv_bfloat16*, const __nv_bfloat16*, double*);
@@ -962,7 +962,7 @@ static int polar_iteration(isoloco_plan* p, int t, int max_iter, float tol, cuda
                                       p->cnt_gram, p->list_step, p->cnt_step, cond, set_cond, p->loopc,
                                       p->fast_steps, p->counters + kLaunchCounters,
                                       make_int4(gp_one(p, 0, 0), gp_one(p, 0, 1), gp_one(p, 1, 0), gp_one(p, 1, 1)),
-                                      make_int4(up_one(p, 0, 0), up_one(p, 0, 1), up_one(p, 1, 0), up_one(p, 1, 1))); }
+                                      make_int4(up_one(p, 0, 0), up_one(p, 0, 1), up_one(p, 1, 0), up_one(p, 1, 1)), gs_on ? 1 : 0); }
         CUDA_TRY(cudaGetLastError());
         // ---- P = a I + b G + c G^2
         LaunchSet poly;

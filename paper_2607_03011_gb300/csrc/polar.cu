@@ -211,7 +211,7 @@ __device__ __forceinline__ const float* sched_row(bool deep, int step) {
 __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatState* __restrict__ state,
                                const float* __restrict__ fin_part, int t, int max_iter, float tol,
                                uint32_t* __restrict__ err, int lane, int fast_steps, int4 gram_one,
-                               int4 upd_one) {
+                               int4 upd_one, int gs_on) {
     MatState& st = state[mi];
     if (st.done) {
         if (lane == 0) st.mode = 0;
@@ -313,7 +313,9 @@ __device__ void control_matrix(const MatDesc* __restrict__ mats, int mi, MatStat
         // (Not from a single-pass Gram: the matrix then takes one more quintic step, and the
         // Gram after it, with a small residual, keeps its passes.)
         st.mode = 2;
-        st.trace_fused = md.gs ? 0 : 1;  // the polish update's epilogue sums tr(Q^T Delta)
+        // the polish update's epilogue sums tr(Q^T Delta) (a Gram-side matrix's polish writes
+        // Z, and its Q = Delta Z launch sums it instead)
+        st.trace_fused = (gs_on && md.gs) ? 0 : 1;
         st.a = 1.5f;
         st.b = static_cast<float>(-0.5 * gscale);
         st.c = 0.f;
@@ -370,11 +372,12 @@ __global__ void __launch_bounds__(kControlThreads) k_control(const MatDesc* __re
                                                              cudaGraphConditionalHandle cond, int set_cond,
                                                              long long* __restrict__ loopc, int fast_steps,
                                                              int* __restrict__ ticket, int4 gram_one,
-                                                             int4 upd_one) {
+                                                             int4 upd_one, int gs_on) {
     constexpr int kWarps = kControlThreads / 32;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     for (int mi = blockIdx.x * kWarps + warp; mi < nmat; mi += gridDim.x * kWarps) {
-        control_matrix(mats, mi, state, fin_part, t, max_iter, tol, err, lane, fast_steps, gram_one, upd_one);
+        control_matrix(mats, mi, state, fin_part, t, max_iter, tol, err, lane, fast_steps, gram_one, upd_one,
+                       gs_on);
         __syncwarp();
     }
     __threadfence();
@@ -423,9 +426,11 @@ __global__ void __launch_bounds__(kControlThreads) k_control(const MatDesc* __re
 }
 
 // Blocks of 256 threads take windows of 32 (matrix, row chunk) entries of `tchunks` (x =
-// matrix, y = first row, z = rows, w = chunk index within the matrix): the first warp checks
-// one entry per lane, and the block then sums the window's chunks whose matrix still needs its
-// trace (no GEMM epilogue summed it: trace_fused), one chunk at a time.  Q comes from the final ping-pong
+// matrix, y = first row, z = rows, w = chunk index within the matrix), window w holding the
+// entries w, w + W, w + 2W, ... (W windows; so one large matrix's chunks spread over many
+// blocks): the first warp checks one entry per lane, and the block then sums the window's
+// chunks whose matrix still needs its trace (no GEMM epilogue summed it: trace_fused), one
+// chunk at a time.  Q comes from the final ping-pong
 // buffer.
 __global__ void __launch_bounds__(256) k_trace_partial(const MatDesc* __restrict__ mats,
                                                        const int4* __restrict__ tchunks, int ntchunks,
@@ -440,9 +445,10 @@ __global__ void __launch_bounds__(256) k_trace_partial(const MatDesc* __restrict
     __shared__ double red[8];
     __shared__ int todo[32];
     __shared__ int ntodo;
-    for (int base = blockIdx.x * 32; base < ntchunks; base += gridDim.x * 32) {
+    const int nwin = (ntchunks + 31) / 32;
+    for (int win = blockIdx.x; win < nwin; win += gridDim.x) {
         if (threadIdx.x < 32) {
-            const int mine = base + static_cast<int>(threadIdx.x);
+            const int mine = win + static_cast<int>(threadIdx.x) * nwin;
             const bool need = mine < ntchunks && !state[tchunks[mine].x].trace_fused;
             const uint32_t m = __ballot_sync(0xffffffffu, need);
             if (need) todo[__popc(m & ((1u << threadIdx.x) - 1u))] = mine;
